@@ -1,0 +1,20 @@
+"""fp64 CPU oracle for the IPD verify step -- TEST INFRASTRUCTURE ONLY.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the ``cpu_baseline`` /
+``--impl reference`` legs of ``bench.py`` may import this package.  The product
+path (``paper_2609_36546_gb300``) never imports it and shares no code with it.
+
+Parity status per function (what pins it is listed in tests/test_oracle_pins.py):
+
+* ``span_attention`` / ``paged_span_attention`` -- pinned (library SDPA in
+  fp64, closed forms, paging invariants).
+* ``log_softmax_row``, ``topk``, ``covered``, ``margin`` -- pinned (scipy,
+  brute-force sort, rank identity).
+* ``topk_kl`` -- pinned (scipy KL on the renormalised support, K=1 closed
+  form, KL >= 0 and symmetry identities).
+* ``verdict`` -- pinned (hand-worked cases from the transition equation and
+  the rollback rules, exhaustive invariants).
+* ``split_loss`` -- pinned (hand-worked fixture, special cases that reduce to
+  pure on-policy and pure off-policy distillation).
+"""
+from .ipd_oracle import *  # noqa: F401,F403

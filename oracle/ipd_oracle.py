@@ -1,0 +1,295 @@
+"""Plain fp64 statement of the IPD verify step (test infrastructure only).
+
+Every function here is the textbook definition or the paper's rule written out
+in the paper's order, with no blocking, fusion or reordering.  numpy's matmul,
+sort, exp and log are the only library steps.  Inputs are bf16 bit patterns
+(uint16) or integers; bf16 -> fp64 conversion is exact.
+
+Notation follows the paper: pi = student, q = teacher, K = top-K width,
+S_t = union of both top-K supports (Sec. 3.1, "Sampled-Token and Top-K OPD";
+Sec. 4.1 fixes the union support and K = 16), m = driver state, z = token
+source (Sec. 3.2.1).
+"""
+from __future__ import annotations
+
+import numpy as np
+
+SRC_STUDENT = 0
+SRC_TEACHER = 1
+SRC_DISCARDED = 255
+
+
+# ----------------------------------------------------------------------------
+# bf16 helpers (exact conversions)
+# ----------------------------------------------------------------------------
+def bf16_to_f64(bits) -> np.ndarray:
+    """bf16 bit patterns (uint16) -> exact fp64 values."""
+    b = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)
+    return b.view(np.float32).astype(np.float64)
+
+
+def f64_to_bf16(x) -> np.ndarray:
+    """fp64 -> bf16 bit patterns, round to nearest even (via the exact fp32
+    value when it is representable; the double rounding is avoided by rounding
+    fp64 straight to 8 significant bits)."""
+    x = np.asarray(x, dtype=np.float64)
+    m, e = np.frexp(x)                       # x = m * 2**e, 0.5 <= |m| < 1
+    r = np.ldexp(np.round(np.ldexp(m, 8)), e - 8)   # np.round is half-to-even
+    return (r.astype(np.float32).view(np.uint32) >> np.uint32(16)).astype(np.uint16)
+
+
+def bf16_ulp(x) -> np.ndarray:
+    """Spacing of bf16 numbers at |x| (normal range)."""
+    x = np.abs(np.asarray(x, dtype=np.float64))
+    _, e = np.frexp(np.maximum(x, np.finfo(np.float32).tiny))
+    return np.ldexp(1.0, e - 8)
+
+
+# ----------------------------------------------------------------------------
+# (a) span-verify attention and (b) proposer decode attention
+# Sec. 3.2.3: the verifier evaluates the k draft tokens of a request in one
+# prefill pass over its own cache (only the new tokens are computed); the
+# proposer decodes one token at a time over its own cache.
+# ----------------------------------------------------------------------------
+def gather_pages(pages: np.ndarray, page_row: np.ndarray, L: int, page_size: int = 16):
+    """Paged cache [num_pages, Hkv, page_size, D] -> contiguous [L, Hkv, D]."""
+    n = (L + page_size - 1) // page_size
+    blocks = [pages[int(page_row[p])] for p in range(n)]          # each [Hkv, ps, D]
+    cont = np.concatenate([b.transpose(1, 0, 2) for b in blocks], axis=0) if n else \
+        np.zeros((0,) + (pages.shape[1], pages.shape[3]))
+    return cont[:L]
+
+
+def span_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float) -> np.ndarray:
+    """Causal attention of n span queries over a contiguous cache of L keys.
+
+    q: [n, Hq, D]; k, v: [L, Hkv, D] (fp64).  Query i sits at absolute position
+    L - n + i and sees keys 0 .. L - n + i.  Query head h reads KV head
+    h // (Hq / Hkv).  Returns [n, Hq, D] fp64.  A decode query is n = 1."""
+    n, Hq, D = q.shape
+    L, Hkv, _ = k.shape
+    G = Hq // Hkv
+    out = np.zeros((n, Hq, D))
+    for i in range(n):
+        visible = L - n + i + 1
+        for h in range(Hq):
+            kh = h // G
+            s = (k[:visible, kh, :] @ q[i, h, :]) * scale          # scores
+            s = s - s.max()
+            p = np.exp(s)
+            out[i, h, :] = (p @ v[:visible, kh, :]) / p.sum()
+    return out
+
+
+def paged_span_attention(q_bits, k_pages_bits, v_pages_bits, page_row, L, scale):
+    """span_attention on a paged cache given as bf16 bit patterns."""
+    k = gather_pages(bf16_to_f64(k_pages_bits), page_row, L)
+    v = gather_pages(bf16_to_f64(v_pages_bits), page_row, L)
+    return span_attention(bf16_to_f64(q_bits), k, v, scale)
+
+
+# ----------------------------------------------------------------------------
+# (c) the vocabulary pass over both models' logits
+# ----------------------------------------------------------------------------
+def log_partition(l: np.ndarray) -> float:
+    """log sum_v exp(l_v), with the maximum taken out first."""
+    m = l.max()
+    return float(m + np.log(np.exp(l - m).sum()))
+
+
+def topk(l: np.ndarray, K: int) -> np.ndarray:
+    """Top_K of Eq. (topk_sets): the K indices of largest probability.
+
+    Probabilities are a monotone function of the logits at temperature 1, so the
+    order is taken on the logits.  Equal logits are ordered by smaller token id
+    first, which makes the set unique."""
+    order = np.lexsort((np.arange(l.size), -l))
+    return order[:K]
+
+
+def covered(l: np.ndarray, x: int, K: int) -> bool:
+    """Coverage test of Eq. (ipd_state_transition): x in Top_K(row)."""
+    return bool(x in set(topk(l, K).tolist()))
+
+
+def margin(l: np.ndarray, x: int, K: int) -> float:
+    """l[x] minus the K-th largest logit (the coverage threshold)."""
+    return float(l[x] - l[topk(l, K)[K - 1]])
+
+
+def topk_kl(l_pi: np.ndarray, l_q: np.ndarray, K: int):
+    """Token-level top-K KL terms on the union support.
+
+    S_t = Top_K(pi) u Top_K(q) (Sec. 4.1 / App. A); pi and q are renormalised on
+    S_t separately (Eq. topk_normalization); then
+      kl_rev = KL(pi_bar || q_bar)   (Eq. topk_opd_on_sequence, l_on of Eq. ipd_off_loss)
+      kl_fwd = KL(q_bar || pi_bar)   (l_off of Eq. ipd_off_loss).
+    The full-vocabulary normaliser cancels in the renormalisation, so the
+    restricted log-sum-exp of the raw logits is used.  Terms with zero mass
+    contribute zero."""
+    S = np.union1d(topk(l_pi, K), topk(l_q, K))
+    a = l_pi[S]
+    b = l_q[S]
+    log_pi_bar = a - log_partition(a)
+    log_q_bar = b - log_partition(b)
+    pi_bar = np.exp(log_pi_bar)
+    q_bar = np.exp(log_q_bar)
+    d = log_pi_bar - log_q_bar
+    kl_rev = float(np.sum(np.where(pi_bar > 0, pi_bar * d, 0.0)))
+    kl_fwd = float(np.sum(np.where(q_bar > 0, q_bar * (-d), 0.0)))
+    return kl_rev, kl_fwd, S
+
+
+def score_position(l_s: np.ndarray, l_t: np.ndarray, x: int, driver: int, K: int) -> dict:
+    """All per-token quantities of one span position.
+
+    l_s, l_t: fp64 logits of the student (pi) and teacher (q) at this position;
+    x: the proposed token; driver 0 = student proposes (teacher verifies),
+    1 = teacher proposes (student verifies)."""
+    logZ_s = log_partition(l_s)
+    logZ_t = log_partition(l_t)
+    logp_s = float(l_s[x] - logZ_s)
+    logp_t = float(l_t[x] - logZ_t)
+    kl_rev, kl_fwd, _ = topk_kl(l_s, l_t, K)
+    ver = l_t if driver == 0 else l_s
+    return dict(
+        logp_s=logp_s, logp_t=logp_t,
+        # token-level teacher feedback: the per-token reward -l_hat^sample =
+        # log q(x) - log pi(x) (Eq. sampled_token_opd and App. B.1)
+        feedback=logp_t - logp_s,
+        kl_rev=kl_rev, kl_fwd=kl_fwd,
+        covered=covered(ver, x, K), margin=margin(ver, x, K))
+
+
+def verdict(cov, tokens, driver: int, prefix_len: int, eos_id: int = -1) -> dict:
+    """Apply Eq. (ipd_state_transition) token by token to one proposed span.
+
+    Student driving (driver 0): a covered proposal is emitted with z = S; the
+    first uncovered one is a takeover: it is rejected (the teacher regenerates
+    that position in its next proposal), both caches roll back to the token
+    before it, and the driver becomes T.  A student EOS ends the request only
+    when covered.
+    Teacher driving (driver 1): every proposal is emitted with z = T; the first
+    covered one is the handback: it is kept, the rest of the span is dropped,
+    and the driver becomes S.  A teacher EOS is accepted directly and ends the
+    request.
+    Both caches end at prefix_len + n_emit (Sec. 3.2.3, verdict stage)."""
+    k = len(cov)
+    m = driver
+    n_emit = 0
+    first_trans = k
+    done = 0
+    source = [SRC_DISCARDED] * k
+    for i in range(k):
+        x = int(tokens[i])
+        if driver == 0:
+            if cov[i]:
+                source[i] = SRC_STUDENT
+                n_emit = i + 1
+                if eos_id >= 0 and x == eos_id:
+                    done = 1
+                    break
+            else:
+                first_trans = i
+                m = 1
+                break
+        else:
+            source[i] = SRC_TEACHER
+            n_emit = i + 1
+            if cov[i]:
+                first_trans = i
+                m = 0
+            if eos_id >= 0 and x == eos_id:
+                done = 1
+            if cov[i] or done:
+                break
+    return dict(first_trans=first_trans, n_emit=n_emit, next_driver=m,
+                new_len=prefix_len + n_emit, done=done, source=source)
+
+
+def score_span(logits_s_bits, logits_t_bits, tokens, cu_span, driver, prefix_len, K, eos_id=-1,
+               requests=None) -> dict:
+    """The whole vocabulary pass + verdict for the requests in ``requests``
+    (default: all).  Per-token arrays are returned in the flat span order, with
+    NaN / -1 at positions of requests that were not evaluated."""
+    T = int(cu_span[-1])
+    R = len(cu_span) - 1
+    reqs = range(R) if requests is None else requests
+    out = {name: np.full(T, np.nan) for name in
+           ("logp_s", "logp_t", "feedback", "kl_rev", "kl_fwd", "margin")}
+    out["covered"] = np.full(T, -1, dtype=np.int64)
+    out["source"] = np.full(T, -1, dtype=np.int64)
+    for name in ("first_trans", "n_emit", "next_driver", "new_len", "done"):
+        out[name] = np.full(R, -1, dtype=np.int64)
+    for r in reqs:
+        t0, t1 = int(cu_span[r]), int(cu_span[r + 1])
+        cov = []
+        for t in range(t0, t1):
+            pos = score_position(bf16_to_f64(logits_s_bits[t]), bf16_to_f64(logits_t_bits[t]),
+                                 int(tokens[t]), int(driver[r]), K)
+            for name in ("logp_s", "logp_t", "feedback", "kl_rev", "kl_fwd", "margin"):
+                out[name][t] = pos[name]
+            out["covered"][t] = int(pos["covered"])
+            cov.append(pos["covered"])
+        v = verdict(cov, tokens[t0:t1], int(driver[r]), int(prefix_len[r]), eos_id)
+        out["source"][t0:t1] = v["source"]
+        for name in ("first_trans", "n_emit", "next_driver", "new_len", "done"):
+            out[name][r] = v[name]
+    return out
+
+
+# ----------------------------------------------------------------------------
+# source-split reduction
+# ----------------------------------------------------------------------------
+DIR_IPD, DIR_PURE_REV, DIR_PURE_FWD, DIR_INVERSE = 0, 1, 2, 3
+
+
+def split_loss(kl_rev, kl_fwd, source, cu_span, n_emit, resp_len=None, agg_mode=0,
+               dir_mode=DIR_IPD) -> dict:
+    """Source-split objective of Eq. (ipd_objective) for one step.
+
+    Student-sourced positions (z = S) take l_on, teacher-sourced ones (z = T)
+    take l_off (Eq. ipd_off_loss).  dir_mode selects the KL direction of each
+    group as in the KL-direction ablation (Sec. 4.3): 0 IPD split (on: reverse,
+    off: forward), 1 pure reverse, 2 pure forward, 3 inverse split.
+    agg_mode 0 is the sequence-mean-token-mean of Eq. (ipd_objective): each
+    request's sum is divided by its length |x_r| (resp_len, or the emitted
+    count when resp_len is None) and requests with |x_r| = 0 are left out of
+    the batch mean; agg_mode 1 is the global token mean (App. B.3).
+    Returns the loss, the per-source sums and counts, the teacher intervention
+    ratio (share of teacher-sourced tokens, Sec. 4.3) and the numerator /
+    denominator whose ratio is the loss (so shards can be combined)."""
+    on_rev = dir_mode in (DIR_IPD, DIR_PURE_REV)
+    off_fwd = dir_mode in (DIR_IPD, DIR_PURE_FWD)
+    R = len(cu_span) - 1
+    sum_on = sum_off = 0.0
+    n_on = n_off = 0
+    per_req = []
+    denoms = []
+    for r in range(R):
+        s_on = s_off = 0.0
+        for t in range(int(cu_span[r]), int(cu_span[r + 1])):
+            if source[t] == SRC_STUDENT:
+                s_on += kl_rev[t] if on_rev else kl_fwd[t]
+                n_on += 1
+            elif source[t] == SRC_TEACHER:
+                s_off += kl_fwd[t] if off_fwd else kl_rev[t]
+                n_off += 1
+        sum_on += s_on
+        sum_off += s_off
+        d = int(n_emit[r]) if resp_len is None else int(resp_len[r])
+        per_req.append(s_on + s_off)
+        denoms.append(d)
+    if agg_mode == 0:
+        terms = [per_req[r] / denoms[r] for r in range(R) if denoms[r] > 0]
+        numer, denom = float(sum(terms)), float(len(terms))
+    else:
+        numer = float(sum(per_req[r] for r in range(R) if denoms[r] > 0))
+        denom = float(sum(d for d in denoms if d > 0))
+    loss = numer / denom if denom > 0 else 0.0
+    ntot = n_on + n_off
+    return dict(loss=loss, sum_on=sum_on, sum_off=sum_off, n_on=float(n_on), n_off=float(n_off),
+                intervention_ratio=(n_off / ntot) if ntot else 0.0, numer=numer, denom=denom)
+
+
+LOSS_FIELDS = ("loss", "sum_on", "sum_off", "n_on", "n_off", "intervention_ratio", "numer", "denom")

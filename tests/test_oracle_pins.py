@@ -1,0 +1,413 @@
+"""Pins of the fp64 oracle to things other than itself (CPU only).
+
+Each test fixes an oracle function against a library routine written by
+someone else, a closed form, a hand-worked fixture from the paper's rules, a
+brute force on tiny inputs, or an invariant the mathematics guarantees.  The
+``test_planted_*`` tests plant a plausible mistake in a copy of the oracle's
+inputs/outputs and check that the pin notices.
+"""
+import itertools
+import math
+import os
+
+import numpy as np
+import pytest
+import scipy.special
+import scipy.stats
+import torch
+
+import oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+RNG = np.random.default_rng(1234)
+
+
+def _bf16_round(x):
+    return O.bf16_to_f64(O.f64_to_bf16(x))
+
+
+# ---------------------------------------------------------------------------
+# bf16 conversions against torch's own
+# ---------------------------------------------------------------------------
+def test_bf16_conversions_match_torch():
+    x = np.concatenate([RNG.normal(size=4000) * 10 ** RNG.uniform(-6, 6, size=4000),
+                        [0.0, -0.0, 1.0, -2.5, 1.00390625, 1.01171875]])
+    ours = O.f64_to_bf16(x)
+    ref = torch.from_numpy(x).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(ours, ref)
+    back = O.bf16_to_f64(ref)
+    assert np.array_equal(back, torch.from_numpy(ref.view(np.int16)).view(torch.bfloat16)
+                          .to(torch.float64).numpy())
+
+
+# ---------------------------------------------------------------------------
+# attention
+# ---------------------------------------------------------------------------
+def _sdpa_reference(q, k, v, scale):
+    """torch's scaled_dot_product_attention in fp64 with an explicit span mask."""
+    n, Hq, D = q.shape
+    L, Hkv, _ = k.shape
+    G = Hq // Hkv
+    qt = torch.from_numpy(q).permute(1, 0, 2)                         # [Hq, n, D]
+    kt = torch.from_numpy(k).permute(1, 0, 2).repeat_interleave(G, 0)  # [Hq, L, D]
+    vt = torch.from_numpy(v).permute(1, 0, 2).repeat_interleave(G, 0)
+    pos_q = torch.arange(n)[:, None] + (L - n)
+    mask = torch.arange(L)[None, :] <= pos_q                          # [n, L]
+    o = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, attn_mask=mask, scale=scale)
+    return o.permute(1, 0, 2).numpy()
+
+
+@pytest.mark.parametrize("n,L,Hq,Hkv", [(1, 1, 4, 2), (1, 37, 8, 4), (4, 40, 32, 4),
+                                        (7, 7, 16, 8), (16, 90, 8, 8)])
+def test_attention_matches_library_sdpa(n, L, Hq, Hkv):
+    q = RNG.normal(size=(n, Hq, 128))
+    k = RNG.normal(size=(L, Hkv, 128))
+    v = RNG.normal(size=(L, Hkv, 128))
+    s = 1 / math.sqrt(128)
+    np.testing.assert_allclose(O.span_attention(q, k, v, s), _sdpa_reference(q, k, v, s),
+                               rtol=1e-12, atol=1e-12)
+
+
+def test_attention_single_key_returns_value():
+    q = RNG.normal(size=(1, 8, 128))
+    k = RNG.normal(size=(1, 2, 128))
+    v = RNG.normal(size=(1, 2, 128))
+    o = O.span_attention(q, k, v, 0.1)
+    for h in range(8):
+        np.testing.assert_array_equal(o[0, h], v[0, h // 4])
+
+
+def test_attention_equal_keys_average_exactly_the_visible_values():
+    n, L = 5, 23
+    q = RNG.normal(size=(n, 4, 128))
+    k = np.repeat(RNG.normal(size=(1, 1, 128)), L, 0).repeat(2, 1)
+    v = RNG.normal(size=(L, 2, 128))
+    o = O.span_attention(q, k, v, 0.3)
+    for i in range(n):
+        vis = L - n + i + 1
+        for h in range(4):
+            np.testing.assert_allclose(o[i, h], v[:vis, h // 2].mean(0), rtol=1e-12, atol=1e-13)
+
+
+def test_attention_gqa_head_mapping():
+    L, Hq, Hkv = 9, 32, 4
+    v = np.zeros((L, Hkv, 128))
+    for j in range(Hkv):
+        v[:, j, :] = j + 1.0
+    o = O.span_attention(RNG.normal(size=(2, Hq, 128)), RNG.normal(size=(L, Hkv, 128)), v, 0.2)
+    for h in range(Hq):
+        np.testing.assert_allclose(o[:, h, :], h // 8 + 1.0, rtol=1e-13)
+
+
+def test_attention_scale_two_keys_closed_form():
+    a, scale = 3.7, 1 / math.sqrt(128)
+    q = np.zeros((1, 1, 128)); q[0, 0, 0] = a
+    k = np.zeros((2, 1, 128)); k[0, 0, 0] = 1.0
+    v = RNG.normal(size=(2, 1, 128))
+    w0 = math.exp(a * scale) / (math.exp(a * scale) + 1.0)
+    np.testing.assert_allclose(O.span_attention(q, k, v, scale)[0, 0],
+                               w0 * v[0, 0] + (1 - w0) * v[1, 0], rtol=1e-13)
+
+
+def test_attention_is_causal_within_span():
+    n, L = 6, 30
+    q = RNG.normal(size=(n, 4, 128)); k = RNG.normal(size=(L, 2, 128)); v = RNG.normal(size=(L, 2, 128))
+    o = O.span_attention(q, k, v, 0.09)
+    k2, v2 = k.copy(), v.copy()
+    k2[-2:] += 5.0; v2[-2:] -= 3.0           # perturb the last two span keys
+    o2 = O.span_attention(q, k2, v2, 0.09)
+    np.testing.assert_array_equal(o[:n - 2], o2[:n - 2])
+    assert np.abs(o[n - 2:] - o2[n - 2:]).min() > 0
+
+
+def _paged(k, v, ps=16, rng=RNG, extra_pages=5):
+    L, Hkv, D = k.shape
+    npg = (L + ps - 1) // ps
+    pool = npg + extra_pages
+    perm = rng.permutation(pool)[:npg]
+    kp = rng.normal(size=(pool, Hkv, ps, D)); vp = rng.normal(size=(pool, Hkv, ps, D))
+    for p in range(npg):
+        seg = slice(p * ps, min(L, (p + 1) * ps))
+        cnt = seg.stop - seg.start
+        kp[perm[p], :, :cnt, :] = k[seg].transpose(1, 0, 2)
+        vp[perm[p], :, :cnt, :] = v[seg].transpose(1, 0, 2)
+    return kp, vp, perm
+
+
+@pytest.mark.parametrize("L", [1, 15, 16, 17, 100])
+def test_paged_equals_contiguous_and_page_permutation_is_invisible(L):
+    n = min(L, 4)
+    q = RNG.normal(size=(n, 8, 128)); k = RNG.normal(size=(L, 4, 128)); v = RNG.normal(size=(L, 4, 128))
+    ref = O.span_attention(q, k, v, 0.088)
+    for seed in (0, 1):
+        kp, vp, row = _paged(k, v, rng=np.random.default_rng(seed))
+        kk = O.gather_pages(kp, row, L); vv = O.gather_pages(vp, row, L)
+        np.testing.assert_array_equal(kk, k)
+        np.testing.assert_array_equal(O.span_attention(q, kk, vv, 0.088), ref)
+
+
+# ---------------------------------------------------------------------------
+# log-softmax, top-K, coverage
+# ---------------------------------------------------------------------------
+def test_log_partition_library_normalisation_and_shift():
+    for V in (5, 4096):
+        l = _bf16_round(RNG.normal(size=V) * 3)
+        lz = O.log_partition(l)
+        assert abs(lz - scipy.special.logsumexp(l)) < 1e-12
+        assert abs(np.exp(l - lz).sum() - 1.0) < 1e-12
+        assert abs(O.log_partition(l + 8.0) - (lz + 8.0)) < 1e-12
+
+
+def _brute_topk(l, K):
+    return [v for _, v in sorted((-l[v], v) for v in range(len(l)))][:K]
+
+
+@pytest.mark.parametrize("quantum", [0.0, 0.5, 2.0])
+def test_topk_matches_brute_force_sort_with_ties(quantum):
+    for _ in range(20):
+        V = int(RNG.integers(33, 300))
+        l = RNG.normal(size=V) * 3
+        if quantum:
+            l = np.round(l / quantum) * quantum
+        l = _bf16_round(l)
+        for K in (1, 4, 16, 32):
+            assert O.topk(l, K).tolist() == _brute_topk(l, K)
+
+
+def test_covered_equals_rank_identity_and_margin_sign():
+    for _ in range(10):
+        V = int(RNG.integers(40, 120))
+        l = _bf16_round(np.round(RNG.normal(size=V) * 2) / 2)
+        for K in (1, 3, 16):
+            top = set(O.topk(l, K).tolist())
+            for x in range(V):
+                rank = int(np.sum(l > l[x]) + np.sum(l[:x] == l[x]))
+                cov = O.covered(l, x, K)
+                assert cov == (rank < K) == (x in top)
+                m = O.margin(l, x, K)
+                if m > 0:
+                    assert cov
+                if m < 0:
+                    assert not cov
+
+
+# ---------------------------------------------------------------------------
+# top-K KL on the union support
+# ---------------------------------------------------------------------------
+def test_topk_kl_matches_scipy_entropy():
+    for _ in range(30):
+        V, K = int(RNG.integers(20, 200)), int(RNG.choice([1, 4, 16]))
+        a = _bf16_round(RNG.normal(size=V) * 2)
+        b = _bf16_round(RNG.normal(size=V) * 2)
+        kl_rev, kl_fwd, S = O.topk_kl(a, b, K)
+        assert K <= len(S) <= 2 * K
+        assert set(S) == set(_brute_topk(a, K)) | set(_brute_topk(b, K))
+        pbar = scipy.special.softmax(a[S]); qbar = scipy.special.softmax(b[S])
+        assert abs(kl_rev - scipy.stats.entropy(pbar, qbar)) < 1e-12
+        assert abs(kl_fwd - scipy.stats.entropy(qbar, pbar)) < 1e-12
+
+
+def test_topk_kl_invariants():
+    for _ in range(20):
+        V = 300
+        a = _bf16_round(RNG.normal(size=V) * 3); b = _bf16_round(RNG.normal(size=V) * 3)
+        r, f, _ = O.topk_kl(a, b, 16)
+        assert r >= 0 and f >= 0
+        r2, f2, _ = O.topk_kl(b, a, 16)
+        assert abs(r - f2) < 1e-12 and abs(f - r2) < 1e-12
+        z = O.topk_kl(a, a, 16)
+        assert z[0] == 0.0 and z[1] == 0.0
+        # a constant shift of one model's row leaves the renormalised KL unchanged
+        s = O.topk_kl(a + 4.0, b, 16)
+        assert abs(s[0] - r) < 1e-12
+
+
+def test_topk_kl_K1_closed_form():
+    for _ in range(50):
+        a = _bf16_round(RNG.normal(size=50) * 2); b = _bf16_round(RNG.normal(size=50) * 2)
+        ia, ib = int(O.topk(a, 1)[0]), int(O.topk(b, 1)[0])
+        r, f, S = O.topk_kl(a, b, 1)
+        if ia == ib:
+            assert len(S) == 1 and r == 0.0 and f == 0.0
+            continue
+        lo, hi = min(ia, ib), max(ia, ib)
+        p = 1 / (1 + math.exp(a[hi] - a[lo]))     # pi_bar(lo)
+        s = 1 / (1 + math.exp(b[hi] - b[lo]))     # q_bar(lo)
+        bern = p * math.log(p / s) + (1 - p) * math.log((1 - p) / (1 - s))
+        assert abs(r - bern) < 1e-12 * max(1.0, abs(bern))
+
+
+def test_sampled_token_estimator_is_unbiased_by_enumeration():
+    """App. B.1: E_{x~pi}[log pi(x) - log q(x)] equals the full-vocabulary reverse
+    KL.  The per-token log-probs of score_position are enumerated over every
+    token of a tiny vocabulary; the feedback term is minus the estimator."""
+    for _ in range(10):
+        V = 7
+        a = _bf16_round(RNG.normal(size=V) * 2); b = _bf16_round(RNG.normal(size=V) * 2)
+        pi = scipy.special.softmax(a)
+        est = 0.0
+        for x in range(V):
+            pos = O.score_position(a, b, x, 0, 3)
+            assert abs(pos["feedback"] + (pos["logp_s"] - pos["logp_t"])) < 1e-15
+            est += pi[x] * (pos["logp_s"] - pos["logp_t"])
+        assert abs(est - scipy.stats.entropy(pi, scipy.special.softmax(b))) < 1e-12
+
+
+# ---------------------------------------------------------------------------
+# verdict
+# ---------------------------------------------------------------------------
+def _load_verdict_cases():
+    cases = []
+    for line in open(os.path.join(GOLDEN, "verdict_cases.txt")):
+        line = line.split("#")[0].strip()
+        if not line:
+            continue
+        lhs, rhs = line.split("|")
+        d, cov, eos, pre = lhs.split()
+        n, ft, nd, nl, done, src = rhs.split()
+        cases.append((d, cov, eos, int(pre), int(n), int(ft), nd, int(nl), int(done), src))
+    return cases
+
+
+@pytest.mark.parametrize("case", _load_verdict_cases())
+def test_verdict_hand_worked_cases(case):
+    d, cov, eos, pre, n, ft, nd, nl, done, src = case
+    EOS = 99
+    k = len(cov)
+    toks = [7] * k
+    if eos != "-":
+        for p in eos.split(","):
+            toks[int(p)] = EOS
+    v = O.verdict([c == "1" for c in cov], toks, 0 if d == "S" else 1, pre, EOS)
+    assert v["n_emit"] == n and v["first_trans"] == ft and v["new_len"] == nl
+    assert v["next_driver"] == (0 if nd == "S" else 1) and v["done"] == done
+    code = {"S": O.SRC_STUDENT, "T": O.SRC_TEACHER, "-": O.SRC_DISCARDED}
+    assert v["source"] == [code[c] for c in src]
+
+
+def test_verdict_exhaustive_invariants():
+    for k in range(1, 9):
+        for bits in itertools.product([0, 1], repeat=k):
+            for d in (0, 1):
+                v = O.verdict(list(bits), [1] * k, d, 10)
+                lead = next((i for i, b in enumerate(bits) if b != (1 if d == 0 else 0)), k)
+                if d == 0:
+                    assert v["n_emit"] == lead and v["first_trans"] == lead
+                else:
+                    assert v["first_trans"] == lead and v["n_emit"] == min(k, lead + 1)
+                assert v["next_driver"] == (1 - d if lead < k else d)
+                assert v["new_len"] == 10 + v["n_emit"] and v["done"] == 0
+                assert v["source"][:v["n_emit"]] == [d] * v["n_emit"]
+                assert all(s == O.SRC_DISCARDED for s in v["source"][v["n_emit"]:])
+
+
+# ---------------------------------------------------------------------------
+# source-split loss
+# ---------------------------------------------------------------------------
+_R0 = dict(src=[0, 0, 255], rev=[0.5, 0.25, 9.0], fwd=[1.0, 2.0, 9.0], n=2)
+_R1 = dict(src=[1, 1, 1], rev=[3.0, 1.0, 2.0], fwd=[0.75, 0.25, 0.5], n=3)
+
+
+def _golden_loss_inputs():
+    src = np.array(_R0["src"] + _R1["src"])
+    return (np.array(_R0["rev"] + _R1["rev"]), np.array(_R0["fwd"] + _R1["fwd"]), src,
+            np.array([0, 3, 6]), np.array([_R0["n"], _R1["n"]]))
+
+
+def _load_loss_cases():
+    out = []
+    for line in open(os.path.join(GOLDEN, "split_loss_cases.txt")):
+        line = line.split("#")[0].strip()
+        if line:
+            lhs, rhs = line.split("|")
+            dm, am, rl = lhs.split()
+            out.append((int(dm), int(am), None if rl == "-" else [int(x) for x in rl.split(",")],
+                        [float(x) for x in rhs.split()]))
+    return out
+
+
+@pytest.mark.parametrize("case", _load_loss_cases())
+def test_split_loss_hand_worked(case):
+    dm, am, rl, expect = case
+    rev, fwd, src, cu, n = _golden_loss_inputs()
+    out = O.split_loss(rev, fwd, src, cu, n, None if rl is None else np.array(rl), am, dm)
+    got = [out[f] for f in O.LOSS_FIELDS[:6]]
+    np.testing.assert_allclose(got, expect, rtol=0, atol=1e-15)
+
+
+def _random_step(rng, R, k, driver, V=64, K=4):
+    ls = rng.normal(size=(R * k, V)) * 2
+    lt = rng.normal(size=(R * k, V)) * 2
+    bits_s = O.f64_to_bf16(ls); bits_t = O.f64_to_bf16(lt)
+    toks = rng.integers(0, V, size=R * k)
+    cu = np.arange(R + 1) * k
+    return bits_s, bits_t, toks, cu
+
+
+def test_never_transfer_reduces_to_reverse_kl_opd():
+    """Sec. 3.2.2: if control never passes to the teacher, the objective is the
+    length-normalised reverse-KL on-policy distillation."""
+    rng = np.random.default_rng(5)
+    R, k, K = 3, 4, 4
+    bs, bt, toks, cu = _random_step(rng, R, k, 0, K=K)
+    # make every proposal covered: raise the teacher's logit of the proposed token
+    lt = O.bf16_to_f64(bt)
+    lt[np.arange(R * k), toks] = 40.0
+    bt = O.f64_to_bf16(lt)
+    out = O.score_span(bs, bt, toks, cu, np.zeros(R, int), np.full(R, 50), K)
+    assert (out["source"] == O.SRC_STUDENT).all()
+    loss = O.split_loss(out["kl_rev"], out["kl_fwd"], out["source"], cu, out["n_emit"])
+    opd = np.mean([np.mean(out["kl_rev"][cu[r]:cu[r + 1]]) for r in range(R)])
+    assert abs(loss["loss"] - opd) < 1e-12 and loss["intervention_ratio"] == 0.0
+
+
+def test_teacher_that_never_hands_back_reduces_to_forward_kl():
+    """Sec. 3.2.2: rejecting the first student token and never handing back
+    gives forward-KL off-policy distillation on teacher tokens."""
+    rng = np.random.default_rng(6)
+    R, k, K = 3, 5, 4
+    bs, bt, toks, cu = _random_step(rng, R, k, 1, K=K)
+    ls = O.bf16_to_f64(bs)
+    ls[np.arange(R * k), toks] = -40.0          # never covered by the student
+    bs = O.f64_to_bf16(ls)
+    out = O.score_span(bs, bt, toks, cu, np.ones(R, int), np.zeros(R, int), K)
+    assert (out["source"] == O.SRC_TEACHER).all()
+    loss = O.split_loss(out["kl_rev"], out["kl_fwd"], out["source"], cu, out["n_emit"])
+    fwd = np.mean([np.mean(out["kl_fwd"][cu[r]:cu[r + 1]]) for r in range(R)])
+    assert abs(loss["loss"] - fwd) < 1e-12 and loss["intervention_ratio"] == 1.0
+
+
+def test_global_mean_equals_seq_mean_for_equal_lengths():
+    rng = np.random.default_rng(7)
+    R, k = 5, 3
+    rev = rng.random(R * k); fwd = rng.random(R * k)
+    src = rng.integers(0, 2, size=R * k)
+    cu = np.arange(R + 1) * k
+    n = np.full(R, k)
+    a = O.split_loss(rev, fwd, src, cu, n, agg_mode=0)
+    b = O.split_loss(rev, fwd, src, cu, n, agg_mode=1)
+    assert abs(a["loss"] - b["loss"]) < 1e-12
+
+
+# ---------------------------------------------------------------------------
+# planted mistakes: each must be caught by a pin above
+# ---------------------------------------------------------------------------
+def test_planted_mistakes_are_caught():
+    q = RNG.normal(size=(3, 8, 128)); k = RNG.normal(size=(20, 4, 128)); v = RNG.normal(size=(20, 4, 128))
+    ref = _sdpa_reference(q, k, v, 0.1)
+    # off-by-one causal window (one extra key) is caught by the library pin
+    bad = np.zeros_like(ref)
+    for i in range(3):
+        vis = 20 - 3 + i + 2
+        for h in range(8):
+            kk = k[:min(vis, 20), h // 2]; s = kk @ q[i, h] * 0.1; p = np.exp(s - s.max())
+            bad[i, h] = p @ v[:min(vis, 20), h // 2] / p.sum()
+    assert not np.allclose(bad, ref, atol=1e-9)
+    # a wrong tie-break (larger index first) is caught by the brute-force sort
+    l = _bf16_round(np.array([1.0, 2.0, 2.0, 0.5, 2.0]))
+    wrong = np.lexsort((-np.arange(5), -l))[:2].tolist()
+    assert wrong != _brute_topk(l, 2) == O.topk(l, 2).tolist()
+    # a swapped KL direction is caught by the scipy pin
+    a = _bf16_round(RNG.normal(size=40)); b = _bf16_round(RNG.normal(size=40) * 3)
+    r, f, S = O.topk_kl(a, b, 4)
+    assert abs(f - scipy.stats.entropy(scipy.special.softmax(a[S]), scipy.special.softmax(b[S]))) > 1e-6
