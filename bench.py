@@ -1,0 +1,462 @@
+"""Verify-step benchmark: verified tokens/s on one GB300 (and N replicas).
+
+One step = the whole hot path on one batch: ipd_verify_attn (span-verify
+attention on the verifier's cache co-launched with the proposer's decode
+attention), ipd_score_span (vocabulary pass + verdict) and ipd_split_loss.
+Inputs are synthetic, seeded, resident in HBM and larger than L2, so every
+step streams its KV pages and logits from DRAM.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config I] [--impl reference]
+
+Prints one JSON line (rank 0).  ``--impl reference`` times the fp64 CPU
+oracle (the only reference that exists for this path) on a bounded sample of
+the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import multiprocessing as mp
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "verified tokens/s on 1 GB300; achieved HBM GB/s as % of peak"
+UNIT = "tokens/s"
+HBM_FALLBACK_GBS = 6800.0
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return HBM_FALLBACK_GBS, "fallback"
+
+
+def _workload_name(cfg: int) -> str:
+    import ipd_synth as S
+    s = S.CONFIGS[cfg]
+    return (f"configs[{cfg}] {s.name}: {s.n_req} requests, ctx {s.ctx}, span {s.span}, "
+            f"direction {s.direction}, teacher 32Q/4KV + student 16Q/8KV heads, head_dim 128, "
+            f"page 16, vocab {s.vocab}, logits '{s.logits}', K={s.K}, one attention layer per model")
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-i", str(index)], stdout=subprocess.PIPE,
+                stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, smax, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax),
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def _smi_index(local_rank: int) -> int:
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+    ids = [v for v in vis.split(",") if v.strip()]
+    if ids and all(v.strip().isdigit() for v in ids) and local_rank < len(ids):
+        return int(ids[local_rank])
+    try:
+        n = len(subprocess.run(["nvidia-smi", "-L"], capture_output=True, text=True,
+                               timeout=10).stdout.strip().splitlines())
+        if n == 1:
+            return 0
+    except Exception:
+        pass
+    return local_rank
+
+
+# ---------------------------------------------------------------------------
+# oracle timing (cpu_baseline and --impl reference)
+# ---------------------------------------------------------------------------
+def _oracle_request(payload):
+    """The oracle's full path for one request: verify + decode attention,
+    the vocabulary pass of every span position, the verdict and the loss."""
+    import numpy as np
+    import oracle as O
+    t0 = time.perf_counter()
+    for q, kp, vp, L in payload["attn"]:
+        O.paged_span_attention(q, kp, vp, np.arange(kp.shape[0]), L, payload["scale"])
+    k = payload["ls"].shape[0]
+    out = O.score_span(payload["ls"], payload["lt"], payload["tokens"], np.array([0, k]),
+                       np.array([payload["driver"]]), np.array([payload["prefix"]]),
+                       payload["K"], payload["eos"])
+    O.split_loss(out["kl_rev"], out["kl_fwd"], out["source"], np.array([0, k]), out["n_emit"])
+    return k, time.perf_counter() - t0
+
+
+def _request_payload(step, w, r):
+    import numpy as np
+    import torch
+    from tests.parity import u16
+    pay = {"attn": [], "scale": step.scale, "K": step.K, "eos": step.eos_id,
+           "driver": int(w.driver[r]), "prefix": int(w.ctx[r] - w.span[r])}
+    for name, b, idx, cache in step.batches:
+        pos = (idx == r).nonzero().flatten()
+        if pos.numel() == 0:
+            continue
+        j = int(pos[0])
+        q, cu_q, seq, ptab, _ = b._keep
+        cu = cu_q.cpu()
+        L = int(seq[j])
+        npg = (L + 15) // 16
+        pages = ptab[j, :npg].to(torch.int64)
+        c = step.cache_t if cache == "teacher" else step.cache_s
+        pay["attn"].append((u16(q[int(cu[j]):int(cu[j + 1])]), u16(c.k_pages.index_select(0, pages)),
+                            u16(c.v_pages.index_select(0, pages)), L))
+    t0, t1 = int(step.cu_span[r]), int(step.cu_span[r + 1])
+    pay["ls"] = u16(step.logits_s[t0:t1])
+    pay["lt"] = u16(step.logits_t[t0:t1])
+    pay["tokens"] = step.tokens[t0:t1].cpu().numpy()
+    return pay
+
+
+def cpu_baseline(step, w, budget_s: float = 25.0) -> dict:
+    """The oracle on the host cores (a spawn pool, one request per task) on a
+    bounded sample of the same workload: whole requests, taken in order."""
+    cores = max(1, min(os.cpu_count() or 1, 32))
+    ctx = mp.get_context("spawn")
+    env_keep = {k: os.environ.get(k) for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS",
+                                               "MKL_NUM_THREADS")}
+    for k in env_keep:
+        os.environ[k] = "1"
+    try:
+        with ctx.Pool(cores) as pool:
+            # one request alone first, to size the sample to the budget
+            first = _request_payload(step, w, 0)
+            k0, t_one = pool.apply(_oracle_request, (first,))
+            n_req = max(1, min(step.R, int(budget_s / max(t_one, 1e-3) * cores * 0.8)))
+            n_req = max(cores, n_req) if step.R >= cores else step.R
+            n_req = min(n_req, step.R)
+            payloads = [_request_payload(step, w, r) for r in range(n_req)]
+            t0 = time.perf_counter()
+            res = pool.map(_oracle_request, payloads, chunksize=1)
+            wall = time.perf_counter() - t0
+    finally:
+        for k, v in env_keep.items():
+            if v is None:
+                os.environ.pop(k, None)
+            else:
+                os.environ[k] = v
+    toks = sum(k for k, _ in res)
+    return {"value": toks / wall, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"first {n_req} of {step.R} requests ({toks} span tokens), whole oracle path "
+                      f"per request (attention of both caches, vocabulary pass, verdict, loss), "
+                      f"numpy fp64, one process per core, BLAS single-threaded; wall {wall:.1f} s"}
+
+
+# ---------------------------------------------------------------------------
+def _init_dist(args):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group("nccl", rank=rank, world_size=world,
+                                device_id=torch.device("cuda", local))
+    return world, rank, local
+
+
+def _barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def _max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def _sum_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def run_reference(args):
+    """--impl reference: the fp64 oracle on the host, one verified token per
+    step (its verifier attention query, the request's decode query, the
+    vocabulary pass of its two logits rows, verdict and loss)."""
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import numpy as np
+    import ipd_synth as S
+    import oracle as O
+    # a small resident sample of the workload, generated on the host
+    spec = S.CONFIGS[args.config]
+    n_req = 2
+    sample_spec = S.Spec(spec.name + " (sample)", n_req, spec.ctx, spec.span, "S" if spec.direction
+                         in ("S", "half", "bernoulli") else "T", spec.vocab, spec.logits,
+                         sigma=spec.sigma, K=spec.K)
+    w = S.make_workload(sample_spec, seed=args.config, device="cpu")
+    from tests.parity import u16
+    scale = 1.0 / math.sqrt(128.0)
+    toks = w.tokens.numpy()
+    cu = w.cu_span.numpy()
+    ls, lt = u16(w.logits_s), u16(w.logits_t)
+
+    def one_token(i):
+        r = i % n_req
+        t = int(cu[r]) + (i // n_req) % int(w.span[r])
+        pos = t - int(cu[r])
+        L = int(w.ctx[r])
+        npg = (L + 15) // 16
+        ver, prop = (w.teacher, w.student) if int(w.driver[r]) == 0 else (w.student, w.teacher)
+        qv = w.q_verify_t if int(w.driver[r]) == 0 else w.q_verify_s
+        qd = w.q_decode_s if int(w.driver[r]) == 0 else w.q_decode_t
+        rows = ver.page_table[r, :npg].long()
+        prow = prop.page_table[r, :npg].long()
+        qi = u16(qv[t:t + 1])
+        O.paged_span_attention(qi, u16(ver.k_pages[rows]), u16(ver.v_pages[rows]),
+                               np.arange(npg), L - int(w.span[r]) + pos + 1, scale)
+        O.paged_span_attention(u16(qd[r:r + 1]), u16(prop.k_pages[prow]), u16(prop.v_pages[prow]),
+                               np.arange(npg), L, scale)
+        out = O.score_span(ls[t:t + 1], lt[t:t + 1], toks[t:t + 1], np.array([0, 1]),
+                           w.driver[r:r + 1].numpy(), np.array([L - 1]), w.spec.K, -1)
+        O.split_loss(out["kl_rev"], out["kl_fwd"], out["source"], np.array([0, 1]), out["n_emit"])
+
+    for i in range(args.warmup):
+        one_token(i)
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        one_token(args.warmup + i)
+    el = time.perf_counter() - t0
+    value = args.steps / el
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * el / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": _workload_name(args.config)},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": "one verified token per step (its verify query over the "
+                                       "verifier cache, the request's decode query, both logits "
+                                       "rows, verdict, loss), 2 host-generated requests of the "
+                                       "workload's shape, cycled"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_gpu(args):
+    import torch
+    world, rank, local = _init_dist(args)
+    torch.cuda.set_device(local)
+    import __graft_entry__
+    __graft_entry__.build()
+    import ipd_synth as S
+    from paper_2609_36546_gb300 import VerifyStep, ipd
+
+    cfg = args.config
+    w = S.make_workload(cfg, seed=cfg + 1000 * rank, device="cuda")
+    step = VerifyStep.from_workload(w, device="cuda")
+    stream = torch.cuda.current_stream()
+    T_tok = step.T
+
+    # warm-up (also yields the verdict used for the algorithmic byte count)
+    for _ in range(max(3, args.warmup)):
+        step.run(stream)
+    torch.cuda.synchronize()
+    if ipd.device_error() != 0:
+        raise RuntimeError("device-side check failed during warm-up")
+    attn_bytes = step.attn_bytes(w.ctx)
+    logits_alg = step.logits_bytes_alg()
+    logits_full = step.logits_bytes_full()
+    accept_rate = float(step.score["covered"].float().mean()) if T_tok else 0.0
+    emitted = int(step.score["n_emit"].sum())
+
+    # ---- timed region: K steps, per-call events on the launching stream ----
+    K = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(_smi_index(local)) if rank == 0 else None
+    time.sleep(0.3 if sampler else 0.0)
+    _barrier(world)
+    torch.cuda.synchronize()
+    t_start.record(stream)
+    for i in range(K):
+        e = ev[i]
+        e[0].record(stream)
+        step.run_attention(stream)
+        e[1].record(stream)
+        step.run_score(stream)
+        e[2].record(stream)
+        step.run_loss(stream)
+        e[3].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    _barrier(world)
+    clocks = sampler.stop() if sampler else None
+    el_ms = t_start.elapsed_time(t_end)
+    attn_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in ev)
+    score_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in ev)
+    loss_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in ev)
+    el_max = _max_over_ranks(el_ms, world)
+    tokens_all = _sum_over_ranks(float(T_tok * K), world)
+    value = tokens_all / (el_max / 1e3)
+    ms_step = el_max / K
+
+    # ---- end to end through host buffers ----
+    e2e = run_e2e(step, w, min(K, args.e2e_steps), stream, world)
+
+    peak, peak_kind = _peaks()
+    if rank != 0:
+        return
+    achieved = attn_bytes / (attn_ms / 1e3) / 1e9
+    traffic = None
+    tr_path = os.path.join(ROOT, "profiles", f"attn_traffic_cfg{cfg}.json")
+    if os.path.exists(tr_path):
+        try:
+            traffic = json.load(open(tr_path)).get("traffic_bytes_per_launch")
+        except Exception:
+            traffic = None
+    step_alg = attn_bytes + logits_alg
+    step_full = attn_bytes + logits_full
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": max(3, args.warmup), "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": _workload_name(cfg), "seed": cfg, "tokens_per_step": T_tok,
+                   "requests": step.R, "l2": "inputs larger than L2 (no flush needed)",
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
+                     "kernel": "ipd_verify_attn (planner + attention launch)",
+                     "bytes_per_launch": attn_bytes, "ms_per_launch": attn_ms},
+        "step_hbm": {"bytes_alg": step_alg, "bytes_full": step_full,
+                     "gbs_alg": step_alg / (ms_step / 1e3) / 1e9,
+                     "gbs_full": step_full / (ms_step / 1e3) / 1e9,
+                     "frac_alg_of_measured": step_alg / (ms_step / 1e3) / 1e9 / peak,
+                     "frac_full_of_nominal_8tbs": step_full / (ms_step / 1e3) / 1e9 / 8000.0},
+        "calls_ms": {"verify_attn": attn_ms, "score_span": score_ms, "split_loss": loss_ms},
+        "acceptance": {"coverage_rate": accept_rate, "emitted_tokens_per_step": emitted},
+        "e2e": e2e, "clocks": clocks,
+        "gpu_launches": 5 * K,
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(step, w)
+    print(json.dumps(line), flush=True)
+
+
+def run_e2e(step, w, K, stream, world):
+    """The same step through host buffers: the per-step inputs (queries, both
+    models' logits, tokens, request metadata) are copied from pinned host
+    memory, the step runs, and its results (per-request verdict, per-token
+    sources, loss record) are copied back; the KV pools stay resident (they
+    are the cache state, not step inputs)."""
+    import torch
+    dev_inputs = []
+    for _, b, _, _ in step.batches:
+        q, cu_q, seq, ptab, _ = b._keep
+        dev_inputs += [q, cu_q, seq, ptab]
+    dev_inputs += [step.logits_s, step.logits_t, step.tokens, step.cu_span, step.driver,
+                   step.prefix_len]
+    host_inputs = [t.cpu().pin_memory() for t in dev_inputs]
+    outs = [step.score[n] for n in ("first_trans", "n_emit", "next_driver", "new_len", "done",
+                                     "source")] + [step.out8]
+    host_outs = [torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs]
+    h2d = sum(t.numel() * t.element_size() for t in host_inputs)
+    d2h = sum(t.numel() * t.element_size() for t in host_outs)
+    for _ in range(2):
+        for d, h in zip(dev_inputs, host_inputs):
+            d.copy_(h, non_blocking=True)
+        step.run(stream)
+        for h, d in zip(host_outs, outs):
+            h.copy_(d, non_blocking=True)
+        torch.cuda.synchronize()
+    _barrier(world)
+    t0 = time.perf_counter()
+    for _ in range(K):
+        for d, h in zip(dev_inputs, host_inputs):
+            d.copy_(h, non_blocking=True)
+        step.run(stream)
+        for h, d in zip(host_outs, outs):
+            h.copy_(d, non_blocking=True)
+        stream.synchronize()          # the engine reads the verdict before the next step
+    el = time.perf_counter() - t0
+    el = _max_over_ranks(el, world)
+    toks = _sum_over_ranks(float(step.T * K), world)
+    return {"value": toks / el, "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "steps": K,
+            "note": "pinned host -> device inputs (Q, logits, tokens, metadata) and device -> "
+                    "host results each step, synchronised per step; KV pools resident"}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--config", type=int, default=1)
+    ap.add_argument("--impl", default="ipd", choices=["ipd", "reference"])
+    ap.add_argument("--e2e-steps", type=int, default=200)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(3, args.warmup)
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

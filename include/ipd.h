@@ -1,0 +1,233 @@
+/*
+ * ipd.h -- C ABI of the IPD verify-step library (libipd.so, sm_103a).
+ *
+ * The verify step of Interactive-Policy Distillation's bidirectional
+ * propose-and-verify rollout (Sec. 3.2.1 and the fused engine of Sec. 3.2.3):
+ * the verifier scores the span of tokens the other model just proposed.
+ *
+ *   ipd_verify_attn  span-causal attention of the verifier's k span queries
+ *                    over its own paged KV cache, co-launched with the
+ *                    proposer's q_len = 1 decode attention over the other
+ *                    model's cache (different GQA shapes, one launch).
+ *   ipd_decode_attn  the decode attention alone.
+ *   ipd_score_span   one pass over both models' logits of every span
+ *                    position: log-softmax, per-token log-probs, the
+ *                    teacher-feedback term, top-K coverage, union-support
+ *                    top-K KL in both directions, the accept / takeover /
+ *                    handback verdict and the new cache lengths.
+ *   ipd_split_loss   the source-split objective of the step.
+ *
+ * Conventions for every call
+ *   - Data pointers are DEVICE pointers owned by the caller; the library never
+ *     allocates.  Scratch memory comes from a caller-provided device workspace
+ *     whose size the matching *_workspace_size query returns (host-only
+ *     arithmetic; the queries never touch the GPU).
+ *   - Every call is asynchronous on the caller's stream and never synchronises.
+ *   - bf16 tensors are passed as uint16_t bit patterns.
+ *   - Arguments are validated on the host before anything is launched; a
+ *     failed check returns a status and launches nothing.  Conditions that
+ *     only the device can see (a page id outside the pool, a length beyond
+ *     the page table) are caught by the kernels, which skip the offending
+ *     access and record a code readable with ipd_get_device_error().
+ *   - Returns IPD_OK or one of the IPD_ERR_* codes below.
+ */
+#ifndef IPD_H_
+#define IPD_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+struct CUstream_st;
+typedef struct CUstream_st *ipd_stream_t; /* same handle as cudaStream_t */
+
+#define IPD_OK 0
+#define IPD_ERR_INVALID_ARG 1 /* null pointer, negative size, inconsistent shape */
+#define IPD_ERR_UNSUPPORTED 2 /* head_dim != 128, page_size != 16, K > 32, ... */
+#define IPD_ERR_WORKSPACE 3   /* workspace null or smaller than the query says */
+#define IPD_ERR_CUDA 4        /* a CUDA runtime call failed (launch, attribute) */
+#define IPD_ERR_TIMEOUT 5     /* a bounded device wait ran out (never expected) */
+#define IPD_ERR_DEVICE 6      /* device-side check recorded an error */
+
+/* Device-side error codes (ipd_get_device_error). */
+#define IPD_DEVERR_NONE 0u
+#define IPD_DEVERR_PAGE_ID 1u    /* page_table entry < 0 or >= num_pages    */
+#define IPD_DEVERR_SEQ_LEN 2u    /* seq_len < q_len or > max_pages*16, or q_len > max_q_len */
+#define IPD_DEVERR_TOKEN 3u      /* proposed token id outside [0, vocab)     */
+#define IPD_DEVERR_PLAN 4u       /* work list larger than the workspace     */
+#define IPD_DEVERR_WAIT 5u       /* a bounded pipeline wait ran out         */
+#define IPD_DEVERR_SPAN 6u       /* cu_span / cu_q not non-decreasing       */
+
+#define IPD_MAX_BATCHES 8
+#define IPD_MAX_K 32
+
+/* One paged KV cache (one attention layer of one model).
+ * k_pages, v_pages: [num_pages][num_kv_heads][page_size][head_dim] bf16,
+ * row-major, 16-byte aligned.  A page holds page_size consecutive token
+ * positions of every KV head (vLLM-style paging, Sec. 3.2.3).
+ * Supported: page_size == 16, head_dim == 128, 1 <= num_kv_heads <= 64. */
+typedef struct ipd_kv_cache {
+  const uint16_t *k_pages;
+  const uint16_t *v_pages;
+  int64_t num_pages;
+  int32_t page_size;
+  int32_t num_kv_heads;
+  int32_t head_dim;
+} ipd_kv_cache;
+
+/* A sub-batch of requests attending one cache.
+ *  cache       host pointer to the cache descriptor.
+ *  num_q_heads multiple of cache->num_kv_heads; query head h reads KV head
+ *              h / (num_q_heads / num_kv_heads) (grouped-query attention).
+ *  q           [total_q][num_q_heads][head_dim] bf16.
+ *  cu_q        [num_reqs + 1] int32 prefix offsets into q; request r has
+ *              q_len = cu_q[r+1] - cu_q[r] queries (the span length k_r for a
+ *              verify batch, 1 for a decode batch).
+ *  seq_len     [num_reqs] int32 KV length L_r in this cache, INCLUDING the
+ *              span (whose K/V are already written at positions L_r-k_r..L_r-1).
+ *              Query i of request r sits at position L_r - q_len + i and sees
+ *              keys 0 .. L_r - q_len + i (causal within the span).
+ *  page_table  [num_reqs][max_pages] int32; entry p of row r is the pool page
+ *              holding positions 16p .. 16p+15 of request r.  Only the first
+ *              ceil(L_r / 16) entries of a row are read.
+ *  total_q, max_q_len, max_seq_len: host-known bounds (total_q must equal
+ *              cu_q[num_reqs]); they size the grid and the workspace without
+ *              a device-to-host read.
+ *  out         [total_q][num_q_heads][head_dim] bf16, written by the call. */
+typedef struct ipd_attn_batch {
+  const ipd_kv_cache *cache;
+  int32_t num_q_heads;
+  int32_t num_reqs;
+  const uint16_t *q;
+  const int32_t *cu_q;
+  const int32_t *seq_len;
+  const int32_t *page_table;
+  int32_t max_pages;
+  int32_t total_q;
+  int32_t max_q_len;
+  int32_t max_seq_len;
+  uint16_t *out;
+} ipd_attn_batch;
+
+/* Workspace bytes for one ipd_verify_attn / ipd_decode_attn call on these
+ * batches (host arithmetic only).  Returns 0 if the batches are invalid. */
+size_t ipd_attn_workspace_size(const ipd_attn_batch *verify, int n_verify,
+                               const ipd_attn_batch *decode, int n_decode);
+
+/* Span-verify attention (Sec. 3.2.3, verification stage: every verifier
+ * prefills the unverified drafts of its sub-batch in one pass over its own
+ * cache) for n_verify batches, together with the proposer decode attention
+ * (proposal stage: each proposer extends only its own cache) for n_decode
+ * batches, in ONE launch.  decode may be NULL when n_decode == 0.
+ * n_verify + n_decode <= IPD_MAX_BATCHES.  softmax_scale is applied to q.k
+ * (1/sqrt(head_dim) for the configurations of this library's tests).
+ * out = softmax(scale * q K^T) V per query and head, fp32 accumulation,
+ * rounded to bf16 once. */
+int ipd_verify_attn(const ipd_attn_batch *verify, int n_verify,
+                    const ipd_attn_batch *decode, int n_decode,
+                    float softmax_scale, void *workspace, size_t workspace_bytes,
+                    ipd_stream_t stream);
+
+/* The decode attention alone (same semantics, q_len = 1 per request). */
+int ipd_decode_attn(const ipd_attn_batch *decode, int n_decode, float softmax_scale,
+                    void *workspace, size_t workspace_bytes, ipd_stream_t stream);
+
+/* Workspace bytes for ipd_score_span. */
+size_t ipd_score_workspace_size(int num_reqs, int total_tokens, int vocab, int K);
+
+/* The vocabulary pass, verdict and cache bookkeeping of one verify step.
+ *
+ * Inputs
+ *  logits_student [total_tokens][vocab] bf16: row t is the student's logits
+ *                 pi(.|c_t) at span position t (flat over requests).
+ *  logits_teacher [total_tokens][vocab] bf16: the teacher's q(.|c_t).
+ *  tokens         [total_tokens] int32: the proposed token at each position.
+ *  cu_span        [num_reqs + 1] int32 prefix offsets of each request's span.
+ *  driver         [num_reqs] uint8: 0 = the student proposed (teacher
+ *                 verifies), 1 = the teacher proposed (student verifies).
+ *  prefix_len     [num_reqs] int32: verified prefix length before the span.
+ *  K              top-K width, 1 <= K <= 32, K <= vocab (Sec. 4.1 uses 16).
+ *  eos_id         end-of-sequence token id, or -1 for none.
+ *
+ * Per-token outputs [total_tokens]
+ *  logp_s, logp_t full-vocabulary log-probabilities of the proposed token
+ *                 under the student and the teacher.
+ *  feedback       log q(x_t) - log pi(x_t): the per-token teacher-feedback
+ *                 reward, minus the sampled-token estimate of Eq.
+ *                 (sampled_token_opd).
+ *  kl_rev         KL(pi_bar || q_bar) on S_t = Top_K(pi) u Top_K(q), both
+ *                 renormalised on S_t (Eq. topk_normalization,
+ *                 topk_opd_on_sequence); the on-policy term of Eq. ipd_off_loss.
+ *  kl_fwd         KL(q_bar || pi_bar) on the same support; the off-policy term.
+ *  covered        1 if the proposed token is in the VERIFIER's Top_K, else 0.
+ *                 Top_K orders by logit, ties broken by smaller token id.
+ *  margin         verifier logit of the proposed token minus the verifier's
+ *                 K-th largest logit (0 on an exact tie at the boundary).
+ *  source         0 = emitted with z = S, 1 = emitted with z = T, 255 = not
+ *                 emitted (rejected or after the transition).
+ * Per-request outputs [num_reqs]
+ *  first_trans    first position whose verdict changes the driver (takeover
+ *                 for driver 0, handback for driver 1), or k_r if none occurs
+ *                 before the span ends or an accepted EOS.
+ *  n_emit         tokens emitted by this step.
+ *  next_driver    driver after the step.
+ *  new_len        prefix_len + n_emit: the length both caches roll back to.
+ *  done           1 if an accepted EOS ended the request.
+ * The verdict follows Eq. (ipd_state_transition) and the verdict-stage rules
+ * of Sec. 3.2.3: a rejected student token is not emitted (the teacher
+ * regenerates it), a handback token is kept, a student EOS counts only when
+ * covered, a teacher EOS is accepted directly. */
+int ipd_score_span(const uint16_t *logits_student, const uint16_t *logits_teacher,
+                   const int32_t *tokens, const int32_t *cu_span, const uint8_t *driver,
+                   const int32_t *prefix_len, int num_reqs, int total_tokens, int vocab,
+                   int K, int eos_id,
+                   float *logp_s, float *logp_t, float *feedback, float *kl_rev,
+                   float *kl_fwd, uint8_t *covered, float *margin, uint8_t *source,
+                   int32_t *first_trans, int32_t *n_emit, uint8_t *next_driver,
+                   int32_t *new_len, uint8_t *done,
+                   void *workspace, size_t workspace_bytes, ipd_stream_t stream);
+
+/* Loss direction per token source (the KL-direction ablation of Sec. 4.3). */
+#define IPD_DIR_SPLIT 0    /* z=S: KL(pi||q), z=T: KL(q||pi)   (IPD default) */
+#define IPD_DIR_REVERSE 1  /* both reverse                                   */
+#define IPD_DIR_FORWARD 2  /* both forward                                   */
+#define IPD_DIR_INVERSE 3  /* z=S: forward, z=T: reverse                     */
+/* Aggregation (Eq. ipd_objective and App. B.3). */
+#define IPD_AGG_SEQ_MEAN_TOKEN_MEAN 0
+#define IPD_AGG_GLOBAL_TOKEN_MEAN 1
+
+/* Workspace bytes for ipd_split_loss (0: it needs none). */
+size_t ipd_loss_workspace_size(int num_reqs);
+
+/* The source-split objective of one step (Eq. ipd_off_loss, ipd_objective).
+ *  kl_rev, kl_fwd, source, n_emit, cu_span: as produced by ipd_score_span.
+ *  resp_len  [num_reqs] int32 response lengths |x_r| for the length
+ *            normalisation, or NULL to use n_emit.  Requests whose length is
+ *            0 are left out of the batch mean.
+ *  out8      8 floats (device): loss, sum_on, sum_off, n_on, n_off,
+ *            intervention_ratio (share of teacher-sourced tokens), numer,
+ *            denom (loss = numer / denom, so shards of a batch can be
+ *            combined by summing numer and denom).
+ * The reduction order is fixed, so the result is bitwise reproducible. */
+int ipd_split_loss(const float *kl_rev, const float *kl_fwd, const uint8_t *source,
+                   const int32_t *cu_span, const int32_t *n_emit, const int32_t *resp_len,
+                   int num_reqs, int agg_mode, int dir_mode, float *out8,
+                   void *workspace, size_t workspace_bytes, ipd_stream_t stream);
+
+/* Reads and clears the device error word of the current device
+ * (synchronises the device).  *code receives an IPD_DEVERR_* value. */
+int ipd_get_device_error(uint32_t *code);
+
+/* Human-readable name of a status code (static storage). */
+const char *ipd_status_string(int status);
+
+/* Library version, e.g. 100 for 0.1.0. */
+int ipd_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* IPD_H_ */

@@ -1,0 +1,218 @@
+"""ctypes binding of libipd.so: argument marshalling only.
+
+Every function here forwards torch tensors (device memory) as raw pointers to
+the C ABI declared in include/ipd.h and raises IpdError on a non-zero status.
+No step of the computation runs in Python, and there is no fallback: if the
+shared library cannot be loaded, importing the binding fails.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_lib", "libipd.so")
+
+IPD_OK = 0
+STATUS = {0: "IPD_OK", 1: "IPD_ERR_INVALID_ARG", 2: "IPD_ERR_UNSUPPORTED", 3: "IPD_ERR_WORKSPACE",
+          4: "IPD_ERR_CUDA", 5: "IPD_ERR_TIMEOUT", 6: "IPD_ERR_DEVICE"}
+STATUS_CODES = {v: k for k, v in STATUS.items()}
+DEVERR = {0: "none", 1: "page id", 2: "seq len", 3: "token id", 4: "plan overflow", 5: "wait",
+          6: "span offsets"}
+
+DIR_SPLIT, DIR_REVERSE, DIR_FORWARD, DIR_INVERSE = 0, 1, 2, 3
+AGG_SEQ_MEAN_TOKEN_MEAN, AGG_GLOBAL_TOKEN_MEAN = 0, 1
+LOSS_FIELDS = ("loss", "sum_on", "sum_off", "n_on", "n_off", "intervention_ratio", "numer", "denom")
+
+# Exported symbols of include/ipd.h (checked by the CPU test suite).
+EXPORTS = ("ipd_attn_workspace_size", "ipd_verify_attn", "ipd_decode_attn",
+           "ipd_score_workspace_size", "ipd_score_span", "ipd_loss_workspace_size",
+           "ipd_split_loss", "ipd_get_device_error", "ipd_status_string", "ipd_version")
+
+
+class IpdError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        super().__init__(f"{what}: {STATUS.get(status, status)}")
+        self.status = status
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"libipd.so not built ({LIB_PATH}); run __graft_entry__.build()")
+    return ctypes.CDLL(LIB_PATH)
+
+
+_lib = _load()
+
+c_p = ctypes.c_void_p
+c_i = ctypes.c_int
+c_sz = ctypes.c_size_t
+
+
+class _KVCache(ctypes.Structure):
+    _fields_ = [("k_pages", c_p), ("v_pages", c_p), ("num_pages", ctypes.c_int64),
+                ("page_size", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32)]
+
+
+class _AttnBatch(ctypes.Structure):
+    _fields_ = [("cache", ctypes.POINTER(_KVCache)), ("num_q_heads", ctypes.c_int32),
+                ("num_reqs", ctypes.c_int32), ("q", c_p), ("cu_q", c_p), ("seq_len", c_p),
+                ("page_table", c_p), ("max_pages", ctypes.c_int32), ("total_q", ctypes.c_int32),
+                ("max_q_len", ctypes.c_int32), ("max_seq_len", ctypes.c_int32), ("out", c_p)]
+
+
+_lib.ipd_attn_workspace_size.restype = c_sz
+_lib.ipd_attn_workspace_size.argtypes = [ctypes.POINTER(_AttnBatch), c_i,
+                                         ctypes.POINTER(_AttnBatch), c_i]
+_lib.ipd_verify_attn.restype = c_i
+_lib.ipd_verify_attn.argtypes = [ctypes.POINTER(_AttnBatch), c_i, ctypes.POINTER(_AttnBatch), c_i,
+                                 ctypes.c_float, c_p, c_sz, c_p]
+_lib.ipd_decode_attn.restype = c_i
+_lib.ipd_decode_attn.argtypes = [ctypes.POINTER(_AttnBatch), c_i, ctypes.c_float, c_p, c_sz, c_p]
+_lib.ipd_score_workspace_size.restype = c_sz
+_lib.ipd_score_workspace_size.argtypes = [c_i, c_i, c_i, c_i]
+_lib.ipd_score_span.restype = c_i
+_lib.ipd_score_span.argtypes = [c_p] * 6 + [c_i] * 5 + [c_p] * 13 + [c_p, c_sz, c_p]
+_lib.ipd_loss_workspace_size.restype = c_sz
+_lib.ipd_loss_workspace_size.argtypes = [c_i]
+_lib.ipd_split_loss.restype = c_i
+_lib.ipd_split_loss.argtypes = [c_p] * 6 + [c_i, c_i, c_i, c_p, c_p, c_sz, c_p]
+_lib.ipd_get_device_error.restype = c_i
+_lib.ipd_get_device_error.argtypes = [ctypes.POINTER(ctypes.c_uint32)]
+_lib.ipd_status_string.restype = ctypes.c_char_p
+_lib.ipd_status_string.argtypes = [c_i]
+_lib.ipd_version.restype = c_i
+
+
+def lib() -> ctypes.CDLL:
+    return _lib
+
+
+def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    if t is None:
+        return None
+    return t.data_ptr()
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream if torch.cuda.is_available() else None
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _check(st: int, what: str):
+    if st != IPD_OK:
+        raise IpdError(st, what)
+
+
+class KVCache:
+    """A paged KV cache: k_pages / v_pages are [num_pages, Hkv, 16, 128] bf16."""
+
+    def __init__(self, k_pages: torch.Tensor, v_pages: torch.Tensor):
+        assert k_pages.shape == v_pages.shape and k_pages.dim() == 4
+        self.k_pages, self.v_pages = k_pages, v_pages
+        self.c = _KVCache(_ptr(k_pages), _ptr(v_pages), k_pages.shape[0], k_pages.shape[2],
+                          k_pages.shape[1], k_pages.shape[3])
+
+    @property
+    def num_kv_heads(self) -> int:
+        return self.k_pages.shape[1]
+
+
+class AttnBatch:
+    """One sub-batch of requests attending one cache (see ipd_attn_batch).
+
+    q [total_q, Hq, 128] bf16, cu_q [R+1] int32, seq_len [R] int32,
+    page_table [R, max_pages] int32, out [total_q, Hq, 128] bf16 (all device);
+    max_q_len / max_seq_len are host-known bounds."""
+
+    def __init__(self, cache: KVCache, q, cu_q, seq_len, page_table, out, max_q_len: int,
+                 max_seq_len: int):
+        self.cache = cache
+        self._keep = (q, cu_q, seq_len, page_table, out)
+        R = seq_len.numel()
+        self.c = _AttnBatch(ctypes.pointer(cache.c), q.shape[1], R, _ptr(q), _ptr(cu_q),
+                            _ptr(seq_len), _ptr(page_table), page_table.shape[1], q.shape[0],
+                            max_q_len, max_seq_len, _ptr(out))
+        self.out = out
+
+
+def _arr(batches: Sequence[AttnBatch]):
+    n = len(batches)
+    if n == 0:
+        return None, 0
+    a = (_AttnBatch * n)(*[b.c for b in batches])
+    return a, n
+
+
+def attn_workspace_size(verify: Sequence[AttnBatch], decode: Sequence[AttnBatch] = ()) -> int:
+    va, nv = _arr(verify)
+    da, nd = _arr(decode)
+    return int(_lib.ipd_attn_workspace_size(va, nv, da, nd))
+
+
+def verify_attn(verify: Sequence[AttnBatch], decode: Sequence[AttnBatch], softmax_scale: float,
+                workspace: torch.Tensor, stream=None):
+    va, nv = _arr(verify)
+    da, nd = _arr(decode)
+    _check(_lib.ipd_verify_attn(va, nv, da, nd, softmax_scale, _ptr(workspace),
+                                workspace.numel() * workspace.element_size(), _stream(stream)),
+           "ipd_verify_attn")
+
+
+def decode_attn(decode: Sequence[AttnBatch], softmax_scale: float, workspace: torch.Tensor,
+                stream=None):
+    da, nd = _arr(decode)
+    _check(_lib.ipd_decode_attn(da, nd, softmax_scale, _ptr(workspace),
+                                workspace.numel() * workspace.element_size(), _stream(stream)),
+           "ipd_decode_attn")
+
+
+def score_workspace_size(num_reqs: int, total_tokens: int, vocab: int, K: int) -> int:
+    return int(_lib.ipd_score_workspace_size(num_reqs, total_tokens, vocab, K))
+
+
+SCORE_TOKEN_OUTPUTS = (("logp_s", torch.float32), ("logp_t", torch.float32),
+                       ("feedback", torch.float32), ("kl_rev", torch.float32),
+                       ("kl_fwd", torch.float32), ("covered", torch.uint8),
+                       ("margin", torch.float32), ("source", torch.uint8))
+SCORE_REQ_OUTPUTS = (("first_trans", torch.int32), ("n_emit", torch.int32),
+                     ("next_driver", torch.uint8), ("new_len", torch.int32), ("done", torch.uint8))
+
+
+def alloc_score_outputs(num_reqs: int, total_tokens: int, device) -> dict:
+    out = {n: torch.empty(total_tokens, dtype=dt, device=device) for n, dt in SCORE_TOKEN_OUTPUTS}
+    out.update({n: torch.empty(num_reqs, dtype=dt, device=device) for n, dt in SCORE_REQ_OUTPUTS})
+    return out
+
+
+def score_span(logits_student, logits_teacher, tokens, cu_span, driver, prefix_len, K: int,
+               eos_id: int, out: dict, workspace: torch.Tensor, stream=None):
+    R = driver.numel()
+    T, V = logits_student.shape
+    _check(_lib.ipd_score_span(
+        _ptr(logits_student), _ptr(logits_teacher), _ptr(tokens), _ptr(cu_span), _ptr(driver),
+        _ptr(prefix_len), R, T, V, K, eos_id,
+        *[_ptr(out[n]) for n, _ in SCORE_TOKEN_OUTPUTS],
+        *[_ptr(out[n]) for n, _ in SCORE_REQ_OUTPUTS],
+        _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)),
+        "ipd_score_span")
+
+
+def split_loss(kl_rev, kl_fwd, source, cu_span, n_emit, resp_len, agg_mode: int, dir_mode: int,
+               out8: torch.Tensor, stream=None):
+    R = cu_span.numel() - 1
+    _check(_lib.ipd_split_loss(_ptr(kl_rev), _ptr(kl_fwd), _ptr(source), _ptr(cu_span),
+                               _ptr(n_emit), _ptr(resp_len), R, agg_mode, dir_mode, _ptr(out8),
+                               None, 0, _stream(stream)), "ipd_split_loss")
+
+
+def device_error() -> int:
+    """Reads and clears the device-side error word (synchronises)."""
+    v = ctypes.c_uint32(0)
+    _check(_lib.ipd_get_device_error(ctypes.byref(v)), "ipd_get_device_error")
+    return int(v.value)

@@ -1,0 +1,157 @@
+"""One verify step of the fused engine, assembled from plain tensors.
+
+Host glue only: it groups requests by verifier (Sec. 3.2.3: requests are
+grouped by their verifier for the verification stage and by their driver for
+the proposal stage), allocates the device buffers, and issues the three C-ABI
+calls on one stream:
+
+  ipd_verify_attn  teacher-verify + student-verify span attention and the
+                   student / teacher decode attention, one launch
+  ipd_score_span   vocabulary pass, verdict and cache bookkeeping
+  ipd_split_loss   source-split objective
+"""
+from __future__ import annotations
+
+import math
+from typing import Optional
+
+import torch
+
+from . import ipd
+
+SCALE = 1.0 / math.sqrt(128.0)
+
+
+def _cu(lengths: torch.Tensor) -> torch.Tensor:
+    out = torch.zeros(lengths.numel() + 1, dtype=torch.int32)
+    out[1:] = torch.cumsum(lengths.to(torch.int64), 0).to(torch.int32)
+    return out
+
+
+class VerifyStep:
+    """Device buffers and calls of one verify step.
+
+    Host inputs (cpu tensors): ctx [R] (KV length of both caches, span
+    included), span [R], driver [R] (0: the student proposed), page tables
+    [R, max_pages] for the teacher and the student cache.  Device inputs:
+    the four paged pools, the span queries for each verifier, the decode
+    queries for each proposer, the proposed tokens and both models' logits.
+    """
+
+    def __init__(self, teacher_k, teacher_v, student_k, student_v, ctx, span, driver,
+                 pt_teacher, pt_student, q_verify_t, q_verify_s, q_decode_s, q_decode_t, tokens,
+                 logits_s, logits_t, K: int = 16, eos_id: int = -1, resp_len=None,
+                 agg_mode: int = ipd.AGG_SEQ_MEAN_TOKEN_MEAN, dir_mode: int = ipd.DIR_SPLIT,
+                 scale: float = SCALE, device="cuda"):
+        dev = torch.device(device)
+        self.device = dev
+        self.K, self.eos_id, self.agg_mode, self.dir_mode, self.scale = K, eos_id, agg_mode, \
+            dir_mode, scale
+        ctx = ctx.to(torch.int32).cpu()
+        span = span.to(torch.int32).cpu()
+        driver = driver.to(torch.uint8).cpu()
+        self.R = int(ctx.numel())
+        self.T = int(span.sum())
+        self.cache_t = ipd.KVCache(teacher_k, teacher_v)
+        self.cache_s = ipd.KVCache(student_k, student_v)
+        idx_s = torch.nonzero(driver == 0).flatten()   # student proposes, teacher verifies
+        idx_t = torch.nonzero(driver == 1).flatten()
+        self.idx_s, self.idx_t = idx_s, idx_t
+
+        def mk(cache, q, idx, q_len, pt):
+            if idx.numel() == 0:
+                return None
+            cu_q = _cu(q_len).to(dev)
+            seq = ctx[idx].contiguous().to(dev)
+            ptab = pt[idx].contiguous().to(dev)
+            out = torch.empty_like(q)
+            return ipd.AttnBatch(cache, q, cu_q, seq, ptab, out, int(q_len.max()),
+                                 int(ctx[idx].max()))
+
+        one = lambda idx: torch.ones(idx.numel(), dtype=torch.int32)
+        # (name, batch, request indices, cache name) for every non-empty sub-batch
+        self.batches = [(n, b, idx, c) for n, b, idx, c in (
+            ("verify_teacher", mk(self.cache_t, q_verify_t, idx_s, span[idx_s], pt_teacher),
+             idx_s, "teacher"),
+            ("verify_student", mk(self.cache_s, q_verify_s, idx_t, span[idx_t], pt_student),
+             idx_t, "student"),
+            ("decode_student", mk(self.cache_s, q_decode_s, idx_s, one(idx_s), pt_student),
+             idx_s, "student"),
+            ("decode_teacher", mk(self.cache_t, q_decode_t, idx_t, one(idx_t), pt_teacher),
+             idx_t, "teacher")) if b is not None]
+        self.verify = [b for n, b, _, _ in self.batches if n.startswith("verify")]
+        self.decode = [b for n, b, _, _ in self.batches if n.startswith("decode")]
+        self.ws_attn = torch.empty(max(256, ipd.attn_workspace_size(self.verify, self.decode)),
+                                   dtype=torch.uint8, device=dev)
+        # scoring
+        self.logits_s, self.logits_t, self.tokens = logits_s, logits_t, tokens
+        self.V = int(logits_s.shape[1])
+        self.cu_span = _cu(span).to(dev)
+        self.driver = driver.to(dev)
+        self.prefix_len = (ctx - span).to(torch.int32).to(dev)
+        self.resp_len = None if resp_len is None else resp_len.to(torch.int32).to(dev)
+        self.score = ipd.alloc_score_outputs(self.R, self.T, dev)
+        self.ws_score = torch.empty(max(256, ipd.score_workspace_size(self.R, self.T, self.V, K)),
+                                    dtype=torch.uint8, device=dev)
+        self.out8 = torch.zeros(8, dtype=torch.float32, device=dev)
+
+    @classmethod
+    def from_workload(cls, w, device="cuda", **kw):
+        """Build from an object with the attributes of a synthetic workload."""
+        dev = torch.device(device)
+        mv = lambda t: t.to(dev)
+        kw.setdefault("K", w.spec.K)
+        kw.setdefault("eos_id", w.spec.eos_id)
+        return cls(mv(w.teacher.k_pages), mv(w.teacher.v_pages), mv(w.student.k_pages),
+                   mv(w.student.v_pages), w.ctx, w.span, w.driver, w.teacher.page_table,
+                   w.student.page_table, mv(w.q_verify_t), mv(w.q_verify_s), mv(w.q_decode_s),
+                   mv(w.q_decode_t), mv(w.tokens), mv(w.logits_s), mv(w.logits_t), device=dev,
+                   **kw)
+
+    # -- the three calls ------------------------------------------------------
+    def run_attention(self, stream=None):
+        ipd.verify_attn(self.verify, self.decode, self.scale, self.ws_attn, stream)
+
+    def run_score(self, stream=None):
+        ipd.score_span(self.logits_s, self.logits_t, self.tokens, self.cu_span, self.driver,
+                       self.prefix_len, self.K, self.eos_id, self.score, self.ws_score, stream)
+
+    def run_loss(self, stream=None):
+        s = self.score
+        ipd.split_loss(s["kl_rev"], s["kl_fwd"], s["source"], self.cu_span, s["n_emit"],
+                       self.resp_len, self.agg_mode, self.dir_mode, self.out8, stream)
+
+    def run(self, stream=None):
+        self.run_attention(stream)
+        self.run_score(stream)
+        self.run_loss(stream)
+
+    # -- bytes the step must move (algorithmic) --------------------------------
+    def attn_bytes(self, ctx: torch.Tensor) -> int:
+        """KV pages read (exact lengths) + Q read + O written, both caches."""
+        total = 0
+        for b in self.verify + self.decode:
+            hkv = b.cache.num_kv_heads
+            seq = b._keep[2].cpu().to(torch.int64)
+            total += int(seq.sum()) * hkv * 128 * 2 * 2          # K and V, bf16
+            q = b._keep[0]
+            total += 2 * q.numel() * q.element_size()              # Q in, O out
+        return total
+
+    def logits_bytes_full(self) -> int:
+        return 2 * self.T * self.V * 2
+
+    def logits_bytes_alg(self) -> int:
+        """Verifier rows for positions 0..first_trans (clipped to the span) and
+        proposer rows for the emitted positions (needs the step's outputs)."""
+        cu = self.cu_span.cpu()
+        ft = self.score["first_trans"].cpu()
+        ne = self.score["n_emit"].cpu()
+        rows = 0
+        for r in range(self.R):
+            k = int(cu[r + 1] - cu[r])
+            rows += min(k, int(ft[r]) + 1) + int(ne[r])
+        return rows * self.V * 2
+
+    def vocab_rows_bytes(self) -> int:
+        return self.logits_bytes_full()

@@ -1,0 +1,180 @@
+"""GPU-vs-oracle comparison of one verify step (used by the -m gpu tests and
+by __graft_entry__.smoke()).
+
+Tolerances (stated once here):
+* attention: every output within 2 bf16 ulp of the fp64 oracle rounded to
+  bf16, the ulp taken at max(|ref|, rowmax/8) where rowmax is the largest
+  magnitude of that (query, head) output vector; the strict ulp at |ref| is
+  reported alongside.  (Reading of "2 bf16 ulp" for near-zero components: an
+  fp32-accumulated average of bf16 values carries an absolute error tied to
+  the scale of the vector, not of one tiny component.)
+* log-probs within 1e-3 absolute; feedback within 2e-3 (difference of two).
+* KL terms within 2e-4 + 1e-4 |ref| (fp32 sums of <= 64 terms of size <= ~40).
+* margin: exact (difference of two bf16 values is exact in fp32).
+* decisions (covered, source, first_trans, n_emit, next_driver, new_len,
+  done): bit-exact; positions with |margin| <= 1e-3 are counted separately.
+* split loss: 1e-4 relative (plus 1e-6 absolute for a zero loss).
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle as O
+
+ATOL_LOGP = 1e-3
+ATOL_FEEDBACK = 2e-3
+KL_ATOL, KL_RTOL = 2e-4, 1e-4
+LOSS_RTOL = 1e-4
+
+
+def u16(t: torch.Tensor) -> np.ndarray:
+    return t.detach().contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
+
+
+def attn_ulp_errors(got_bits: np.ndarray, ref: np.ndarray):
+    """(floored-ulp error, strict-ulp error) arrays, in bf16 ulps."""
+    got = O.bf16_to_f64(got_bits)
+    ref_b = O.bf16_to_f64(O.f64_to_bf16(ref))
+    rowmax = np.abs(ref).max(axis=-1, keepdims=True)
+    ulp_floor = O.bf16_ulp(np.maximum(np.abs(ref), rowmax / 8.0))
+    ulp_strict = O.bf16_ulp(np.maximum(np.abs(ref_b), 1e-30))
+    err = np.abs(got - ref_b)
+    return err / ulp_floor, err / ulp_strict
+
+
+def check_attention(step, requests=None, max_reqs_per_batch=None, rng=None):
+    """Compare every sub-batch's output for the chosen requests."""
+    stats = dict(attn_rows=0, attn_max_ulp=0.0, attn_max_ulp_strict=0.0, attn_frac_strict_le2=1.0,
+                 attn_bad=0)
+    n_strict_ok = n_all = 0
+    for name, b, idx, cache in step.batches:
+        q, cu_q, seq, ptab, out = b._keep
+        cu = cu_q.cpu().numpy()
+        seqh = seq.cpu().numpy()
+        pth = ptab.cpu().numpy()
+        pool_k, pool_v = (step.cache_t if cache == "teacher" else step.cache_s).k_pages, \
+            (step.cache_t if cache == "teacher" else step.cache_s).v_pages
+        local = range(len(idx))
+        if requests is not None:
+            sel = set(int(r) for r in requests)
+            local = [j for j in range(len(idx)) if int(idx[j]) in sel]
+        if max_reqs_per_batch is not None and len(local) > max_reqs_per_batch:
+            local = sorted((rng or np.random.default_rng(0)).choice(list(local), max_reqs_per_batch,
+                                                                   replace=False).tolist())
+        for j in local:
+            L = int(seqh[j])
+            npg = (L + 15) // 16
+            pages = torch.from_numpy(pth[j, :npg].astype(np.int64)).to(pool_k.device)
+            kp = u16(pool_k.index_select(0, pages))
+            vp = u16(pool_v.index_select(0, pages))
+            qb = u16(q[cu[j]:cu[j + 1]])
+            ref = O.paged_span_attention(qb, kp, vp, np.arange(npg), L, step.scale)
+            got = u16(out[cu[j]:cu[j + 1]])
+            e_floor, e_strict = attn_ulp_errors(got, ref)
+            stats["attn_rows"] += ref.shape[0] * ref.shape[1]
+            stats["attn_max_ulp"] = max(stats["attn_max_ulp"], float(e_floor.max()))
+            stats["attn_max_ulp_strict"] = max(stats["attn_max_ulp_strict"], float(e_strict.max()))
+            stats["attn_bad"] += int((e_floor > 2.0).sum())
+            n_strict_ok += int((e_strict <= 2.0).sum())
+            n_all += e_strict.size
+    if n_all:
+        stats["attn_frac_strict_le2"] = n_strict_ok / n_all
+    stats["attn_ok"] = stats["attn_bad"] == 0
+    return stats
+
+
+def oracle_scores(step, requests):
+    cu = step.cu_span.cpu().numpy()
+    drv = step.driver.cpu().numpy()
+    pre = step.prefix_len.cpu().numpy()
+    toks = step.tokens.cpu().numpy()
+    res = {}
+    for r in requests:
+        t0, t1 = int(cu[r]), int(cu[r + 1])
+        ls = u16(step.logits_s[t0:t1]) if t1 > t0 else np.zeros((0, step.V), np.uint16)
+        lt = u16(step.logits_t[t0:t1]) if t1 > t0 else np.zeros((0, step.V), np.uint16)
+        sub = O.score_span(ls, lt, toks[t0:t1], np.array([0, t1 - t0]), drv[r:r + 1],
+                           pre[r:r + 1], step.K, step.eos_id)
+        res[int(r)] = (t0, t1, sub)
+    return res
+
+
+def check_scores(step, requests=None):
+    R = step.R
+    reqs = list(range(R)) if requests is None else [int(r) for r in requests]
+    orc = oracle_scores(step, reqs)
+    g = {k: v.cpu().numpy() for k, v in step.score.items()}
+    st = dict(score_positions=0, max_logp_err=0.0, max_fb_err=0.0, max_kl_err=0.0,
+              max_margin_err=0.0, decision_mismatch=0, near_threshold=0, near_threshold_mismatch=0,
+              coverage_rate=0.0)
+    ncov = 0
+    for r in reqs:
+        t0, t1, o = orc[r]
+        sl = slice(t0, t1)
+        st["score_positions"] += t1 - t0
+        if t1 > t0:
+            st["max_logp_err"] = max(st["max_logp_err"],
+                                     float(np.abs(g["logp_s"][sl] - o["logp_s"]).max()),
+                                     float(np.abs(g["logp_t"][sl] - o["logp_t"]).max()))
+            st["max_fb_err"] = max(st["max_fb_err"],
+                                   float(np.abs(g["feedback"][sl] - o["feedback"]).max()))
+            for name in ("kl_rev", "kl_fwd"):
+                err = np.abs(g[name][sl] - o[name]) - KL_RTOL * np.abs(o[name])
+                st["max_kl_err"] = max(st["max_kl_err"], float(err.max()))
+            st["max_margin_err"] = max(st["max_margin_err"],
+                                       float(np.abs(g["margin"][sl] - o["margin"]).max()))
+            near = np.abs(o["margin"]) <= 1e-3
+            cov_mis = g["covered"][sl].astype(np.int64) != o["covered"]
+            src_mis = g["source"][sl].astype(np.int64) != o["source"]
+            st["near_threshold"] += int(near.sum())
+            st["near_threshold_mismatch"] += int((near & cov_mis).sum())
+            st["decision_mismatch"] += int(cov_mis.sum() + src_mis.sum())
+            ncov += int(o["covered"].sum())
+        for name in ("first_trans", "n_emit", "next_driver", "new_len", "done"):
+            if int(g[name][r]) != int(o[name][0]):
+                st["decision_mismatch"] += 1
+    if st["score_positions"]:
+        st["coverage_rate"] = ncov / st["score_positions"]
+    st["score_ok"] = (st["max_logp_err"] <= ATOL_LOGP and st["max_fb_err"] <= ATOL_FEEDBACK and
+                      st["max_kl_err"] <= KL_ATOL and st["max_margin_err"] <= 1e-6 and
+                      st["decision_mismatch"] == 0)
+    return st, orc
+
+
+def check_loss(step, orc):
+    """Full-batch loss check (needs the oracle scores of every request)."""
+    T = step.T
+    rev = np.zeros(T); fwd = np.zeros(T); src = np.zeros(T, np.int64)
+    n_emit = np.zeros(step.R, np.int64)
+    for r, (t0, t1, o) in orc.items():
+        rev[t0:t1] = o["kl_rev"]; fwd[t0:t1] = o["kl_fwd"]; src[t0:t1] = o["source"]
+        n_emit[r] = o["n_emit"][0]
+    rl = None if step.resp_len is None else step.resp_len.cpu().numpy()
+    ref = O.split_loss(rev, fwd, src, step.cu_span.cpu().numpy(), n_emit, rl, step.agg_mode,
+                       step.dir_mode)
+    got = step.out8.cpu().numpy()
+    st = dict(loss_gpu=float(got[0]), loss_ref=ref["loss"], loss_rel_err=0.0)
+    ok = True
+    for i, name in enumerate(O.LOSS_FIELDS):
+        a, b = float(got[i]), float(ref[name])
+        if abs(a - b) > LOSS_RTOL * abs(b) + 1e-6:
+            ok = False
+        if name == "loss":
+            st["loss_rel_err"] = abs(a - b) / max(abs(b), 1e-30)
+    st["loss_ok"] = ok
+    return st
+
+
+def check_step(step, w=None, requests=None, attn_max_reqs=None, rng=None):
+    """Full comparison; requests=None checks every request and the loss."""
+    rep = {}
+    rep.update(check_attention(step, requests, attn_max_reqs, rng))
+    s, orc = check_scores(step, requests)
+    rep.update(s)
+    if requests is None:
+        rep.update(check_loss(step, orc))
+    else:
+        rep["loss_ok"] = True
+    rep["ok"] = bool(rep["attn_ok"] and rep["score_ok"] and rep["loss_ok"])
+    return rep

@@ -1,0 +1,87 @@
+"""The C ABI on the host: the library loads, exports every function that
+include/ipd.h declares, and rejects bad arguments before launching anything
+(these calls never reach the GPU)."""
+import ctypes
+import os
+import re
+
+import pytest
+import torch
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def ipd():
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_36546_gb300 import ipd as m
+    return m
+
+
+def _header_functions():
+    src = open(os.path.join(ROOT, "include", "ipd.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(ipd_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_library_exports_every_declared_function(ipd):
+    names = _header_functions()
+    assert len(names) >= 10
+    for n in names:
+        assert hasattr(ipd.lib(), n), n
+    assert sorted(ipd.EXPORTS) == names
+
+
+def test_status_strings_and_version(ipd):
+    assert ipd.lib().ipd_status_string(0) == b"IPD_OK"
+    assert ipd.lib().ipd_status_string(3) == b"IPD_ERR_WORKSPACE"
+    assert ipd.lib().ipd_status_string(99) == b"IPD_ERR_UNKNOWN"
+    assert ipd.lib().ipd_version() == 100
+
+
+def _fake_batch(ipd, hd=128, ps=16, hkv=4, hq=32, R=2, maxq=4, maxs=100):
+    c = ipd._KVCache(16, 16, 10, ps, hkv, hd)
+    b = ipd._AttnBatch(ctypes.pointer(c), hq, R, 16, 16, 16, 16, (maxs + 15) // 16, R * maxq,
+                       maxq, maxs, 16)
+    return c, b
+
+
+def test_attn_host_validation(ipd):
+    L = ipd.lib()
+    c, b = _fake_batch(ipd)
+    arr = (ipd._AttnBatch * 1)(b)
+    assert L.ipd_attn_workspace_size(arr, 1, None, 0) > 0
+    # too small a workspace is refused before any device call
+    assert L.ipd_verify_attn(arr, 1, None, 0, 0.088, 256, 16, None) == ipd.STATUS_CODES["IPD_ERR_WORKSPACE"]
+    for kw, code in ((dict(hd=64), "IPD_ERR_UNSUPPORTED"), (dict(ps=32), "IPD_ERR_UNSUPPORTED"),
+                     (dict(hq=30), "IPD_ERR_INVALID_ARG"), (dict(maxs=2, maxq=4), "IPD_ERR_INVALID_ARG")):
+        c2, b2 = _fake_batch(ipd, **kw)
+        a2 = (ipd._AttnBatch * 1)(b2)
+        assert L.ipd_verify_attn(a2, 1, None, 0, 0.088, 256, 1 << 30, None) == ipd.STATUS_CODES[code], kw
+        assert L.ipd_attn_workspace_size(a2, 1, None, 0) == 0
+    many = (ipd._AttnBatch * 9)(*([b] * 9))
+    assert L.ipd_verify_attn(many, 9, None, 0, 0.088, 256, 1 << 30, None) == ipd.STATUS_CODES["IPD_ERR_INVALID_ARG"]
+    assert L.ipd_verify_attn(arr, 1, None, 0, -1.0, 256, 1 << 30, None) == ipd.STATUS_CODES["IPD_ERR_INVALID_ARG"]
+    # no batches at all: nothing to do
+    assert L.ipd_verify_attn(None, 0, None, 0, 0.088, None, 0, None) == 0
+
+
+def test_score_and_loss_host_validation(ipd):
+    L = ipd.lib()
+    p = [16] * 6
+    outs = [16] * 13
+    bad = ipd.STATUS_CODES
+    args = lambda R, T, V, K: p + [R, T, V, K, -1] + outs + [16, 1 << 30, None]
+    assert L.ipd_score_span(*args(2, 4, 4096, 33)) == bad["IPD_ERR_UNSUPPORTED"]
+    assert L.ipd_score_span(*args(2, 4, 4096, 0)) == bad["IPD_ERR_UNSUPPORTED"]
+    assert L.ipd_score_span(*args(2, 4, 4100, 16)) == bad["IPD_ERR_UNSUPPORTED"]
+    assert L.ipd_score_span(*args(2, 4, 8, 16)) == bad["IPD_ERR_UNSUPPORTED"]
+    assert L.ipd_score_span(*args(-1, 4, 4096, 16)) == bad["IPD_ERR_INVALID_ARG"]
+    small_ws = p + [2, 4, 4096, 16, -1] + outs + [16, 8, None]
+    assert L.ipd_score_span(*small_ws) == bad["IPD_ERR_WORKSPACE"]
+    assert L.ipd_score_workspace_size(2, 4, 4096, 16) >= 8 * 2 * 4
+    assert L.ipd_loss_workspace_size(10) == 0
+    assert L.ipd_split_loss(16, 16, 16, 16, 16, None, 3, 2, 0, 16, None, 0, None) == bad["IPD_ERR_INVALID_ARG"]
+    assert L.ipd_split_loss(16, 16, 16, 16, 16, None, 3, 0, 7, 16, None, 0, None) == bad["IPD_ERR_INVALID_ARG"]
+    assert L.ipd_split_loss(16, 16, 16, 16, 16, None, 3, 0, 0, None, None, 0, None) == bad["IPD_ERR_INVALID_ARG"]

@@ -1,0 +1,179 @@
+"""CUDA path vs the fp64 oracle, through the C ABI (needs a GB300)."""
+import numpy as np
+import pytest
+import torch
+
+import ipd_synth as S
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_36546_gb300 import ipd
+    return ipd
+
+
+def _run(spec, seed, device="cuda", **kw):
+    from paper_2609_36546_gb300 import VerifyStep
+    w = S.make_workload(spec, seed=seed, device="cpu")
+    step = VerifyStep.from_workload(w, device=device, **kw)
+    step.run()
+    torch.cuda.synchronize()
+    return w, step
+
+
+SMALL = [
+    ("mixed", S.small_spec(), 0),
+    ("short-ctx", S.small_spec(n_req=8, ctx=(1, 40), span=(1, 8)), 1),
+    ("one-page", S.small_spec(n_req=5, ctx=(16, 16), span=(1, 4)), 2),
+    ("long-split-128rows", S.small_spec(n_req=3, ctx=(1000, 3000), span=(16, 16), direction="S"), 3),
+    ("teacher-driving", S.small_spec(n_req=6, direction="T", span=(1, 16), ctx=(20, 700)), 4),
+    ("ties", S.small_spec(n_req=6, vocab=4096, sigma=3.0, tie_quantum=0.5, span=(2, 6)), 5),
+    ("accept-all", S.small_spec(n_req=5, force="accept", span=(3, 9)), 6),
+    ("reject-all", S.small_spec(n_req=5, force="reject", span=(3, 9)), 7),
+    ("mixed-eos", S.small_spec(n_req=10, force="mixed", eos_id=5, eos_prob=0.3, span=(2, 10)), 8),
+    ("K1", S.small_spec(n_req=4, K=1), 9),
+    ("K32", S.small_spec(n_req=4, K=32, vocab=8192), 10),
+    ("V-equals-K", S.small_spec(n_req=3, K=8, vocab=8, ctx=(1, 50)), 11),
+    ("wide-vocab", S.small_spec(n_req=2, vocab=151936, sigma=3.0, logits="boost", span=(4, 8),
+                                ctx=(100, 400)), 12),
+]
+
+
+@pytest.mark.parametrize("name,spec,seed", SMALL, ids=[c[0] for c in SMALL])
+def test_small_cases_match_oracle(lib, name, spec, seed):
+    from tests import parity
+    w, step = _run(spec, seed)
+    rep = parity.check_step(step, w)
+    assert lib.device_error() == 0
+    assert rep["ok"], rep
+
+
+@pytest.mark.parametrize("agg,dirm", [(0, 0), (1, 0), (0, 1), (0, 2), (0, 3)])
+def test_loss_modes_and_resp_len(lib, agg, dirm):
+    from tests import parity
+    spec = S.small_spec(n_req=7, force="mixed", span=(1, 8))
+    w0 = S.make_workload(spec, seed=21, device="cpu")
+    resp = torch.randint(5, 60, (7,), generator=torch.Generator().manual_seed(1), dtype=torch.int32)
+    resp[2] = 0
+    for rl in (None, resp):
+        from paper_2609_36546_gb300 import VerifyStep
+        step = VerifyStep.from_workload(w0, device="cuda", agg_mode=agg, dir_mode=dirm,
+                                        resp_len=rl)
+        step.run()
+        torch.cuda.synchronize()
+        rep = parity.check_step(step, w0)
+        assert rep["ok"], rep
+
+
+def test_config0_full(lib):
+    from tests import parity
+    w, step = _run(0, 0)
+    rep = parity.check_step(step, w)
+    assert rep["ok"], rep
+
+
+def test_outputs_are_deterministic(lib):
+    spec = S.small_spec(n_req=6, ctx=(200, 3000), span=(1, 16))
+    w, step = _run(spec, 31)
+    first = {k: v.clone() for k, v in step.score.items()}
+    outs = [b.out.clone() for _, b, _, _ in step.batches]
+    o8 = step.out8.clone()
+    step.run()
+    torch.cuda.synchronize()
+    for k, v in step.score.items():
+        assert torch.equal(first[k].view(torch.uint8), v.view(torch.uint8)), k
+    for a, (_, b, _, _) in zip(outs, step.batches):
+        assert torch.equal(a.view(torch.int16), b.out.view(torch.int16))
+    assert torch.equal(o8, step.out8)
+
+
+def test_decode_alone_equals_colaunched(lib):
+    spec = S.small_spec(n_req=6, ctx=(10, 900))
+    w, step = _run(spec, 41)
+    ref = [b.out.clone() for b in step.decode]
+    for b in step.decode:
+        b.out.zero_()
+    ws = torch.empty(max(256, lib.attn_workspace_size([], step.decode)), dtype=torch.uint8,
+                     device="cuda")
+    lib.decode_attn(step.decode, step.scale, ws)
+    torch.cuda.synchronize()
+    for a, b in zip(ref, step.decode):
+        assert torch.equal(a.view(torch.int16), b.out.view(torch.int16))
+
+
+def test_device_checks_report_bad_page_ids_and_tokens(lib):
+    from paper_2609_36546_gb300 import VerifyStep
+    spec = S.small_spec(n_req=3, ctx=(40, 60))
+    w = S.make_workload(spec, seed=5, device="cpu")
+    w.teacher.page_table[0, 0] = 10 ** 6          # outside the pool: skipped and reported
+    w.student.page_table[0, 0] = 10 ** 6
+    step = VerifyStep.from_workload(w, device="cuda")
+    step.run_attention()
+    assert lib.device_error() == 1                 # IPD_DEVERR_PAGE_ID
+    assert lib.device_error() == 0                 # read-and-clear
+    w2 = S.make_workload(spec, seed=6, device="cpu")
+    w2.tokens[0] = spec.vocab + 3
+    step2 = VerifyStep.from_workload(w2, device="cuda")
+    step2.run_score()
+    assert lib.device_error() == 3                 # IPD_DEVERR_TOKEN
+
+
+def test_empty_spans(lib):
+    """Requests with a zero-length span: nothing emitted, caches keep their length."""
+    R, V = 3, 64
+    dev = "cuda"
+    ls = torch.zeros((0, V), dtype=torch.bfloat16, device=dev)
+    out = lib.alloc_score_outputs(R, 0, dev)
+    cu = torch.zeros(R + 1, dtype=torch.int32, device=dev)
+    drv = torch.tensor([0, 1, 0], dtype=torch.uint8, device=dev)
+    pre = torch.tensor([5, 6, 7], dtype=torch.int32, device=dev)
+    ws = torch.empty(256, dtype=torch.uint8, device=dev)
+    toks = torch.zeros(0, dtype=torch.int32, device=dev)
+    lib.score_span(ls, ls, toks, cu, drv, pre, 4, -1, out, ws)
+    torch.cuda.synchronize()
+    assert out["n_emit"].tolist() == [0, 0, 0]
+    assert out["first_trans"].tolist() == [0, 0, 0]
+    assert out["new_len"].tolist() == [5, 6, 7]
+    assert out["next_driver"].tolist() == [0, 1, 0]
+
+
+def _sampled(idx, n=3, seed=0):
+    rng = np.random.default_rng(seed)
+    return sorted(rng.choice(idx, min(n, len(idx)), replace=False).tolist())
+
+
+@pytest.mark.parametrize("cfg", [1, 2, 3, 4])
+def test_full_size_configs_sampled(lib, cfg):
+    """Full-size workloads (generated on the device, launch configuration of
+    the benchmark); outputs of a sample of requests are recomputed by the
+    oracle one by one, and batch-level properties are checked on all of them."""
+    from paper_2609_36546_gb300 import VerifyStep
+    from tests import parity
+    w = S.make_workload(cfg, device="cuda")
+    step = VerifyStep.from_workload(w, device="cuda")
+    step.run()
+    torch.cuda.synchronize()
+    assert lib.device_error() == 0
+    reqs = sorted(set(_sampled(step.idx_s.numpy(), 2, cfg)) | set(_sampled(step.idx_t.numpy(), 2, cfg)))
+    rep = parity.check_step(step, w, requests=reqs, attn_max_reqs=None)
+    assert rep["ok"], rep
+    # properties over the whole batch
+    sc = {k: v.cpu() for k, v in step.score.items()}
+    o8 = step.out8.cpu()
+    emitted = sc["source"] != 255
+    assert int(emitted.sum()) == int(sc["n_emit"].sum())
+    assert float(o8[3] + o8[4]) == float(emitted.sum())
+    assert torch.all(sc["kl_rev"] >= -1e-5) and torch.all(sc["kl_fwd"] >= -1e-5)
+    assert torch.all(sc["logp_s"] <= 1e-6) and torch.all(sc["logp_t"] <= 1e-6)
+    assert torch.all(sc["new_len"] == step.prefix_len.cpu() + sc["n_emit"])
+    print(f"cfg{cfg}:", {k: rep[k] for k in ("attn_max_ulp", "attn_max_ulp_strict",
+                                              "attn_frac_strict_le2", "max_logp_err", "max_kl_err",
+                                              "near_threshold", "coverage_rate")})
+    del step, w
+    torch.cuda.empty_cache()
