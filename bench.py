@@ -41,6 +41,20 @@ def _peaks():
         return HBM_FALLBACK_GBS, "fallback"
 
 
+def _committed_traffic(cfg: int):
+    """DRAM bytes per attention launch from the committed ncu capture, or None
+    when the kernel source has changed since that capture."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", f"attn_traffic_cfg{cfg}.json")
+    src = os.path.join(ROOT, "paper_2609_36546_gb300", "csrc", "attn.cu")
+    try:
+        rec = json.load(open(path))
+        h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        return rec["traffic_bytes_per_launch"] if rec.get("source_sha256_16") == h else None
+    except Exception:
+        return None
+
+
 def _workload_name(cfg: int) -> str:
     import ipd_synth as S
     s = S.CONFIGS[cfg]
@@ -362,13 +376,7 @@ def run_gpu(args):
     if rank != 0:
         return
     achieved = attn_bytes / (attn_ms / 1e3) / 1e9
-    traffic = None
-    tr_path = os.path.join(ROOT, "profiles", f"attn_traffic_cfg{cfg}.json")
-    if os.path.exists(tr_path):
-        try:
-            traffic = json.load(open(tr_path)).get("traffic_bytes_per_launch")
-        except Exception:
-            traffic = None
+    traffic = _committed_traffic(cfg)
     step_alg = attn_bytes + logits_alg
     step_full = attn_bytes + logits_full
     line = {

@@ -7,15 +7,30 @@
 // one persistent launch over both caches, whose GQA shapes differ.
 //
 // Work decomposition (device side, no host round trip):
-//   task  = (batch, request, kv head, row block of <= kRowsCuda query rows)
+//   task  = (batch, request, kv head, row block); a row is one (span query,
+//           query head) pair, row = i * G + j for query i and head kvh*G + j.
 //   item  = (task, KV chunk); long tasks are split into chunks so that the
-//           work list has about kTargetItems items, and split partials are
-//           merged by the last CTA to finish a task (atomic ticket, no wait).
-// A row is one (query, query head) pair of a task: row = i * G + j for span
-// query i and head kvh * G + j.
+//           work list has about 8 items per SM; split partials are merged by
+//           the last CTA to finish a task (atomic ticket, no waiting).
+// Two compute paths, chosen per task by its row count:
+//   tensor path (rows >= kTcMinRows): a 128-row tile.  S = Q K^T and
+//     O += P V run on tcgen05 (bf16 operands in 128-byte-swizzled shared
+//     memory, fp32 accumulators in TMEM); one thread per row does the online
+//     softmax.  O stays in TMEM for the whole item and is rescaled only when
+//     a row maximum grows by more than 2^8 (exponentials are taken against a
+//     stale maximum until then).  P is passed as two bf16 terms (value and
+//     rounded residual), so the P V product keeps about 16 bits of each
+//     probability.  S and P are double-buffered: the softmax of chunk j
+//     overlaps the P V product of chunk j-1 and the Q K^T product of j+1.
+//   CUDA-core path (fewer rows: GQA group 2 decode): fp32 FMA, one page of 16
+//     keys per warp, two lanes per key.
+// Warp roles: warps 0-3 compute, warp 4 streams KV pages with 2-D TMA into a
+// 3-stage mbarrier ring, warp 5 issues the tensor-core instructions.
+#include <cuda.h>
 #include <cuda_runtime.h>
+#include <cudaTypedefs.h>
 #include <stdint.h>
-#include <stdio.h>
+#include <string.h>
 
 #include <algorithm>
 
@@ -27,16 +42,27 @@ namespace {
 
 constexpr int kPage = 16;
 constexpr int kD = 128;
-constexpr int kTileBytes = kPage * kD * 2;  // one page of one KV head: 4 KB
-constexpr int kRowsCuda = 64;               // rows per item
-constexpr int kPPS = 8;                     // pages per pipeline stage
-constexpr int kStages = 2;
-constexpr int kCW = 8;                      // consumer warps
-constexpr int kThreads = (kCW + 1) * 32;    // + one producer warp
-constexpr int kTargetItems = 2048;
+constexpr int kStagePages = 4;                    // 64 keys per stage
+constexpr int kStageKeys = kStagePages * kPage;
+constexpr int kStages = 3;
+constexpr int kHalfBytes = kStageKeys * 128;      // one 64-dim half of 64 key rows: 8 KB
+constexpr int kStageBytes = 4 * kHalfBytes;       // K and V, two halves each: 32 KB
+constexpr int kTcRows = 128;                      // rows of a tensor-core tile (M)
+constexpr int kTcMinRows = 8;                     // tasks with at least this many rows use it
+constexpr int kCcRows = kTcMinRows - 1;           // CUDA-core tasks have fewer rows
+constexpr int kCW = 4;                            // compute warps
+constexpr int kProducerWarp = 4;
+constexpr int kMmaWarp = 5;
+constexpr int kThreads = 6 * 32;
+constexpr int kTargetItemsPerSm = 8;
+constexpr int kMaxTargetItems = 4096;            // bound used for workspace sizing
 constexpr int kMinChunkPages = 16;
 constexpr int kSplitMax = 16;
-constexpr int kPStride = 132;               // floats per partial row: o[128], m, l, pad
+constexpr int kPStride = 132;                     // floats per partial row: o[128], m, l, pad
+constexpr uint32_t kTmemCols = 512;
+// TMEM columns: S double buffer at 0 and 64, the O accumulator at 128..255
+__device__ __forceinline__ uint32_t col_s(uint32_t b) { return b * 64u; }
+__device__ __forceinline__ uint32_t col_o(uint32_t b) { return 128u + b * 128u; }
 
 struct BatchDev {
   const uint16_t *q;
@@ -44,19 +70,18 @@ struct BatchDev {
   const int *cu_q;
   const int *seq_len;
   const int *page_table;
-  const uint16_t *k_pages;
-  const uint16_t *v_pages;
   long long num_pages;
-  int num_reqs, hq, hkv, group, max_pages, max_q_len, total_q;
+  int num_reqs, hq, hkv, group, max_pages, max_q_len, total_q, cache;
 };
 
 struct Item {
   int b, r, kvh, rb;
   int split, n_split, page_lo, page_hi;
-  int task, pbase, rows, pad;
+  int task, pbase, rows, path;  // path: 1 = tensor cores, 0 = CUDA cores
 };
 
 struct AttnParams {
+  CUtensorMap tmap[2 * IPD_MAX_BATCHES];  // K and V map of every distinct cache
   BatchDev b[IPD_MAX_BATCHES];
   int req_base[IPD_MAX_BATCHES + 1];
   int n_batches;
@@ -69,6 +94,7 @@ struct AttnParams {
   float *partials;
   int item_cap, task_cap;
   long long prow_cap;
+  int target_items;  // work-list size the planner aims for (a multiple of the SM count)
 };
 
 struct StageMeta {
@@ -77,7 +103,8 @@ struct StageMeta {
   int npages;
   int flags;        // 1 = first stage of its item, 2 = last stage
   uint32_t invalid; // pages of the stage whose id failed validation
-  int pad[3];
+  int path;
+  int pad[2];
 };
 
 // --------------------------------------------------------------------------
@@ -97,13 +124,14 @@ int validate_batch(const ipd_attn_batch *b) {
   if (c->page_size != kPage || c->head_dim != kD) return IPD_ERR_UNSUPPORTED;
   if (c->num_kv_heads < 1 || c->num_kv_heads > 64) return IPD_ERR_UNSUPPORTED;
   if (b->num_q_heads < 1 || b->num_q_heads % c->num_kv_heads) return IPD_ERR_INVALID_ARG;
-  if (b->num_q_heads / c->num_kv_heads > kRowsCuda) return IPD_ERR_UNSUPPORTED;
+  if (b->num_q_heads / c->num_kv_heads > kTcRows) return IPD_ERR_UNSUPPORTED;
   if (b->num_reqs < 0 || b->total_q < 0 || b->max_q_len < 0 || b->max_seq_len < 0)
     return IPD_ERR_INVALID_ARG;
   if (b->num_reqs == 0) return IPD_OK;
   if (b->max_q_len < 1 || b->max_seq_len < b->max_q_len) return IPD_ERR_INVALID_ARG;
   if ((long long)b->max_pages * kPage < b->max_seq_len) return IPD_ERR_INVALID_ARG;
   if (c->num_pages < 1) return IPD_ERR_INVALID_ARG;
+  if (c->num_pages * c->num_kv_heads * (long long)kPage >= (1LL << 31)) return IPD_ERR_UNSUPPORTED;
   if (!b->q || !b->out || !b->cu_q || !b->seq_len || !b->page_table || !c->k_pages ||
       !c->v_pages)
     return IPD_ERR_INVALID_ARG;
@@ -121,10 +149,15 @@ int collect(const ipd_attn_batch *verify, int nv, const ipd_attn_batch *decode, 
   for (int i = 0; i < nv; ++i) out[n++] = &verify[i];
   for (int i = 0; i < nd; ++i) out[n++] = &decode[i];
   for (int i = 0; i < n; ++i) {
-    int st = validate_batch(out[i]);
+    const int st = validate_batch(out[i]);
     if (st != IPD_OK) return st;
   }
   return IPD_OK;
+}
+
+// rows per row block of a task with `rows` rows
+__host__ __device__ inline int rows_per_block(int rows) {
+  return rows >= kTcMinRows ? kTcRows : kCcRows;
 }
 
 WsLayout layout(const ipd_attn_batch *const *bs, int n) {
@@ -133,14 +166,18 @@ WsLayout layout(const ipd_attn_batch *const *bs, int n) {
   int reqs = 0;
   for (int i = 0; i < n; ++i) {
     const ipd_attn_batch *b = bs[i];
-    int G = b->num_q_heads / b->cache->num_kv_heads;
-    long long nrb = ((long long)b->max_q_len * G + kRowsCuda - 1) / kRowsCuda;
+    const int G = b->num_q_heads / b->cache->num_kv_heads;
+    // a task with r rows has ceil(r / rows_per_block(r)) row blocks; the
+    // largest r = max_q_len * G bounds every request of the batch
+    const long long rmax = (long long)b->max_q_len * G;
+    const long long nrb = rmax >= kTcMinRows ? (rmax + kTcRows - 1) / kTcRows : 1;
     task_cap += (long long)b->num_reqs * b->cache->num_kv_heads * nrb;
     rows_all += (long long)b->total_q * b->num_q_heads;
     reqs += b->num_reqs;
   }
-  long long item_cap = task_cap + 2LL * kTargetItems;
-  long long prow_cap = std::min<long long>(2LL * kTargetItems * kRowsCuda, kSplitMax * rows_all);
+  const long long item_cap = task_cap + 2LL * kMaxTargetItems;
+  const long long prow_cap =
+      std::min<long long>(2LL * kMaxTargetItems * kTcRows, (long long)kSplitMax * rows_all);
   L.item_cap = (int)std::min<long long>(item_cap, 1LL << 30);
   L.task_cap = (int)std::min<long long>(task_cap, 1LL << 30);
   L.prow_cap = prow_cap;
@@ -170,13 +207,13 @@ __device__ __forceinline__ int find_batch(const AttnParams &p, int gi) {
 }
 
 struct ReqShape {
-  int ql, L, pages, rows, nrb, ok;
+  int ql, L, pages, rows, nrb, rpb, ok;
 };
 
 __device__ ReqShape req_shape(const AttnParams &p, int b, int r) {
   const BatchDev &B = p.b[b];
   ReqShape s{};
-  int c0 = B.cu_q[r], c1 = B.cu_q[r + 1];
+  const int c0 = B.cu_q[r], c1 = B.cu_q[r + 1];
   s.ql = c1 - c0;
   s.L = B.seq_len[r];
   s.ok = 1;
@@ -188,18 +225,19 @@ __device__ ReqShape req_shape(const AttnParams &p, int b, int r) {
     s.ok = 0;
   }
   if (!s.ok || s.ql == 0) {
-    s.ql = 0; s.L = 0; s.pages = 0; s.rows = 0; s.nrb = 0;
+    s.ql = 0; s.L = 0; s.pages = 0; s.rows = 0; s.nrb = 0; s.rpb = 1;
     return s;
   }
   s.pages = (s.L + kPage - 1) / kPage;
   s.rows = s.ql * B.group;
-  s.nrb = (s.rows + kRowsCuda - 1) / kRowsCuda;
+  s.rpb = rows_per_block(s.rows);
+  s.nrb = (s.rows + s.rpb - 1) / s.rpb;
   return s;
 }
 
 template <typename T>
 __device__ T block_sum(T v, T *red) {
-  int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   __syncthreads();
@@ -213,13 +251,13 @@ __device__ T block_sum(T v, T *red) {
 
 // exclusive scan of three ints across the block; returns totals in tot
 __device__ void block_scan3(int3 v, int3 &excl, int3 &tot, int3 *sh) {
-  int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
   int3 inc = v;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
-    int x = __shfl_up_sync(0xffffffffu, inc.x, o);
-    int y = __shfl_up_sync(0xffffffffu, inc.y, o);
-    int z = __shfl_up_sync(0xffffffffu, inc.z, o);
+    const int x = __shfl_up_sync(0xffffffffu, inc.x, o);
+    const int y = __shfl_up_sync(0xffffffffu, inc.y, o);
+    const int z = __shfl_up_sync(0xffffffffu, inc.z, o);
     if (lane >= o) { inc.x += x; inc.y += y; inc.z += z; }
   }
   __syncthreads();
@@ -244,26 +282,26 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const __grid_constant__
 
   long long w = 0;
   for (int gi = tid; gi < p.total_reqs; gi += blockDim.x) {
-    int b = find_batch(p, gi);
-    ReqShape s = req_shape(p, b, gi - p.req_base[b]);
+    const int b = find_batch(p, gi);
+    const ReqShape s = req_shape(p, b, gi - p.req_base[b]);
     w += (long long)s.pages * p.b[b].hkv * s.nrb;
   }
-  long long W = block_sum<long long>(w, red);
-  long long chunk = (W + kTargetItems - 1) / kTargetItems;
+  const long long W = block_sum<long long>(w, red);
+  long long chunk = (W + p.target_items - 1) / p.target_items;
   if (chunk < kMinChunkPages) chunk = kMinChunkPages;
 
   int3 carry = make_int3(0, 0, 0);
   for (int base = 0; base < p.total_reqs; base += blockDim.x) {
-    int gi = base + tid;
+    const int gi = base + tid;
     int3 cnt = make_int3(0, 0, 0);
     int nsplit = 1;
     if (gi < p.total_reqs) {
-      int b = find_batch(p, gi);
-      ReqShape s = req_shape(p, b, gi - p.req_base[b]);
+      const int b = find_batch(p, gi);
+      const ReqShape s = req_shape(p, b, gi - p.req_base[b]);
       if (s.pages > 0) {
-        long long ns = (s.pages + chunk - 1) / chunk;
+        const long long ns = (s.pages + chunk - 1) / chunk;
         nsplit = (int)(ns < kSplitMax ? ns : kSplitMax);
-        int tasks = p.b[b].hkv * s.nrb;
+        const int tasks = p.b[b].hkv * s.nrb;
         cnt = make_int3(tasks * nsplit, tasks, nsplit > 1 ? nsplit * p.b[b].hkv * s.rows : 0);
       }
     }
@@ -287,17 +325,18 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const __grid_constant__
   if (s_fail) return;
 
   for (int gi = tid; gi < p.total_reqs; gi += blockDim.x) {
-    int b = find_batch(p, gi);
-    int r = gi - p.req_base[b];
-    ReqShape s = req_shape(p, b, r);
+    const int b = find_batch(p, gi);
+    const int r = gi - p.req_base[b];
+    const ReqShape s = req_shape(p, b, r);
     if (s.pages == 0) continue;
-    int4 info = p.reqinfo[gi];
-    int item = info.x, task = info.y, ns = info.w;
-    int per = (s.pages + ns - 1) / ns;
+    const int4 info = p.reqinfo[gi];
+    int item = info.x, task = info.y;
+    const int ns = info.w;
+    const int per = (s.pages + ns - 1) / ns;
     for (int kvh = 0; kvh < p.b[b].hkv; ++kvh) {
       for (int rb = 0; rb < s.nrb; ++rb) {
-        int rows = min(kRowsCuda, s.rows - rb * kRowsCuda);
-        int pbase = ns > 1 ? info.z + ns * (kvh * s.rows + rb * kRowsCuda) : -1;
+        const int rows = min(s.rpb, s.rows - rb * s.rpb);
+        const int pbase = ns > 1 ? info.z + ns * (kvh * s.rows + rb * s.rpb) : -1;
         p.tickets[task] = 0;
         for (int sp = 0; sp < ns; ++sp) {
           Item it;
@@ -305,10 +344,8 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const __grid_constant__
           it.split = sp; it.n_split = ns;
           it.page_lo = sp * per;
           it.page_hi = min(s.pages, (sp + 1) * per);
-          it.task = task; it.pbase = pbase; it.rows = rows; it.pad = 0;
-          if (it.page_lo >= it.page_hi) {  // cannot happen with per = ceil(pages/ns); kept safe
-            it.page_lo = it.page_hi = 0;
-          }
+          it.task = task; it.pbase = pbase; it.rows = rows;
+          it.path = s.rows >= kTcMinRows ? 1 : 0;
           p.items[item++] = it;
         }
         ++task;
@@ -318,170 +355,420 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const __grid_constant__
 }
 
 // --------------------------------------------------------------------------
-// attention kernel (CUDA cores)
+// the attention kernel
 // --------------------------------------------------------------------------
-struct SmemLayout {
-  static constexpr int kStageBytes = kPPS * 2 * kTileBytes;             // 64 KB
-  static constexpr int off_stage = 0;
-  static constexpr int off_q = off_stage + kStages * kStageBytes;       // fp32 [64][128]
-  static constexpr int off_p = off_q + kRowsCuda * kD * 4;              // fp32 [8 warps][8][16]
-  static constexpr int off_merge = off_p + kCW * 8 * 16 * 4;            // fp32 [8][8][132]
-  static constexpr int off_meta = off_merge + kCW * 8 * kPStride * 4;
+struct Smem {
+  static constexpr int off_stage = 0;                              // 3 x 32 KB, 1024-aligned
+  static constexpr int off_q = off_stage + kStages * kStageBytes;  // 32 KB
+  static constexpr int off_p = off_q + 2 * kTcRows * 128;          // 2 buffers x (hi, lo) x 16 KB
+  static constexpr int kPBytes = kTcRows * 128;                    // one 128 x 64 bf16 operand
+  static constexpr int off_meta = off_p + 4 * kPBytes;
   static constexpr int off_bar = off_meta + kStages * (int)sizeof(StageMeta);
-  static constexpr int off_misc = off_bar + 2 * kStages * 8;
+  static constexpr int n_bars = 2 * kStages + 1 + 2 + 2 + 2 + 1 + 1;
+  static constexpr int off_misc = off_bar + n_bars * 8;
   static constexpr int total = off_misc + 64;
+  // CUDA-core path scratch (inside the Q and P regions, unused by that path)
+  static constexpr int off_ccq = off_q;                              // fp32 [7][128]
+  static constexpr int off_merge = off_p;                            // fp32 [4][8][132]
+  static constexpr int off_ps = off_merge + kCW * 8 * kPStride * 4;  // fp32 [4][8][16]
+  // split-merge scratch (P region, free once an item's last P V product landed)
+  static constexpr int off_msc = off_p;                              // fp32 [128][16] + [128]
+};
+static_assert(Smem::off_ps + kCW * 8 * 16 * 4 <= Smem::off_meta, "CUDA-core scratch overflow");
+static_assert(Smem::total <= 227 * 1024, "shared memory");
+
+struct Bars {
+  uint64_t *full, *empty;     // KV ring
+  uint64_t *q_ready;          // Q tile written (one phase per tensor item)
+  uint64_t *s_full, *p_full;  // S = Q K^T landed / P written, per buffer
+  uint64_t *p_free;           // P V product done reading P, per buffer
+  uint64_t *o_full;           // P V product of a chunk landed in O (one phase per chunk)
+  uint64_t *o_free;           // O read out (one phase per tensor item)
 };
 
-__device__ __forceinline__ uint8_t *stage_tile(uint8_t *smem, int s, int page, int kv) {
-  return smem + SmemLayout::off_stage + s * SmemLayout::kStageBytes + (page * 2 + kv) * kTileBytes;
+__device__ __forceinline__ Bars bars(uint8_t *smem) {
+  uint64_t *b = reinterpret_cast<uint64_t *>(smem + Smem::off_bar);
+  Bars r;
+  r.full = b;
+  r.empty = b + kStages;
+  r.q_ready = b + 2 * kStages;
+  r.s_full = r.q_ready + 1;
+  r.p_full = r.s_full + 2;
+  r.p_free = r.p_full + 2;
+  r.o_full = r.p_free + 2;
+  r.o_free = r.o_full + 1;
+  return r;
 }
 
-// fp32 Q layout in shared memory: for a row, dim d = half*64 + c*8 + sub*4 + e is
-// stored at half*64 + sub*32 + c*4 + e, so that eight lanes reading chunk
-// (c + lane) & 7 of the same row touch eight different bank groups.
+// byte offset of 16-byte chunk c (0..7) of row `row` in a 128-byte-swizzled
+// block of 128-byte rows (the layout TMA writes with SWIZZLE_128B)
+__device__ __forceinline__ uint32_t sw128(int row, int c) {
+  return (uint32_t)(row * 128 + ((c ^ (row & 7)) << 4));
+}
+
+__device__ __forceinline__ uint8_t *stage_k(uint8_t *smem, int s) {
+  return smem + Smem::off_stage + s * kStageBytes;
+}
+__device__ __forceinline__ uint8_t *stage_v(uint8_t *smem, int s) {
+  return stage_k(smem, s) + 2 * kHalfBytes;
+}
+
+// fp32 Q layout of the CUDA-core path: dim d = half*64 + c*8 + sub*4 + e is
+// stored at half*64 + sub*32 + c*4 + e (conflict-free float4 reads below).
 __device__ __forceinline__ int q_slot(int d) {
-  int half = d >> 6, c = (d >> 3) & 7, sub = (d >> 2) & 1, e = d & 3;
+  const int half = d >> 6, c = (d >> 3) & 7, sub = (d >> 2) & 1, e = d & 3;
   return half * 64 + sub * 32 + c * 4 + e;
 }
 
-__global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant__ AttnParams p) {
-  extern __shared__ __align__(1024) uint8_t smem[];
-  float *qs = reinterpret_cast<float *>(smem + SmemLayout::off_q);
-  float *ps = reinterpret_cast<float *>(smem + SmemLayout::off_p);
-  float *mg = reinterpret_cast<float *>(smem + SmemLayout::off_merge);
-  StageMeta *meta = reinterpret_cast<StageMeta *>(smem + SmemLayout::off_meta);
-  uint64_t *full = reinterpret_cast<uint64_t *>(smem + SmemLayout::off_bar);
-  uint64_t *empty = full + kStages;
-  int *misc = reinterpret_cast<int *>(smem + SmemLayout::off_misc);
 
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], kCW);
+struct CompCtx {
+  uint8_t *smem;
+  Bars B;
+  StageMeta *meta;
+  uint32_t *misc;  // [0] TMEM base, [1] abort flag, [2] ticket broadcast
+  uint32_t tmem;
+  int warp, lane, ctid;
+};
+
+__device__ __forceinline__ bool wait_or_abort(const CompCtx &X, uint64_t *bar, uint32_t par) {
+  if (mbar_wait_bounded(bar, par)) return true;
+  ipd_set_error(&g_attn_err, IPD_DEVERR_WAIT);
+  atomicExch(&X.misc[1], 1u);
+  return false;
+}
+
+struct ItemGeom {
+  const BatchDev *Bt;
+  int q0, ql, L, G, hq;
+};
+
+__device__ __forceinline__ ItemGeom item_geom(const AttnParams &p, const Item &I) {
+  ItemGeom g;
+  g.Bt = &p.b[I.b];
+  g.q0 = g.Bt->cu_q[I.r];
+  g.ql = g.Bt->cu_q[I.r + 1] - g.q0;
+  g.L = g.Bt->seq_len[I.r];
+  g.G = g.Bt->group;
+  g.hq = g.Bt->hq;
+  return g;
+}
+
+// query / output row of task row `grow` (query grow / G, head kvh * G + grow % G)
+__device__ __forceinline__ size_t row_off(const ItemGeom &g, const Item &I, int grow) {
+  const int qi = grow / g.G, j = grow % g.G;
+  return ((size_t)(g.q0 + qi) * g.hq + I.kvh * g.G + j) * kD;
+}
+__device__ __forceinline__ uint16_t *out_row(const ItemGeom &g, const Item &I, int grow) {
+  return g.Bt->out + row_off(g, I, grow);
+}
+__device__ __forceinline__ const uint16_t *q_row(const ItemGeom &g, const Item &I, int grow) {
+  return g.Bt->q + row_off(g, I, grow);
+}
+
+// The last CTA of a split task merges the partials of all its splits.
+// Step 1 (thread = row): scale factors of every split.  Step 2 (warp = 4 rows
+// at a time, lane = 4 dims): weighted sums, all split loads in flight at once.
+__device__ void merge_splits(const AttnParams &p, const CompCtx &X, const Item &I,
+                             const ItemGeom &g) {
+  float *sc = reinterpret_cast<float *>(X.smem + Smem::off_msc);  // [128][kSplitMax]
+  float *inv_l = sc + kTcRows * kSplitMax;                         // [128]
+  const int ns = I.n_split;
+  const size_t sstr = (size_t)I.rows * kPStride;
+  const int rpb = I.path ? kTcRows : kCcRows;
+  for (int r = X.ctid; r < I.rows; r += kCW * 32) {
+    const float *base = p.partials + (size_t)(I.pbase + r) * kPStride;
+    float mv[kSplitMax], lv[kSplitMax];
+#pragma unroll
+    for (int sp = 0; sp < kSplitMax; ++sp) {
+      mv[sp] = sp < ns ? __ldcg(base + sp * sstr + 128) : -INFINITY;
+      lv[sp] = sp < ns ? __ldcg(base + sp * sstr + 129) : 0.f;
     }
-    misc[0] = 0;  // abort flag
-    fence_mbar_init();
+    float Mx = -INFINITY;
+#pragma unroll
+    for (int sp = 0; sp < kSplitMax; ++sp) Mx = fmaxf(Mx, mv[sp]);
+    float Ls = 0.f;
+#pragma unroll
+    for (int sp = 0; sp < kSplitMax; ++sp) {
+      const float f = mv[sp] == -INFINITY ? 0.f : ex2_approx(mv[sp] - Mx);
+      sc[r * kSplitMax + sp] = f;
+      Ls = fmaf(lv[sp], f, Ls);
+    }
+    inv_l[r] = Ls > 0.f ? 1.f / Ls : 0.f;
   }
-  __syncthreads();
-  const int n_items = p.ctrl[0];
-
-  if (warp == kCW) {
-    // ------------------------------ producer ------------------------------
-    const uint64_t policy = l2_policy_evict_first();
-    uint32_t it = 0;
-    bool aborted = false;
-    for (;;) {
-      int idx = 0;
-      if (lane == 0) idx = atomicAdd(&p.ctrl[1], 1);
-      idx = __shfl_sync(0xffffffffu, idx, 0);
-      if (idx >= n_items) break;
-      const Item I = p.items[idx];
-      const BatchDev &B = p.b[I.b];
-      const int *prow = B.page_table + (long long)I.r * B.max_pages;
-      for (int page = I.page_lo; page < I.page_hi && !aborted; page += kPPS) {
-        const int np = min(kPPS, I.page_hi - page);
-        const int s = it % kStages;
-        const uint32_t ph = (it / kStages) & 1;
-        if (!mbar_wait_bounded(&empty[s], ph ^ 1)) {
-          ipd_set_error(&g_attn_err, IPD_DEVERR_WAIT);
-          aborted = true;
-          break;
+  named_bar_sync(1, kCW * 32);
+  for (int r0 = X.warp * 4; r0 < I.rows; r0 += kCW * 4) {
+    float4 acc[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int r = r0 + u;
+      if (r < I.rows) {
+        const float *base = p.partials + (size_t)(I.pbase + r) * kPStride;
+#pragma unroll
+        for (int sp = 0; sp < kSplitMax; ++sp) {
+          if (sp < ns) {
+            const float f = sc[r * kSplitMax + sp];
+            const float4 ov = __ldcg(reinterpret_cast<const float4 *>(base + sp * sstr) + X.lane);
+            acc[u].x = fmaf(ov.x, f, acc[u].x);
+            acc[u].y = fmaf(ov.y, f, acc[u].y);
+            acc[u].z = fmaf(ov.z, f, acc[u].z);
+            acc[u].w = fmaf(ov.w, f, acc[u].w);
+          }
         }
-        int pid = -1;
-        bool ok = false;
-        if (lane < np) {
-          pid = prow[page + lane];
-          ok = pid >= 0 && (long long)pid < B.num_pages;
-          if (!ok) ipd_set_error(&g_attn_err, IPD_DEVERR_PAGE_ID);
-        }
-        const uint32_t okmask = __ballot_sync(0xffffffffu, ok);
-        if (lane == 0) {
-          StageMeta m;
-          m.item = idx;
-          m.page0 = page;
-          m.npages = np;
-          m.flags = (page == I.page_lo ? 1 : 0) | (page + np >= I.page_hi ? 2 : 0);
-          m.invalid = (~okmask) & ((1u << np) - 1u);
-          meta[s] = m;
-          mbar_arrive_expect_tx(&full[s], (uint32_t)__popc(okmask) * 2u * kTileBytes);
-        }
-        __syncwarp();
-        if (ok) {
-          const size_t off = ((size_t)pid * B.hkv + I.kvh) * (size_t)(kPage * kD);
-          bulk_g2s_evict_first(stage_tile(smem, s, lane, 0), B.k_pages + off, kTileBytes, &full[s],
-                               policy);
-          bulk_g2s_evict_first(stage_tile(smem, s, lane, 1), B.v_pages + off, kTileBytes, &full[s],
-                               policy);
-        }
-        ++it;
       }
-      if (aborted) break;
     }
-    if (!aborted) {
-      // end-of-work marker in the next slot, once the consumers have freed it
-      const int s = it % kStages;
-      const uint32_t ph = (it / kStages) & 1;
-      if (mbar_wait_bounded(&empty[s], ph ^ 1)) {
-        if (lane == 0) {
-          meta[s].item = -1;
-          mbar_arrive(&full[s]);
-        }
-        return;  // the consumers wait for every copy still in flight
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int r = r0 + u;
+      if (r < I.rows) {
+        const float inv = inv_l[r];
+        uint2 pk;
+        pk.x = pack_bf16x2(acc[u].x * inv, acc[u].y * inv);
+        pk.y = pack_bf16x2(acc[u].z * inv, acc[u].w * inv);
+        *reinterpret_cast<uint2 *>(out_row(g, I, I.rb * rpb + r) + X.lane * 4) = pk;
       }
-      ipd_set_error(&g_attn_err, IPD_DEVERR_WAIT);
     }
-    // time-out path: the consumers stopped; make sure no copy issued by this
-    // CTA is still landing in shared memory before the CTA exits.  No slot
-    // was reused after stage it-1, so the parities below are unambiguous.
-    if (lane == 0) atomicExch(&misc[0], 1);
-    for (uint32_t k = (it > (uint32_t)kStages ? it - kStages : 0); k < it; ++k)
-      (void)mbar_wait_bounded(&full[k % kStages], (k / kStages) & 1);
-    return;
   }
+}
 
-  // -------------------------------- consumers --------------------------------
-  const int ctid = threadIdx.x;  // 0 .. 255
-  uint32_t it = 0;
-  // item context (warp-uniform)
-  Item I{};
-  int ql = 0, L = 0, G = 1, hq = 1, q0 = 0, rows = 0;
-  int n_rg = 1, pw_count = 1, rg = 0, pw = 0, nrow_g = 0;
-  bool active = false;
-  float m[8], l[8], o[8][4];
+// Zero the V rows of stage s at or past the end of the sequence: unwritten
+// cache slots may hold non-finite bits, and a zero probability times NaN is NaN.
+__device__ __forceinline__ void zero_tail(const CompCtx &X, int s, int page0, int L) {
+  const int tail0 = max(L - page0 * kPage, 0);  // first key slot at or past L
+  if (tail0 >= kStageKeys) return;
+  uint8_t *vb = stage_v(X.smem, s);
+  for (int e = X.ctid; e < (kStageKeys - tail0) * 16; e += kCW * 32) {
+    const int row = tail0 + e / 16, cpart = e % 16;
+    *reinterpret_cast<uint4 *>(vb + (cpart >> 3) * kHalfBytes + row * 128 + (cpart & 7) * 16) =
+        make_uint4(0, 0, 0, 0);
+  }
+  fence_proxy_async_smem();
+  named_bar_sync(1, kCW * 32);
+}
 
-  for (;;) {
+// After this CTA wrote its split partial: take a ticket; the last CTA of the
+// task merges every split (compute warps; all threads call it).
+__device__ __forceinline__ void ticket_merge(const AttnParams &p, const CompCtx &X, const Item &I,
+                                             const ItemGeom &g) {
+  __threadfence();
+  named_bar_sync(1, kCW * 32);
+  if (X.ctid == 0) X.misc[2] = (atomicAdd(&p.tickets[I.task], 1) == I.n_split - 1);
+  named_bar_sync(1, kCW * 32);
+  if (X.misc[2]) {
+    __threadfence();
+    merge_splits(p, X, I, g);
+  }
+}
+
+// ============================ tensor-core path ============================
+// One 128-row tile over the item's KV chunks; thread = row.  Returns false on
+// a wait time-out.  `it` (stage counter) and `c` (chunk counter) advance.
+__device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, const Item &I,
+                                        uint32_t &it, uint32_t &c) {
+  const ItemGeom g = item_geom(p, I);
+  const Bars &B = X.B;
+  const int warp = X.warp, lane = X.lane;
+  const int row = warp * 32 + lane;
+  const bool real = row < I.rows;
+  const bool warp_rows = warp * 32 < I.rows;  // the warp owns at least one real row
+  const uint32_t tl = X.tmem + ((uint32_t)(warp * 32) << 16);
+  const int lim = g.L - g.ql + (I.rb * kTcRows + row) / g.G;  // last key this row sees
+  const int lim_all = g.L - g.ql;                             // every row sees up to here
+  const float sl2 = p.scale_log2;
+  float m_used = -INFINITY;  // maximum the exponentials are taken against (log2 units)
+  float l_run = 0.f;
+
+  for (bool first = true;; first = false) {
     const int s = it % kStages;
-    const uint32_t ph = (it / kStages) & 1;
-    if (!mbar_wait_bounded(&full[s], ph)) {
-      ipd_set_error(&g_attn_err, IPD_DEVERR_WAIT);
-      atomicExch(&misc[0], 1);
-      break;
+    if (!wait_or_abort(X, &B.full[s], (it / kStages) & 1)) return false;
+    const StageMeta M = X.meta[s];
+    zero_tail(X, s, M.page0, g.L);
+    if (first) {
+      // Q tile: rows rb*128 .. +127 of the task, bf16, swizzled, zero padded
+      uint8_t *qb = X.smem + Smem::off_q;
+      for (int e = X.ctid; e < kTcRows * 16; e += kCW * 32) {
+        const int r = e >> 4, cpart = e & 15;
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (r < I.rows) v = *reinterpret_cast<const uint4 *>(q_row(g, I, I.rb * kTcRows + r) + cpart * 8);
+        *reinterpret_cast<uint4 *>(qb + (cpart >> 3) * (kTcRows * 128) + sw128(r, cpart & 7)) = v;
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(B.q_ready);
     }
-    const StageMeta M = meta[s];
-    if (M.item < 0 || *(volatile int *)&misc[0]) break;
-    if (M.flags & 1) {
-      I = p.items[M.item];
-      const BatchDev &B = p.b[I.b];
-      q0 = B.cu_q[I.r];
-      ql = B.cu_q[I.r + 1] - q0;
-      L = B.seq_len[I.r];
-      G = B.group;
-      hq = B.hq;
-      rows = I.rows;
-      n_rg = (rows + 7) >> 3;
-      pw_count = kCW / n_rg;
-      rg = warp % n_rg;
-      pw = warp / n_rg;
-      active = pw < pw_count;
-      nrow_g = active ? min(8, rows - rg * 8) : 0;
-      // stage the item's query rows (fp32) into shared memory
-      for (int e = ctid; e < rows * (kD / 8); e += kCW * 32) {
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&B.empty[s]);  // this warp is done with the stage
+
+    const uint32_t b = c & 1;
+    if (!wait_or_abort(X, &B.s_full[b], (c >> 1) & 1)) return false;
+    tc_fence_after();
+    const int kp0 = M.page0 * kPage;
+    const bool full_vis =
+        M.npages == kStagePages && M.invalid == 0 && kp0 + kStageKeys - 1 <= lim_all;
+    uint32_t sr[2][32];
+    float mc = -INFINITY;  // chunk maximum of the raw scores
+    if (warp_rows) {
+      tc_ld_32x32b_x32(tl + col_s(b), sr[0]);
+      tc_ld_32x32b_x32(tl + col_s(b) + 32, sr[1]);
+      tc_wait_ld();
+      if (!full_vis) {
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            const int col = h * 32 + e;
+            const bool vis = (col >> 4) < M.npages && !((M.invalid >> (col >> 4)) & 1u) &&
+                             kp0 + col <= lim;
+            if (!vis) sr[h][e] = 0xff800000u;  // -inf
+          }
+      }
+#pragma unroll
+      for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int e = 0; e < 32; ++e) mc = fmaxf(mc, __uint_as_float(sr[h][e]));
+    }
+    // lazy rescale: keep the old maximum unless the new one is 2^8 larger
+    const float mcs = mc * sl2;
+    float alpha = 1.f;
+    bool resc = false;
+    if (real && mcs != -INFINITY) {
+      if (m_used == -INFINITY) {
+        m_used = mcs;
+      } else if (mcs > m_used + 8.f) {
+        alpha = ex2_approx(m_used - mcs);
+        m_used = mcs;
+        resc = true;
+      }
+    }
+    if (warp_rows && __any_sync(0xffffffffu, resc)) {
+      // O holds the P V products of earlier chunks of this item: let them land
+      if (!wait_or_abort(X, B.o_full, (c - 1) & 1)) return false;
+      tc_fence_after();
+#pragma unroll
+      for (int q4 = 0; q4 < kD / 32; ++q4) {
+        uint32_t r[32];
+        tc_ld_32x32b_x32(tl + col_o(0) + q4 * 32, r);
+        tc_wait_ld();
+#pragma unroll
+        for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
+        tc_st_32x32b_x32(tl + col_o(0) + q4 * 32, r);
+      }
+      tc_wait_st();
+    }
+    l_run *= alpha;
+    // probabilities, as bf16 value + bf16 residual, into P buffer b
+    if (!wait_or_abort(X, &B.p_free[b], ((c >> 1) & 1) ^ 1)) return false;
+    if (warp_rows) {
+      uint8_t *pb = X.smem + Smem::off_p + b * 2 * Smem::kPBytes;
+      const float moff = (!real || m_used == -INFINITY) ? -INFINITY : -m_used;  // -inf: p = 0
+      float lsum = 0.f;
+#pragma unroll
+      for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int cch = 0; cch < 4; ++cch) {
+          uint32_t whi[4], wlo[4];
+#pragma unroll
+          for (int t = 0; t < 4; ++t) {
+            const int e = cch * 8 + 2 * t;
+            const float p0 = ex2_approx(fmaf(__uint_as_float(sr[h][e]), sl2, moff));
+            const float p1 = ex2_approx(fmaf(__uint_as_float(sr[h][e + 1]), sl2, moff));
+            const uint32_t hi = pack_bf16x2(p0, p1);
+            whi[t] = hi;
+            wlo[t] = pack_bf16x2(p0 - bf16lo(hi), p1 - bf16hi(hi));
+            lsum += p0 + p1;
+          }
+          if (real) {
+            *reinterpret_cast<uint4 *>(pb + sw128(row, h * 4 + cch)) =
+                make_uint4(whi[0], whi[1], whi[2], whi[3]);
+            *reinterpret_cast<uint4 *>(pb + Smem::kPBytes + sw128(row, h * 4 + cch)) =
+                make_uint4(wlo[0], wlo[1], wlo[2], wlo[3]);
+          }
+        }
+      if (real) l_run += lsum;
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&B.p_full[b]);
+    ++it;
+    ++c;
+    if (M.flags & 2) break;
+  }
+
+  // ---- the tile is done once the last P V product has landed in O ----
+  if (!wait_or_abort(X, B.o_full, (c - 1) & 1)) return false;
+  tc_fence_after();
+  const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+  if (warp_rows) {
+    uint16_t *orow = real ? out_row(g, I, I.rb * kTcRows + row) : nullptr;
+    float *prow = (real && I.n_split > 1)
+                      ? p.partials + ((size_t)I.pbase + (size_t)I.split * I.rows + row) * kPStride
+                      : nullptr;
+#pragma unroll
+    for (int q4 = 0; q4 < kD / 32; ++q4) {
+      uint32_t r[32];
+      tc_ld_32x32b_x32(tl + col_o(0) + q4 * 32, r);
+      tc_wait_ld();
+      if (real) {
+        if (I.n_split == 1) {
+#pragma unroll
+          for (int c8 = 0; c8 < 4; ++c8) {
+            uint4 v;
+            v.x = pack_bf16x2(__uint_as_float(r[8 * c8 + 0]) * inv, __uint_as_float(r[8 * c8 + 1]) * inv);
+            v.y = pack_bf16x2(__uint_as_float(r[8 * c8 + 2]) * inv, __uint_as_float(r[8 * c8 + 3]) * inv);
+            v.z = pack_bf16x2(__uint_as_float(r[8 * c8 + 4]) * inv, __uint_as_float(r[8 * c8 + 5]) * inv);
+            v.w = pack_bf16x2(__uint_as_float(r[8 * c8 + 6]) * inv, __uint_as_float(r[8 * c8 + 7]) * inv);
+            reinterpret_cast<uint4 *>(orow + q4 * 32)[c8] = v;
+          }
+        } else {
+#pragma unroll
+          for (int c4 = 0; c4 < 8; ++c4)
+            __stcg(reinterpret_cast<float4 *>(prow + q4 * 32) + c4,
+                   make_float4(__uint_as_float(r[4 * c4]), __uint_as_float(r[4 * c4 + 1]),
+                               __uint_as_float(r[4 * c4 + 2]), __uint_as_float(r[4 * c4 + 3])));
+        }
+      }
+    }
+    if (real && I.n_split > 1) {
+      __stcg(prow + 128, m_used);
+      __stcg(prow + 129, l_run);
+    }
+  }
+  tc_fence_before();
+  __syncwarp();
+  if (lane == 0) mbar_arrive(B.o_free);
+  if (I.n_split > 1) ticket_merge(p, X, I, g);
+  named_bar_sync(1, kCW * 32);
+  return true;
+}
+
+// ============================ CUDA-core path ============================
+// Fewer than kTcMinRows rows; warp w takes page w of every stage, lanes split
+// a page's 16 keys in halves of the head dimension.
+__device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, const Item &I,
+                                     uint32_t &it) {
+  const ItemGeom g = item_geom(p, I);
+  const Bars &B = X.B;
+  const int warp = X.warp, lane = X.lane;
+  float *qs = reinterpret_cast<float *>(X.smem + Smem::off_ccq);
+  float *mg = reinterpret_cast<float *>(X.smem + Smem::off_merge);
+  float *ps = reinterpret_cast<float *>(X.smem + Smem::off_ps);
+  const int nrow = I.rows;
+  float cm[kCcRows], cl[kCcRows], co[kCcRows][4];
+
+  for (bool first = true;; first = false) {
+    const int s = it % kStages;
+    if (!wait_or_abort(X, &B.full[s], (it / kStages) & 1)) return false;
+    const StageMeta M = X.meta[s];
+    zero_tail(X, s, M.page0, g.L);
+    if (first) {
+      for (int e = X.ctid; e < nrow * (kD / 8); e += kCW * 32) {
         const int rho = e / (kD / 8), c8 = e % (kD / 8);
-        const int grow = I.rb * kRowsCuda + rho;
-        const int qi = grow / G, j = grow % G;
+        const int grow = I.rb * kCcRows + rho;
+        const int qi = grow / g.G, j = grow % g.G;
         const uint4 raw = *reinterpret_cast<const uint4 *>(
-            B.q + ((size_t)(q0 + qi) * hq + I.kvh * G + j) * kD + c8 * 8);
+            g.Bt->q + ((size_t)(g.q0 + qi) * g.hq + I.kvh * g.G + j) * kD + c8 * 8);
         float *dst = qs + rho * kD;
         const int d0 = c8 * 8;
         dst[q_slot(d0 + 0)] = bf16lo(raw.x);
@@ -494,211 +781,380 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
         dst[q_slot(d0 + 7)] = bf16hi(raw.w);
       }
 #pragma unroll
-      for (int g = 0; g < 8; ++g) {
-        m[g] = -INFINITY;
-        l[g] = 0.f;
-        o[g][0] = o[g][1] = o[g][2] = o[g][3] = 0.f;
+      for (int r = 0; r < kCcRows; ++r) {
+        cm[r] = -INFINITY;
+        cl[r] = 0.f;
+        co[r][0] = co[r][1] = co[r][2] = co[r][3] = 0.f;
       }
       named_bar_sync(1, kCW * 32);
     }
-
-    if (active) {
+    const int pg = warp;  // one page per compute warp
+    if (pg < M.npages) {
       const int key = lane >> 1, half = lane & 1;
-      for (int pg = pw; pg < M.npages; pg += pw_count) {
-        const uint8_t *Kp = stage_tile(smem, s, pg, 0);
-        const uint8_t *Vp = stage_tile(smem, s, pg, 1);
-        const int kpos = (M.page0 + pg) * kPage + key;
-        const bool page_ok = !((M.invalid >> pg) & 1u);
-        uint4 kr[8];
+      const int R = pg * kPage + key;  // key row within the stage
+      const uint8_t *kb = stage_k(X.smem, s) + half * kHalfBytes + R * 128;
+      const uint8_t *vb = stage_v(X.smem, s);
+      const int kpos = (M.page0 + pg) * kPage + key;
+      const bool page_ok = !((M.invalid >> pg) & 1u);
+      uint4 kr[8];
 #pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          const int cc = (c + lane) & 7;
-          kr[c] = *reinterpret_cast<const uint4 *>(Kp + key * 256 + half * 128 + cc * 16);
+      for (int cc = 0; cc < 8; ++cc) {
+        const int lc = (cc + 4 * half) & 7;  // logical chunk, rotated per half
+        kr[cc] = *reinterpret_cast<const uint4 *>(kb + ((lc ^ (R & 7)) << 4));
+      }
+#pragma unroll
+      for (int r = 0; r < kCcRows; ++r) {
+        if (r < nrow) {
+          const float *qrow = qs + r * kD + half * 64;
+          float pa[4] = {0.f, 0.f, 0.f, 0.f};  // four independent partial sums
+#pragma unroll
+          for (int cc = 0; cc < 8; ++cc) {
+            const int lc = (cc + 4 * half) & 7;
+            const float4 a = *reinterpret_cast<const float4 *>(qrow + lc * 4);
+            const float4 b2 = *reinterpret_cast<const float4 *>(qrow + 32 + lc * 4);
+            float &acc = pa[cc & 3];
+            acc = fmaf(bf16lo(kr[cc].x), a.x, acc);
+            acc = fmaf(bf16hi(kr[cc].x), a.y, acc);
+            acc = fmaf(bf16lo(kr[cc].y), a.z, acc);
+            acc = fmaf(bf16hi(kr[cc].y), a.w, acc);
+            acc = fmaf(bf16lo(kr[cc].z), b2.x, acc);
+            acc = fmaf(bf16hi(kr[cc].z), b2.y, acc);
+            acc = fmaf(bf16lo(kr[cc].w), b2.z, acc);
+            acc = fmaf(bf16hi(kr[cc].w), b2.w, acc);
+          }
+          float acc = (pa[0] + pa[1]) + (pa[2] + pa[3]);
+          acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+          const int qi = (I.rb * kCcRows + r) / g.G;
+          const bool vis = page_ok && kpos < g.L && kpos <= g.L - g.ql + qi;
+          const float sc = vis ? acc * p.scale_log2 : -INFINITY;
+          float mx = sc;
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+          const float mnew = fmaxf(cm[r], mx);
+          float alpha = 1.f, pr = 0.f;
+          if (mnew != -INFINITY) {
+            alpha = exp2f(cm[r] - mnew);
+            pr = exp2f(sc - mnew);
+          }
+          cl[r] = cl[r] * alpha + (half == 0 ? pr : 0.f);
+          co[r][0] *= alpha;
+          co[r][1] *= alpha;
+          co[r][2] *= alpha;
+          co[r][3] *= alpha;
+          cm[r] = mnew;
+          if (half == 0) ps[(warp * 8 + r) * 16 + key] = pr;
         }
+      }
+      __syncwarp();
+      // P V: lane owns dims 4*lane .. 4*lane+3
+      const int vhalf = lane >> 4, vc = (lane & 15) >> 1, vsub = (lane & 1) * 8;
 #pragma unroll
-        for (int g = 0; g < 8; ++g) {
-          if (g < nrow_g) {
-            const int rho = rg * 8 + g;
-            const float *qrow = qs + rho * kD + half * 64;
-            float acc = 0.f;
+      for (int jk = 0; jk < kPage; ++jk) {
+        const int Rv = pg * kPage + jk;
+        const uint2 vv = *reinterpret_cast<const uint2 *>(vb + vhalf * kHalfBytes + Rv * 128 +
+                                                          ((vc ^ (Rv & 7)) << 4) + vsub);
+        const float v0 = bf16lo(vv.x), v1 = bf16hi(vv.x), v2 = bf16lo(vv.y), v3 = bf16hi(vv.y);
 #pragma unroll
-            for (int c = 0; c < 8; ++c) {
-              const int cc = (c + lane) & 7;
-              const float4 a = *reinterpret_cast<const float4 *>(qrow + cc * 4);
-              const float4 b2 = *reinterpret_cast<const float4 *>(qrow + 32 + cc * 4);
-              acc = fmaf(bf16lo(kr[c].x), a.x, acc);
-              acc = fmaf(bf16hi(kr[c].x), a.y, acc);
-              acc = fmaf(bf16lo(kr[c].y), a.z, acc);
-              acc = fmaf(bf16hi(kr[c].y), a.w, acc);
-              acc = fmaf(bf16lo(kr[c].z), b2.x, acc);
-              acc = fmaf(bf16hi(kr[c].z), b2.y, acc);
-              acc = fmaf(bf16lo(kr[c].w), b2.z, acc);
-              acc = fmaf(bf16hi(kr[c].w), b2.w, acc);
-            }
-            acc += __shfl_xor_sync(0xffffffffu, acc, 1);
-            const int qi = (I.rb * kRowsCuda + rho) / G;
-            const bool vis = page_ok && kpos < L && kpos <= L - ql + qi;
-            const float sc = vis ? acc * p.scale_log2 : -INFINITY;
-            float mx = sc;
-            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
-            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
-            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
-            const float mnew = fmaxf(m[g], mx);
-            float alpha = 1.f, pr = 0.f;
-            if (mnew != -INFINITY) {
-              alpha = exp2f(m[g] - mnew);
-              pr = exp2f(sc - mnew);
-            }
-            l[g] = l[g] * alpha + (half == 0 ? pr : 0.f);
-            o[g][0] *= alpha;
-            o[g][1] *= alpha;
-            o[g][2] *= alpha;
-            o[g][3] *= alpha;
-            m[g] = mnew;
-            if (half == 0) ps[(warp * 8 + g) * 16 + key] = pr;
+        for (int r = 0; r < kCcRows; ++r) {
+          if (r < nrow) {
+            const float pj = ps[(warp * 8 + r) * 16 + jk];
+            co[r][0] = fmaf(pj, v0, co[r][0]);
+            co[r][1] = fmaf(pj, v1, co[r][1]);
+            co[r][2] = fmaf(pj, v2, co[r][2]);
+            co[r][3] = fmaf(pj, v3, co[r][3]);
           }
         }
-        __syncwarp();
-#pragma unroll 4
-        for (int jk = 0; jk < 16; ++jk) {
-          const uint2 vv = *reinterpret_cast<const uint2 *>(Vp + jk * 256 + lane * 8);
-          const float v0 = bf16lo(vv.x), v1 = bf16hi(vv.x), v2 = bf16lo(vv.y), v3 = bf16hi(vv.y);
-#pragma unroll
-          for (int g = 0; g < 8; ++g) {
-            if (g < nrow_g) {
-              const float pj = ps[(warp * 8 + g) * 16 + jk];
-              o[g][0] = fmaf(pj, v0, o[g][0]);
-              o[g][1] = fmaf(pj, v1, o[g][1]);
-              o[g][2] = fmaf(pj, v2, o[g][2]);
-              o[g][3] = fmaf(pj, v3, o[g][3]);
-            }
-          }
-        }
-        __syncwarp();
       }
     }
     __syncwarp();
-    if (lane == 0) mbar_arrive(&empty[s]);
+    if (lane == 0) mbar_arrive(&B.empty[s]);
+    ++it;
+    if (M.flags & 2) break;
+  }
 
-    if (M.flags & 2) {
-      // ------------------------------ finalize ------------------------------
-      const BatchDev &B = p.b[I.b];
+  // ---- finalize: merge the four warps' page subsets ----
 #pragma unroll
-      for (int g = 0; g < 8; ++g)
-        if (g < nrow_g) l[g] = warp_sum(l[g]);
-      if (pw_count > 1) {
-        if (active) {
+  for (int r = 0; r < kCcRows; ++r)
+    if (r < nrow) cl[r] = warp_sum(cl[r]);
 #pragma unroll
-          for (int g = 0; g < 8; ++g) {
-            if (g < nrow_g) {
-              float *dst = mg + (warp * 8 + g) * kPStride;
-              *reinterpret_cast<float4 *>(dst + lane * 4) =
-                  make_float4(o[g][0], o[g][1], o[g][2], o[g][3]);
-              if (lane == 0) {
-                dst[128] = m[g];
-                dst[129] = l[g];
-              }
-            }
-          }
+  for (int r = 0; r < kCcRows; ++r) {
+    if (r < nrow) {
+      float *dst = mg + (warp * 8 + r) * kPStride;
+      *reinterpret_cast<float4 *>(dst + lane * 4) = make_float4(co[r][0], co[r][1], co[r][2], co[r][3]);
+      if (lane == 0) {
+        dst[128] = cm[r];
+        dst[129] = cl[r];
+      }
+    }
+  }
+  named_bar_sync(1, kCW * 32);
+  if (warp == 0) {
+#pragma unroll
+    for (int r = 0; r < kCcRows; ++r) {
+      if (r < nrow) {
+        float Mx = -INFINITY;
+        for (int w2 = 0; w2 < kCW; ++w2) Mx = fmaxf(Mx, mg[(w2 * 8 + r) * kPStride + 128]);
+        float Ls = 0.f, O0 = 0.f, O1 = 0.f, O2 = 0.f, O3 = 0.f;
+        for (int w2 = 0; w2 < kCW; ++w2) {
+          const float *src = mg + (w2 * 8 + r) * kPStride;
+          const float sc = (src[128] == -INFINITY) ? 0.f : exp2f(src[128] - Mx);
+          const float4 ov = *reinterpret_cast<const float4 *>(src + lane * 4);
+          Ls += src[129] * sc;
+          O0 += ov.x * sc;
+          O1 += ov.y * sc;
+          O2 += ov.z * sc;
+          O3 += ov.w * sc;
         }
-        named_bar_sync(1, kCW * 32);
-        if (active && pw == 0) {
-#pragma unroll
-          for (int g = 0; g < 8; ++g) {
-            if (g < nrow_g) {
-              float Mx = -INFINITY;
-              for (int w2 = 0; w2 < pw_count; ++w2)
-                Mx = fmaxf(Mx, mg[((rg + w2 * n_rg) * 8 + g) * kPStride + 128]);
-              float Ls = 0.f, O0 = 0.f, O1 = 0.f, O2 = 0.f, O3 = 0.f;
-              for (int w2 = 0; w2 < pw_count; ++w2) {
-                const float *src = mg + ((rg + w2 * n_rg) * 8 + g) * kPStride;
-                const float sc = (src[128] == -INFINITY) ? 0.f : exp2f(src[128] - Mx);
-                const float4 ov = *reinterpret_cast<const float4 *>(src + lane * 4);
-                Ls += src[129] * sc;
-                O0 += ov.x * sc;
-                O1 += ov.y * sc;
-                O2 += ov.z * sc;
-                O3 += ov.w * sc;
-              }
-              m[g] = Mx;
-              l[g] = Ls;
-              o[g][0] = O0; o[g][1] = O1; o[g][2] = O2; o[g][3] = O3;
-            }
+        const int grow = I.rb * kCcRows + r;
+        const int qi = grow / g.G, j = grow % g.G;
+        if (I.n_split == 1) {
+          const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+          uint2 pk;
+          pk.x = (uint32_t)f2bf16(O0 * inv) | ((uint32_t)f2bf16(O1 * inv) << 16);
+          pk.y = (uint32_t)f2bf16(O2 * inv) | ((uint32_t)f2bf16(O3 * inv) << 16);
+          *reinterpret_cast<uint2 *>(g.Bt->out + ((size_t)(g.q0 + qi) * g.hq + I.kvh * g.G + j) * kD +
+                                     lane * 4) = pk;
+        } else {
+          float *dst = p.partials + ((size_t)I.pbase + (size_t)I.split * I.rows + r) * kPStride;
+          __stcg(reinterpret_cast<float4 *>(dst + lane * 4), make_float4(O0, O1, O2, O3));
+          if (lane == 0) {
+            __stcg(dst + 128, Mx);
+            __stcg(dst + 129, Ls);
           }
         }
       }
-      const bool owner = active && pw == 0;
-      if (I.n_split == 1) {
-        if (owner) {
-#pragma unroll
-          for (int g = 0; g < 8; ++g) {
-            if (g < nrow_g) {
-              const int grow = I.rb * kRowsCuda + rg * 8 + g;
-              const int qi = grow / G, j = grow % G;
-              const float inv = l[g] > 0.f ? 1.f / l[g] : 0.f;
-              uint2 pk;
-              pk.x = (uint32_t)f2bf16(o[g][0] * inv) | ((uint32_t)f2bf16(o[g][1] * inv) << 16);
-              pk.y = (uint32_t)f2bf16(o[g][2] * inv) | ((uint32_t)f2bf16(o[g][3] * inv) << 16);
-              *reinterpret_cast<uint2 *>(B.out + ((size_t)(q0 + qi) * hq + I.kvh * G + j) * kD +
-                                         lane * 4) = pk;
-            }
-          }
+    }
+  }
+  if (I.n_split > 1) ticket_merge(p, X, I, g);
+  named_bar_sync(1, kCW * 32);
+  return true;
+}
+
+__global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant__ AttnParams p) {
+  extern __shared__ __align__(1024) uint8_t smem[];
+  const Bars B = bars(smem);
+  StageMeta *meta = reinterpret_cast<StageMeta *>(smem + Smem::off_meta);
+  // misc[0] TMEM base, [1] abort flag, [2] ticket broadcast
+  uint32_t *misc = reinterpret_cast<uint32_t *>(smem + Smem::off_misc);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // the 128-byte swizzle atoms of TMA and tcgen05 assume 1024-byte alignment
+  if (smem_u32(smem) & 1023u) {
+    if (threadIdx.x == 0) ipd_set_error(&g_attn_err, IPD_DEVERR_PLAN);
+    return;
+  }
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&B.full[s], 1);
+      mbar_init(&B.empty[s], 1 + kCW);  // the MMA warp and every compute warp
+    }
+    mbar_init(B.q_ready, kCW);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&B.s_full[i], 1);
+      mbar_init(&B.p_full[i], kCW);
+      mbar_init(&B.p_free[i], 1);
+    }
+    mbar_init(B.o_full, 1);
+    mbar_init(B.o_free, kCW);
+    misc[1] = 0;
+    fence_mbar_init();
+  }
+  if (warp == kMmaWarp) {
+    tc_alloc(&misc[0], kTmemCols);
+    tc_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = misc[0];
+  const int n_items = p.ctrl[0];
+
+  if (warp == kProducerWarp) {
+    // ------------------------------ producer ------------------------------
+    const uint64_t policy = l2_policy_evict_first();
+    uint32_t it = 0;
+    bool aborted = false;
+    for (;;) {
+      int idx = 0;
+      if (lane == 0) idx = atomicAdd(&p.ctrl[1], 1);
+      idx = __shfl_sync(0xffffffffu, idx, 0);
+      if (idx >= n_items) break;
+      const Item I = p.items[idx];
+      const BatchDev &Bt = p.b[I.b];
+      const int *prow = Bt.page_table + (long long)I.r * Bt.max_pages;
+      const void *tk = &p.tmap[2 * Bt.cache];
+      const void *tv = &p.tmap[2 * Bt.cache + 1];
+      const int oob_row = (int)(Bt.num_pages * Bt.hkv * kPage);  // a box here reads zeros
+      for (int page = I.page_lo; page < I.page_hi; page += kStagePages) {
+        const int np = min(kStagePages, I.page_hi - page);
+        const int s = it % kStages;
+        const uint32_t ph = (it / kStages) & 1;
+        if (!mbar_wait_bounded(&B.empty[s], ph ^ 1)) {
+          ipd_set_error(&g_attn_err, IPD_DEVERR_WAIT);
+          aborted = true;
+          break;
+        }
+        int y = oob_row;
+        bool ok = false;
+        if (lane < np) {
+          const int pid = prow[page + lane];
+          ok = pid >= 0 && (long long)pid < Bt.num_pages;
+          if (!ok) ipd_set_error(&g_attn_err, IPD_DEVERR_PAGE_ID);
+          else y = (pid * Bt.hkv + I.kvh) * kPage;
+        }
+        const uint32_t okmask = __ballot_sync(0xffffffffu, ok);
+        if (lane == 0) {
+          StageMeta m;
+          m.item = idx;
+          m.page0 = page;
+          m.npages = np;
+          m.flags = (page == I.page_lo ? 1 : 0) | (page + np >= I.page_hi ? 2 : 0);
+          m.invalid = (~okmask) & ((1u << np) - 1u);
+          m.path = I.path;
+          meta[s] = m;
+          mbar_arrive_expect_tx(&B.full[s], kStageBytes);
+        }
+        __syncwarp();
+        if (lane < kStagePages) {  // every page slot is written (zeros past the item)
+          uint8_t *kd = stage_k(smem, s) + lane * kPage * 128;
+          uint8_t *vd = stage_v(smem, s) + lane * kPage * 128;
+          tma_load_2d(kd, tk, 0, y, &B.full[s], policy);
+          tma_load_2d(kd + kHalfBytes, tk, 64, y, &B.full[s], policy);
+          tma_load_2d(vd, tv, 0, y, &B.full[s], policy);
+          tma_load_2d(vd + kHalfBytes, tv, 64, y, &B.full[s], policy);
+        }
+        ++it;
+      }
+      if (aborted) break;
+    }
+    if (!aborted) {
+      const int s = it % kStages;
+      const uint32_t ph = (it / kStages) & 1;
+      if (mbar_wait_bounded(&B.empty[s], ph ^ 1)) {
+        if (lane == 0) {
+          meta[s].item = -1;
+          mbar_arrive(&B.full[s]);
         }
       } else {
-        if (owner) {
-#pragma unroll
-          for (int g = 0; g < 8; ++g) {
-            if (g < nrow_g) {
-              float *dst = p.partials +
-                           ((size_t)I.pbase + (size_t)I.split * rows + rg * 8 + g) * kPStride;
-              __stcg(reinterpret_cast<float4 *>(dst + lane * 4),
-                     make_float4(o[g][0], o[g][1], o[g][2], o[g][3]));
-              if (lane == 0) {
-                __stcg(dst + 128, m[g]);
-                __stcg(dst + 129, l[g]);
-              }
-            }
-          }
-        }
-        __threadfence();
-        named_bar_sync(1, kCW * 32);
-        if (ctid == 0) misc[1] = (atomicAdd(&p.tickets[I.task], 1) == I.n_split - 1);
-        named_bar_sync(1, kCW * 32);
-        if (misc[1]) {
-          __threadfence();
-          for (int rho = warp; rho < rows; rho += kCW) {
-            float Mx = -INFINITY;
-            for (int sp = 0; sp < I.n_split; ++sp)
-              Mx = fmaxf(Mx, __ldcg(p.partials + ((size_t)I.pbase + (size_t)sp * rows + rho) *
-                                                     kPStride + 128));
-            float Ls = 0.f, O0 = 0.f, O1 = 0.f, O2 = 0.f, O3 = 0.f;
-            for (int sp = 0; sp < I.n_split; ++sp) {
-              const float *src = p.partials + ((size_t)I.pbase + (size_t)sp * rows + rho) * kPStride;
-              const float mm = __ldcg(src + 128);
-              const float sc = (mm == -INFINITY) ? 0.f : exp2f(mm - Mx);
-              const float4 ov = __ldcg(reinterpret_cast<const float4 *>(src + lane * 4));
-              Ls += __ldcg(src + 129) * sc;
-              O0 += ov.x * sc;
-              O1 += ov.y * sc;
-              O2 += ov.z * sc;
-              O3 += ov.w * sc;
-            }
-            const int grow = I.rb * kRowsCuda + rho;
-            const int qi = grow / G, j = grow % G;
-            const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
-            uint2 pk;
-            pk.x = (uint32_t)f2bf16(O0 * inv) | ((uint32_t)f2bf16(O1 * inv) << 16);
-            pk.y = (uint32_t)f2bf16(O2 * inv) | ((uint32_t)f2bf16(O3 * inv) << 16);
-            *reinterpret_cast<uint2 *>(B.out + ((size_t)(q0 + qi) * hq + I.kvh * G + j) * kD +
-                                       lane * 4) = pk;
-          }
-        }
+        ipd_set_error(&g_attn_err, IPD_DEVERR_WAIT);
+        aborted = true;
       }
-      named_bar_sync(1, kCW * 32);
     }
-    ++it;
+    if (aborted) {
+      // the consumers stopped: let this CTA's copies land before exiting
+      if (lane == 0) atomicExch(&misc[1], 1u);
+      for (uint32_t k = (it > (uint32_t)kStages ? it - kStages : 0); k < it; ++k)
+        (void)mbar_wait_bounded(&B.full[k % kStages], (k / kStages) & 1);
+    }
+    return;
   }
+
+  if (warp == kMmaWarp) {
+    // ------------------------------ MMA issuer -----------------------------
+    constexpr uint32_t idesc_s = idesc_bf16_f32(kTcRows, kStageKeys, 0);
+    constexpr uint32_t idesc_o = idesc_bf16_f32(kTcRows, kD, 1);
+    const uint32_t sq = smem_u32(smem + Smem::off_q);
+    uint32_t it = 0, c = 0, nq = 0, cur_item = 0;
+    bool pend = false, pend_first = false;
+    uint32_t pend_c = 0, pend_s = 0, pend_item = 0;
+    bool ok = true;
+    // O (+)= P[cc & 1] V[stage ss], with P = P_hi + P_lo; the first chunk of
+    // an item overwrites O (after the previous item's O was read out).
+    auto issue_pv = [&](uint32_t cc, uint32_t ss, bool firstc, uint32_t item) -> bool {
+      const uint32_t bb = cc & 1;
+      if (!mbar_wait_bounded(&B.p_full[bb], (cc >> 1) & 1)) return false;
+      if (firstc && !mbar_wait_bounded(B.o_free, (item & 1) ^ 1)) return false;
+      tc_fence_after();
+      if (lane == 0) {
+        const uint32_t pa = smem_u32(smem + Smem::off_p + bb * 2 * Smem::kPBytes);
+        const uint32_t va = smem_u32(stage_v(smem, ss));
+#pragma unroll
+        for (int kk = 0; kk < kStageKeys / 16; ++kk) {
+          const uint64_t bd = sdesc_sw128(va + kk * 16 * 128, kHalfBytes, 1024);
+          tc_mma_bf16(tmem + col_o(0), sdesc_sw128(pa + kk * 32, 16, 1024), bd, idesc_o,
+                      (firstc && kk == 0) ? 0u : 1u);
+          tc_mma_bf16(tmem + col_o(0), sdesc_sw128(pa + Smem::kPBytes + kk * 32, 16, 1024), bd,
+                      idesc_o, 1u);
+        }
+        tc_commit(B.o_full);
+        tc_commit(&B.p_free[bb]);
+        tc_commit(&B.empty[ss]);
+      }
+      __syncwarp();
+      return true;
+    };
+    for (;;) {
+      const int s = it % kStages;
+      if (!mbar_wait_bounded(&B.full[s], (it / kStages) & 1)) { ok = false; break; }
+      const StageMeta M = meta[s];
+      if (M.item < 0) break;
+      if (!M.path) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&B.empty[s]);
+        ++it;
+        continue;
+      }
+      const bool firstc = M.flags & 1;
+      if (firstc) {
+        if (!mbar_wait_bounded(B.q_ready, nq & 1)) { ok = false; break; }
+        cur_item = nq++;
+      }
+      tc_fence_after();
+      const uint32_t b = c & 1;
+      if (lane == 0) {
+        const uint32_t ka = smem_u32(stage_k(smem, s));
+#pragma unroll
+        for (int kk = 0; kk < kD / 16; ++kk) {
+          const uint32_t qoff = (kk >> 2) * (kTcRows * 128) + (kk & 3) * 32;
+          const uint32_t koff = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
+          tc_mma_bf16(tmem + col_s(b), sdesc_sw128(sq + qoff, 16, 1024),
+                      sdesc_sw128(ka + koff, 16, 1024), idesc_s, kk > 0);
+        }
+        tc_commit(&B.s_full[b]);
+      }
+      __syncwarp();
+      if (pend) {
+        if (!issue_pv(pend_c, pend_s, pend_first, pend_item)) { ok = false; break; }
+        pend = false;
+      }
+      if (M.flags & 2) {
+        if (!issue_pv(c, s, firstc, cur_item)) { ok = false; break; }
+      } else {
+        pend = true;
+        pend_c = c;
+        pend_s = s;
+        pend_first = firstc;
+        pend_item = cur_item;
+      }
+      ++c;
+      ++it;
+    }
+    if (!ok) {
+      ipd_set_error(&g_attn_err, IPD_DEVERR_WAIT);
+      atomicExch(&misc[1], 1u);
+    }
+    // every tensor-core op and TMEM access is finished before TMEM is released
+    named_bar_sync(2, (kCW + 1) * 32);
+    tc_fence_after();
+    tc_dealloc(tmem, kTmemCols);
+    return;
+  }
+
+  // -------------------------------- compute warps --------------------------------
+  const CompCtx X{smem, B, meta, misc, tmem, warp, lane, (int)threadIdx.x};
+  uint32_t it = 0, c = 0;
+  for (;;) {
+    const int s = it % kStages;
+    if (!wait_or_abort(X, &B.full[s], (it / kStages) & 1)) break;
+    const StageMeta M = meta[s];
+    if (M.item < 0 || *(volatile uint32_t *)&misc[1]) break;
+    const Item I = p.items[M.item];
+    const bool ok = I.path ? tc_item(p, X, I, it, c) : cc_item(p, X, I, it);
+    if (!ok) break;
+  }
+  named_bar_sync(2, (kCW + 1) * 32);
 }
 
 // --------------------------------------------------------------------------
@@ -710,10 +1166,38 @@ struct DevInfo {
 };
 DevInfo g_dev[64];
 
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+int get_encoder() {
+  if (g_encode) return IPD_OK;
+  void *fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                       &q) != cudaSuccess ||
+      q != cudaDriverEntryPointSuccess || !fn)
+    return IPD_ERR_CUDA;
+  g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  return IPD_OK;
+}
+
+// A pool [num_pages][Hkv][16][128] bf16 seen as a 2-D tensor of 128-element
+// rows; boxes of 64 elements x 16 rows, 128-byte swizzle.
+int encode_pool(CUtensorMap *m, const void *base, long long rows) {
+  cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)kD * 2};
+  cuuint32_t box[2] = {64, (cuuint32_t)kPage};
+  cuuint32_t estr[2] = {1, 1};
+  const CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base),
+                              dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                              CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? IPD_OK : IPD_ERR_CUDA;
+}
+
 int launch(const ipd_attn_batch *const *bs, int n, float scale, void *ws, size_t ws_bytes,
            cudaStream_t stream) {
   if (!(scale > 0.f) || scale != scale) return IPD_ERR_INVALID_ARG;
-  WsLayout W = layout(bs, n);
+  const WsLayout W = layout(bs, n);
   if (W.total_reqs == 0) return IPD_OK;
   if (!ws || ws_bytes < W.total || ((uintptr_t)ws & 255)) return IPD_ERR_WORKSPACE;
   int dev = 0;
@@ -723,31 +1207,47 @@ int launch(const ipd_attn_batch *const *bs, int n, float scale, void *ws, size_t
     if (cudaDeviceGetAttribute(&D.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
       return IPD_ERR_CUDA;
     if (cudaFuncSetAttribute(attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             SmemLayout::total) != cudaSuccess)
+                             Smem::total) != cudaSuccess)
       return IPD_ERR_CUDA;
     D.attr_set = true;
   }
-  AttnParams P{};
+  if (get_encoder() != IPD_OK) return IPD_ERR_CUDA;
+  AttnParams P;
+  memset(&P, 0, sizeof(P));
   P.n_batches = n;
+  const ipd_kv_cache *caches[IPD_MAX_BATCHES];
+  int n_caches = 0;
   int base = 0;
   for (int i = 0; i < n; ++i) {
     const ipd_attn_batch *b = bs[i];
-    BatchDev &B = P.b[i];
-    B.q = b->q;
-    B.out = b->out;
-    B.cu_q = b->cu_q;
-    B.seq_len = b->seq_len;
-    B.page_table = b->page_table;
-    B.k_pages = b->cache->k_pages;
-    B.v_pages = b->cache->v_pages;
-    B.num_pages = b->cache->num_pages;
-    B.num_reqs = b->num_reqs;
-    B.hq = b->num_q_heads;
-    B.hkv = b->cache->num_kv_heads;
-    B.group = B.hq / B.hkv;
-    B.max_pages = b->max_pages;
-    B.max_q_len = b->max_q_len;
-    B.total_q = b->total_q;
+    int ci = 0;
+    while (ci < n_caches && !(caches[ci]->k_pages == b->cache->k_pages &&
+                              caches[ci]->v_pages == b->cache->v_pages &&
+                              caches[ci]->num_pages == b->cache->num_pages &&
+                              caches[ci]->num_kv_heads == b->cache->num_kv_heads))
+      ++ci;
+    if (ci == n_caches) {
+      caches[n_caches++] = b->cache;
+      const long long rows = b->cache->num_pages * b->cache->num_kv_heads * kPage;
+      if (encode_pool(&P.tmap[2 * ci], b->cache->k_pages, rows) != IPD_OK ||
+          encode_pool(&P.tmap[2 * ci + 1], b->cache->v_pages, rows) != IPD_OK)
+        return IPD_ERR_CUDA;
+    }
+    BatchDev &Bd = P.b[i];
+    Bd.q = b->q;
+    Bd.out = b->out;
+    Bd.cu_q = b->cu_q;
+    Bd.seq_len = b->seq_len;
+    Bd.page_table = b->page_table;
+    Bd.num_pages = b->cache->num_pages;
+    Bd.num_reqs = b->num_reqs;
+    Bd.hq = b->num_q_heads;
+    Bd.hkv = b->cache->num_kv_heads;
+    Bd.group = Bd.hq / Bd.hkv;
+    Bd.max_pages = b->max_pages;
+    Bd.max_q_len = b->max_q_len;
+    Bd.total_q = b->total_q;
+    Bd.cache = ci;
     P.req_base[i] = base;
     base += b->num_reqs;
   }
@@ -763,11 +1263,12 @@ int launch(const ipd_attn_batch *const *bs, int n, float scale, void *ws, size_t
   P.item_cap = W.item_cap;
   P.task_cap = W.task_cap;
   P.prow_cap = W.prow_cap;
+  P.target_items = std::min(kMaxTargetItems, kTargetItemsPerSm * D.sms);
 
   attn_plan_kernel<<<1, 1024, 0, stream>>>(P);
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   const int grid = std::max(1, std::min(D.sms, W.item_cap));
-  attn_kernel<<<grid, kThreads, SmemLayout::total, stream>>>(P);
+  attn_kernel<<<grid, kThreads, Smem::total, stream>>>(P);
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   return IPD_OK;
 }
@@ -792,7 +1293,7 @@ extern "C" int ipd_verify_attn(const ipd_attn_batch *verify, int n_verify,
                                const ipd_attn_batch *decode, int n_decode, float softmax_scale,
                                void *workspace, size_t workspace_bytes, ipd_stream_t stream) {
   const ipd_attn_batch *bs[IPD_MAX_BATCHES];
-  int st = collect(verify, n_verify, decode, n_decode, bs);
+  const int st = collect(verify, n_verify, decode, n_decode, bs);
   if (st != IPD_OK) return st;
   return launch(bs, n_verify + n_decode, softmax_scale, workspace, workspace_bytes,
                 reinterpret_cast<cudaStream_t>(stream));
