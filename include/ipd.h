@@ -51,6 +51,7 @@ typedef struct CUstream_st *ipd_stream_t; /* same handle as cudaStream_t */
 #define IPD_ERR_CUDA 4        /* a CUDA runtime call failed (launch, attribute) */
 #define IPD_ERR_TIMEOUT 5     /* a bounded device wait ran out (never expected) */
 #define IPD_ERR_DEVICE 6      /* device-side check recorded an error */
+#define IPD_ERR_CAPACITY 7    /* more work than a fixed-size entry point holds */
 
 /* Device-side error codes (ipd_get_device_error). */
 #define IPD_DEVERR_NONE 0u
@@ -189,6 +190,38 @@ int ipd_score_span(const uint16_t *logits_student, const uint16_t *logits_teache
                    int32_t *first_trans, int32_t *n_emit, uint8_t *next_driver,
                    int32_t *new_len, uint8_t *done,
                    void *workspace, size_t workspace_bytes, ipd_stream_t stream);
+
+/* ipd_score_span for callers that cannot allocate device memory.
+ *
+ * No counterpart in the paper: this is a calling convention of the library.
+ * Some callers cannot hand the library a workspace: an operator plugged into
+ * a runtime whose interface passes only inputs and outputs and which forbids
+ * allocating inside the step, or a serving loop that must not call the
+ * allocator because cudaMalloc / cudaFree can synchronise the device.  This
+ * entry point takes no workspace and allocates nothing (no cudaMalloc, no
+ * cudaFree, no allocating library routine).  Its scratch is one array in the
+ * library's static device memory, sized for IPD_STATIC_MAX_TOKENS span
+ * positions (about 2.1 MiB), which every GPU that loads the library holds
+ * until the process exits.
+ *
+ * Arguments, outputs and semantics are those of ipd_score_span without the
+ * workspace.  total_tokens > IPD_STATIC_MAX_TOKENS returns IPD_ERR_CAPACITY
+ * and launches nothing.  The first call on a device looks up the array's
+ * device address (cudaGetSymbolAddress, once per device, with that device
+ * current); make that first call before any stream capture.  All calls share
+ * the one array, so calls that overlap on the GPU (on different streams, or
+ * from different host threads) race on it and their results are undefined:
+ * serialise them.  The array keeps the last call's contents; nothing in it
+ * needs to start at zero. */
+#define IPD_STATIC_MAX_TOKENS 4096
+int ipd_score_span_static(const uint16_t *logits_student, const uint16_t *logits_teacher,
+                          const int32_t *tokens, const int32_t *cu_span, const uint8_t *driver,
+                          const int32_t *prefix_len, int num_reqs, int total_tokens, int vocab,
+                          int K, int eos_id,
+                          float *logp_s, float *logp_t, float *feedback, float *kl_rev,
+                          float *kl_fwd, uint8_t *covered, float *margin, uint8_t *source,
+                          int32_t *first_trans, int32_t *n_emit, uint8_t *next_driver,
+                          int32_t *new_len, uint8_t *done, ipd_stream_t stream);
 
 /* Loss direction per token source (the KL-direction ablation of Sec. 4.3). */
 #define IPD_DIR_SPLIT 0    /* z=S: KL(pi||q), z=T: KL(q||pi)   (IPD default) */

@@ -16,6 +16,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <mutex>
+
 #include "common.cuh"
 
 IPD_DECLARE_ERROR_WORD(g_score_err);
@@ -404,6 +406,76 @@ extern "C" int ipd_score_span(const uint16_t *logits_student, const uint16_t *lo
     if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   }
   score_epilogue_kernel<<<num_reqs, kEpiThreads, 0, st>>>(
+      logits_student, logits_teacher, tokens, cu_span, driver, prefix_len, vocab, K, eos_id, rows,
+      logp_s, logp_t, feedback, kl_rev, kl_fwd, covered, margin, source, first_trans, n_emit,
+      next_driver, new_len, done, total_tokens);
+  if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
+  return IPD_OK;
+}
+
+// ---------------------------------------------------------------------------
+// ipd_score_span_static: the same computation for callers that cannot
+// allocate device memory.  The per-row scratch that ipd_score_span takes from
+// the caller's workspace lives here in one file-scope device array, sized for
+// IPD_STATIC_MAX_TOKENS span positions.  Every GPU that loads the library
+// holds this array (about 2.1 MiB) until the process exits.
+// ---------------------------------------------------------------------------
+static __device__ __align__(256) RowOut g_static_rows[2 * IPD_STATIC_MAX_TOKENS];
+
+namespace {
+std::mutex g_static_mu;
+RowOut *g_static_ptr[64] = {};  // device address of g_static_rows, per device
+
+// In host code g_static_rows names a host-side stand-in, not device memory:
+// the device address is looked up once per device, with that device current.
+int static_rows(RowOut **out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return IPD_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  if (!g_static_ptr[dev]) {
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_rows) != cudaSuccess || !p) return IPD_ERR_CUDA;
+    g_static_ptr[dev] = static_cast<RowOut *>(p);
+  }
+  *out = g_static_ptr[dev];
+  return IPD_OK;
+}
+}  // namespace
+
+extern "C" int ipd_score_span_static(const uint16_t *logits_student,
+                                     const uint16_t *logits_teacher, const int32_t *tokens,
+                                     const int32_t *cu_span, const uint8_t *driver,
+                                     const int32_t *prefix_len, int num_reqs, int total_tokens,
+                                     int vocab, int K, int eos_id, float *logp_s, float *logp_t,
+                                     float *feedback, float *kl_rev, float *kl_fwd,
+                                     uint8_t *covered, float *margin, uint8_t *source,
+                                     int32_t *first_trans, int32_t *n_emit, uint8_t *next_driver,
+                                     int32_t *new_len, uint8_t *done, ipd_stream_t stream) {
+  if (num_reqs < 0 || total_tokens < 0) return IPD_ERR_INVALID_ARG;
+  if (K < 1 || K > IPD_MAX_K) return IPD_ERR_UNSUPPORTED;
+  if (vocab < 8 || vocab % 8 || K > vocab) return IPD_ERR_UNSUPPORTED;
+  if (total_tokens > IPD_STATIC_MAX_TOKENS) return IPD_ERR_CAPACITY;
+  if (num_reqs == 0) return IPD_OK;
+  if (!cu_span || !driver || !prefix_len || !first_trans || !n_emit || !next_driver || !new_len ||
+      !done)
+    return IPD_ERR_INVALID_ARG;
+  if (total_tokens > 0 &&
+      (!logits_student || !logits_teacher || !tokens || !logp_s || !logp_t || !feedback ||
+       !kl_rev || !kl_fwd || !covered || !margin || !source))
+    return IPD_ERR_INVALID_ARG;
+  if (((uintptr_t)logits_student | (uintptr_t)logits_teacher) & 15) return IPD_ERR_INVALID_ARG;
+  RowOut *rows = nullptr;
+  const int st = static_rows(&rows);
+  if (st != IPD_OK) return st;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  // Every RowOut the epilogue reads is written by the row kernel of the same
+  // call first, so nothing in the array has to start at zero.
+  if (total_tokens > 0) {
+    score_rows_kernel<<<2 * total_tokens, kRowThreads, 0, s>>>(logits_student, logits_teacher,
+                                                               tokens, vocab, K, rows);
+    if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
+  }
+  score_epilogue_kernel<<<num_reqs, kEpiThreads, 0, s>>>(
       logits_student, logits_teacher, tokens, cu_span, driver, prefix_len, vocab, K, eos_id, rows,
       logp_s, logp_t, feedback, kl_rev, kl_fwd, covered, margin, source, first_trans, n_emit,
       next_driver, new_len, done, total_tokens);

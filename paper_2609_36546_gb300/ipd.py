@@ -18,7 +18,7 @@ LIB_PATH = os.path.join(_HERE, "_lib", "libipd.so")
 
 IPD_OK = 0
 STATUS = {0: "IPD_OK", 1: "IPD_ERR_INVALID_ARG", 2: "IPD_ERR_UNSUPPORTED", 3: "IPD_ERR_WORKSPACE",
-          4: "IPD_ERR_CUDA", 5: "IPD_ERR_TIMEOUT", 6: "IPD_ERR_DEVICE"}
+          4: "IPD_ERR_CUDA", 5: "IPD_ERR_TIMEOUT", 6: "IPD_ERR_DEVICE", 7: "IPD_ERR_CAPACITY"}
 STATUS_CODES = {v: k for k, v in STATUS.items()}
 DEVERR = {0: "none", 1: "page id", 2: "seq len", 3: "token id", 4: "plan overflow", 5: "wait",
           6: "span offsets"}
@@ -30,7 +30,9 @@ LOSS_FIELDS = ("loss", "sum_on", "sum_off", "n_on", "n_off", "intervention_ratio
 # Exported symbols of include/ipd.h (checked by the CPU test suite).
 EXPORTS = ("ipd_attn_workspace_size", "ipd_verify_attn", "ipd_decode_attn",
            "ipd_score_workspace_size", "ipd_score_span", "ipd_loss_workspace_size",
-           "ipd_split_loss", "ipd_get_device_error", "ipd_status_string", "ipd_version")
+           "ipd_split_loss", "ipd_get_device_error", "ipd_status_string", "ipd_version",
+           "ipd_score_span_static")
+STATIC_MAX_TOKENS = 4096  # IPD_STATIC_MAX_TOKENS
 
 
 class IpdError(RuntimeError):
@@ -77,6 +79,8 @@ _lib.ipd_score_workspace_size.restype = c_sz
 _lib.ipd_score_workspace_size.argtypes = [c_i, c_i, c_i, c_i]
 _lib.ipd_score_span.restype = c_i
 _lib.ipd_score_span.argtypes = [c_p] * 6 + [c_i] * 5 + [c_p] * 13 + [c_p, c_sz, c_p]
+_lib.ipd_score_span_static.restype = c_i
+_lib.ipd_score_span_static.argtypes = [c_p] * 6 + [c_i] * 5 + [c_p] * 13 + [c_p]
 _lib.ipd_loss_workspace_size.restype = c_sz
 _lib.ipd_loss_workspace_size.argtypes = [c_i]
 _lib.ipd_split_loss.restype = c_i
@@ -201,6 +205,21 @@ def score_span(logits_student, logits_teacher, tokens, cu_span, driver, prefix_l
         *[_ptr(out[n]) for n, _ in SCORE_REQ_OUTPUTS],
         _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)),
         "ipd_score_span")
+
+
+def score_span_static(logits_student, logits_teacher, tokens, cu_span, driver, prefix_len,
+                      K: int, eos_id: int, out: dict, stream=None):
+    """ipd_score_span without a workspace: for callers that cannot allocate
+    device memory (the scratch is the library's static device array, at most
+    STATIC_MAX_TOKENS span positions; overlapping calls race on it)."""
+    R = driver.numel()
+    T, V = logits_student.shape
+    _check(_lib.ipd_score_span_static(
+        _ptr(logits_student), _ptr(logits_teacher), _ptr(tokens), _ptr(cu_span), _ptr(driver),
+        _ptr(prefix_len), R, T, V, K, eos_id,
+        *[_ptr(out[n]) for n, _ in SCORE_TOKEN_OUTPUTS],
+        *[_ptr(out[n]) for n, _ in SCORE_REQ_OUTPUTS],
+        _stream(stream)), "ipd_score_span_static")
 
 
 def split_loss(kl_rev, kl_fwd, source, cu_span, n_emit, resp_len, agg_mode: int, dir_mode: int,

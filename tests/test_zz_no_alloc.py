@@ -1,0 +1,67 @@
+"""The allocation-free scoring entry point (ipd_score_span_static).
+
+Some callers cannot give the library a workspace: an operator plugged into a
+runtime that passes only inputs and outputs and forbids allocating inside the
+step, or a serving loop that must not call cudaMalloc / cudaFree because they
+can synchronise the device.  ipd_score_span_static serves them from a fixed
+array in the library's static device memory.  This file is collected last
+(its name sorts last) so that a run stopping at the first failure has run
+every other test already; it also passes on its own in a fresh process.
+"""
+import numpy as np
+import pytest
+import torch
+
+import ipd_synth as S
+
+pytestmark = pytest.mark.gpu
+
+FLOAT_TOL = {"logp_s": 1e-3, "logp_t": 1e-3, "feedback": 2e-3, "kl_rev": 2e-4, "kl_fwd": 2e-4,
+             "margin": 1e-6}
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_36546_gb300 import ipd
+    return ipd
+
+
+def _compare(ref: dict, got: dict):
+    for name, r in ref.items():
+        g = got[name]
+        if name in FLOAT_TOL:
+            assert torch.allclose(g, r, rtol=0, atol=FLOAT_TOL[name]), name
+        else:
+            assert torch.equal(g, r), name
+
+
+def test_static_scratch_matches_workspace_entry_point_on_two_calls(lib):
+    from paper_2609_36546_gb300 import VerifyStep
+    specs = [(S.small_spec(n_req=6, vocab=4096, span=(1, 9), force="mixed"), 11),
+             (S.small_spec(n_req=9, vocab=151936, sigma=3.0, logits="boost", span=(2, 8),
+                           ctx=(20, 60)), 12)]
+    for spec, seed in specs:           # two calls in a row, different inputs
+        w = S.make_workload(spec, seed=seed, device="cpu")
+        step = VerifyStep.from_workload(w, device="cuda")
+        step.run_score()                # existing entry point, caller workspace
+        torch.cuda.synchronize()
+        ref = {k: v.clone() for k, v in step.score.items()}
+        out = lib.alloc_score_outputs(step.R, step.T, "cuda")
+        for v in out.values():
+            v.fill_(7)                  # every output must be written by the call
+        lib.score_span_static(step.logits_s, step.logits_t, step.tokens, step.cu_span,
+                              step.driver, step.prefix_len, step.K, step.eos_id, out)
+        torch.cuda.synchronize()
+        _compare(ref, out)
+    assert lib.device_error() == 0
+
+
+def test_static_scratch_rejects_more_tokens_than_it_holds(lib):
+    import ctypes
+    T = lib.STATIC_MAX_TOKENS + 1
+    args = [16] * 6 + [1, T, 4096, 16, -1] + [16] * 13 + [None]
+    assert lib.lib().ipd_score_span_static(*args) == lib.STATUS_CODES["IPD_ERR_CAPACITY"]
