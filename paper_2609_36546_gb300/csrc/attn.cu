@@ -25,7 +25,7 @@
 //   CUDA-core path (fewer rows: GQA group 2 decode): fp32 FMA, one page of 16
 //     keys per warp, two lanes per key.
 // Warp roles: warps 0-3 compute, warp 4 streams KV pages with 2-D TMA into a
-// 3-stage mbarrier ring, warp 5 issues the tensor-core instructions.
+// 4-stage mbarrier ring, warp 5 issues the tensor-core instructions.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
@@ -44,7 +44,7 @@ constexpr int kPage = 16;
 constexpr int kD = 128;
 constexpr int kStagePages = 4;                    // 64 keys per stage
 constexpr int kStageKeys = kStagePages * kPage;
-constexpr int kStages = 3;
+constexpr int kStages = 4;
 constexpr int kHalfBytes = kStageKeys * 128;      // one 64-dim half of 64 key rows: 8 KB
 constexpr int kStageBytes = 4 * kHalfBytes;       // K and V, two halves each: 32 KB
 constexpr int kTcRows = 128;                      // rows of a tensor-core tile (M)
@@ -358,13 +358,13 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const __grid_constant__
 // the attention kernel
 // --------------------------------------------------------------------------
 struct Smem {
-  static constexpr int off_stage = 0;                              // 3 x 32 KB, 1024-aligned
+  static constexpr int off_stage = 0;                              // 4 x 32 KB, 1024-aligned
   static constexpr int off_q = off_stage + kStages * kStageBytes;  // 32 KB
   static constexpr int off_p = off_q + 2 * kTcRows * 128;          // 2 buffers x (hi, lo) x 16 KB
   static constexpr int kPBytes = kTcRows * 128;                    // one 128 x 64 bf16 operand
   static constexpr int off_meta = off_p + 4 * kPBytes;
   static constexpr int off_bar = off_meta + kStages * (int)sizeof(StageMeta);
-  static constexpr int n_bars = 2 * kStages + 1 + 2 + 2 + 2 + 1 + 1;
+  static constexpr int n_bars = 2 * kStages + 1 + 2 + 2 + 2 + 1;
   static constexpr int off_misc = off_bar + n_bars * 8;
   static constexpr int total = off_misc + 64;
   // CUDA-core path scratch (inside the Q and P regions, unused by that path)
@@ -381,8 +381,7 @@ struct Bars {
   uint64_t *full, *empty;     // KV ring
   uint64_t *q_ready;          // Q tile written (one phase per tensor item)
   uint64_t *s_full, *p_full;  // S = Q K^T landed / P written, per buffer
-  uint64_t *p_free;           // P V product done reading P, per buffer
-  uint64_t *o_full;           // P V product of a chunk landed in O (one phase per chunk)
+  uint64_t *p_free;           // P V product done (P read, O written), per buffer
   uint64_t *o_free;           // O read out (one phase per tensor item)
 };
 
@@ -395,8 +394,7 @@ __device__ __forceinline__ Bars bars(uint8_t *smem) {
   r.s_full = r.q_ready + 1;
   r.p_full = r.s_full + 2;
   r.p_free = r.p_full + 2;
-  r.o_full = r.p_free + 2;
-  r.o_free = r.o_full + 1;
+  r.o_free = r.p_free + 2;
   return r;
 }
 
@@ -578,6 +576,13 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
   const float sl2 = p.scale_log2;
   float m_used = -INFINITY;  // maximum the exponentials are taken against (log2 units)
   float l_run = 0.f;
+  // "the P V product of chunk k has landed in O": p_free[k & 1] completes
+  // with that product (same commit).  Each buffer's phases are waited in
+  // order (chunk k waits for k - 2 before writing P), so this wait is never
+  // more than one phase ahead of the barrier and its parity cannot alias.
+  auto wait_pv_done = [&](uint32_t k) -> bool {
+    return wait_or_abort(X, &B.p_free[k & 1], (k >> 1) & 1);
+  };
 
   for (bool first = true;; first = false) {
     const int s = it % kStages;
@@ -643,7 +648,7 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
     }
     if (warp_rows && __any_sync(0xffffffffu, resc)) {
       // O holds the P V products of earlier chunks of this item: let them land
-      if (!wait_or_abort(X, B.o_full, (c - 1) & 1)) return false;
+      if (!wait_pv_done(c - 1)) return false;
       tc_fence_after();
 #pragma unroll
       for (int q4 = 0; q4 < kD / 32; ++q4) {
@@ -697,7 +702,7 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
   }
 
   // ---- the tile is done once the last P V product has landed in O ----
-  if (!wait_or_abort(X, B.o_full, (c - 1) & 1)) return false;
+  if (!wait_pv_done(c - 1)) return false;
   tc_fence_after();
   const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
   if (warp_rows) {
@@ -746,16 +751,18 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
 // ============================ CUDA-core path ============================
 // Fewer than kTcMinRows rows; warp w takes page w of every stage, lanes split
 // a page's 16 keys in halves of the head dimension.
+template <int NR>
 __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, const Item &I,
-                                     uint32_t &it) {
+                                        uint32_t &it) {
   const ItemGeom g = item_geom(p, I);
   const Bars &B = X.B;
   const int warp = X.warp, lane = X.lane;
   float *qs = reinterpret_cast<float *>(X.smem + Smem::off_ccq);
   float *mg = reinterpret_cast<float *>(X.smem + Smem::off_merge);
   float *ps = reinterpret_cast<float *>(X.smem + Smem::off_ps);
-  const int nrow = I.rows;
-  float cm[kCcRows], cl[kCcRows], co[kCcRows][4];
+  // NR rows known at compile time, or up to NR with run-time guards when NR == kCcRows
+  const int nrow = NR < kCcRows ? NR : I.rows;
+  float cm[NR], cl[NR], co[NR][4];
 
   for (bool first = true;; first = false) {
     const int s = it % kStages;
@@ -781,7 +788,7 @@ __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, c
         dst[q_slot(d0 + 7)] = bf16hi(raw.w);
       }
 #pragma unroll
-      for (int r = 0; r < kCcRows; ++r) {
+      for (int r = 0; r < NR; ++r) {
         cm[r] = -INFINITY;
         cl[r] = 0.f;
         co[r][0] = co[r][1] = co[r][2] = co[r][3] = 0.f;
@@ -803,7 +810,7 @@ __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, c
         kr[cc] = *reinterpret_cast<const uint4 *>(kb + ((lc ^ (R & 7)) << 4));
       }
 #pragma unroll
-      for (int r = 0; r < kCcRows; ++r) {
+      for (int r = 0; r < NR; ++r) {
         if (r < nrow) {
           const float *qrow = qs + r * kD + half * 64;
           float pa[4] = {0.f, 0.f, 0.f, 0.f};  // four independent partial sums
@@ -857,7 +864,7 @@ __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, c
                                                           ((vc ^ (Rv & 7)) << 4) + vsub);
         const float v0 = bf16lo(vv.x), v1 = bf16hi(vv.x), v2 = bf16lo(vv.y), v3 = bf16hi(vv.y);
 #pragma unroll
-        for (int r = 0; r < kCcRows; ++r) {
+        for (int r = 0; r < NR; ++r) {
           if (r < nrow) {
             const float pj = ps[(warp * 8 + r) * 16 + jk];
             co[r][0] = fmaf(pj, v0, co[r][0]);
@@ -876,10 +883,10 @@ __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, c
 
   // ---- finalize: merge the four warps' page subsets ----
 #pragma unroll
-  for (int r = 0; r < kCcRows; ++r)
+  for (int r = 0; r < NR; ++r)
     if (r < nrow) cl[r] = warp_sum(cl[r]);
 #pragma unroll
-  for (int r = 0; r < kCcRows; ++r) {
+  for (int r = 0; r < NR; ++r) {
     if (r < nrow) {
       float *dst = mg + (warp * 8 + r) * kPStride;
       *reinterpret_cast<float4 *>(dst + lane * 4) = make_float4(co[r][0], co[r][1], co[r][2], co[r][3]);
@@ -892,7 +899,7 @@ __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, c
   named_bar_sync(1, kCW * 32);
   if (warp == 0) {
 #pragma unroll
-    for (int r = 0; r < kCcRows; ++r) {
+    for (int r = 0; r < NR; ++r) {
       if (r < nrow) {
         float Mx = -INFINITY;
         for (int w2 = 0; w2 < kCW; ++w2) Mx = fmaxf(Mx, mg[(w2 * 8 + r) * kPStride + 128]);
@@ -956,7 +963,6 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
       mbar_init(&B.p_full[i], kCW);
       mbar_init(&B.p_free[i], 1);
     }
-    mbar_init(B.o_full, 1);
     mbar_init(B.o_free, kCW);
     misc[1] = 0;
     fence_mbar_init();
@@ -973,24 +979,55 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
 
   if (warp == kProducerWarp) {
     // ------------------------------ producer ------------------------------
+    // Page ids are read 32 at a time (one coalesced load per warp), one batch
+    // ahead of use, and the next item's descriptor is fetched while the
+    // current one streams, so no TMA issue waits on a global load.
     const uint64_t policy = l2_policy_evict_first();
     uint32_t it = 0;
     bool aborted = false;
-    for (;;) {
-      int idx = 0;
-      if (lane == 0) idx = atomicAdd(&p.ctrl[1], 1);
-      idx = __shfl_sync(0xffffffffu, idx, 0);
-      if (idx >= n_items) break;
-      const Item I = p.items[idx];
+    auto claim = [&]() -> int {
+      int v = 0;
+      if (lane == 0) v = atomicAdd(&p.ctrl[1], 1);
+      return __shfl_sync(0xffffffffu, v, 0);
+    };
+    // page id of page `page_lo + 32 * batch + lane`, or -1 past the item
+    auto load_ids = [&](const Item &I, int batch) -> int {
+      const int pg = I.page_lo + 32 * batch + lane;
+      if (pg >= I.page_hi) return -1;
+      const BatchDev &Bp = p.b[I.b];
+      return __ldg(Bp.page_table + (long long)I.r * Bp.max_pages + pg);
+    };
+    int idx = claim();
+    Item I{};
+    int ids = -1;
+    if (idx < n_items) {
+      I = p.items[idx];
+      ids = load_ids(I, 0);
+    }
+    while (idx < n_items) {
+      const int nxt = claim();
+      Item In = I;
+      if (nxt < n_items) In = p.items[nxt];  // consumed at the next item
       const BatchDev &Bt = p.b[I.b];
-      const int *prow = Bt.page_table + (long long)I.r * Bt.max_pages;
       const void *tk = &p.tmap[2 * Bt.cache];
       const void *tv = &p.tmap[2 * Bt.cache + 1];
       const int oob_row = (int)(Bt.num_pages * Bt.hkv * kPage);  // a box here reads zeros
-      for (int page = I.page_lo; page < I.page_hi; page += kStagePages) {
-        const int np = min(kStagePages, I.page_hi - page);
+      const int npages = I.page_hi - I.page_lo;
+      const int nst = (npages + kStagePages - 1) / kStagePages;
+      int ids_next = (npages > 32) ? load_ids(I, 1) : -1;
+      int ids_item_next = -1;
+      for (int st = 0; st < nst; ++st) {
+        if (st == max(0, nst - 2) && nxt < n_items) ids_item_next = load_ids(In, 0);
+        const int rel = st * kStagePages;  // first page of the stage, relative to page_lo
+        if (rel > 0 && (rel & 31) == 0) {   // move to the next batch of 32 ids
+          ids = ids_next;
+          ids_next = (rel + 32 < npages) ? load_ids(I, (rel >> 5) + 1) : -1;
+        }
+        const int page = I.page_lo + rel;
+        const int np = min(kStagePages, npages - rel);
         const int s = it % kStages;
         const uint32_t ph = (it / kStages) & 1;
+        const int pid = __shfl_sync(0xffffffffu, ids, (rel & 31) + (lane & (kStagePages - 1)));
         if (!mbar_wait_bounded(&B.empty[s], ph ^ 1)) {
           ipd_set_error(&g_attn_err, IPD_DEVERR_WAIT);
           aborted = true;
@@ -999,7 +1036,6 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
         int y = oob_row;
         bool ok = false;
         if (lane < np) {
-          const int pid = prow[page + lane];
           ok = pid >= 0 && (long long)pid < Bt.num_pages;
           if (!ok) ipd_set_error(&g_attn_err, IPD_DEVERR_PAGE_ID);
           else y = (pid * Bt.hkv + I.kvh) * kPage;
@@ -1010,7 +1046,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
           m.item = idx;
           m.page0 = page;
           m.npages = np;
-          m.flags = (page == I.page_lo ? 1 : 0) | (page + np >= I.page_hi ? 2 : 0);
+          m.flags = (st == 0 ? 1 : 0) | (st == nst - 1 ? 2 : 0);
           m.invalid = (~okmask) & ((1u << np) - 1u);
           m.path = I.path;
           meta[s] = m;
@@ -1028,6 +1064,11 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
         ++it;
       }
       if (aborted) break;
+      idx = nxt;
+      if (idx < n_items) {
+        I = In;
+        ids = ids_item_next;
+      }
     }
     if (!aborted) {
       const int s = it % kStages;
@@ -1053,83 +1094,102 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
 
   if (warp == kMmaWarp) {
     // ------------------------------ MMA issuer -----------------------------
+    // Event loop: P V of the oldest pending chunk is issued as soon as its P
+    // is written, and Q K^T of the next chunk as soon as its stage has landed
+    // and an S buffer is free, so neither waits for the other's inputs.
     constexpr uint32_t idesc_s = idesc_bf16_f32(kTcRows, kStageKeys, 0);
     constexpr uint32_t idesc_o = idesc_bf16_f32(kTcRows, kD, 1);
     const uint32_t sq = smem_u32(smem + Smem::off_q);
     uint32_t it = 0, c = 0, nq = 0, cur_item = 0;
-    bool pend = false, pend_first = false;
-    uint32_t pend_c = 0, pend_s = 0, pend_item = 0;
-    bool ok = true;
-    // O (+)= P[cc & 1] V[stage ss], with P = P_hi + P_lo; the first chunk of
-    // an item overwrites O (after the previous item's O was read out).
-    auto issue_pv = [&](uint32_t cc, uint32_t ss, bool firstc, uint32_t item) -> bool {
-      const uint32_t bb = cc & 1;
-      if (!mbar_wait_bounded(&B.p_full[bb], (cc >> 1) & 1)) return false;
-      if (firstc && !mbar_wait_bounded(B.o_free, (item & 1) ^ 1)) return false;
-      tc_fence_after();
-      if (lane == 0) {
-        const uint32_t pa = smem_u32(smem + Smem::off_p + bb * 2 * Smem::kPBytes);
-        const uint32_t va = smem_u32(stage_v(smem, ss));
+    uint32_t pc[2], ps_[2], pitem[2];  // chunks with S issued and P V pending, oldest first
+    bool pfirst[2];
+    int qn = 0;
+    bool done = false, ok = true;
+    long long t_last = clock64();
+    while (!done || qn > 0) {
+      bool progress = false;
+      if (qn > 0) {
+        const uint32_t cc = pc[0], bb = cc & 1;
+        if (warp_test(&B.p_full[bb], (cc >> 1) & 1) &&
+            (!pfirst[0] || warp_test(B.o_free, (pitem[0] & 1) ^ 1))) {
+          tc_fence_after();
+          if (lane == 0) {
+            // O (+)= P V with P = P_hi + P_lo; the first chunk of an item overwrites O
+            const uint32_t pa = smem_u32(smem + Smem::off_p + bb * 2 * Smem::kPBytes);
+            const uint32_t va = smem_u32(stage_v(smem, ps_[0]));
 #pragma unroll
-        for (int kk = 0; kk < kStageKeys / 16; ++kk) {
-          const uint64_t bd = sdesc_sw128(va + kk * 16 * 128, kHalfBytes, 1024);
-          tc_mma_bf16(tmem + col_o(0), sdesc_sw128(pa + kk * 32, 16, 1024), bd, idesc_o,
-                      (firstc && kk == 0) ? 0u : 1u);
-          tc_mma_bf16(tmem + col_o(0), sdesc_sw128(pa + Smem::kPBytes + kk * 32, 16, 1024), bd,
-                      idesc_o, 1u);
+            for (int kk = 0; kk < kStageKeys / 16; ++kk) {
+              const uint64_t bd = sdesc_sw128(va + kk * 16 * 128, kHalfBytes, 1024);
+              tc_mma_bf16(tmem + col_o(0), sdesc_sw128(pa + kk * 32, 16, 1024), bd, idesc_o,
+                          (pfirst[0] && kk == 0) ? 0u : 1u);
+              tc_mma_bf16(tmem + col_o(0), sdesc_sw128(pa + Smem::kPBytes + kk * 32, 16, 1024),
+                          bd, idesc_o, 1u);
+            }
+            tc_commit(&B.p_free[bb]);
+            tc_commit(&B.empty[ps_[0]]);
+          }
+          __syncwarp();
+          pc[0] = pc[1]; ps_[0] = ps_[1]; pitem[0] = pitem[1]; pfirst[0] = pfirst[1];
+          --qn;
+          progress = true;
         }
-        tc_commit(B.o_full);
-        tc_commit(&B.p_free[bb]);
-        tc_commit(&B.empty[ss]);
       }
-      __syncwarp();
-      return true;
-    };
-    for (;;) {
-      const int s = it % kStages;
-      if (!mbar_wait_bounded(&B.full[s], (it / kStages) & 1)) { ok = false; break; }
-      const StageMeta M = meta[s];
-      if (M.item < 0) break;
-      if (!M.path) {
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&B.empty[s]);
-        ++it;
-        continue;
-      }
-      const bool firstc = M.flags & 1;
-      if (firstc) {
-        if (!mbar_wait_bounded(B.q_ready, nq & 1)) { ok = false; break; }
-        cur_item = nq++;
-      }
-      tc_fence_after();
-      const uint32_t b = c & 1;
-      if (lane == 0) {
-        const uint32_t ka = smem_u32(stage_k(smem, s));
+      if (!progress && !done && qn < 2) {
+        const int s = it % kStages;
+        if (warp_test(&B.full[s], (it / kStages) & 1)) {
+          int item = 0, flags = 0, path = 0;
+          if (lane == 0) {
+            item = meta[s].item;
+            flags = meta[s].flags;
+            path = meta[s].path;
+          }
+          item = __shfl_sync(0xffffffffu, item, 0);
+          flags = __shfl_sync(0xffffffffu, flags, 0);
+          path = __shfl_sync(0xffffffffu, path, 0);
+          if (item < 0) {
+            done = true;
+            progress = true;
+          } else if (!path) {
+            if (lane == 0) mbar_arrive(&B.empty[s]);
+            __syncwarp();
+            ++it;
+            progress = true;
+          } else {
+            const bool firstc = flags & 1;
+            if (!firstc || warp_test(B.q_ready, nq & 1)) {
+              if (firstc) cur_item = nq++;
+              tc_fence_after();
+              const uint32_t b = c & 1;
+              if (lane == 0) {
+                const uint32_t ka = smem_u32(stage_k(smem, s));
 #pragma unroll
-        for (int kk = 0; kk < kD / 16; ++kk) {
-          const uint32_t qoff = (kk >> 2) * (kTcRows * 128) + (kk & 3) * 32;
-          const uint32_t koff = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
-          tc_mma_bf16(tmem + col_s(b), sdesc_sw128(sq + qoff, 16, 1024),
-                      sdesc_sw128(ka + koff, 16, 1024), idesc_s, kk > 0);
+                for (int kk = 0; kk < kD / 16; ++kk) {
+                  const uint32_t qoff = (kk >> 2) * (kTcRows * 128) + (kk & 3) * 32;
+                  const uint32_t koff = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
+                  tc_mma_bf16(tmem + col_s(b), sdesc_sw128(sq + qoff, 16, 1024),
+                              sdesc_sw128(ka + koff, 16, 1024), idesc_s, kk > 0);
+                }
+                tc_commit(&B.s_full[b]);
+              }
+              __syncwarp();
+              pc[qn] = c; ps_[qn] = s; pitem[qn] = cur_item; pfirst[qn] = firstc;
+              ++qn;
+              ++c;
+              ++it;
+              progress = true;
+            }
+          }
         }
-        tc_commit(&B.s_full[b]);
       }
-      __syncwarp();
-      if (pend) {
-        if (!issue_pv(pend_c, pend_s, pend_first, pend_item)) { ok = false; break; }
-        pend = false;
-      }
-      if (M.flags & 2) {
-        if (!issue_pv(c, s, firstc, cur_item)) { ok = false; break; }
+      if (progress) {
+        t_last = clock64();
       } else {
-        pend = true;
-        pend_c = c;
-        pend_s = s;
-        pend_first = firstc;
-        pend_item = cur_item;
+        if (*(volatile uint32_t *)&misc[1] || clock64() - t_last > kWaitLimitCycles) {
+          ok = false;
+          break;
+        }
+        __nanosleep(32);
       }
-      ++c;
-      ++it;
     }
     if (!ok) {
       ipd_set_error(&g_attn_err, IPD_DEVERR_WAIT);
@@ -1151,7 +1211,15 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
     const StageMeta M = meta[s];
     if (M.item < 0 || *(volatile uint32_t *)&misc[1]) break;
     const Item I = p.items[M.item];
-    const bool ok = I.path ? tc_item(p, X, I, it, c) : cc_item(p, X, I, it);
+    bool ok;
+    if (I.path) {
+      ok = tc_item(p, X, I, it, c);
+    } else {
+      // GQA-2 decode (two rows) gets straight-line code; other sizes take
+      // the guarded loop (more instances overflow the register budget)
+      if (I.rows == 2) ok = cc_item<2>(p, X, I, it);
+      else ok = cc_item<kCcRows>(p, X, I, it);
+    }
     if (!ok) break;
   }
   named_bar_sync(2, (kCW + 1) * 32);

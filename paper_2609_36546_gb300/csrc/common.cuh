@@ -268,3 +268,26 @@ IPD_DEVINL uint32_t pack_bf16x2(float lo, float hi) {
   asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(d) : "f"(hi), "f"(lo));
   return d;
 }
+
+// Non-blocking test of an mbarrier phase.
+IPD_DEVINL bool mbar_test(uint64_t *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// Lane 0 tests the phase and the warp follows its answer; on success every
+// lane then observes the (completed, so immediate) phase itself.
+IPD_DEVINL bool warp_test(uint64_t *bar, uint32_t parity) {
+  uint32_t r = 0;
+  if ((threadIdx.x & 31) == 0) r = mbar_test(bar, parity) ? 1u : 0u;
+  r = __shfl_sync(0xffffffffu, r, 0);
+  if (r) (void)mbar_try_wait(bar, parity);
+  return r != 0;
+}
