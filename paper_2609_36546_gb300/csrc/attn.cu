@@ -9,23 +9,27 @@
 // Work decomposition (device side, no host round trip):
 //   task  = (batch, request, kv head, row block); a row is one (span query,
 //           query head) pair, row = i * G + j for query i and head kvh*G + j.
-//   item  = (task, KV chunk); long tasks are split into chunks so that the
-//           work list has about 8 items per SM; split partials are merged by
-//           the last CTA to finish a task (atomic ticket, no waiting).
+//   item  = (task, KV chunk); tasks longer than about a quarter of an SM's
+//           share are split, items are claimed longest first, and a small
+//           follow-up kernel merges the partials of split tasks.
+// KV pages stream through a 3-stage ring of 128-key stages (64 KB: K and V,
+// each as two 64-dim halves of 128 swizzled rows), written by 2-D TMA.
 // Two compute paths, chosen per task by its row count:
-//   tensor path (rows >= kTcMinRows): a 128-row tile.  S = Q K^T and
-//     O += P V run on tcgen05 (bf16 operands in 128-byte-swizzled shared
-//     memory, fp32 accumulators in TMEM); one thread per row does the online
-//     softmax.  O stays in TMEM for the whole item and is rescaled only when
-//     a row maximum grows by more than 2^8 (exponentials are taken against a
-//     stale maximum until then).  P is passed as two bf16 terms (value and
-//     rounded residual), so the P V product keeps about 16 bits of each
-//     probability.  S and P are double-buffered: the softmax of chunk j
-//     overlaps the P V product of chunk j-1 and the Q K^T product of j+1.
-//   CUDA-core path (fewer rows: GQA group 2 decode): fp32 FMA, one page of 16
-//     keys per warp, two lanes per key.
-// Warp roles: warps 0-3 compute, warp 4 streams KV pages with 2-D TMA into a
-// 4-stage mbarrier ring, warp 5 issues the tensor-core instructions.
+//   tensor path (rows >= kTcMinRows): a 128-lane tile.  S = Q K^T (Q read
+//     from TMEM, K from shared memory, N = 128 keys) and O += P V run on
+//     tcgen05 with fp32 accumulators in TMEM.  O stays in TMEM for the whole
+//     item and is rescaled only when a row maximum grows by more than 2^8.
+//     P is passed as two bf16 terms (its upper 16 bits and the truncated
+//     residual), so the P V product keeps about 16 bits of each probability.
+//     Tiles of at most 64 rows give each row two threads (one per half of the
+//     chunk's keys) and stack the two P terms in the two 64-row halves of one
+//     operand; larger tiles keep one thread per row.  S is double-buffered,
+//     so the softmax of chunk j overlaps Q K^T of j+1 and P V of j-1.
+//   CUDA-core path (fewer rows: GQA group 2 decode): fp32 FMA, two pages of
+//     16 keys per warp and stage, two lanes per key.
+// Warp roles: warps 0-3 compute, warp 4 streams KV pages, warp 5 issues the
+// tensor-core instructions in a fixed order (Q K^T of chunk j, then P V of
+// chunk j-1).
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
@@ -42,27 +46,35 @@ namespace {
 
 constexpr int kPage = 16;
 constexpr int kD = 128;
-constexpr int kStagePages = 4;                    // 64 keys per stage
+constexpr int kStagePages = 8;                    // 128 keys per stage
 constexpr int kStageKeys = kStagePages * kPage;
-constexpr int kStages = 4;
-constexpr int kHalfBytes = kStageKeys * 128;      // one 64-dim half of 64 key rows: 8 KB
-constexpr int kStageBytes = 4 * kHalfBytes;       // K and V, two halves each: 32 KB
-constexpr int kTcRows = 128;                      // rows of a tensor-core tile (M)
+constexpr int kStages = 3;
+constexpr int kHalfBytes = kStageKeys * 128;      // one 64-dim half of 128 key rows: 16 KB
+constexpr int kStageBytes = 4 * kHalfBytes;       // K and V, two halves each: 64 KB
+constexpr int kTcRows = 128;                      // TMEM lanes of a tensor-core tile (M)
+constexpr int kTcSplitRows = 64;                  // tiles up to this size split rows over two threads
 constexpr int kTcMinRows = 8;                     // tasks with at least this many rows use it
 constexpr int kCcRows = kTcMinRows - 1;           // CUDA-core tasks have fewer rows
 constexpr int kCW = 4;                            // compute warps
 constexpr int kProducerWarp = 4;
 constexpr int kMmaWarp = 5;
 constexpr int kThreads = 6 * 32;
-constexpr int kTargetItemsPerSm = 8;
+constexpr int kTargetItemsPerSm = 4;               // items of about a quarter of an SM's share
+constexpr int kSizesPerBatch = 32;                // claim order: batch by batch, and within a
+constexpr int kSizeBuckets = IPD_MAX_BATCHES * kSizesPerBatch;  // batch the longest items first
 constexpr int kMaxTargetItems = 4096;            // bound used for workspace sizing
 constexpr int kMinChunkPages = 16;
 constexpr int kSplitMax = 16;
 constexpr int kPStride = 132;                     // floats per partial row: o[128], m, l, pad
 constexpr uint32_t kTmemCols = 512;
-// TMEM columns: S double buffer at 0 and 64, the O accumulator at 128..255
-__device__ __forceinline__ uint32_t col_s(uint32_t b) { return b * 64u; }
-__device__ __forceinline__ uint32_t col_o(uint32_t b) { return 128u + b * 128u; }
+// TMEM columns: the S double buffer at 0 and 128 (fp32, one column per key;
+// 128-row tiles later overwrite a consumed buffer with their P residual),
+// the O accumulator at 256, the Q tile at 384 (64 columns of bf16 pairs).
+__device__ __forceinline__ uint32_t col_s(uint32_t b) { return b * 128u; }
+constexpr uint32_t kColO = 256;
+constexpr uint32_t kColQ = 384;
+// item paths
+constexpr int kPathCc = 0, kPathTcSplit = 1, kPathTcFull = 2;
 
 struct BatchDev {
   const uint16_t *q;
@@ -77,7 +89,7 @@ struct BatchDev {
 struct Item {
   int b, r, kvh, rb;
   int split, n_split, page_lo, page_hi;
-  int task, pbase, rows, path;  // path: 1 = tensor cores, 0 = CUDA cores
+  int task, pbase, rows, path;  // path: kPathCc, kPathTcSplit or kPathTcFull
 };
 
 struct AttnParams {
@@ -90,11 +102,11 @@ struct AttnParams {
   int *ctrl;       // [0] n_items, [1] dynamic item counter, [2] n_tasks, [3] partial rows
   int4 *reqinfo;   // per flattened request: item offset, task offset, partial offset, n_split
   Item *items;
-  int *tickets;
   float *partials;
   int item_cap, task_cap;
   long long prow_cap;
   int target_items;  // work-list size the planner aims for (a multiple of the SM count)
+  int n_sms;
 };
 
 struct StageMeta {
@@ -111,7 +123,7 @@ struct StageMeta {
 // host-side sizes
 // --------------------------------------------------------------------------
 struct WsLayout {
-  size_t off_ctrl, off_reqinfo, off_items, off_tickets, off_partials, total;
+  size_t off_ctrl, off_reqinfo, off_items, off_partials, total;
   int item_cap, task_cap, total_reqs;
   long long prow_cap;
 };
@@ -189,8 +201,6 @@ WsLayout layout(const ipd_attn_batch *const *bs, int n) {
   off = align_up(off + (size_t)reqs * sizeof(int4), 256);
   L.off_items = off;
   off = align_up(off + (size_t)L.item_cap * sizeof(Item), 256);
-  L.off_tickets = off;
-  off = align_up(off + (size_t)L.task_cap * sizeof(int), 256);
   L.off_partials = off;
   off = align_up(off + (size_t)prow_cap * kPStride * sizeof(float), 256);
   L.total = off;
@@ -273,12 +283,38 @@ __device__ void block_scan3(int3 v, int3 &excl, int3 &tot, int3 *sh) {
   __syncthreads();
 }
 
+// Pages per split of a request with `pages` pages, for a target chunk size:
+// a whole number of stages, so only a request's last split ends mid-stage.
+__device__ __forceinline__ int split_pages(int pages, long long chunk) {
+  long long ns = (pages + chunk - 1) / chunk;
+  if (ns > kSplitMax) ns = kSplitMax;
+  const int per = (int)((pages + ns - 1) / ns);
+  return (per + kStagePages - 1) / kStagePages * kStagePages;
+}
+__device__ __forceinline__ int split_count(int pages, long long chunk) {
+  const int per = split_pages(pages, chunk);
+  return (pages + per - 1) / per;
+}
+
+// Claim-order bucket of an item of batch `b` with `n` pages; higher buckets
+// are claimed first.  Streaming one cache at a time measured faster than
+// interleaving both (every CTA streams more slowly when the two pools are
+// read at once), and longest-first within a batch keeps the tail short.
+__device__ __forceinline__ int size_bucket(int b, int n_batches, int n, long long chunk) {
+  const long long top = (chunk + kStagePages - 1) / kStagePages * kStagePages;  // usual largest
+  long long k = (long long)n * (kSizesPerBatch - 1) / top;
+  if (k > kSizesPerBatch - 1) k = kSizesPerBatch - 1;
+  return (n_batches - 1 - b) * kSizesPerBatch + (int)k;
+}
+
 __global__ void __launch_bounds__(1024) attn_plan_kernel(const __grid_constant__ AttnParams p) {
   __shared__ long long red[32];
   __shared__ int3 sh3[32];
   __shared__ int s_fail;
+  __shared__ int s_slot[kSizeBuckets];  // items per size bucket, then each bucket's next slot
   const int tid = threadIdx.x;
   if (tid == 0) s_fail = 0;
+  for (int i = tid; i < kSizeBuckets; i += blockDim.x) s_slot[i] = 0;
 
   long long w = 0;
   for (int gi = tid; gi < p.total_reqs; gi += blockDim.x) {
@@ -290,6 +326,8 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const __grid_constant__
   long long chunk = (W + p.target_items - 1) / p.target_items;
   if (chunk < kMinChunkPages) chunk = kMinChunkPages;
 
+  // per request: split count, partial-row offset (exclusive scans), and the
+  // size histogram of its items
   int3 carry = make_int3(0, 0, 0);
   for (int base = 0; base < p.total_reqs; base += blockDim.x) {
     const int gi = base + tid;
@@ -299,10 +337,13 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const __grid_constant__
       const int b = find_batch(p, gi);
       const ReqShape s = req_shape(p, b, gi - p.req_base[b]);
       if (s.pages > 0) {
-        const long long ns = (s.pages + chunk - 1) / chunk;
-        nsplit = (int)(ns < kSplitMax ? ns : kSplitMax);
+        nsplit = split_count(s.pages, chunk);
+        const int per = split_pages(s.pages, chunk);
         const int tasks = p.b[b].hkv * s.nrb;
         cnt = make_int3(tasks * nsplit, tasks, nsplit > 1 ? nsplit * p.b[b].hkv * s.rows : 0);
+        for (int sp = 0; sp < nsplit; ++sp)
+          atomicAdd(&s_slot[size_bucket(b, p.n_batches, min(s.pages, (sp + 1) * per) - sp * per, chunk)],
+                    tasks);
       }
     }
     int3 ex, tot;
@@ -315,6 +356,13 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const __grid_constant__
     if (carry.x > p.item_cap || carry.y > p.task_cap || carry.z > p.prow_cap) {
       ipd_set_error(&g_attn_err, IPD_DEVERR_PLAN);
       s_fail = 1;
+    }
+    // largest bucket first
+    int off = 0;
+    for (int k = kSizeBuckets - 1; k >= 0; --k) {
+      const int n = s_slot[k];
+      s_slot[k] = off;
+      off += n;
     }
     p.ctrl[0] = s_fail ? 0 : carry.x;
     p.ctrl[1] = 0;
@@ -330,14 +378,13 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const __grid_constant__
     const ReqShape s = req_shape(p, b, r);
     if (s.pages == 0) continue;
     const int4 info = p.reqinfo[gi];
-    int item = info.x, task = info.y;
+    int task = info.y;
     const int ns = info.w;
-    const int per = (s.pages + ns - 1) / ns;
+    const int per = split_pages(s.pages, chunk);
     for (int kvh = 0; kvh < p.b[b].hkv; ++kvh) {
       for (int rb = 0; rb < s.nrb; ++rb) {
         const int rows = min(s.rpb, s.rows - rb * s.rpb);
         const int pbase = ns > 1 ? info.z + ns * (kvh * s.rows + rb * s.rpb) : -1;
-        p.tickets[task] = 0;
         for (int sp = 0; sp < ns; ++sp) {
           Item it;
           it.b = b; it.r = r; it.kvh = kvh; it.rb = rb;
@@ -345,11 +392,64 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const __grid_constant__
           it.page_lo = sp * per;
           it.page_hi = min(s.pages, (sp + 1) * per);
           it.task = task; it.pbase = pbase; it.rows = rows;
-          it.path = s.rows >= kTcMinRows ? 1 : 0;
-          p.items[item++] = it;
+          it.path = s.rows < kTcMinRows ? kPathCc : (rows <= kTcSplitRows ? kPathTcSplit : kPathTcFull);
+          const int slot =
+              atomicAdd(&s_slot[size_bucket(b, p.n_batches, it.page_hi - it.page_lo, chunk)], 1);
+          p.items[slot] = it;
         }
         ++task;
       }
+    }
+  }
+}
+
+// Split-KV merge: each task split over several items combines its splits'
+// partial rows (unnormalised O, maximum m, sum l, all in log2 units) into the
+// output rows.  Work unit = (item, group of 8 rows); warp = row, lane = 4
+// dims, every split's loads in flight at once.
+__global__ void __launch_bounds__(256) attn_merge_kernel(const __grid_constant__ AttnParams p) {
+  constexpr int kGroups = kTcRows / 8;  // row groups of 8 (one per warp) per item
+  const int n_units = p.ctrl[0] * kGroups;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int u = blockIdx.x; u < n_units; u += gridDim.x) {
+    const Item I = p.items[u / kGroups];
+    const int r = (u % kGroups) * 8 + warp;
+    if (I.n_split < 2 || I.split != 0 || (u % kGroups) * 8 >= I.rows) continue;
+    if (r < I.rows) {
+      const BatchDev &Bt = p.b[I.b];
+      const int q0 = Bt.cu_q[I.r], G = Bt.group;
+      const int rpb = I.path != kPathCc ? kTcRows : kCcRows;
+      const int ns = I.n_split;
+      const size_t sstr = (size_t)I.rows * kPStride;
+      const float *base = p.partials + (size_t)(I.pbase + r) * kPStride;
+      const float mv = lane < ns ? __ldcg(base + lane * sstr + 128) : -INFINITY;
+      const float lv = lane < ns ? __ldcg(base + lane * sstr + 129) : 0.f;
+      float4 ov[kSplitMax];
+#pragma unroll
+      for (int sp = 0; sp < kSplitMax; ++sp)
+        if (sp < ns) ov[sp] = __ldcg(reinterpret_cast<const float4 *>(base + sp * sstr) + lane);
+      const float Mx = warp_max(mv);
+      const float f = mv == -INFINITY ? 0.f : ex2_approx(mv - Mx);
+      const float Ls = warp_sum(lv * f);
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int sp = 0; sp < kSplitMax; ++sp) {
+        if (sp < ns) {
+          const float fs = __shfl_sync(0xffffffffu, f, sp);
+          acc.x = fmaf(ov[sp].x, fs, acc.x);
+          acc.y = fmaf(ov[sp].y, fs, acc.y);
+          acc.z = fmaf(ov[sp].z, fs, acc.z);
+          acc.w = fmaf(ov[sp].w, fs, acc.w);
+        }
+      }
+      const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+      const int grow = I.rb * rpb + r;
+      const int qi = grow / G, j = grow % G;
+      uint2 pk;
+      pk.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+      pk.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+      *reinterpret_cast<uint2 *>(Bt.out + ((size_t)(q0 + qi) * Bt.hq + I.kvh * G + j) * kD +
+                                 lane * 4) = pk;
     }
   }
 }
@@ -358,31 +458,31 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const __grid_constant__
 // the attention kernel
 // --------------------------------------------------------------------------
 struct Smem {
-  static constexpr int off_stage = 0;                              // 4 x 32 KB, 1024-aligned
-  static constexpr int off_q = off_stage + kStages * kStageBytes;  // 32 KB
-  static constexpr int off_p = off_q + 2 * kTcRows * 128;          // 2 buffers x (hi, lo) x 16 KB
-  static constexpr int kPBytes = kTcRows * 128;                    // one 128 x 64 bf16 operand
-  static constexpr int off_meta = off_p + 4 * kPBytes;
+  static constexpr int off_stage = 0;                              // 3 x 64 KB, 1024-aligned
+  static constexpr int off_p = off_stage + kStages * kStageBytes;  // P: two blocks of 128 rows x 64 keys
+  static constexpr int kPBlock = kTcRows * 128;                    // 16 KB
+  static constexpr int off_x = off_p + 2 * kPBlock;                // row-max exchange [2][128], l [128]
+  static constexpr int off_meta = off_x + 3 * kTcRows * 4;
   static constexpr int off_bar = off_meta + kStages * (int)sizeof(StageMeta);
-  static constexpr int n_bars = 2 * kStages + 1 + 2 + 2 + 2 + 1;
+  static constexpr int n_bars = 2 * kStages + 5;
   static constexpr int off_misc = off_bar + n_bars * 8;
   static constexpr int total = off_misc + 64;
-  // CUDA-core path scratch (inside the Q and P regions, unused by that path)
-  static constexpr int off_ccq = off_q;                              // fp32 [7][128]
-  static constexpr int off_merge = off_p;                            // fp32 [4][8][132]
+  // CUDA-core path scratch (inside the P region, unused by that path)
+  static constexpr int off_ccq = off_p;                              // fp32 [7][128]
+  static constexpr int off_merge = off_ccq + kCcRows * kD * 4;       // fp32 [4][8][132]
   static constexpr int off_ps = off_merge + kCW * 8 * kPStride * 4;  // fp32 [4][8][16]
-  // split-merge scratch (P region, free once an item's last P V product landed)
-  static constexpr int off_msc = off_p;                              // fp32 [128][16] + [128]
 };
-static_assert(Smem::off_ps + kCW * 8 * 16 * 4 <= Smem::off_meta, "CUDA-core scratch overflow");
+static_assert(Smem::off_ps + kCW * 8 * 16 * 4 <= Smem::off_x, "CUDA-core scratch overflow");
+static_assert(kTcSplitRows * kD * 4 <= 2 * Smem::kPBlock, "O exchange overflow");
+static_assert(Smem::off_bar % 8 == 0, "mbarrier alignment");
 static_assert(Smem::total <= 227 * 1024, "shared memory");
 
 struct Bars {
-  uint64_t *full, *empty;     // KV ring
-  uint64_t *q_ready;          // Q tile written (one phase per tensor item)
-  uint64_t *s_full, *p_full;  // S = Q K^T landed / P written, per buffer
-  uint64_t *p_free;           // P V product done (P read, O written), per buffer
-  uint64_t *o_free;           // O read out (one phase per tensor item)
+  uint64_t *full, *empty;  // KV ring
+  uint64_t *q_ready;       // Q tile written to TMEM (one phase per tensor item)
+  uint64_t *s_full;        // S = Q K^T landed, per S buffer (one phase per use)
+  uint64_t *p_full;        // P of a chunk written (one phase per chunk)
+  uint64_t *p_free;        // P V product of a chunk done: P read, O written (one phase per chunk)
 };
 
 __device__ __forceinline__ Bars bars(uint8_t *smem) {
@@ -393,8 +493,7 @@ __device__ __forceinline__ Bars bars(uint8_t *smem) {
   r.q_ready = b + 2 * kStages;
   r.s_full = r.q_ready + 1;
   r.p_full = r.s_full + 2;
-  r.p_free = r.p_full + 2;
-  r.o_free = r.p_free + 2;
+  r.p_free = r.p_full + 1;
   return r;
 }
 
@@ -423,7 +522,7 @@ struct CompCtx {
   uint8_t *smem;
   Bars B;
   StageMeta *meta;
-  uint32_t *misc;  // [0] TMEM base, [1] abort flag, [2] ticket broadcast
+  uint32_t *misc;  // [0] TMEM base, [1] abort flag
   uint32_t tmem;
   int warp, lane, ctid;
 };
@@ -463,73 +562,6 @@ __device__ __forceinline__ const uint16_t *q_row(const ItemGeom &g, const Item &
   return g.Bt->q + row_off(g, I, grow);
 }
 
-// The last CTA of a split task merges the partials of all its splits.
-// Step 1 (thread = row): scale factors of every split.  Step 2 (warp = 4 rows
-// at a time, lane = 4 dims): weighted sums, all split loads in flight at once.
-__device__ void merge_splits(const AttnParams &p, const CompCtx &X, const Item &I,
-                             const ItemGeom &g) {
-  float *sc = reinterpret_cast<float *>(X.smem + Smem::off_msc);  // [128][kSplitMax]
-  float *inv_l = sc + kTcRows * kSplitMax;                         // [128]
-  const int ns = I.n_split;
-  const size_t sstr = (size_t)I.rows * kPStride;
-  const int rpb = I.path ? kTcRows : kCcRows;
-  for (int r = X.ctid; r < I.rows; r += kCW * 32) {
-    const float *base = p.partials + (size_t)(I.pbase + r) * kPStride;
-    float mv[kSplitMax], lv[kSplitMax];
-#pragma unroll
-    for (int sp = 0; sp < kSplitMax; ++sp) {
-      mv[sp] = sp < ns ? __ldcg(base + sp * sstr + 128) : -INFINITY;
-      lv[sp] = sp < ns ? __ldcg(base + sp * sstr + 129) : 0.f;
-    }
-    float Mx = -INFINITY;
-#pragma unroll
-    for (int sp = 0; sp < kSplitMax; ++sp) Mx = fmaxf(Mx, mv[sp]);
-    float Ls = 0.f;
-#pragma unroll
-    for (int sp = 0; sp < kSplitMax; ++sp) {
-      const float f = mv[sp] == -INFINITY ? 0.f : ex2_approx(mv[sp] - Mx);
-      sc[r * kSplitMax + sp] = f;
-      Ls = fmaf(lv[sp], f, Ls);
-    }
-    inv_l[r] = Ls > 0.f ? 1.f / Ls : 0.f;
-  }
-  named_bar_sync(1, kCW * 32);
-  for (int r0 = X.warp * 4; r0 < I.rows; r0 += kCW * 4) {
-    float4 acc[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) acc[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int r = r0 + u;
-      if (r < I.rows) {
-        const float *base = p.partials + (size_t)(I.pbase + r) * kPStride;
-#pragma unroll
-        for (int sp = 0; sp < kSplitMax; ++sp) {
-          if (sp < ns) {
-            const float f = sc[r * kSplitMax + sp];
-            const float4 ov = __ldcg(reinterpret_cast<const float4 *>(base + sp * sstr) + X.lane);
-            acc[u].x = fmaf(ov.x, f, acc[u].x);
-            acc[u].y = fmaf(ov.y, f, acc[u].y);
-            acc[u].z = fmaf(ov.z, f, acc[u].z);
-            acc[u].w = fmaf(ov.w, f, acc[u].w);
-          }
-        }
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int r = r0 + u;
-      if (r < I.rows) {
-        const float inv = inv_l[r];
-        uint2 pk;
-        pk.x = pack_bf16x2(acc[u].x * inv, acc[u].y * inv);
-        pk.y = pack_bf16x2(acc[u].z * inv, acc[u].w * inv);
-        *reinterpret_cast<uint2 *>(out_row(g, I, I.rb * rpb + r) + X.lane * 4) = pk;
-      }
-    }
-  }
-}
-
 // Zero the V rows of stage s at or past the end of the sequence: unwritten
 // cache slots may hold non-finite bits, and a zero probability times NaN is NaN.
 __device__ __forceinline__ void zero_tail(const CompCtx &X, int s, int page0, int L) {
@@ -545,44 +577,42 @@ __device__ __forceinline__ void zero_tail(const CompCtx &X, int s, int page0, in
   named_bar_sync(1, kCW * 32);
 }
 
-// After this CTA wrote its split partial: take a ticket; the last CTA of the
-// task merges every split (compute warps; all threads call it).
-__device__ __forceinline__ void ticket_merge(const AttnParams &p, const CompCtx &X, const Item &I,
-                                             const ItemGeom &g) {
-  __threadfence();
-  named_bar_sync(1, kCW * 32);
-  if (X.ctid == 0) X.misc[2] = (atomicAdd(&p.tickets[I.task], 1) == I.n_split - 1);
-  named_bar_sync(1, kCW * 32);
-  if (X.misc[2]) {
-    __threadfence();
-    merge_splits(p, X, I, g);
-  }
-}
-
 // ============================ tensor-core path ============================
-// One 128-row tile over the item's KV chunks; thread = row.  Returns false on
-// a wait time-out.  `it` (stage counter) and `c` (chunk counter) advance.
+// One 128-lane tile over the item's KV chunks of 128 keys.
+//   kSplit (at most 64 rows): TMEM lanes 64..127 repeat rows 0..63 (the Q
+//     tile is written twice), and thread t takes row t mod 64 and keys
+//     [64 h, 64 h + 64) of every chunk, h = t / 64, so the exponentials are
+//     spread over all four warps; the two threads of a row agree on the
+//     chunk maximum through shared memory.  P goes to shared memory with its
+//     upper bf16 term in rows 0..63 and its residual in rows 64..127 of one
+//     128-row operand: one MMA per 16 keys leaves P_hi V in O rows 0..63 and
+//     P_lo V in O rows 64..127, which the finalize adds.
+//   otherwise (65..128 rows): thread t takes row t and all 128 keys.  The
+//     upper term of P goes to shared memory, the residual to the TMEM columns
+//     of the chunk's own (already consumed) S buffer, and P V takes two MMAs
+//     per 16 keys.
+// Returns false on a wait time-out.  `it` (stage counter) and `c` (chunk
+// counter) advance.
+template <bool kSplit>
 __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, const Item &I,
                                         uint32_t &it, uint32_t &c) {
   const ItemGeom g = item_geom(p, I);
   const Bars &B = X.B;
-  const int warp = X.warp, lane = X.lane;
-  const int row = warp * 32 + lane;
+  const int t = X.ctid;                                   // TMEM lane
+  const int row = kSplit ? (t & (kTcSplitRows - 1)) : t;  // tile row
+  const int h = kSplit ? (t >> 6) : 0;                    // key half (split rows)
   const bool real = row < I.rows;
-  const bool warp_rows = warp * 32 < I.rows;  // the warp owns at least one real row
-  const uint32_t tl = X.tmem + ((uint32_t)(warp * 32) << 16);
+  const uint32_t tl = X.tmem + ((uint32_t)(X.warp * 32) << 16);
   const int lim = g.L - g.ql + (I.rb * kTcRows + row) / g.G;  // last key this row sees
   const int lim_all = g.L - g.ql;                             // every row sees up to here
   const float sl2 = p.scale_log2;
+  float *xbuf = reinterpret_cast<float *>(X.smem + Smem::off_x);
   float m_used = -INFINITY;  // maximum the exponentials are taken against (log2 units)
-  float l_run = 0.f;
-  // "the P V product of chunk k has landed in O": p_free[k & 1] completes
-  // with that product (same commit).  Each buffer's phases are waited in
-  // order (chunk k waits for k - 2 before writing P), so this wait is never
-  // more than one phase ahead of the barrier and its parity cannot alias.
-  auto wait_pv_done = [&](uint32_t k) -> bool {
-    return wait_or_abort(X, &B.p_free[k & 1], (k >> 1) & 1);
-  };
+  float l_run = 0.f;         // this thread's share of the row sum
+  // "P V of chunk k has landed in O" is completion k of p_free.  Chunk k waits
+  // for completion k - 1 before it writes P, so the barrier is never more than
+  // one phase behind a wait and the parity cannot alias.
+  auto wait_pv_done = [&](uint32_t k) -> bool { return wait_or_abort(X, B.p_free, k & 1); };
 
   for (bool first = true;; first = false) {
     const int s = it % kStages;
@@ -590,20 +620,27 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
     const StageMeta M = X.meta[s];
     zero_tail(X, s, M.page0, g.L);
     if (first) {
-      // Q tile: rows rb*128 .. +127 of the task, bf16, swizzled, zero padded
-      uint8_t *qb = X.smem + Smem::off_q;
-      for (int e = X.ctid; e < kTcRows * 16; e += kCW * 32) {
-        const int r = e >> 4, cpart = e & 15;
+      // Q: lane t <- tile row `row` as 64 columns of bf16 pairs (zeros past the rows)
+      uint32_t qw[2][32];
+      const uint4 *src = reinterpret_cast<const uint4 *>(q_row(g, I, I.rb * kTcRows + row));
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
         uint4 v = make_uint4(0, 0, 0, 0);
-        if (r < I.rows) v = *reinterpret_cast<const uint4 *>(q_row(g, I, I.rb * kTcRows + r) + cpart * 8);
-        *reinterpret_cast<uint4 *>(qb + (cpart >> 3) * (kTcRows * 128) + sw128(r, cpart & 7)) = v;
+        if (real) v = __ldg(src + j);
+        qw[j >> 3][(j & 7) * 4 + 0] = v.x;
+        qw[j >> 3][(j & 7) * 4 + 1] = v.y;
+        qw[j >> 3][(j & 7) * 4 + 2] = v.z;
+        qw[j >> 3][(j & 7) * 4 + 3] = v.w;
       }
-      fence_proxy_async_smem();
+      tc_st_32x32b_x32(tl + kColQ, qw[0]);
+      tc_st_32x32b_x32(tl + kColQ + 32, qw[1]);
+      tc_wait_st();
+      tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(B.q_ready);
+      if (X.lane == 0) mbar_arrive(B.q_ready);
     }
     __syncwarp();
-    if (lane == 0) mbar_arrive(&B.empty[s]);  // this warp is done with the stage
+    if (X.lane == 0) mbar_arrive(&B.empty[s]);  // this warp is done with the stage
 
     const uint32_t b = c & 1;
     if (!wait_or_abort(X, &B.s_full[b], (c >> 1) & 1)) return false;
@@ -611,91 +648,140 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
     const int kp0 = M.page0 * kPage;
     const bool full_vis =
         M.npages == kStagePages && M.invalid == 0 && kp0 + kStageKeys - 1 <= lim_all;
-    uint32_t sr[2][32];
-    float mc = -INFINITY;  // chunk maximum of the raw scores
-    if (warp_rows) {
-      tc_ld_32x32b_x32(tl + col_s(b), sr[0]);
-      tc_ld_32x32b_x32(tl + col_s(b) + 32, sr[1]);
-      tc_wait_ld();
+    // -inf for the keys of the stage this row does not see
+    auto mask32 = [&](uint32_t (&v)[32], int col0) {
       if (!full_vis) {
 #pragma unroll
-        for (int h = 0; h < 2; ++h)
-#pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            const int col = h * 32 + e;
-            const bool vis = (col >> 4) < M.npages && !((M.invalid >> (col >> 4)) & 1u) &&
-                             kp0 + col <= lim;
-            if (!vis) sr[h][e] = 0xff800000u;  // -inf
-          }
+        for (int e = 0; e < 32; ++e) {
+          const int col = col0 + e;
+          const bool vis = (col >> 4) < M.npages && !((M.invalid >> (col >> 4)) & 1u) &&
+                           kp0 + col <= lim;
+          if (!vis) v[e] = 0xff800000u;
+        }
       }
+    };
+    auto max32 = [](const uint32_t (&v)[32], float m) {
 #pragma unroll
-      for (int h = 0; h < 2; ++h)
-#pragma unroll
-        for (int e = 0; e < 32; ++e) mc = fmaxf(mc, __uint_as_float(sr[h][e]));
-    }
-    // lazy rescale: keep the old maximum unless the new one is 2^8 larger
-    const float mcs = mc * sl2;
-    float alpha = 1.f;
-    bool resc = false;
-    if (real && mcs != -INFINITY) {
-      if (m_used == -INFINITY) {
-        m_used = mcs;
-      } else if (mcs > m_used + 8.f) {
-        alpha = ex2_approx(m_used - mcs);
-        m_used = mcs;
-        resc = true;
+      for (int e = 0; e < 32; ++e) m = fmaxf(m, __uint_as_float(v[e]));
+      return m;
+    };
+    // the lazy rescale: keep the old maximum unless the chunk's is 2^8 larger
+    auto rescale = [&](float mc) -> bool {
+      const float mcs = mc * sl2;
+      float alpha = 1.f;
+      bool resc = false;
+      if (real && mcs != -INFINITY) {
+        if (m_used == -INFINITY) {
+          m_used = mcs;
+        } else if (mcs > m_used + 8.f) {
+          alpha = ex2_approx(m_used - mcs);
+          m_used = mcs;
+          resc = true;
+        }
       }
-    }
-    if (warp_rows && __any_sync(0xffffffffu, resc)) {
-      // O holds the P V products of earlier chunks of this item: let them land
+      if (__any_sync(0xffffffffu, resc)) {
+        // O holds the P V products of earlier chunks of this item: let them land
+        if (!wait_pv_done(c - 1)) return false;
+        tc_fence_after();
+#pragma unroll
+        for (int q4 = 0; q4 < kD / 32; ++q4) {
+          uint32_t r[32];
+          tc_ld_32x32b_x32(tl + kColO + q4 * 32, r);
+          tc_wait_ld();
+#pragma unroll
+          for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
+          tc_st_32x32b_x32(tl + kColO + q4 * 32, r);
+        }
+        tc_wait_st();
+      }
+      l_run *= alpha;
+      return true;
+    };
+    // p = 2^(s*scale - m) as a truncated bf16 pair and the truncated residual
+    float lsum = 0.f;
+    auto exp_pairs = [&](const uint32_t (&v)[32], float moff, uint32_t *hi, uint32_t *lo) {
+#pragma unroll
+      for (int e = 0; e < 32; e += 2) {
+        const float p0 = ex2_approx(fmaf(__uint_as_float(v[e]), sl2, moff));
+        const float p1 = ex2_approx(fmaf(__uint_as_float(v[e + 1]), sl2, moff));
+        const float h0 = __uint_as_float(__float_as_uint(p0) & 0xffff0000u);
+        const float h1 = __uint_as_float(__float_as_uint(p1) & 0xffff0000u);
+        hi[e >> 1] = pack_bf16x2_trunc(p0, p1);
+        lo[e >> 1] = pack_bf16x2_trunc(p0 - h0, p1 - h1);
+        lsum += p0 + p1;
+      }
+    };
+
+    if constexpr (kSplit) {
+      uint32_t sr[2][32];
+      tc_ld_32x32b_x32(tl + col_s(b) + 64 * h, sr[0]);
+      tc_ld_32x32b_x32(tl + col_s(b) + 64 * h + 32, sr[1]);
+      tc_wait_ld();
+      mask32(sr[0], 64 * h);
+      mask32(sr[1], 64 * h + 32);
+      float mc = max32(sr[1], max32(sr[0], -INFINITY));
+      // the partner thread (other key half of the same row) holds the rest
+      float *xm = xbuf + (c & 1) * kTcRows;
+      xm[t] = mc;
+      named_bar_sync(1, kCW * 32);
+      mc = fmaxf(mc, xm[t ^ kTcSplitRows]);
+      if (!rescale(mc)) return false;
+      const float moff = (!real || m_used == -INFINITY) ? -INFINITY : -m_used;  // -inf: p = 0
+      uint32_t ph[32], pl[32];
+      exp_pairs(sr[0], moff, ph, pl);
+      exp_pairs(sr[1], moff, ph + 16, pl + 16);
+      // the P buffer is free once the previous chunk's P V product is done
       if (!wait_pv_done(c - 1)) return false;
-      tc_fence_after();
+      uint8_t *pb = X.smem + Smem::off_p + h * Smem::kPBlock;
 #pragma unroll
-      for (int q4 = 0; q4 < kD / 32; ++q4) {
-        uint32_t r[32];
-        tc_ld_32x32b_x32(tl + col_o(0) + q4 * 32, r);
+      for (int j = 0; j < 8; ++j) {
+        *reinterpret_cast<uint4 *>(pb + sw128(row, j)) =
+            make_uint4(ph[4 * j], ph[4 * j + 1], ph[4 * j + 2], ph[4 * j + 3]);
+        *reinterpret_cast<uint4 *>(pb + sw128(row + kTcSplitRows, j)) =
+            make_uint4(pl[4 * j], pl[4 * j + 1], pl[4 * j + 2], pl[4 * j + 3]);
+      }
+    } else {
+      float mc = -INFINITY;
+#pragma unroll
+      for (int q2 = 0; q2 < kStageKeys / 64; ++q2) {
+        uint32_t sr[2][32];
+        tc_ld_32x32b_x32(tl + col_s(b) + 64 * q2, sr[0]);
+        tc_ld_32x32b_x32(tl + col_s(b) + 64 * q2 + 32, sr[1]);
         tc_wait_ld();
+        mask32(sr[0], 64 * q2);
+        mask32(sr[1], 64 * q2 + 32);
+        mc = max32(sr[1], max32(sr[0], mc));
+      }
+      if (!rescale(mc)) return false;
+      const float moff = (!real || m_used == -INFINITY) ? -INFINITY : -m_used;
+      uint32_t ph[64];
 #pragma unroll
-        for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
-        tc_st_32x32b_x32(tl + col_o(0) + q4 * 32, r);
+      for (int q4 = 0; q4 < kStageKeys / 32; ++q4) {
+        uint32_t sr[32], pl[16];
+        tc_ld_32x32b_x32(tl + col_s(b) + 32 * q4, sr);
+        tc_wait_ld();
+        mask32(sr, 32 * q4);
+        exp_pairs(sr, moff, ph + 16 * q4, pl);
+        // the residual overwrites S columns 16 q4 .. that this thread has already read
+        tc_st_32x32b_x16(tl + col_s(b) + 16 * q4, pl);
       }
       tc_wait_st();
-    }
-    l_run *= alpha;
-    // probabilities, as bf16 value + bf16 residual, into P buffer b
-    if (!wait_or_abort(X, &B.p_free[b], ((c >> 1) & 1) ^ 1)) return false;
-    if (warp_rows) {
-      uint8_t *pb = X.smem + Smem::off_p + b * 2 * Smem::kPBytes;
-      const float moff = (!real || m_used == -INFINITY) ? -INFINITY : -m_used;  // -inf: p = 0
-      float lsum = 0.f;
+      if (!wait_pv_done(c - 1)) return false;
 #pragma unroll
-      for (int h = 0; h < 2; ++h)
+      for (int blk = 0; blk < 2; ++blk) {
+        uint8_t *pb = X.smem + Smem::off_p + blk * Smem::kPBlock;
 #pragma unroll
-        for (int cch = 0; cch < 4; ++cch) {
-          uint32_t whi[4], wlo[4];
-#pragma unroll
-          for (int t = 0; t < 4; ++t) {
-            const int e = cch * 8 + 2 * t;
-            const float p0 = ex2_approx(fmaf(__uint_as_float(sr[h][e]), sl2, moff));
-            const float p1 = ex2_approx(fmaf(__uint_as_float(sr[h][e + 1]), sl2, moff));
-            const uint32_t hi = pack_bf16x2(p0, p1);
-            whi[t] = hi;
-            wlo[t] = pack_bf16x2(p0 - bf16lo(hi), p1 - bf16hi(hi));
-            lsum += p0 + p1;
-          }
-          if (real) {
-            *reinterpret_cast<uint4 *>(pb + sw128(row, h * 4 + cch)) =
-                make_uint4(whi[0], whi[1], whi[2], whi[3]);
-            *reinterpret_cast<uint4 *>(pb + Smem::kPBytes + sw128(row, h * 4 + cch)) =
-                make_uint4(wlo[0], wlo[1], wlo[2], wlo[3]);
-          }
+        for (int j = 0; j < 8; ++j) {
+          const uint32_t *w = ph + 32 * blk + 4 * j;
+          *reinterpret_cast<uint4 *>(pb + sw128(row, j)) = make_uint4(w[0], w[1], w[2], w[3]);
         }
-      if (real) l_run += lsum;
+      }
     }
+    if (real) l_run += lsum;
     fence_proxy_async_smem();
     tc_fence_before();
     __syncwarp();
-    if (lane == 0) mbar_arrive(&B.p_full[b]);
+    if (X.lane == 0) mbar_arrive(B.p_full);
     ++it;
     ++c;
     if (M.flags & 2) break;
@@ -704,8 +790,30 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
   // ---- the tile is done once the last P V product has landed in O ----
   if (!wait_pv_done(c - 1)) return false;
   tc_fence_after();
-  const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-  if (warp_rows) {
+  float *ox = reinterpret_cast<float *>(X.smem + Smem::off_p);  // [64][128] fp32, O exchange
+  float *xl = xbuf + 2 * kTcRows;
+  // 16-byte chunk j of exchange row r sits at chunk j ^ (r & 7) (conflict-free)
+  auto ox_at = [&](int r, int j) { return reinterpret_cast<float4 *>(ox + r * kD) + (j ^ (r & 7)); };
+  if constexpr (kSplit) {
+    if (h == 1) {
+#pragma unroll
+      for (int q4 = 0; q4 < kD / 32; ++q4) {
+        uint32_t r[32];
+        tc_ld_32x32b_x32(tl + kColO + q4 * 32, r);
+        tc_wait_ld();
+#pragma unroll
+        for (int c4 = 0; c4 < 8; ++c4)
+          *ox_at(row, q4 * 8 + c4) =
+              make_float4(__uint_as_float(r[4 * c4]), __uint_as_float(r[4 * c4 + 1]),
+                          __uint_as_float(r[4 * c4 + 2]), __uint_as_float(r[4 * c4 + 3]));
+      }
+      xl[row] = l_run;
+    }
+    named_bar_sync(1, kCW * 32);
+  }
+  if (h == 0) {
+    const float l_tot = kSplit ? l_run + xl[row] : l_run;
+    const float inv = l_tot > 0.f ? 1.f / l_tot : 0.f;
     uint16_t *orow = real ? out_row(g, I, I.rb * kTcRows + row) : nullptr;
     float *prow = (real && I.n_split > 1)
                       ? p.partials + ((size_t)I.pbase + (size_t)I.split * I.rows + row) * kPStride
@@ -713,44 +821,54 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
 #pragma unroll
     for (int q4 = 0; q4 < kD / 32; ++q4) {
       uint32_t r[32];
-      tc_ld_32x32b_x32(tl + col_o(0) + q4 * 32, r);
+      tc_ld_32x32b_x32(tl + kColO + q4 * 32, r);
       tc_wait_ld();
+      float o[32];
+#pragma unroll
+      for (int e = 0; e < 32; ++e) o[e] = __uint_as_float(r[e]);
+      if (kSplit) {
+#pragma unroll
+        for (int c4 = 0; c4 < 8; ++c4) {
+          const float4 v = *ox_at(row, q4 * 8 + c4);
+          o[4 * c4] += v.x;
+          o[4 * c4 + 1] += v.y;
+          o[4 * c4 + 2] += v.z;
+          o[4 * c4 + 3] += v.w;
+        }
+      }
       if (real) {
         if (I.n_split == 1) {
 #pragma unroll
           for (int c8 = 0; c8 < 4; ++c8) {
             uint4 v;
-            v.x = pack_bf16x2(__uint_as_float(r[8 * c8 + 0]) * inv, __uint_as_float(r[8 * c8 + 1]) * inv);
-            v.y = pack_bf16x2(__uint_as_float(r[8 * c8 + 2]) * inv, __uint_as_float(r[8 * c8 + 3]) * inv);
-            v.z = pack_bf16x2(__uint_as_float(r[8 * c8 + 4]) * inv, __uint_as_float(r[8 * c8 + 5]) * inv);
-            v.w = pack_bf16x2(__uint_as_float(r[8 * c8 + 6]) * inv, __uint_as_float(r[8 * c8 + 7]) * inv);
+            v.x = pack_bf16x2(o[8 * c8 + 0] * inv, o[8 * c8 + 1] * inv);
+            v.y = pack_bf16x2(o[8 * c8 + 2] * inv, o[8 * c8 + 3] * inv);
+            v.z = pack_bf16x2(o[8 * c8 + 4] * inv, o[8 * c8 + 5] * inv);
+            v.w = pack_bf16x2(o[8 * c8 + 6] * inv, o[8 * c8 + 7] * inv);
             reinterpret_cast<uint4 *>(orow + q4 * 32)[c8] = v;
           }
         } else {
 #pragma unroll
           for (int c4 = 0; c4 < 8; ++c4)
             __stcg(reinterpret_cast<float4 *>(prow + q4 * 32) + c4,
-                   make_float4(__uint_as_float(r[4 * c4]), __uint_as_float(r[4 * c4 + 1]),
-                               __uint_as_float(r[4 * c4 + 2]), __uint_as_float(r[4 * c4 + 3])));
+                   make_float4(o[4 * c4], o[4 * c4 + 1], o[4 * c4 + 2], o[4 * c4 + 3]));
         }
       }
     }
     if (real && I.n_split > 1) {
       __stcg(prow + 128, m_used);
-      __stcg(prow + 129, l_run);
+      __stcg(prow + 129, l_tot);
     }
   }
+  // TMEM O and the exchange area are free again once every thread is here
   tc_fence_before();
-  __syncwarp();
-  if (lane == 0) mbar_arrive(B.o_free);
-  if (I.n_split > 1) ticket_merge(p, X, I, g);
   named_bar_sync(1, kCW * 32);
   return true;
 }
 
 // ============================ CUDA-core path ============================
-// Fewer than kTcMinRows rows; warp w takes page w of every stage, lanes split
-// a page's 16 keys in halves of the head dimension.
+// Fewer than kTcMinRows rows; warp w takes pages w and w + 4 of every stage,
+// lanes split a page's 16 keys in halves of the head dimension.
 template <int NR>
 __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, const Item &I,
                                         uint32_t &it) {
@@ -795,87 +913,90 @@ __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, c
       }
       named_bar_sync(1, kCW * 32);
     }
-    const int pg = warp;  // one page per compute warp
-    if (pg < M.npages) {
-      const int key = lane >> 1, half = lane & 1;
-      const int R = pg * kPage + key;  // key row within the stage
-      const uint8_t *kb = stage_k(X.smem, s) + half * kHalfBytes + R * 128;
-      const uint8_t *vb = stage_v(X.smem, s);
-      const int kpos = (M.page0 + pg) * kPage + key;
-      const bool page_ok = !((M.invalid >> pg) & 1u);
-      uint4 kr[8];
+#pragma unroll 1
+    for (int jp = 0; jp < kStagePages / kCW; ++jp) {
+      const int pg = warp + kCW * jp;  // pages warp, warp + 4 of the stage
+      if (pg < M.npages) {
+        const int key = lane >> 1, half = lane & 1;
+        const int R = pg * kPage + key;  // key row within the stage
+        const uint8_t *kb = stage_k(X.smem, s) + half * kHalfBytes + R * 128;
+        const uint8_t *vb = stage_v(X.smem, s);
+        const int kpos = (M.page0 + pg) * kPage + key;
+        const bool page_ok = !((M.invalid >> pg) & 1u);
+        uint4 kr[8];
 #pragma unroll
-      for (int cc = 0; cc < 8; ++cc) {
-        const int lc = (cc + 4 * half) & 7;  // logical chunk, rotated per half
-        kr[cc] = *reinterpret_cast<const uint4 *>(kb + ((lc ^ (R & 7)) << 4));
-      }
-#pragma unroll
-      for (int r = 0; r < NR; ++r) {
-        if (r < nrow) {
-          const float *qrow = qs + r * kD + half * 64;
-          float pa[4] = {0.f, 0.f, 0.f, 0.f};  // four independent partial sums
-#pragma unroll
-          for (int cc = 0; cc < 8; ++cc) {
-            const int lc = (cc + 4 * half) & 7;
-            const float4 a = *reinterpret_cast<const float4 *>(qrow + lc * 4);
-            const float4 b2 = *reinterpret_cast<const float4 *>(qrow + 32 + lc * 4);
-            float &acc = pa[cc & 3];
-            acc = fmaf(bf16lo(kr[cc].x), a.x, acc);
-            acc = fmaf(bf16hi(kr[cc].x), a.y, acc);
-            acc = fmaf(bf16lo(kr[cc].y), a.z, acc);
-            acc = fmaf(bf16hi(kr[cc].y), a.w, acc);
-            acc = fmaf(bf16lo(kr[cc].z), b2.x, acc);
-            acc = fmaf(bf16hi(kr[cc].z), b2.y, acc);
-            acc = fmaf(bf16lo(kr[cc].w), b2.z, acc);
-            acc = fmaf(bf16hi(kr[cc].w), b2.w, acc);
-          }
-          float acc = (pa[0] + pa[1]) + (pa[2] + pa[3]);
-          acc += __shfl_xor_sync(0xffffffffu, acc, 1);
-          const int qi = (I.rb * kCcRows + r) / g.G;
-          const bool vis = page_ok && kpos < g.L && kpos <= g.L - g.ql + qi;
-          const float sc = vis ? acc * p.scale_log2 : -INFINITY;
-          float mx = sc;
-          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
-          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
-          mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
-          const float mnew = fmaxf(cm[r], mx);
-          float alpha = 1.f, pr = 0.f;
-          if (mnew != -INFINITY) {
-            alpha = exp2f(cm[r] - mnew);
-            pr = exp2f(sc - mnew);
-          }
-          cl[r] = cl[r] * alpha + (half == 0 ? pr : 0.f);
-          co[r][0] *= alpha;
-          co[r][1] *= alpha;
-          co[r][2] *= alpha;
-          co[r][3] *= alpha;
-          cm[r] = mnew;
-          if (half == 0) ps[(warp * 8 + r) * 16 + key] = pr;
+        for (int cc = 0; cc < 8; ++cc) {
+          const int lc = (cc + 4 * half) & 7;  // logical chunk, rotated per half
+          kr[cc] = *reinterpret_cast<const uint4 *>(kb + ((lc ^ (R & 7)) << 4));
         }
-      }
-      __syncwarp();
-      // P V: lane owns dims 4*lane .. 4*lane+3
-      const int vhalf = lane >> 4, vc = (lane & 15) >> 1, vsub = (lane & 1) * 8;
-#pragma unroll
-      for (int jk = 0; jk < kPage; ++jk) {
-        const int Rv = pg * kPage + jk;
-        const uint2 vv = *reinterpret_cast<const uint2 *>(vb + vhalf * kHalfBytes + Rv * 128 +
-                                                          ((vc ^ (Rv & 7)) << 4) + vsub);
-        const float v0 = bf16lo(vv.x), v1 = bf16hi(vv.x), v2 = bf16lo(vv.y), v3 = bf16hi(vv.y);
 #pragma unroll
         for (int r = 0; r < NR; ++r) {
           if (r < nrow) {
-            const float pj = ps[(warp * 8 + r) * 16 + jk];
-            co[r][0] = fmaf(pj, v0, co[r][0]);
-            co[r][1] = fmaf(pj, v1, co[r][1]);
-            co[r][2] = fmaf(pj, v2, co[r][2]);
-            co[r][3] = fmaf(pj, v3, co[r][3]);
+            const float *qrow = qs + r * kD + half * 64;
+            float pa[4] = {0.f, 0.f, 0.f, 0.f};  // four independent partial sums
+#pragma unroll
+            for (int cc = 0; cc < 8; ++cc) {
+              const int lc = (cc + 4 * half) & 7;
+              const float4 a = *reinterpret_cast<const float4 *>(qrow + lc * 4);
+              const float4 b2 = *reinterpret_cast<const float4 *>(qrow + 32 + lc * 4);
+              float &acc = pa[cc & 3];
+              acc = fmaf(bf16lo(kr[cc].x), a.x, acc);
+              acc = fmaf(bf16hi(kr[cc].x), a.y, acc);
+              acc = fmaf(bf16lo(kr[cc].y), a.z, acc);
+              acc = fmaf(bf16hi(kr[cc].y), a.w, acc);
+              acc = fmaf(bf16lo(kr[cc].z), b2.x, acc);
+              acc = fmaf(bf16hi(kr[cc].z), b2.y, acc);
+              acc = fmaf(bf16lo(kr[cc].w), b2.z, acc);
+              acc = fmaf(bf16hi(kr[cc].w), b2.w, acc);
+            }
+            float acc = (pa[0] + pa[1]) + (pa[2] + pa[3]);
+            acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+            const int qi = (I.rb * kCcRows + r) / g.G;
+            const bool vis = page_ok && kpos < g.L && kpos <= g.L - g.ql + qi;
+            const float sc = vis ? acc * p.scale_log2 : -INFINITY;
+            float mx = sc;
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+            const float mnew = fmaxf(cm[r], mx);
+            float alpha = 1.f, pr = 0.f;
+            if (mnew != -INFINITY) {
+              alpha = exp2f(cm[r] - mnew);
+              pr = exp2f(sc - mnew);
+            }
+            cl[r] = cl[r] * alpha + (half == 0 ? pr : 0.f);
+            co[r][0] *= alpha;
+            co[r][1] *= alpha;
+            co[r][2] *= alpha;
+            co[r][3] *= alpha;
+            cm[r] = mnew;
+            if (half == 0) ps[(warp * 8 + r) * 16 + key] = pr;
+          }
+        }
+        __syncwarp();
+        // P V: lane owns dims 4*lane .. 4*lane+3
+        const int vhalf = lane >> 4, vc = (lane & 15) >> 1, vsub = (lane & 1) * 8;
+#pragma unroll
+        for (int jk = 0; jk < kPage; ++jk) {
+          const int Rv = pg * kPage + jk;
+          const uint2 vv = *reinterpret_cast<const uint2 *>(vb + vhalf * kHalfBytes + Rv * 128 +
+                                                            ((vc ^ (Rv & 7)) << 4) + vsub);
+          const float v0 = bf16lo(vv.x), v1 = bf16hi(vv.x), v2 = bf16lo(vv.y), v3 = bf16hi(vv.y);
+#pragma unroll
+          for (int r = 0; r < NR; ++r) {
+            if (r < nrow) {
+              const float pj = ps[(warp * 8 + r) * 16 + jk];
+              co[r][0] = fmaf(pj, v0, co[r][0]);
+              co[r][1] = fmaf(pj, v1, co[r][1]);
+              co[r][2] = fmaf(pj, v2, co[r][2]);
+              co[r][3] = fmaf(pj, v3, co[r][3]);
+            }
           }
         }
       }
+      __syncwarp();  // ps is rewritten by the next page
     }
-    __syncwarp();
     if (lane == 0) mbar_arrive(&B.empty[s]);
     ++it;
     if (M.flags & 2) break;
@@ -934,7 +1055,6 @@ __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, c
       }
     }
   }
-  if (I.n_split > 1) ticket_merge(p, X, I, g);
   named_bar_sync(1, kCW * 32);
   return true;
 }
@@ -943,7 +1063,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
   extern __shared__ __align__(1024) uint8_t smem[];
   const Bars B = bars(smem);
   StageMeta *meta = reinterpret_cast<StageMeta *>(smem + Smem::off_meta);
-  // misc[0] TMEM base, [1] abort flag, [2] ticket broadcast
+  // misc[0] TMEM base, [1] abort flag
   uint32_t *misc = reinterpret_cast<uint32_t *>(smem + Smem::off_misc);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -958,12 +1078,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
       mbar_init(&B.empty[s], 1 + kCW);  // the MMA warp and every compute warp
     }
     mbar_init(B.q_ready, kCW);
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&B.s_full[i], 1);
-      mbar_init(&B.p_full[i], kCW);
-      mbar_init(&B.p_free[i], 1);
-    }
-    mbar_init(B.o_free, kCW);
+    for (int i = 0; i < 2; ++i) mbar_init(&B.s_full[i], 1);
+    mbar_init(B.p_full, kCW);
+    mbar_init(B.p_free, 1);
     misc[1] = 0;
     fence_mbar_init();
   }
@@ -1094,102 +1211,86 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
 
   if (warp == kMmaWarp) {
     // ------------------------------ MMA issuer -----------------------------
-    // Event loop: P V of the oldest pending chunk is issued as soon as its P
-    // is written, and Q K^T of the next chunk as soon as its stage has landed
-    // and an S buffer is free, so neither waits for the other's inputs.
+    // Fixed order per tensor chunk j: Q K^T of j into S buffer j & 1, then
+    // P V of chunk j-1 (once its P is written); an item's last chunk also
+    // issues its own P V, so no product waits on the next item's stages.
     constexpr uint32_t idesc_s = idesc_bf16_f32(kTcRows, kStageKeys, 0);
     constexpr uint32_t idesc_o = idesc_bf16_f32(kTcRows, kD, 1);
-    const uint32_t sq = smem_u32(smem + Smem::off_q);
-    uint32_t it = 0, c = 0, nq = 0, cur_item = 0;
-    uint32_t pc[2], ps_[2], pitem[2];  // chunks with S issued and P V pending, oldest first
-    bool pfirst[2];
-    int qn = 0;
-    bool done = false, ok = true;
-    long long t_last = clock64();
-    while (!done || qn > 0) {
-      bool progress = false;
-      if (qn > 0) {
-        const uint32_t cc = pc[0], bb = cc & 1;
-        if (warp_test(&B.p_full[bb], (cc >> 1) & 1) &&
-            (!pfirst[0] || warp_test(B.o_free, (pitem[0] & 1) ^ 1))) {
-          tc_fence_after();
-          if (lane == 0) {
-            // O (+)= P V with P = P_hi + P_lo; the first chunk of an item overwrites O
-            const uint32_t pa = smem_u32(smem + Smem::off_p + bb * 2 * Smem::kPBytes);
-            const uint32_t va = smem_u32(stage_v(smem, ps_[0]));
+    const uint32_t pa = smem_u32(smem + Smem::off_p);
+    uint32_t it = 0, c = 0, nq = 0;
+    bool ok = true, pend = false;
+    uint32_t pc = 0;  // pending chunk
+    int pstage = 0, pfirst = 0, ppath = 0;
+    auto mwait = [&](uint64_t *bar, uint32_t par) -> bool {
+      if (mbar_wait_bounded(bar, par)) return true;
+      ok = false;
+      return false;
+    };
+    // O (+)= P V of the pending chunk; the first chunk of an item overwrites O
+    auto issue_pv = [&]() -> bool {
+      if (!mwait(B.p_full, pc & 1)) return false;
+      tc_fence_after();
+      if (lane == 0) {
+        const uint32_t va = smem_u32(stage_v(smem, pstage));
 #pragma unroll
-            for (int kk = 0; kk < kStageKeys / 16; ++kk) {
-              const uint64_t bd = sdesc_sw128(va + kk * 16 * 128, kHalfBytes, 1024);
-              tc_mma_bf16(tmem + col_o(0), sdesc_sw128(pa + kk * 32, 16, 1024), bd, idesc_o,
-                          (pfirst[0] && kk == 0) ? 0u : 1u);
-              tc_mma_bf16(tmem + col_o(0), sdesc_sw128(pa + Smem::kPBytes + kk * 32, 16, 1024),
-                          bd, idesc_o, 1u);
-            }
-            tc_commit(&B.p_free[bb]);
-            tc_commit(&B.empty[ps_[0]]);
-          }
-          __syncwarp();
-          pc[0] = pc[1]; ps_[0] = ps_[1]; pitem[0] = pitem[1]; pfirst[0] = pfirst[1];
-          --qn;
-          progress = true;
+        for (int kk = 0; kk < kStageKeys / 16; ++kk) {
+          // V rows 16kk.. as an MN-major operand: the two 64-dim halves kHalfBytes apart
+          const uint64_t bd = sdesc_sw128(va + kk * 16 * 128, kHalfBytes, 1024);
+          const uint64_t ad = sdesc_sw128(pa + (kk >> 2) * Smem::kPBlock + (kk & 3) * 32, 16, 1024);
+          tc_mma_bf16(tmem + kColO, ad, bd, idesc_o, (pfirst && kk == 0) ? 0u : 1u);
+          if (ppath == kPathTcFull)  // residual of P, from the chunk's S buffer
+            tc_mma_bf16_ta(tmem + kColO, tmem + col_s(pc & 1) + 8 * kk, bd, idesc_o, 1u);
         }
+        tc_commit(B.p_free);
+        tc_commit(&B.empty[pstage]);
       }
-      if (!progress && !done && qn < 2) {
-        const int s = it % kStages;
-        if (warp_test(&B.full[s], (it / kStages) & 1)) {
-          int item = 0, flags = 0, path = 0;
-          if (lane == 0) {
-            item = meta[s].item;
-            flags = meta[s].flags;
-            path = meta[s].path;
-          }
-          item = __shfl_sync(0xffffffffu, item, 0);
-          flags = __shfl_sync(0xffffffffu, flags, 0);
-          path = __shfl_sync(0xffffffffu, path, 0);
-          if (item < 0) {
-            done = true;
-            progress = true;
-          } else if (!path) {
-            if (lane == 0) mbar_arrive(&B.empty[s]);
-            __syncwarp();
-            ++it;
-            progress = true;
-          } else {
-            const bool firstc = flags & 1;
-            if (!firstc || warp_test(B.q_ready, nq & 1)) {
-              if (firstc) cur_item = nq++;
-              tc_fence_after();
-              const uint32_t b = c & 1;
-              if (lane == 0) {
-                const uint32_t ka = smem_u32(stage_k(smem, s));
+      __syncwarp();
+      pend = false;
+      return true;
+    };
+    for (;;) {
+      const int s = it % kStages;
+      if (!mwait(&B.full[s], (it / kStages) & 1)) break;
+      int item = 0, flags = 0, path = 0;
+      if (lane == 0) {
+        item = meta[s].item;
+        flags = meta[s].flags;
+        path = meta[s].path;
+      }
+      item = __shfl_sync(0xffffffffu, item, 0);
+      flags = __shfl_sync(0xffffffffu, flags, 0);
+      path = __shfl_sync(0xffffffffu, path, 0);
+      if (item < 0 || *(volatile uint32_t *)&misc[1]) break;
+      if (path == kPathCc) {
+        if (lane == 0) mbar_arrive(&B.empty[s]);
+        __syncwarp();
+        ++it;
+        continue;
+      }
+      if (flags & 1) {  // a new tensor item: its Q tile must be in TMEM
+        if (!mwait(B.q_ready, nq & 1)) break;
+        ++nq;
+      }
+      tc_fence_after();
+      if (lane == 0) {
+        const uint32_t ka = smem_u32(stage_k(smem, s));
 #pragma unroll
-                for (int kk = 0; kk < kD / 16; ++kk) {
-                  const uint32_t qoff = (kk >> 2) * (kTcRows * 128) + (kk & 3) * 32;
-                  const uint32_t koff = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
-                  tc_mma_bf16(tmem + col_s(b), sdesc_sw128(sq + qoff, 16, 1024),
-                              sdesc_sw128(ka + koff, 16, 1024), idesc_s, kk > 0);
-                }
-                tc_commit(&B.s_full[b]);
-              }
-              __syncwarp();
-              pc[qn] = c; ps_[qn] = s; pitem[qn] = cur_item; pfirst[qn] = firstc;
-              ++qn;
-              ++c;
-              ++it;
-              progress = true;
-            }
-          }
+        for (int kk = 0; kk < kD / 16; ++kk) {
+          const uint64_t bd = sdesc_sw128(ka + (kk >> 2) * kHalfBytes + (kk & 3) * 32, 16, 1024);
+          tc_mma_bf16_ta(tmem + col_s(c & 1), tmem + kColQ + 8 * kk, bd, idesc_s, kk > 0);
         }
+        tc_commit(&B.s_full[c & 1]);
       }
-      if (progress) {
-        t_last = clock64();
-      } else {
-        if (*(volatile uint32_t *)&misc[1] || clock64() - t_last > kWaitLimitCycles) {
-          ok = false;
-          break;
-        }
-        __nanosleep(32);
-      }
+      __syncwarp();
+      if (pend && !issue_pv()) break;
+      pend = true;
+      pc = c;
+      pstage = s;
+      pfirst = flags & 1;
+      ppath = path;
+      ++c;
+      ++it;
+      if ((flags & 2) && !issue_pv()) break;
     }
     if (!ok) {
       ipd_set_error(&g_attn_err, IPD_DEVERR_WAIT);
@@ -1212,8 +1313,10 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
     if (M.item < 0 || *(volatile uint32_t *)&misc[1]) break;
     const Item I = p.items[M.item];
     bool ok;
-    if (I.path) {
-      ok = tc_item(p, X, I, it, c);
+    if (I.path == kPathTcSplit) {
+      ok = tc_item<true>(p, X, I, it, c);
+    } else if (I.path == kPathTcFull) {
+      ok = tc_item<false>(p, X, I, it, c);
     } else {
       // GQA-2 decode (two rows) gets straight-line code; other sizes take
       // the guarded loop (more instances overflow the register budget)
@@ -1326,17 +1429,19 @@ int launch(const ipd_attn_batch *const *bs, int n, float scale, void *ws, size_t
   P.ctrl = reinterpret_cast<int *>(w + W.off_ctrl);
   P.reqinfo = reinterpret_cast<int4 *>(w + W.off_reqinfo);
   P.items = reinterpret_cast<Item *>(w + W.off_items);
-  P.tickets = reinterpret_cast<int *>(w + W.off_tickets);
   P.partials = reinterpret_cast<float *>(w + W.off_partials);
   P.item_cap = W.item_cap;
   P.task_cap = W.task_cap;
   P.prow_cap = W.prow_cap;
   P.target_items = std::min(kMaxTargetItems, kTargetItemsPerSm * D.sms);
+  P.n_sms = D.sms;
 
   attn_plan_kernel<<<1, 1024, 0, stream>>>(P);
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   const int grid = std::max(1, std::min(D.sms, W.item_cap));
   attn_kernel<<<grid, kThreads, Smem::total, stream>>>(P);
+  if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
+  attn_merge_kernel<<<8 * D.sms, 256, 0, stream>>>(P);
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   return IPD_OK;
 }

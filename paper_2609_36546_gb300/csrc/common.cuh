@@ -190,6 +190,19 @@ IPD_DEVINL void tc_mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uin
       : "memory");
 }
 
+// D[tmem] (+)= A[tmem] * B[smem]: A is read from TMEM (lane = row of A, each
+// 32-bit column holds two consecutive K elements, the lower one in the low
+// half), B from shared memory as above.
+IPD_DEVINL void tc_mma_bf16_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                               uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
 // Arrive once on an mbarrier when every tcgen05 op issued so far by this
 // thread has completed.
 IPD_DEVINL void tc_commit(uint64_t *bar) {
@@ -253,6 +266,23 @@ IPD_DEVINL void tc_st_32x32b_x32(uint32_t taddr, const uint32_t (&r)[32]) {
       "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
       "r"(r[29]), "r"(r[30]), "r"(r[31])
       : "memory");
+}
+
+// Each lane of the warp writes 16 consecutive 32-bit TMEM columns of its lane.
+IPD_DEVINL void tc_st_32x32b_x16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15,%16};" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+      "r"(r[15])
+      : "memory");
+}
+
+// Two floats truncated to their upper 16 bits (bf16 rounded toward zero) and
+// packed, the first in the low half.  Integer byte permute only.
+IPD_DEVINL uint32_t pack_bf16x2_trunc(float lo, float hi) {
+  return __byte_perm(__float_as_uint(lo), __float_as_uint(hi), 0x7632);
 }
 
 // 2^x on the special-function unit (hardware approximation, about 2 ulp).
