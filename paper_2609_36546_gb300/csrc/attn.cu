@@ -12,8 +12,8 @@
 //   item  = (task, KV chunk); tasks longer than about a quarter of an SM's
 //           share are split, items are claimed longest first, and a small
 //           follow-up kernel merges the partials of split tasks.
-// KV pages stream through a 3-stage ring of 128-key stages (64 KB: K and V,
-// each as two 64-dim halves of 128 swizzled rows), written by 2-D TMA.
+// KV pages stream through a 3-stage ring of 128-key stages (64 KB), one
+// 4 KB 4-D TMA box per page and tensor.
 // Two compute paths, chosen per task by its row count:
 //   tensor path (rows >= kTcMinRows): a 128-lane tile.  S = Q K^T (Q read
 //     from TMEM, K from shared memory, N = 128 keys) and O += P V run on
@@ -49,8 +49,17 @@ constexpr int kD = 128;
 constexpr int kStagePages = 8;                    // 128 keys per stage
 constexpr int kStageKeys = kStagePages * kPage;
 constexpr int kStages = 3;
-constexpr int kHalfBytes = kStageKeys * 128;      // one 64-dim half of 128 key rows: 16 KB
-constexpr int kStageBytes = 4 * kHalfBytes;       // K and V, two halves each: 64 KB
+// A stage holds the K pages then the V pages.  One page (16 keys x 128 dims
+// of one kv head) is one 4 KB TMA box laid out as two 8-key groups of 2 KB,
+// each group as its 64-dim halves, each half one 128-byte-swizzled 1 KB atom
+// (8 rows x 128 B).  Key row R, half h of a tensor sits at
+// (R / 8) * 2048 + h * 1024 + (R % 8) * 128: a K-major operand with 8-row
+// groups 2048 B apart, or an MN-major one with halves 1024 B apart.
+constexpr int kPageBytes = kPage * kD * 2;        // 4 KB
+constexpr int kGroupBytes = 2048;                 // 8 keys, both halves
+constexpr int kAtomBytes = 1024;                  // 8 keys, one 64-dim half
+constexpr int kTensorBytes = kStagePages * kPageBytes;  // 32 KB of K (or V) per stage
+constexpr int kStageBytes = 2 * kTensorBytes;     // 64 KB
 constexpr int kTcRows = 128;                      // TMEM lanes of a tensor-core tile (M)
 constexpr int kTcSplitRows = 64;                  // tiles up to this size split rows over two threads
 constexpr int kTcMinRows = 8;                     // tasks with at least this many rows use it
@@ -470,7 +479,7 @@ struct Smem {
   // CUDA-core path scratch (inside the P region, unused by that path)
   static constexpr int off_ccq = off_p;                              // fp32 [7][128]
   static constexpr int off_merge = off_ccq + kCcRows * kD * 4;       // fp32 [4][8][132]
-  static constexpr int off_ps = off_merge + kCW * 8 * kPStride * 4;  // fp32 [4][8][16]
+  static constexpr int off_ps = off_merge + kCW * 8 * kPStride * 4;  // fp32 [4][8][16] / [4][32][2]
 };
 static_assert(Smem::off_ps + kCW * 8 * 16 * 4 <= Smem::off_x, "CUDA-core scratch overflow");
 static_assert(kTcSplitRows * kD * 4 <= 2 * Smem::kPBlock, "O exchange overflow");
@@ -507,7 +516,12 @@ __device__ __forceinline__ uint8_t *stage_k(uint8_t *smem, int s) {
   return smem + Smem::off_stage + s * kStageBytes;
 }
 __device__ __forceinline__ uint8_t *stage_v(uint8_t *smem, int s) {
-  return stage_k(smem, s) + 2 * kHalfBytes;
+  return stage_k(smem, s) + kTensorBytes;
+}
+// row R (key of the stage), 64-dim half h of a staged K or V tensor; its
+// 16-byte chunk c sits at ((c ^ (R & 7)) << 4)
+__device__ __forceinline__ const uint8_t *kv_row(const uint8_t *t, int R, int h) {
+  return t + (R >> 3) * kGroupBytes + h * kAtomBytes + (R & 7) * 128;
 }
 
 // fp32 Q layout of the CUDA-core path: dim d = half*64 + c*8 + sub*4 + e is
@@ -570,7 +584,7 @@ __device__ __forceinline__ void zero_tail(const CompCtx &X, int s, int page0, in
   uint8_t *vb = stage_v(X.smem, s);
   for (int e = X.ctid; e < (kStageKeys - tail0) * 16; e += kCW * 32) {
     const int row = tail0 + e / 16, cpart = e % 16;
-    *reinterpret_cast<uint4 *>(vb + (cpart >> 3) * kHalfBytes + row * 128 + (cpart & 7) * 16) =
+    *reinterpret_cast<uint4 *>(const_cast<uint8_t *>(kv_row(vb, row, cpart >> 3)) + (cpart & 7) * 16) =
         make_uint4(0, 0, 0, 0);
   }
   fence_proxy_async_smem();
@@ -919,7 +933,7 @@ __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, c
       if (pg < M.npages) {
         const int key = lane >> 1, half = lane & 1;
         const int R = pg * kPage + key;  // key row within the stage
-        const uint8_t *kb = stage_k(X.smem, s) + half * kHalfBytes + R * 128;
+        const uint8_t *kb = kv_row(stage_k(X.smem, s), R, half);
         const uint8_t *vb = stage_v(X.smem, s);
         const int kpos = (M.page0 + pg) * kPage + key;
         const bool page_ok = !((M.invalid >> pg) & 1u);
@@ -980,7 +994,7 @@ __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, c
 #pragma unroll
         for (int jk = 0; jk < kPage; ++jk) {
           const int Rv = pg * kPage + jk;
-          const uint2 vv = *reinterpret_cast<const uint2 *>(vb + vhalf * kHalfBytes + Rv * 128 +
+          const uint2 vv = *reinterpret_cast<const uint2 *>(kv_row(vb, Rv, vhalf) +
                                                             ((vc ^ (Rv & 7)) << 4) + vsub);
           const float v0 = bf16lo(vv.x), v1 = bf16hi(vv.x), v2 = bf16lo(vv.y), v3 = bf16hi(vv.y);
 #pragma unroll
@@ -1059,6 +1073,199 @@ __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, c
   return true;
 }
 
+// Two-row tasks (GQA group 2 decode), the bulk of the CUDA-core work.  Warp
+// w takes pages w and w + 4 of every stage (32 keys); lane = (k, q) with
+// k = lane / 4 and q = lane % 4.
+//   Q K^T: the lane holds dims 32q .. 32q + 31 of both query rows in fp32
+//     registers and takes them against keys g * 8 + k, g = 0..3 (all K loads
+//     in flight together); a butterfly over the four quarter lanes leaves lane
+//     (k, q) with both rows' scores of key q * 8 + k (six shuffles).
+//   P V: lane owns output dims 4 lane .. 4 lane + 3 of both rows; the
+//     probabilities come back from shared memory as broadcasts.
+// The warps' partial (m, l, O) are merged at the end of the item.
+__device__ __forceinline__ bool cc2_item(const AttnParams &p, const CompCtx &X, const Item &I,
+                                         uint32_t &it) {
+  constexpr int NR = 2;
+  const ItemGeom g = item_geom(p, I);
+  const Bars &B = X.B;
+  const int warp = X.warp, lane = X.lane;
+  const int kq = lane >> 2, qq = lane & 3;
+  float *mg = reinterpret_cast<float *>(X.smem + Smem::off_merge);
+  float *pw = reinterpret_cast<float *>(X.smem + Smem::off_ps) + warp * 32 * NR;  // [32 keys][2]
+  float qv[NR][32];
+  int lim[NR];
+#pragma unroll
+  for (int r = 0; r < NR; ++r) {
+    const int grow = I.rb * kCcRows + r;
+    lim[r] = g.L - g.ql + grow / g.G;
+    const uint4 *src = reinterpret_cast<const uint4 *>(q_row(g, I, grow) + qq * 32);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint4 v = __ldg(src + j);
+      qv[r][8 * j + 0] = bf16lo(v.x);
+      qv[r][8 * j + 1] = bf16hi(v.x);
+      qv[r][8 * j + 2] = bf16lo(v.y);
+      qv[r][8 * j + 3] = bf16hi(v.y);
+      qv[r][8 * j + 4] = bf16lo(v.z);
+      qv[r][8 * j + 5] = bf16hi(v.z);
+      qv[r][8 * j + 6] = bf16lo(v.w);
+      qv[r][8 * j + 7] = bf16hi(v.w);
+    }
+  }
+  float cm[NR], cl[NR], co[NR][4];
+#pragma unroll
+  for (int r = 0; r < NR; ++r) {
+    cm[r] = -INFINITY;
+    cl[r] = 0.f;
+    co[r][0] = co[r][1] = co[r][2] = co[r][3] = 0.f;
+  }
+  const int vhalf = lane >> 4, vc = (lane & 15) >> 1, vsub = (lane & 1) * 8;
+
+  for (;;) {
+    const int s = it % kStages;
+    if (!wait_or_abort(X, &B.full[s], (it / kStages) & 1)) return false;
+    const StageMeta M = X.meta[s];
+    zero_tail(X, s, M.page0, g.L);
+    const uint8_t *kst = stage_k(X.smem, s);
+    const uint8_t *vb = stage_v(X.smem, s);
+    // ---- partial dot products of this lane's quarter for keys g * 8 + k ----
+    float part[4][NR];
+#pragma unroll
+    for (int gg = 0; gg < 4; ++gg) {
+      const int R = (warp + kCW * (gg >> 1)) * kPage + (gg & 1) * 8 + kq;
+      const uint8_t *kb = kv_row(kst, R, qq >> 1);
+      uint4 kr[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        kr[j] = *reinterpret_cast<const uint4 *>(kb + (((4 * (qq & 1) + j) ^ (R & 7)) << 4));
+#pragma unroll
+      for (int r = 0; r < NR; ++r) {
+        float a0 = 0.f, a1 = 0.f;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          a0 = fmaf(bf16lo(kr[j].x), qv[r][8 * j + 0], a0);
+          a1 = fmaf(bf16hi(kr[j].x), qv[r][8 * j + 1], a1);
+          a0 = fmaf(bf16lo(kr[j].y), qv[r][8 * j + 2], a0);
+          a1 = fmaf(bf16hi(kr[j].y), qv[r][8 * j + 3], a1);
+          a0 = fmaf(bf16lo(kr[j].z), qv[r][8 * j + 4], a0);
+          a1 = fmaf(bf16hi(kr[j].z), qv[r][8 * j + 5], a1);
+          a0 = fmaf(bf16lo(kr[j].w), qv[r][8 * j + 6], a0);
+          a1 = fmaf(bf16hi(kr[j].w), qv[r][8 * j + 7], a1);
+        }
+        part[gg][r] = a0 + a1;
+      }
+    }
+    // ---- butterfly over the quarters: lane keeps group qq ----
+    const bool odd = qq & 1, up = qq >> 1;
+    float half_sum[2][NR];
+#pragma unroll
+    for (int i = 0; i < 2; ++i)
+#pragma unroll
+      for (int r = 0; r < NR; ++r) {
+        const float send = odd ? part[2 * i][r] : part[2 * i + 1][r];
+        const float keep = odd ? part[2 * i + 1][r] : part[2 * i][r];
+        half_sum[i][r] = keep + __shfl_xor_sync(0xffffffffu, send, 1);
+      }
+    float sc[NR];
+    const int pg = warp + kCW * up;
+    const int kpos = (M.page0 + pg) * kPage + (int)odd * 8 + kq;
+    const bool page_ok = pg < M.npages && !((M.invalid >> pg) & 1u);
+#pragma unroll
+    for (int r = 0; r < NR; ++r) {
+      const float send = up ? half_sum[0][r] : half_sum[1][r];
+      const float keep = up ? half_sum[1][r] : half_sum[0][r];
+      const float tot = keep + __shfl_xor_sync(0xffffffffu, send, 2);
+      sc[r] = (page_ok && kpos <= lim[r]) ? tot * p.scale_log2 : -INFINITY;
+    }
+    // ---- online softmax over the warp's 32 keys ----
+    float pr[NR];
+#pragma unroll
+    for (int r = 0; r < NR; ++r) {
+      const float mnew = fmaxf(cm[r], warp_max(sc[r]));
+      const float alpha = mnew == -INFINITY ? 1.f : ex2_approx(cm[r] - mnew);
+      pr[r] = mnew == -INFINITY ? 0.f : ex2_approx(sc[r] - mnew);
+      cl[r] = fmaf(cl[r], alpha, pr[r]);
+      co[r][0] *= alpha;
+      co[r][1] *= alpha;
+      co[r][2] *= alpha;
+      co[r][3] *= alpha;
+      cm[r] = mnew;
+    }
+    *reinterpret_cast<float2 *>(pw + (qq * 8 + kq) * NR) = make_float2(pr[0], pr[1]);
+    __syncwarp();
+    // ---- P V: 32 keys into this lane's 4 dims of both rows ----
+#pragma unroll 8
+    for (int key = 0; key < 32; ++key) {
+      const int R = (warp + kCW * (key >> 4)) * kPage + (key & 15);
+      const uint2 vv = *reinterpret_cast<const uint2 *>(kv_row(vb, R, vhalf) +
+                                                        ((vc ^ (R & 7)) << 4) + vsub);
+      const float2 pk = *reinterpret_cast<const float2 *>(pw + key * NR);
+      const float v0 = bf16lo(vv.x), v1 = bf16hi(vv.x), v2 = bf16lo(vv.y), v3 = bf16hi(vv.y);
+      co[0][0] = fmaf(pk.x, v0, co[0][0]);
+      co[0][1] = fmaf(pk.x, v1, co[0][1]);
+      co[0][2] = fmaf(pk.x, v2, co[0][2]);
+      co[0][3] = fmaf(pk.x, v3, co[0][3]);
+      co[1][0] = fmaf(pk.y, v0, co[1][0]);
+      co[1][1] = fmaf(pk.y, v1, co[1][1]);
+      co[1][2] = fmaf(pk.y, v2, co[1][2]);
+      co[1][3] = fmaf(pk.y, v3, co[1][3]);
+    }
+    __syncwarp();  // pw is rewritten at the next stage
+    if (lane == 0) mbar_arrive(&B.empty[s]);
+    ++it;
+    if (M.flags & 2) break;
+  }
+
+  // ---- finalize: merge the four warps' partial results ----
+#pragma unroll
+  for (int r = 0; r < NR; ++r) cl[r] = warp_sum(cl[r]);
+#pragma unroll
+  for (int r = 0; r < NR; ++r) {
+    float *dst = mg + (warp * 8 + r) * kPStride;
+    *reinterpret_cast<float4 *>(dst + lane * 4) = make_float4(co[r][0], co[r][1], co[r][2], co[r][3]);
+    if (lane == 0) {
+      dst[128] = cm[r];
+      dst[129] = cl[r];
+    }
+  }
+  named_bar_sync(1, kCW * 32);
+  if (warp < NR) {  // warp r merges row r
+    const int r = warp;
+    float Mx = -INFINITY;
+#pragma unroll
+    for (int w2 = 0; w2 < kCW; ++w2) Mx = fmaxf(Mx, mg[(w2 * 8 + r) * kPStride + 128]);
+    float Ls = 0.f, O0 = 0.f, O1 = 0.f, O2 = 0.f, O3 = 0.f;
+#pragma unroll
+    for (int w2 = 0; w2 < kCW; ++w2) {
+      const float *src = mg + (w2 * 8 + r) * kPStride;
+      const float sc = (src[128] == -INFINITY) ? 0.f : ex2_approx(src[128] - Mx);
+      const float4 ov = *reinterpret_cast<const float4 *>(src + lane * 4);
+      Ls = fmaf(src[129], sc, Ls);
+      O0 = fmaf(ov.x, sc, O0);
+      O1 = fmaf(ov.y, sc, O1);
+      O2 = fmaf(ov.z, sc, O2);
+      O3 = fmaf(ov.w, sc, O3);
+    }
+    const int grow = I.rb * kCcRows + r;
+    if (I.n_split == 1) {
+      const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+      uint2 pk;
+      pk.x = pack_bf16x2(O0 * inv, O1 * inv);
+      pk.y = pack_bf16x2(O2 * inv, O3 * inv);
+      *reinterpret_cast<uint2 *>(out_row(g, I, grow) + lane * 4) = pk;
+    } else {
+      float *dst = p.partials + ((size_t)I.pbase + (size_t)I.split * I.rows + r) * kPStride;
+      __stcg(reinterpret_cast<float4 *>(dst + lane * 4), make_float4(O0, O1, O2, O3));
+      if (lane == 0) {
+        __stcg(dst + 128, Mx);
+        __stcg(dst + 129, Ls);
+      }
+    }
+  }
+  named_bar_sync(1, kCW * 32);
+  return true;
+}
+
 __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant__ AttnParams p) {
   extern __shared__ __align__(1024) uint8_t smem[];
   const Bars B = bars(smem);
@@ -1128,7 +1335,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
       const BatchDev &Bt = p.b[I.b];
       const void *tk = &p.tmap[2 * Bt.cache];
       const void *tv = &p.tmap[2 * Bt.cache + 1];
-      const int oob_row = (int)(Bt.num_pages * Bt.hkv * kPage);  // a box here reads zeros
+      const int oob_w = (int)(Bt.num_pages * Bt.hkv * 2);  // a box here reads zeros
       const int npages = I.page_hi - I.page_lo;
       const int nst = (npages + kStagePages - 1) / kStagePages;
       int ids_next = (npages > 32) ? load_ids(I, 1) : -1;
@@ -1150,12 +1357,12 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
           aborted = true;
           break;
         }
-        int y = oob_row;
+        int w = oob_w;
         bool ok = false;
         if (lane < np) {
           ok = pid >= 0 && (long long)pid < Bt.num_pages;
           if (!ok) ipd_set_error(&g_attn_err, IPD_DEVERR_PAGE_ID);
-          else y = (pid * Bt.hkv + I.kvh) * kPage;
+          else w = (pid * Bt.hkv + I.kvh) * 2;
         }
         const uint32_t okmask = __ballot_sync(0xffffffffu, ok);
         if (lane == 0) {
@@ -1171,12 +1378,8 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
         }
         __syncwarp();
         if (lane < kStagePages) {  // every page slot is written (zeros past the item)
-          uint8_t *kd = stage_k(smem, s) + lane * kPage * 128;
-          uint8_t *vd = stage_v(smem, s) + lane * kPage * 128;
-          tma_load_2d(kd, tk, 0, y, &B.full[s], policy);
-          tma_load_2d(kd + kHalfBytes, tk, 64, y, &B.full[s], policy);
-          tma_load_2d(vd, tv, 0, y, &B.full[s], policy);
-          tma_load_2d(vd + kHalfBytes, tv, 64, y, &B.full[s], policy);
+          tma_load_4d(stage_k(smem, s) + lane * kPageBytes, tk, 0, 0, 0, w, &B.full[s], policy);
+          tma_load_4d(stage_v(smem, s) + lane * kPageBytes, tv, 0, 0, 0, w, &B.full[s], policy);
         }
         ++it;
       }
@@ -1234,8 +1437,8 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
         const uint32_t va = smem_u32(stage_v(smem, pstage));
 #pragma unroll
         for (int kk = 0; kk < kStageKeys / 16; ++kk) {
-          // V rows 16kk.. as an MN-major operand: the two 64-dim halves kHalfBytes apart
-          const uint64_t bd = sdesc_sw128(va + kk * 16 * 128, kHalfBytes, 1024);
+          // V keys 16kk.. as an MN-major operand: 64-dim halves 1 KB apart, 8-key groups 2 KB
+          const uint64_t bd = sdesc_sw128(va + kk * 2 * kGroupBytes, kAtomBytes, kGroupBytes);
           const uint64_t ad = sdesc_sw128(pa + (kk >> 2) * Smem::kPBlock + (kk & 3) * 32, 16, 1024);
           tc_mma_bf16(tmem + kColO, ad, bd, idesc_o, (pfirst && kk == 0) ? 0u : 1u);
           if (ppath == kPathTcFull)  // residual of P, from the chunk's S buffer
@@ -1276,7 +1479,8 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
         const uint32_t ka = smem_u32(stage_k(smem, s));
 #pragma unroll
         for (int kk = 0; kk < kD / 16; ++kk) {
-          const uint64_t bd = sdesc_sw128(ka + (kk >> 2) * kHalfBytes + (kk & 3) * 32, 16, 1024);
+          const uint64_t bd =
+              sdesc_sw128(ka + (kk >> 2) * kAtomBytes + (kk & 3) * 32, 16, kGroupBytes);
           tc_mma_bf16_ta(tmem + col_s(c & 1), tmem + kColQ + 8 * kk, bd, idesc_s, kk > 0);
         }
         tc_commit(&B.s_full[c & 1]);
@@ -1318,9 +1522,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
     } else if (I.path == kPathTcFull) {
       ok = tc_item<false>(p, X, I, it, c);
     } else {
-      // GQA-2 decode (two rows) gets straight-line code; other sizes take
-      // the guarded loop (more instances overflow the register budget)
-      if (I.rows == 2) ok = cc_item<2>(p, X, I, it);
+      // GQA-2 decode (two rows) has its own layout; other sizes take the
+      // guarded loop
+      if (I.rows == 2) ok = cc2_item(p, X, I, it);
       else ok = cc_item<kCcRows>(p, X, I, it);
     }
     if (!ok) break;
@@ -1351,14 +1555,16 @@ int get_encoder() {
   return IPD_OK;
 }
 
-// A pool [num_pages][Hkv][16][128] bf16 seen as a 2-D tensor of 128-element
-// rows; boxes of 64 elements x 16 rows, 128-byte swizzle.
+// A pool [num_pages][Hkv][16][128] bf16 seen as a 4-D tensor (x: 64 dims,
+// y: 8 rows 256 B apart, z: 2 halves 128 B apart, w: 8-row groups 2 KB
+// apart), 128-byte swizzle; a box (64, 8, 2, 2) is one page of one kv head
+// in the stage layout (two groups, each as its two halves).
 int encode_pool(CUtensorMap *m, const void *base, long long rows) {
-  cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)rows};
-  cuuint64_t strides[1] = {(cuuint64_t)kD * 2};
-  cuuint32_t box[2] = {64, (cuuint32_t)kPage};
-  cuuint32_t estr[2] = {1, 1};
-  const CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base),
+  cuuint64_t dims[4] = {64, 8, 2, (cuuint64_t)(rows / 8)};
+  cuuint64_t strides[3] = {(cuuint64_t)kD * 2, 128, (cuuint64_t)kGroupBytes};
+  cuuint32_t box[4] = {64, 8, 2, 2};
+  cuuint32_t estr[4] = {1, 1, 1, 1};
+  const CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base),
                               dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                               CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);

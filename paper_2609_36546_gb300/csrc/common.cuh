@@ -155,6 +155,16 @@ IPD_DEVINL void tma_load_2d(void *dst_smem, const void *tmap, int x, int y, uint
       : "memory");
 }
 
+// 4-D tiled TMA load (coordinates x, y, z, w), same conventions as above.
+IPD_DEVINL void tma_load_4d(void *dst_smem, const void *tmap, int x, int y, int z, int w,
+                            uint64_t *bar, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3, %4, %5}], [%6], %7;" ::"r"(smem_u32(dst_smem)),
+      "l"(tmap), "r"(x), "r"(y), "r"(z), "r"(w), "r"(smem_u32(bar)), "l"(policy)
+      : "memory");
+}
+
 // Orders this thread's generic-proxy shared-memory writes before later
 // async-proxy reads (tcgen05.mma operands written by threads).
 IPD_DEVINL void fence_proxy_async_smem() {
