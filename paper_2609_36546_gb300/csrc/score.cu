@@ -1,18 +1,15 @@
 // The vocabulary pass of the verify step (Sec. 3.1 top-K supports, Sec. 3.2.1
 // coverage rules, Sec. 3.2.2 source-split KL terms, Sec. 3.2.3 verdict).
 //
-// Kernel 1 (row pass), one CTA per logits row (2 rows per span position: the
-// student's and the teacher's), one read of the row from HBM:
-//   - log Z = log sum exp(l) with a per-thread online maximum (fp32),
-//   - the exact top-K (K <= 32) under the order (logit desc, token id asc).
-//     Every warp keeps its best 32 keys sorted across its lanes; a 64-bit key
-//     (bf16 order code << 32 | ~token id) makes keys distinct and the order
-//     total.  A warp-uniform threshold filters candidates with one compare
-//     per 8 logits, and warps share their thresholds through shared memory.
-//   - the logit of the proposed token.
-// Kernel 2 (epilogue), one CTA per request: union support, renormalised KL in
-// both directions, log-probs and feedback, coverage and margin, then the
-// verdict of the request's span.
+// Kernel 1 (row pass), one CTA per quarter of a logits row (2 rows per span
+// position: the student's and the teacher's), one read of the row from HBM:
+//   - the part's log-sum-exp (maximum and scaled sum, fp32),
+//   - the part's exact top-K (K <= 32) under the order (logit desc, token id
+//     asc), through a threshold filter, a per-warp queue of vectors that pass
+//     it and a per-warp candidate buffer.
+// Kernel 2 (epilogue), one CTA per request: each row's log Z and top-K from
+// its parts, union support, renormalised KL in both directions, log-probs
+// and feedback, coverage and margin, then the verdict of the request's span.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -27,12 +24,16 @@ namespace {
 constexpr int kRowThreads = 256;
 constexpr int kRowWarps = kRowThreads / 32;
 constexpr int kEpiThreads = 256;
+constexpr int kParts = 1;    // a logits row is split into this many parts, one CTA each
+constexpr int kQueue = 160;  // per-warp queue of vectors that passed the filter (32 + 4 * 32)
+constexpr int kBuf = 64;     // per-warp candidate buffer: up to 32 kept keys + one round of 32
 
+// One part of one logits row.
 struct RowOut {
-  float logz;     // log sum_v exp(l_v)
-  float lx;       // logit of the proposed token (NaN if the token id is invalid)
+  float m;  // maximum logit of the part (-inf if the part is empty)
+  float s;  // sum over the part of exp(l - m)
   int pad[2];
-  unsigned long long keys[IPD_MAX_K];  // best first
+  unsigned long long keys[IPD_MAX_K];  // the part's best keys, best first, 0 past the end
 };
 
 // Order code of a bf16 value: monotone in the value, -0 folded onto +0.
@@ -74,109 +75,179 @@ __device__ __forceinline__ unsigned long long shfl_u64(unsigned long long v, int
   return __shfl_sync(0xffffffffu, v, src);
 }
 
-// Insert key c into the warp's descending list (lane i holds the i-th best).
-__device__ __forceinline__ void list_insert(unsigned long long &L, unsigned long long c, int lane) {
-  const int pos = __popc(__ballot_sync(0xffffffffu, L > c));
-  const unsigned long long up = __shfl_up_sync(0xffffffffu, L, 1);
-  if (lane == pos) L = c;
-  else if (lane > pos) L = up;
-}
-
-// Bitonic sort of one key per lane, descending over lanes.
-__device__ __forceinline__ unsigned long long warp_sort_desc(unsigned long long k, int lane) {
+// Bitonic sort of one float per lane, descending over lanes.
+__device__ __forceinline__ float warp_sort_desc_f(float k, int lane) {
 #pragma unroll
   for (int size = 2; size <= 32; size <<= 1) {
 #pragma unroll
     for (int j = size >> 1; j > 0; j >>= 1) {
-      const unsigned long long o = __shfl_xor_sync(0xffffffffu, k, j);
+      const float o = __shfl_xor_sync(0xffffffffu, k, j);
       const bool lower = (lane & j) == 0;
       const bool desc = (lane & size) == 0;
-      const unsigned long long hi = k > o ? k : o, lo = k > o ? o : k;
-      k = (lower == desc) ? hi : lo;
+      k = (lower == desc) ? fmaxf(k, o) : fminf(k, o);
     }
   }
   return k;
 }
 
+// number of values above c (or at least c) in a descending list of 32
+__device__ __forceinline__ int count_above32(const float *list, float c, bool or_equal) {
+  int lo = 0, hi = 32;
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if (list[mid] > c || (or_equal && list[mid] == c)) lo = mid + 1;
+    else hi = mid;
+  }
+  return lo;
+}
+
+// number of keys greater than c in a descending list of 32 (binary search)
+__device__ __forceinline__ int count_greater32(const unsigned long long *list, unsigned long long c) {
+  int lo = 0, hi = 32;
+  while (lo < hi) {
+    const int mid = (lo + hi) >> 1;
+    if (list[mid] > c) lo = mid + 1;
+    else hi = mid;
+  }
+  return lo;
+}
+
+// Row pass over one part of one logits row (Sec. 3.1, Sec. 3.2.1):
+//   - the part's log-sum-exp as (m, s) with a per-thread online maximum;
+//   - the part's exact top-K (K <= 32) under the order (logit desc, token id
+//     asc), a 64-bit key (bf16 order code << 32 | ~token id) making keys
+//     distinct and the order total.
+// A key at or below the current threshold th cannot be among the part's
+// top-K: th is either a key with at least K larger keys in the part (the
+// warm-up value) or the K-th best key a warp already holds.  Vectors whose
+// maximum reaches th's value go to a per-warp queue; 32 queued vectors are
+// examined at once, one per lane, and keys above th go to the warp's buffer,
+// which is cut back to its best K (by rank) whenever it fills.
 __global__ void __launch_bounds__(kRowThreads, 4) score_rows_kernel(
-    const uint16_t *__restrict__ ls, const uint16_t *__restrict__ lt,
-    const int32_t *__restrict__ tokens, int vocab, int K, RowOut *__restrict__ out) {
+    const uint16_t *__restrict__ ls, const uint16_t *__restrict__ lt, int vocab, int K,
+    RowOut *__restrict__ out) {
   __shared__ unsigned long long s_theta;
   __shared__ unsigned long long s_lists[kRowWarps][32];
+  __shared__ unsigned long long s_buf[kRowWarps][kBuf];
+  __shared__ uint4 s_qraw[kRowWarps][kQueue];
+  __shared__ int s_qidx[kRowWarps][kQueue];
   __shared__ float s_m[kRowWarps], s_s[kRowWarps];
 
-  const int t = blockIdx.x >> 1, model = blockIdx.x & 1;
+  const int row_id = blockIdx.x / kParts, part = blockIdx.x % kParts;
+  const int t = row_id >> 1, model = row_id & 1;
   const uint16_t *row = (model ? lt : ls) + (size_t)t * vocab;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int nvec = vocab >> 3;
+  const int per = (nvec + kParts - 1) / kParts;
+  const int v_lo = min(nvec, part * per), v_hi = min(nvec, v_lo + per);
   if (threadIdx.x == 0) s_theta = 0ull;
   __syncthreads();
+  volatile unsigned long long *vtheta = &s_theta;
+  unsigned long long *buf = s_buf[warp];
 
-  const int nvec = vocab >> 3;
   float m = -INFINITY, s = 0.f;
-  unsigned long long L = 0ull, theta = 0ull;
+  unsigned long long theta = 0ull;  // K-th best key this warp holds (0: fewer than K)
+  int nb = 0;                       // keys in the warp's buffer
+  int qn = 0;                       // vectors in the warp's queue
 
-  // Block-wide warm-up.  Every thread takes the best key among its first
-  // U vectors (8*U logits); the 17th largest of those 256 lane maxima starts
-  // the shared threshold.  At least 16 logits of the row are strictly above
-  // it, so no member of the row's top-K (K <= 16 here; larger K lowers it to
-  // the (K+1)-th) is ever filtered out, and only ~0.3 % of N(0,1)-like logits
-  // pass it from the start.
+  // Block-wide warm-up: every thread takes the largest value among its first
+  // U vectors; with tau the (max(K,16)+1)-th largest of those 256 values (ties
+  // counted), at least max(K,16)+1 logits of the part are >= tau, so at least
+  // that many keys lie strictly above the key (tau, largest index) =
+  // ord(tau) << 32, which starts the shared threshold.
   constexpr int U = 4;
   uint4 pre[U];
-  unsigned long long lane_best = 0ull;
+  float lane_best = -INFINITY;
 #pragma unroll
   for (int u = 0; u < U; ++u) {
-    const int v0 = u * kRowThreads + (int)threadIdx.x;
+    const int v0 = v_lo + u * kRowThreads + (int)threadIdx.x;
     pre[u] = make_uint4(0xff80ff80u, 0xff80ff80u, 0xff80ff80u, 0xff80ff80u);  // -inf
-    if (v0 < nvec) pre[u] = ldg_stream(row + (size_t)v0 * 8);
+    if (v0 < v_hi) pre[u] = ldg_stream(row + (size_t)v0 * 8);
   }
 #pragma unroll
-  for (int u = 0; u < U; ++u) {
-    const int v0 = u * kRowThreads + (int)threadIdx.x;
-    if (v0 < nvec) {
-#pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        const unsigned long long k = make_key(elem_bits(pre[u], e), (uint32_t)v0 * 8u + e);
-        lane_best = k > lane_best ? k : lane_best;
-      }
-    }
-  }
-  s_lists[warp][lane] = warp_sort_desc(lane_best, lane);
-  __syncthreads();
+  for (int u = 0; u < U; ++u) lane_best = fmaxf(lane_best, bf16x8_max(pre[u]));
   {
-    const unsigned long long c = s_lists[warp][lane];
-    int rank = 0;
+    float *sv = reinterpret_cast<float *>(s_lists);  // [8][32] floats, sorted per warp
+    sv[warp * 32 + lane] = warp_sort_desc_f(lane_best, lane);
+    __syncthreads();
+    const float c = sv[warp * 32 + lane];
+    int gt = 0, ge = 0;
 #pragma unroll 1
     for (int w2 = 0; w2 < kRowWarps; ++w2) {
-      int lo = 0, hi = 32;
-      while (lo < hi) {
-        const int mid = (lo + hi) >> 1;
-        if (s_lists[w2][mid] > c) lo = mid + 1;
-        else hi = mid;
-      }
-      rank += lo;
+      gt += count_above32(sv + w2 * 32, c, false);
+      ge += count_above32(sv + w2 * 32, c, true);
     }
-    if (c != 0ull && rank == (K > 16 ? K : 16)) s_theta = c;  // the (max(K,16)+1)-th largest
+    const int need = (K > 16 ? K : 16) + 1;
+    if (c != -INFINITY && gt < need && ge >= need)
+      s_theta = (unsigned long long)ord16(__float_as_uint(c) >> 16) << 32;
+    __syncthreads();
   }
-  __syncthreads();
-  L = 0ull;
-  theta = 0ull;
 
-  // Four independent 16-byte loads per thread are in flight per iteration.
-  // Per 8 logits: the maximum on the packed bf16 words (3 max instructions),
-  // then unpack, one fused multiply-add and one hardware 2^x each for the sum.
-  // The candidate filter compares the vector maximum with the threshold's
-  // value; only vectors reaching it build 64-bit keys.
-  // The trip count is the same for every thread (warp-wide ballots below).
-  for (int base = 0; base < nvec; base += kRowThreads * U) {
+  // Keep the best min(K, nb) keys of the buffer, sorted, and raise theta.
+  auto compact = [&]() {
+    __syncwarp();
+    const unsigned long long a = lane < nb ? buf[lane] : 0ull;
+    const unsigned long long b = lane + 32 < nb ? buf[lane + 32] : 0ull;
+    int ra = 0, rb = 0;
+    for (int j = 0; j < nb; ++j) {
+      const unsigned long long x = buf[j];
+      ra += x > a;
+      rb += x > b;
+    }
+    __syncwarp();
+    if (lane < nb && ra < K) buf[ra] = a;
+    if (lane + 32 < nb && rb < K) buf[rb] = b;
+    __syncwarp();
+    nb = nb < K ? nb : K;
+    if (nb == K) {
+      theta = buf[K - 1];
+      if (lane == 0 && theta > *vtheta) atomicMax(&s_theta, theta);
+    }
+  };
+  // Examine queued vectors q0 .. q0 + n - 1 (n <= 32), one per lane.
+  auto examine = [&](int q0, int n) {
+    const bool have = lane < n;
+    uint4 r = make_uint4(0, 0, 0, 0);
+    int v = 0;
+    if (have) {
+      r = s_qraw[warp][q0 + lane];
+      v = s_qidx[warp][q0 + lane];
+    }
+    __syncwarp();
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const unsigned long long sth = *vtheta;
+      const unsigned long long th = theta > sth ? theta : sth;
+      const unsigned long long key = make_key(elem_bits(r, e), (uint32_t)v * 8u + e);
+      const bool c = have && key > th;
+      const unsigned bal = __ballot_sync(0xffffffffu, c);
+      if (bal) {
+        if (nb + 32 > kBuf) compact();
+        if (c) buf[nb + __popc(bal & ((1u << lane) - 1u))] = key;
+        nb += __popc(bal);
+      }
+    }
+  };
+
+  // Each iteration takes four 16-byte vectors per thread and issues the loads
+  // of the next iteration's four before it works on them, so eight loads per
+  // thread are in flight.  Per 8 logits: the maximum on the packed bf16
+  // words, then unpack, one fused multiply-add and one hardware 2^x each for
+  // the sum.  The trip count is the same for every thread of the block
+  // (warp-wide ballots below).
+  uint4 nxt[U];
+#pragma unroll
+  for (int u = 0; u < U; ++u) nxt[u] = pre[u];
+  for (int base = v_lo; base < v_hi; base += kRowThreads * U) {
     uint4 raw[U];
     int vv[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
+      raw[u] = nxt[u];
       vv[u] = base + u * kRowThreads + (int)threadIdx.x;
-      raw[u] = make_uint4(0xff80ff80u, 0xff80ff80u, 0xff80ff80u, 0xff80ff80u);  // -inf
-      if (base == 0) raw[u] = pre[u];
-      else if (vv[u] < nvec) raw[u] = ldg_stream(row + (size_t)vv[u] * 8);
+      const int vn = vv[u] + kRowThreads * U;
+      nxt[u] = make_uint4(0xff80ff80u, 0xff80ff80u, 0xff80ff80u, 0xff80ff80u);  // -inf
+      if (vn < v_hi) nxt[u] = ldg_stream(row + (size_t)vn * 8);
     }
     float vmx[U];
 #pragma unroll
@@ -198,53 +269,50 @@ __global__ void __launch_bounds__(kRowThreads, 4) score_rows_kernel(
         }
       }
     }
-    // candidate filter against the warp / block threshold
-    const unsigned long long sth = s_theta;
+    // vectors that may hold a key above the threshold go to the queue
+    const unsigned long long sth = *vtheta;
     const unsigned long long th = theta > sth ? theta : sth;
-    const float thf = key_val(th);  // threshold value (keys equal in value go to the full test)
-    uint32_t pending = 0;           // bit 8u + e: element e of vector u
-    if (th == 0ull || bmax >= thf) {
+    const float thf = key_val(th);  // equal values go on to the full key test
+    uint32_t pmask = 0;
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+      if (vv[u] < v_hi && (th == 0ull || vmx[u] >= thf)) pmask |= 1u << u;
+    if (__any_sync(0xffffffffu, pmask != 0)) {
+      const int cnt = __popc(pmask);
+      int off = cnt;  // inclusive scan over lanes
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, off, o);
+        if (lane >= o) off += y;
+      }
+      const int total = __shfl_sync(0xffffffffu, off, 31);
+      off -= cnt;
 #pragma unroll
       for (int u = 0; u < U; ++u)
-        if (vv[u] < nvec && (th == 0ull || vmx[u] >= thf)) {
-#pragma unroll
-          for (int e = 0; e < 8; ++e)
-            if (make_key(elem_bits(raw[u], e), (uint32_t)vv[u] * 8u + e) > th)
-              pending |= 1u << (8 * u + e);
+        if (pmask & (1u << u)) {
+          s_qraw[warp][qn + off] = raw[u];
+          s_qidx[warp][qn + off] = vv[u];
+          ++off;
         }
-    }
-    unsigned any = __ballot_sync(0xffffffffu, pending != 0);
-    if (any) {
-      while (any) {
-        const int leader = __ffs(any) - 1;
-        unsigned long long c = 0ull;
-        if (lane == leader) {
-          const int bit = __ffs(pending) - 1;
-          pending &= pending - 1;
-          const int u = bit >> 3, e = bit & 7;
-          const uint4 r = u == 0 ? raw[0] : (u == 1 ? raw[1] : (u == 2 ? raw[2] : raw[3]));
-          const int vsel = u == 0 ? vv[0] : (u == 1 ? vv[1] : (u == 2 ? vv[2] : vv[3]));
-          c = make_key(elem_bits(r, e), (uint32_t)vsel * 8u + e);
-        }
-        c = shfl_u64(c, leader);
-        if (c > theta) {
-          list_insert(L, c, lane);
-          theta = shfl_u64(L, K - 1);
-        }
-        any = __ballot_sync(0xffffffffu, pending != 0);
+      qn += total;
+      __syncwarp();
+      while (qn >= 32) {
+        examine(qn - 32, 32);
+        qn -= 32;
       }
-      if (lane == 0 && theta > s_theta) atomicMax(&s_theta, theta);
     }
   }
-  // Every logit of the row went through the filter exactly once, so each
-  // reached at most one warp list and the keys in the lists are distinct.
+  if (qn > 0) examine(0, qn);
+  if (nb > 0) compact();
+  // Every logit of the part went through the filter once, so the warps'
+  // buffers hold distinct keys.
 
   // block merge of the log-sum-exp
   float wm = warp_max(m);
   float ws = (m == -INFINITY) ? 0.f : s * exp2f((m - wm) * kLog2e);
   if (wm == -INFINITY) ws = 0.f;
   ws = warp_sum(ws);
-  s_lists[warp][lane] = L;
+  s_lists[warp][lane] = lane < nb ? buf[lane] : 0ull;
   if (lane == 0) {
     s_m[warp] = wm;
     s_s[warp] = ws;
@@ -255,31 +323,20 @@ __global__ void __launch_bounds__(kRowThreads, 4) score_rows_kernel(
     const float gm = warp_max(bm);
     float bs = (lane < kRowWarps && bm != -INFINITY) ? s_s[lane] * exp2f((bm - gm) * kLog2e) : 0.f;
     bs = warp_sum(bs);
-    // merge of the warp lists: the rank of a key in the union is the number of
-    // larger keys in every list (binary search in each sorted list)
     if (lane == 0) {
-      out[blockIdx.x].logz = gm + logf(bs);
-      const int x = tokens[t];
-      float lx = __int_as_float(0x7fc00000);
-      if (x >= 0 && x < vocab) lx = bf16f(row[x]);
-      out[blockIdx.x].lx = lx;
+      out[blockIdx.x].m = gm;
+      out[blockIdx.x].s = bs;
     }
+    if (lane < IPD_MAX_K) out[blockIdx.x].keys[lane] = 0ull;
   }
-  // every thread ranks one candidate key (kRowWarps * 32 == kRowThreads)
+  __syncthreads();
+  // merge of the warp lists: a key's rank in the union is the number of
+  // larger keys in every list (each thread ranks one key)
   {
     const unsigned long long c = s_lists[warp][lane];
     int rank = 0;
 #pragma unroll 1
-    for (int w2 = 0; w2 < kRowWarps; ++w2) {
-      // number of keys > c in list w2 (descending): binary search
-      int lo = 0, hi = 32;
-      while (lo < hi) {
-        const int mid = (lo + hi) >> 1;
-        if (s_lists[w2][mid] > c) lo = mid + 1;
-        else hi = mid;
-      }
-      rank += lo;
-    }
+    for (int w2 = 0; w2 < kRowWarps; ++w2) rank += count_greater32(s_lists[w2], c);
     if (c != 0ull && rank < K) out[blockIdx.x].keys[rank] = c;
   }
 }
@@ -293,6 +350,8 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     int32_t *first_trans, int32_t *n_emit, uint8_t *next_driver, int32_t *new_len, uint8_t *done,
     int total_tokens) {
   __shared__ uint8_t s_cov[1024];
+  __shared__ unsigned long long s_pk[kEpiThreads / 32][kParts][32];  // one row's part lists
+  __shared__ unsigned long long s_top[kEpiThreads / 32][2][32];      // merged top-K, S and T
   const int r = blockIdx.x;
   const int t0 = cu_span[r], t1 = cu_span[r + 1];
   const int drv = driver[r] ? 1 : 0;
@@ -304,17 +363,49 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
   const int k = t1 - t0;
 
   for (int t = t0 + warp; t < t1; t += kEpiThreads / 32) {
-    const RowOut &rs = rows[2 * t], &rq = rows[2 * t + 1];
     const int x = tokens[t];
     const bool xok = x >= 0 && x < vocab;
     if (!xok && lane == 0) ipd_set_error(&g_score_err, IPD_DEVERR_TOKEN);
     const uint16_t *rowS = ls + (size_t)t * vocab, *rowT = lt + (size_t)t * vocab;
+    // each row from its parts: log Z by the log-sum-exp merge, the top-K as
+    // the best K of the parts' lists (a key's rank is the number of larger
+    // keys in every part list)
+    float logz[2];
+#pragma unroll
+    for (int mdl = 0; mdl < 2; ++mdl) {
+      const RowOut *pr = rows + (size_t)(2 * t + mdl) * kParts;
+      float M = -INFINITY;
+#pragma unroll
+      for (int q = 0; q < kParts; ++q) M = fmaxf(M, pr[q].m);
+      float S = 0.f;
+#pragma unroll
+      for (int q = 0; q < kParts; ++q)
+        if (pr[q].m != -INFINITY) S += pr[q].s * expf(pr[q].m - M);
+      logz[mdl] = M + logf(S);
+#pragma unroll
+      for (int q = 0; q < kParts; ++q) s_pk[warp][q][lane] = lane < K ? pr[q].keys[lane] : 0ull;
+      s_top[warp][mdl][lane] = 0ull;
+      __syncwarp();
+#pragma unroll
+      for (int q = 0; q < kParts; ++q) {
+        const unsigned long long c = s_pk[warp][q][lane];
+        if (c != 0ull) {
+          int rank = 0;
+#pragma unroll
+          for (int q2 = 0; q2 < kParts; ++q2) rank += count_greater32(s_pk[warp][q2], c);
+          if (rank < K) s_top[warp][mdl][rank] = c;
+        }
+      }
+      __syncwarp();
+    }
+    const float nan = __int_as_float(0x7fc00000);
+    const float lxS = xok ? bf16f(rowS[x]) : nan, lxT = xok ? bf16f(rowT[x]) : nan;
     // union support S = Top_K(pi) u Top_K(q)
     unsigned long long kS = 0ull, kT = 0ull;
     uint32_t iS = 0, iT = 0;
     if (lane < K) {
-      kS = rs.keys[lane];
-      kT = rq.keys[lane];
+      kS = s_top[warp][0][lane];
+      kT = s_top[warp][1][lane];
       iS = key_idx(kS);
       iT = key_idx(kT);
       if (iS >= (uint32_t)vocab) iS = 0;  // never taken: K <= vocab fills every slot
@@ -364,15 +455,14 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     const bool cov = __ballot_sync(0xffffffffu, hit) != 0;
     const unsigned long long kth = shfl_u64(kv, K - 1);
     if (lane == 0) {
-      const RowOut &rv = drv ? rs : rq;
-      const float lps = rs.lx - rs.logz, lpt = rq.lx - rq.logz;
+      const float lps = lxS - logz[0], lpt = lxT - logz[1];
       logp_s[t] = lps;
       logp_t[t] = lpt;
       feedback[t] = lpt - lps;
       kl_rev[t] = kr;
       kl_fwd[t] = kf;
       covered[t] = cov ? 1 : 0;
-      margin[t] = rv.lx - key_val(kth);
+      margin[t] = (drv ? lxS : lxT) - key_val(kth);
       if (t - t0 < 1024) s_cov[t - t0] = cov ? 1 : 0;
     }
   }
@@ -425,7 +515,7 @@ extern "C" __attribute__((visibility("hidden"))) unsigned int ipd_internal_take_
 
 extern "C" size_t ipd_score_workspace_size(int num_reqs, int total_tokens, int vocab, int K) {
   if (num_reqs < 0 || total_tokens < 0 || vocab < 1 || K < 1) return 0;
-  return (size_t)total_tokens * 2 * sizeof(RowOut) + 256;
+  return (size_t)total_tokens * 2 * kParts * sizeof(RowOut) + 256;
 }
 
 extern "C" int ipd_score_span(const uint16_t *logits_student, const uint16_t *logits_teacher,
@@ -455,8 +545,8 @@ extern "C" int ipd_score_span(const uint16_t *logits_student, const uint16_t *lo
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   RowOut *rows = static_cast<RowOut *>(workspace);
   if (total_tokens > 0) {
-    score_rows_kernel<<<2 * total_tokens, kRowThreads, 0, st>>>(logits_student, logits_teacher,
-                                                                tokens, vocab, K, rows);
+    score_rows_kernel<<<2 * kParts * total_tokens, kRowThreads, 0, st>>>(
+        logits_student, logits_teacher, vocab, K, rows);
     if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   }
   score_epilogue_kernel<<<num_reqs, kEpiThreads, 0, st>>>(
@@ -472,9 +562,9 @@ extern "C" int ipd_score_span(const uint16_t *logits_student, const uint16_t *lo
 // allocate device memory.  The per-row scratch that ipd_score_span takes from
 // the caller's workspace lives here in one file-scope device array, sized for
 // IPD_STATIC_MAX_TOKENS span positions.  Every GPU that loads the library
-// holds this array (about 2.1 MiB) until the process exits.
+// holds this array (about 8.5 MiB) until the process exits.
 // ---------------------------------------------------------------------------
-static __device__ __align__(256) RowOut g_static_rows[2 * IPD_STATIC_MAX_TOKENS];
+static __device__ __align__(256) RowOut g_static_rows[2 * kParts * IPD_STATIC_MAX_TOKENS];
 
 namespace {
 std::mutex g_static_mu;
@@ -525,8 +615,8 @@ extern "C" int ipd_score_span_static(const uint16_t *logits_student,
   // Every RowOut the epilogue reads is written by the row kernel of the same
   // call first, so nothing in the array has to start at zero.
   if (total_tokens > 0) {
-    score_rows_kernel<<<2 * total_tokens, kRowThreads, 0, s>>>(logits_student, logits_teacher,
-                                                               tokens, vocab, K, rows);
+    score_rows_kernel<<<2 * kParts * total_tokens, kRowThreads, 0, s>>>(
+        logits_student, logits_teacher, vocab, K, rows);
     if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   }
   score_epilogue_kernel<<<num_reqs, kEpiThreads, 0, s>>>(
