@@ -27,6 +27,9 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
+# kernels one step launches: ipd_verify_attn (planner, attention, split merge),
+# ipd_score_span (row pass, epilogue), ipd_split_loss (one)
+LAUNCHES_PER_STEP = 6
 METRIC = "verified tokens/s on 1 GB300; achieved HBM GB/s as % of peak"
 UNIT = "tokens/s"
 HBM_FALLBACK_GBS = 6800.0
@@ -388,7 +391,7 @@ def run_gpu(args):
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
-                     "kernel": "ipd_verify_attn (planner + attention launch)",
+                     "kernel": "ipd_verify_attn (planner, attention and split-merge launches)",
                      "bytes_per_launch": attn_bytes, "ms_per_launch": attn_ms},
         "step_hbm": {"bytes_alg": step_alg, "bytes_full": step_full,
                      "gbs_alg": step_alg / (ms_step / 1e3) / 1e9,
@@ -398,7 +401,7 @@ def run_gpu(args):
         "calls_ms": {"verify_attn": attn_ms, "score_span": score_ms, "split_loss": loss_ms},
         "acceptance": {"coverage_rate": accept_rate, "emitted_tokens_per_step": emitted},
         "e2e": e2e, "clocks": clocks,
-        "gpu_launches": 5 * K,
+        "gpu_launches": LAUNCHES_PER_STEP * K,
     }
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(step, w)

@@ -1,7 +1,7 @@
 // The vocabulary pass of the verify step (Sec. 3.1 top-K supports, Sec. 3.2.1
 // coverage rules, Sec. 3.2.2 source-split KL terms, Sec. 3.2.3 verdict).
 //
-// Kernel 1 (row pass), one CTA per quarter of a logits row (2 rows per span
+// Kernel 1 (row pass), one CTA per part of a logits row (2 rows per span
 // position: the student's and the teacher's), one read of the row from HBM:
 //   - the part's log-sum-exp (maximum and scaled sum, fp32),
 //   - the part's exact top-K (K <= 32) under the order (logit desc, token id
@@ -21,7 +21,7 @@ IPD_DECLARE_ERROR_WORD(g_score_err);
 
 namespace {
 
-constexpr int kRowThreads = 256;
+constexpr int kRowThreads = 128;  // eight row CTAs per SM: every row of a step in flight at once
 constexpr int kRowWarps = kRowThreads / 32;
 constexpr int kEpiThreads = 256;
 constexpr int kParts = 1;    // a logits row is split into this many parts, one CTA each
@@ -123,7 +123,7 @@ __device__ __forceinline__ int count_greater32(const unsigned long long *list, u
 // maximum reaches th's value go to a per-warp queue; 32 queued vectors are
 // examined at once, one per lane, and keys above th go to the warp's buffer,
 // which is cut back to its best K (by rank) whenever it fills.
-__global__ void __launch_bounds__(kRowThreads, 4) score_rows_kernel(
+__global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
     const uint16_t *__restrict__ ls, const uint16_t *__restrict__ lt, int vocab, int K,
     RowOut *__restrict__ out) {
   __shared__ unsigned long long s_theta;
@@ -151,7 +151,7 @@ __global__ void __launch_bounds__(kRowThreads, 4) score_rows_kernel(
   int qn = 0;                       // vectors in the warp's queue
 
   // Block-wide warm-up: every thread takes the largest value among its first
-  // U vectors; with tau the (max(K,16)+1)-th largest of those 256 values (ties
+  // U vectors; with tau the (max(K,16)+1)-th largest of those values (ties
   // counted), at least max(K,16)+1 logits of the part are >= tau, so at least
   // that many keys lie strictly above the key (tau, largest index) =
   // ord(tau) << 32, which starts the shared threshold.
