@@ -108,11 +108,13 @@ struct AttnParams {
   int n_batches;
   int total_reqs;
   float scale_log2;
-  int *ctrl;       // [0] n_items, [1] dynamic item counter, [2] n_tasks, [3] partial rows
-  int4 *reqinfo;   // per flattened request: item offset, task offset, partial offset, n_split
+  int *ctrl;       // [0] n_items, [1] dynamic item counter, [2] n_tasks, [3] partial rows,
+                   // [4] merge entries
+  int4 *reqinfo;   // per flattened request: merge-entry offset, task offset, partial offset, n_split
   Item *items;
+  int2 *merges;    // merge entries: (work-list slot of a split task's first item, 8-row group)
   float *partials;
-  int item_cap, task_cap;
+  int item_cap, task_cap, merge_cap;
   long long prow_cap;
   int target_items;  // work-list size the planner aims for (a multiple of the SM count)
   int n_sms;
@@ -132,8 +134,8 @@ struct StageMeta {
 // host-side sizes
 // --------------------------------------------------------------------------
 struct WsLayout {
-  size_t off_ctrl, off_reqinfo, off_items, off_partials, total;
-  int item_cap, task_cap, total_reqs;
+  size_t off_ctrl, off_reqinfo, off_items, off_merges, off_partials, total;
+  int item_cap, task_cap, merge_cap, total_reqs;
   long long prow_cap;
 };
 
@@ -210,6 +212,12 @@ WsLayout layout(const ipd_attn_batch *const *bs, int n) {
   off = align_up(off + (size_t)reqs * sizeof(int4), 256);
   L.off_items = off;
   off = align_up(off + (size_t)L.item_cap * sizeof(Item), 256);
+  // a split task has more pages than the chunk, and the chunk is at least
+  // 1 / kMaxTargetItems of all pages, so fewer than kMaxTargetItems tasks are
+  // split; each has at most kTcRows / 8 row groups
+  L.merge_cap = (int)std::min<long long>(prow_cap / 2 + 1, (long long)kMaxTargetItems * (kTcRows / 8));
+  L.off_merges = off;
+  off = align_up(off + (size_t)L.merge_cap * sizeof(int2), 256);
   L.off_partials = off;
   off = align_up(off + (size_t)prow_cap * kPStride * sizeof(float), 256);
   L.total = off;
@@ -268,27 +276,29 @@ __device__ T block_sum(T v, T *red) {
   return t;
 }
 
-// exclusive scan of three ints across the block; returns totals in tot
-__device__ void block_scan3(int3 v, int3 &excl, int3 &tot, int3 *sh) {
+// exclusive scan of four ints across the block; returns totals in tot
+__device__ void block_scan4(int4 v, int4 &excl, int4 &tot, int4 *sh) {
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  int3 inc = v;
+  int4 inc = v;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
     const int x = __shfl_up_sync(0xffffffffu, inc.x, o);
     const int y = __shfl_up_sync(0xffffffffu, inc.y, o);
     const int z = __shfl_up_sync(0xffffffffu, inc.z, o);
-    if (lane >= o) { inc.x += x; inc.y += y; inc.z += z; }
+    const int q = __shfl_up_sync(0xffffffffu, inc.w, o);
+    if (lane >= o) { inc.x += x; inc.y += y; inc.z += z; inc.w += q; }
   }
   __syncthreads();
   if (lane == 31) sh[w] = inc;
   __syncthreads();
-  int3 base = make_int3(0, 0, 0);
-  tot = make_int3(0, 0, 0);
+  int4 base = make_int4(0, 0, 0, 0);
+  tot = make_int4(0, 0, 0, 0);
   for (int i = 0; i < nw; ++i) {
-    if (i < w) { base.x += sh[i].x; base.y += sh[i].y; base.z += sh[i].z; }
-    tot.x += sh[i].x; tot.y += sh[i].y; tot.z += sh[i].z;
+    if (i < w) { base.x += sh[i].x; base.y += sh[i].y; base.z += sh[i].z; base.w += sh[i].w; }
+    tot.x += sh[i].x; tot.y += sh[i].y; tot.z += sh[i].z; tot.w += sh[i].w;
   }
-  excl = make_int3(base.x + inc.x - v.x, base.y + inc.y - v.y, base.z + inc.z - v.z);
+  excl = make_int4(base.x + inc.x - v.x, base.y + inc.y - v.y, base.z + inc.z - v.z,
+                   base.w + inc.w - v.w);
   __syncthreads();
 }
 
@@ -316,78 +326,126 @@ __device__ __forceinline__ int size_bucket(int b, int n_batches, int n, long lon
   return (n_batches - 1 - b) * kSizesPerBatch + (int)k;
 }
 
-__global__ void __launch_bounds__(1024) attn_plan_kernel(const __grid_constant__ AttnParams p) {
+// merge entries (8-row groups) of one kv head of a split request
+__device__ __forceinline__ int merge_groups(const ReqShape &s) {
+  int n = 0;
+  for (int rb = 0; rb < s.nrb; ++rb) n += (min(s.rpb, s.rows - rb * s.rpb) + 7) / 8;
+  return n;
+}
+
+// One block of 1024 threads.  Each thread owns requests tid, tid + 1024, ...;
+// the first kPlanCache of them keep their shape (two loads each) in
+// registers across the three passes: total work, per-request counts with
+// their block scan, and the items.
+constexpr int kPlanThreads = 1024;
+constexpr int kPlanCache = 4;
+
+__global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_constant__ AttnParams p) {
   __shared__ long long red[32];
-  __shared__ int3 sh3[32];
+  __shared__ int4 sh4[32];
   __shared__ int s_fail;
   __shared__ int s_slot[kSizeBuckets];  // items per size bucket, then each bucket's next slot
   const int tid = threadIdx.x;
   if (tid == 0) s_fail = 0;
-  for (int i = tid; i < kSizeBuckets; i += blockDim.x) s_slot[i] = 0;
+  for (int i = tid; i < kSizeBuckets; i += kPlanThreads) s_slot[i] = 0;
+
+  ReqShape cs[kPlanCache];
+  int cbat[kPlanCache];
+#pragma unroll
+  for (int k = 0; k < kPlanCache; ++k) {
+    const int gi = tid + k * kPlanThreads;
+    cbat[k] = 0;
+    cs[k] = ReqShape{};
+    if (gi < p.total_reqs) {
+      cbat[k] = find_batch(p, gi);
+      cs[k] = req_shape(p, cbat[k], gi - p.req_base[cbat[k]]);
+    }
+  }
+  // the k-th request of this thread (k < kPlanCache from registers)
+  auto shape_of = [&](int k, int gi, int &b) -> ReqShape {
+#pragma unroll
+    for (int j = 0; j < kPlanCache; ++j)
+      if (k == j) {
+        b = cbat[j];
+        return cs[j];
+      }
+    b = find_batch(p, gi);
+    return req_shape(p, b, gi - p.req_base[b]);
+  };
+  const int n_rounds = (p.total_reqs + kPlanThreads - 1) / kPlanThreads;
 
   long long w = 0;
-  for (int gi = tid; gi < p.total_reqs; gi += blockDim.x) {
-    const int b = find_batch(p, gi);
-    const ReqShape s = req_shape(p, b, gi - p.req_base[b]);
-    w += (long long)s.pages * p.b[b].hkv * s.nrb;
+  for (int k = 0; k < n_rounds; ++k) {
+    const int gi = tid + k * kPlanThreads;
+    if (gi < p.total_reqs) {
+      int b;
+      const ReqShape s = shape_of(k, gi, b);
+      w += (long long)s.pages * p.b[b].hkv * s.nrb;
+    }
   }
   const long long W = block_sum<long long>(w, red);
   long long chunk = (W + p.target_items - 1) / p.target_items;
   if (chunk < kMinChunkPages) chunk = kMinChunkPages;
 
-  // per request: split count, partial-row offset (exclusive scans), and the
-  // size histogram of its items
-  int3 carry = make_int3(0, 0, 0);
-  for (int base = 0; base < p.total_reqs; base += blockDim.x) {
-    const int gi = base + tid;
-    int3 cnt = make_int3(0, 0, 0);
+  // per request: split count, merge-entry, task and partial-row offsets
+  // (exclusive scans), and the size histogram of its items
+  int4 carry = make_int4(0, 0, 0, 0);  // merge entries, tasks, partial rows, items
+  for (int k = 0; k < n_rounds; ++k) {
+    const int gi = tid + k * kPlanThreads;
+    int4 cnt = make_int4(0, 0, 0, 0);
     int nsplit = 1;
     if (gi < p.total_reqs) {
-      const int b = find_batch(p, gi);
-      const ReqShape s = req_shape(p, b, gi - p.req_base[b]);
+      int b;
+      const ReqShape s = shape_of(k, gi, b);
       if (s.pages > 0) {
         nsplit = split_count(s.pages, chunk);
         const int per = split_pages(s.pages, chunk);
-        const int tasks = p.b[b].hkv * s.nrb;
-        cnt = make_int3(tasks * nsplit, tasks, nsplit > 1 ? nsplit * p.b[b].hkv * s.rows : 0);
+        const int hkv = p.b[b].hkv;
+        const int tasks = hkv * s.nrb;
+        cnt = make_int4(nsplit > 1 ? hkv * merge_groups(s) : 0, tasks,
+                        nsplit > 1 ? nsplit * hkv * s.rows : 0, tasks * nsplit);
         for (int sp = 0; sp < nsplit; ++sp)
           atomicAdd(&s_slot[size_bucket(b, p.n_batches, min(s.pages, (sp + 1) * per) - sp * per, chunk)],
                     tasks);
       }
     }
-    int3 ex, tot;
-    block_scan3(cnt, ex, tot, sh3);
+    int4 ex, tot;
+    block_scan4(cnt, ex, tot, sh4);
     if (gi < p.total_reqs)
       p.reqinfo[gi] = make_int4(carry.x + ex.x, carry.y + ex.y, carry.z + ex.z, nsplit);
-    carry.x += tot.x; carry.y += tot.y; carry.z += tot.z;
+    carry.x += tot.x; carry.y += tot.y; carry.z += tot.z; carry.w += tot.w;
   }
   if (tid == 0) {
-    if (carry.x > p.item_cap || carry.y > p.task_cap || carry.z > p.prow_cap) {
+    if (carry.w > p.item_cap || carry.y > p.task_cap || carry.z > p.prow_cap ||
+        carry.x > p.merge_cap) {
       ipd_set_error(&g_attn_err, IPD_DEVERR_PLAN);
       s_fail = 1;
     }
     // largest bucket first
     int off = 0;
-    for (int k = kSizeBuckets - 1; k >= 0; --k) {
-      const int n = s_slot[k];
-      s_slot[k] = off;
+    for (int q = kSizeBuckets - 1; q >= 0; --q) {
+      const int n = s_slot[q];
+      s_slot[q] = off;
       off += n;
     }
-    p.ctrl[0] = s_fail ? 0 : carry.x;
+    p.ctrl[0] = s_fail ? 0 : carry.w;
     p.ctrl[1] = 0;
     p.ctrl[2] = carry.y;
     p.ctrl[3] = carry.z;
+    p.ctrl[4] = s_fail ? 0 : carry.x;
   }
   __syncthreads();
   if (s_fail) return;
 
-  for (int gi = tid; gi < p.total_reqs; gi += blockDim.x) {
-    const int b = find_batch(p, gi);
-    const int r = gi - p.req_base[b];
-    const ReqShape s = req_shape(p, b, r);
+  for (int k = 0; k < n_rounds; ++k) {
+    const int gi = tid + k * kPlanThreads;
+    if (gi >= p.total_reqs) continue;
+    int b;
+    const ReqShape s = shape_of(k, gi, b);
     if (s.pages == 0) continue;
+    const int r = gi - p.req_base[b];
     const int4 info = p.reqinfo[gi];
-    int task = info.y;
+    int task = info.y, mrg = info.x;
     const int ns = info.w;
     const int per = split_pages(s.pages, chunk);
     for (int kvh = 0; kvh < p.b[b].hkv; ++kvh) {
@@ -405,6 +463,8 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const __grid_constant__
           const int slot =
               atomicAdd(&s_slot[size_bucket(b, p.n_batches, it.page_hi - it.page_lo, chunk)], 1);
           p.items[slot] = it;
+          if (ns > 1 && sp == 0)
+            for (int g8 = 0; g8 < (rows + 7) / 8; ++g8) p.merges[mrg++] = make_int2(slot, g8);
         }
         ++task;
       }
@@ -414,52 +474,50 @@ __global__ void __launch_bounds__(1024) attn_plan_kernel(const __grid_constant__
 
 // Split-KV merge: each task split over several items combines its splits'
 // partial rows (unnormalised O, maximum m, sum l, all in log2 units) into the
-// output rows.  Work unit = (item, group of 8 rows); warp = row, lane = 4
-// dims, every split's loads in flight at once.
+// output rows.  The planner lists one entry per (split task, group of 8
+// rows); warp = row, lane = 4 dims, every split's loads in flight at once.
 __global__ void __launch_bounds__(256) attn_merge_kernel(const __grid_constant__ AttnParams p) {
-  constexpr int kGroups = kTcRows / 8;  // row groups of 8 (one per warp) per item
-  const int n_units = p.ctrl[0] * kGroups;
+  const int n_entries = p.ctrl[4];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int u = blockIdx.x; u < n_units; u += gridDim.x) {
-    const Item I = p.items[u / kGroups];
-    const int r = (u % kGroups) * 8 + warp;
-    if (I.n_split < 2 || I.split != 0 || (u % kGroups) * 8 >= I.rows) continue;
-    if (r < I.rows) {
-      const BatchDev &Bt = p.b[I.b];
-      const int q0 = Bt.cu_q[I.r], G = Bt.group;
-      const int rpb = I.path != kPathCc ? kTcRows : kCcRows;
-      const int ns = I.n_split;
-      const size_t sstr = (size_t)I.rows * kPStride;
-      const float *base = p.partials + (size_t)(I.pbase + r) * kPStride;
-      const float mv = lane < ns ? __ldcg(base + lane * sstr + 128) : -INFINITY;
-      const float lv = lane < ns ? __ldcg(base + lane * sstr + 129) : 0.f;
-      float4 ov[kSplitMax];
+  for (int e = blockIdx.x; e < n_entries; e += gridDim.x) {
+    const int2 me = p.merges[e];
+    const Item I = p.items[me.x];
+    const int r = me.y * 8 + warp;
+    if (r >= I.rows) continue;
+    const BatchDev &Bt = p.b[I.b];
+    const int q0 = Bt.cu_q[I.r], G = Bt.group;
+    const int rpb = I.path != kPathCc ? kTcRows : kCcRows;
+    const int ns = I.n_split;
+    const size_t sstr = (size_t)I.rows * kPStride;
+    const float *base = p.partials + (size_t)(I.pbase + r) * kPStride;
+    const float mv = lane < ns ? __ldcg(base + lane * sstr + 128) : -INFINITY;
+    const float lv = lane < ns ? __ldcg(base + lane * sstr + 129) : 0.f;
+    float4 ov[kSplitMax];
 #pragma unroll
-      for (int sp = 0; sp < kSplitMax; ++sp)
-        if (sp < ns) ov[sp] = __ldcg(reinterpret_cast<const float4 *>(base + sp * sstr) + lane);
-      const float Mx = warp_max(mv);
-      const float f = mv == -INFINITY ? 0.f : ex2_approx(mv - Mx);
-      const float Ls = warp_sum(lv * f);
-      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int sp = 0; sp < kSplitMax; ++sp)
+      if (sp < ns) ov[sp] = __ldcg(reinterpret_cast<const float4 *>(base + sp * sstr) + lane);
+    const float Mx = warp_max(mv);
+    const float f = mv == -INFINITY ? 0.f : ex2_approx(mv - Mx);
+    const float Ls = warp_sum(lv * f);
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-      for (int sp = 0; sp < kSplitMax; ++sp) {
-        if (sp < ns) {
-          const float fs = __shfl_sync(0xffffffffu, f, sp);
-          acc.x = fmaf(ov[sp].x, fs, acc.x);
-          acc.y = fmaf(ov[sp].y, fs, acc.y);
-          acc.z = fmaf(ov[sp].z, fs, acc.z);
-          acc.w = fmaf(ov[sp].w, fs, acc.w);
-        }
+    for (int sp = 0; sp < kSplitMax; ++sp) {
+      if (sp < ns) {
+        const float fs = __shfl_sync(0xffffffffu, f, sp);
+        acc.x = fmaf(ov[sp].x, fs, acc.x);
+        acc.y = fmaf(ov[sp].y, fs, acc.y);
+        acc.z = fmaf(ov[sp].z, fs, acc.z);
+        acc.w = fmaf(ov[sp].w, fs, acc.w);
       }
-      const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
-      const int grow = I.rb * rpb + r;
-      const int qi = grow / G, j = grow % G;
-      uint2 pk;
-      pk.x = pack_bf16x2(acc.x * inv, acc.y * inv);
-      pk.y = pack_bf16x2(acc.z * inv, acc.w * inv);
-      *reinterpret_cast<uint2 *>(Bt.out + ((size_t)(q0 + qi) * Bt.hq + I.kvh * G + j) * kD +
-                                 lane * 4) = pk;
     }
+    const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+    const int grow = I.rb * rpb + r;
+    const int qi = grow / G, j = grow % G;
+    uint2 pk;
+    pk.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+    pk.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+    *reinterpret_cast<uint2 *>(Bt.out + ((size_t)(q0 + qi) * Bt.hq + I.kvh * G + j) * kD +
+                               lane * 4) = pk;
   }
 }
 
@@ -1635,6 +1693,8 @@ int launch(const ipd_attn_batch *const *bs, int n, float scale, void *ws, size_t
   P.ctrl = reinterpret_cast<int *>(w + W.off_ctrl);
   P.reqinfo = reinterpret_cast<int4 *>(w + W.off_reqinfo);
   P.items = reinterpret_cast<Item *>(w + W.off_items);
+  P.merges = reinterpret_cast<int2 *>(w + W.off_merges);
+  P.merge_cap = W.merge_cap;
   P.partials = reinterpret_cast<float *>(w + W.off_partials);
   P.item_cap = W.item_cap;
   P.task_cap = W.task_cap;
@@ -1642,12 +1702,12 @@ int launch(const ipd_attn_batch *const *bs, int n, float scale, void *ws, size_t
   P.target_items = std::min(kMaxTargetItems, kTargetItemsPerSm * D.sms);
   P.n_sms = D.sms;
 
-  attn_plan_kernel<<<1, 1024, 0, stream>>>(P);
+  attn_plan_kernel<<<1, kPlanThreads, 0, stream>>>(P);
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   const int grid = std::max(1, std::min(D.sms, W.item_cap));
   attn_kernel<<<grid, kThreads, Smem::total, stream>>>(P);
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
-  attn_merge_kernel<<<8 * D.sms, 256, 0, stream>>>(P);
+  attn_merge_kernel<<<4 * D.sms, 256, 0, stream>>>(P);
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   return IPD_OK;
 }
