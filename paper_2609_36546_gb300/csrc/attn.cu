@@ -769,18 +769,26 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
       l_run *= alpha;
       return true;
     };
-    // p = 2^(s*scale - m) as a truncated bf16 pair and the truncated residual
-    float lsum = 0.f;
+    // p = 2^(s*scale - m) as a truncated bf16 pair and the truncated residual;
+    // the scaling, residual and row sum run on packed fp32 pairs
+    unsigned long long lsum2 = 0ull;  // {0.f, 0.f}
     auto exp_pairs = [&](const uint32_t (&v)[32], float moff, uint32_t *hi, uint32_t *lo) {
+      const unsigned long long sl2x2 = f2_pack(sl2, sl2), moffx2 = f2_pack(moff, moff);
 #pragma unroll
       for (int e = 0; e < 32; e += 2) {
-        const float p0 = ex2_approx(fmaf(__uint_as_float(v[e]), sl2, moff));
-        const float p1 = ex2_approx(fmaf(__uint_as_float(v[e + 1]), sl2, moff));
-        const float h0 = __uint_as_float(__float_as_uint(p0) & 0xffff0000u);
-        const float h1 = __uint_as_float(__float_as_uint(p1) & 0xffff0000u);
+        float x0, x1;
+        f2_unpack(f2_fma(f2_pack(__uint_as_float(v[e]), __uint_as_float(v[e + 1])), sl2x2, moffx2),
+                  x0, x1);
+        const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+        const unsigned long long pp = f2_pack(p0, p1);
+        const unsigned long long hh =
+            f2_pack(__uint_as_float(__float_as_uint(p0) & 0xffff0000u),
+                    __uint_as_float(__float_as_uint(p1) & 0xffff0000u));
+        float l0, l1;
+        f2_unpack(f2_sub(pp, hh), l0, l1);
         hi[e >> 1] = pack_bf16x2_trunc(p0, p1);
-        lo[e >> 1] = pack_bf16x2_trunc(p0 - h0, p1 - h1);
-        lsum += p0 + p1;
+        lo[e >> 1] = pack_bf16x2_trunc(l0, l1);
+        lsum2 = f2_add(lsum2, pp);
       }
     };
 
@@ -826,16 +834,21 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
       }
       if (!rescale(mc)) return false;
       const float moff = (!real || m_used == -INFINITY) ? -INFINITY : -m_used;
+      // four groups of 32 keys; the TMEM load of group g+1 is in flight while
+      // group g is worked on
       uint32_t ph[64];
+      uint32_t sr[2][32];
+      tc_ld_32x32b_x32(tl + col_s(b), sr[0]);
+      tc_wait_ld();
 #pragma unroll
       for (int q4 = 0; q4 < kStageKeys / 32; ++q4) {
-        uint32_t sr[32], pl[16];
-        tc_ld_32x32b_x32(tl + col_s(b) + 32 * q4, sr);
-        tc_wait_ld();
-        mask32(sr, 32 * q4);
-        exp_pairs(sr, moff, ph + 16 * q4, pl);
+        if (q4 + 1 < kStageKeys / 32) tc_ld_32x32b_x32(tl + col_s(b) + 32 * (q4 + 1), sr[(q4 + 1) & 1]);
+        uint32_t pl[16];
+        mask32(sr[q4 & 1], 32 * q4);
+        exp_pairs(sr[q4 & 1], moff, ph + 16 * q4, pl);
         // the residual overwrites S columns 16 q4 .. that this thread has already read
         tc_st_32x32b_x16(tl + col_s(b) + 16 * q4, pl);
+        if (q4 + 1 < kStageKeys / 32) tc_wait_ld();
       }
       tc_wait_st();
       if (!wait_pv_done(c - 1)) return false;
@@ -849,7 +862,11 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
         }
       }
     }
-    if (real) l_run += lsum;
+    {
+      float a0, a1;
+      f2_unpack(lsum2, a0, a1);
+      if (real) l_run += a0 + a1;
+    }
     fence_proxy_async_smem();
     tc_fence_before();
     __syncwarp();

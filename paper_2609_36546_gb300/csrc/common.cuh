@@ -295,6 +295,33 @@ IPD_DEVINL uint32_t pack_bf16x2_trunc(float lo, float hi) {
   return __byte_perm(__float_as_uint(lo), __float_as_uint(hi), 0x7632);
 }
 
+// Packed fp32 pairs (Blackwell f32x2 arithmetic): a 64-bit register holds
+// {lo, hi}; each instruction does two round-to-nearest fp32 operations.
+IPD_DEVINL unsigned long long f2_pack(float lo, float hi) {
+  unsigned long long r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+IPD_DEVINL void f2_unpack(unsigned long long v, float &lo, float &hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+IPD_DEVINL unsigned long long f2_fma(unsigned long long a, unsigned long long b,
+                                     unsigned long long c) {
+  unsigned long long d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+IPD_DEVINL unsigned long long f2_add(unsigned long long a, unsigned long long b) {
+  unsigned long long d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+IPD_DEVINL unsigned long long f2_sub(unsigned long long a, unsigned long long b) {
+  unsigned long long d;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+
 // 2^x on the special-function unit (hardware approximation, about 2 ulp).
 IPD_DEVINL float ex2_approx(float x) {
   float y;
