@@ -562,7 +562,7 @@ extern "C" int ipd_score_span(const uint16_t *logits_student, const uint16_t *lo
 // allocate device memory.  The per-row scratch that ipd_score_span takes from
 // the caller's workspace lives here in one file-scope device array, sized for
 // IPD_STATIC_MAX_TOKENS span positions.  Every GPU that loads the library
-// holds this array (about 8.5 MiB) until the process exits.
+// holds this array (about 2.1 MiB) until the process exits.
 // ---------------------------------------------------------------------------
 static __device__ __align__(256) RowOut g_static_rows[2 * kParts * IPD_STATIC_MAX_TOKENS];
 
