@@ -71,6 +71,7 @@ constexpr int kThreads = 6 * 32;
 constexpr int kTargetItemsPerSm = 4;               // items of about a quarter of an SM's share
 constexpr int kSizesPerBatch = 32;                // claim order: batch by batch, and within a
 constexpr int kSizeBuckets = IPD_MAX_BATCHES * kSizesPerBatch;  // batch the longest items first
+static_assert(kSizeBuckets % 32 == 0, "bucket prefix: whole lanes");
 constexpr int kMaxTargetItems = 4096;            // bound used for workspace sizing
 constexpr int kMinChunkPages = 16;
 constexpr int kSplitMax = 16;
@@ -95,11 +96,12 @@ struct BatchDev {
   int num_reqs, hq, hkv, group, max_pages, max_q_len, total_q, cache;
 };
 
-struct Item {
+struct __align__(16) Item {
   int b, r, kvh, rb;
   int split, n_split, page_lo, page_hi;
   int task, pbase, rows, path;  // path: kPathCc, kPathTcSplit or kPathTcFull
 };
+static_assert(sizeof(Item) == 48, "items are written as three 16-byte vectors");
 
 struct AttnParams {
   CUtensorMap tmap[2 * IPD_MAX_BATCHES];  // K and V map of every distinct cache
@@ -113,6 +115,7 @@ struct AttnParams {
   int4 *reqinfo;   // per flattened request: merge-entry offset, task offset, partial offset, n_split
   Item *items;
   int2 *merges;    // merge entries: (work-list slot of a split task's first item, 8-row group)
+  int2 *reqslot;   // per flattened request: slot offsets of its full-size and last splits
   float *partials;
   int item_cap, task_cap, merge_cap;
   long long prow_cap;
@@ -134,7 +137,7 @@ struct StageMeta {
 // host-side sizes
 // --------------------------------------------------------------------------
 struct WsLayout {
-  size_t off_ctrl, off_reqinfo, off_items, off_merges, off_partials, total;
+  size_t off_ctrl, off_reqinfo, off_reqslot, off_items, off_merges, off_partials, total;
   int item_cap, task_cap, merge_cap, total_reqs;
   long long prow_cap;
 };
@@ -210,6 +213,8 @@ WsLayout layout(const ipd_attn_batch *const *bs, int n) {
   off = align_up(off + 64, 256);
   L.off_reqinfo = off;
   off = align_up(off + (size_t)reqs * sizeof(int4), 256);
+  L.off_reqslot = off;
+  off = align_up(off + (size_t)reqs * sizeof(int2), 256);
   L.off_items = off;
   off = align_up(off + (size_t)L.item_cap * sizeof(Item), 256);
   // a split task has more pages than the chunk, and the chunk is at least
@@ -304,13 +309,13 @@ __device__ void block_scan4(int4 v, int4 &excl, int4 &tot, int4 *sh) {
 
 // Pages per split of a request with `pages` pages, for a target chunk size:
 // a whole number of stages, so only a request's last split ends mid-stage.
-__device__ __forceinline__ int split_pages(int pages, long long chunk) {
-  long long ns = (pages + chunk - 1) / chunk;
+__device__ __forceinline__ int split_pages(int pages, int chunk) {
+  int ns = (int)(((unsigned)pages + (unsigned)chunk - 1u) / (unsigned)chunk);
   if (ns > kSplitMax) ns = kSplitMax;
-  const int per = (int)((pages + ns - 1) / ns);
+  const int per = (int)(((unsigned)pages + (unsigned)ns - 1u) / (unsigned)ns);
   return (per + kStagePages - 1) / kStagePages * kStagePages;
 }
-__device__ __forceinline__ int split_count(int pages, long long chunk) {
+__device__ __forceinline__ int split_count(int pages, int chunk) {
   const int per = split_pages(pages, chunk);
   return (pages + per - 1) / per;
 }
@@ -319,11 +324,37 @@ __device__ __forceinline__ int split_count(int pages, long long chunk) {
 // are claimed first.  Streaming one cache at a time measured faster than
 // interleaving both (every CTA streams more slowly when the two pools are
 // read at once), and longest-first within a batch keeps the tail short.
-__device__ __forceinline__ int size_bucket(int b, int n_batches, int n, long long chunk) {
-  const long long top = (chunk + kStagePages - 1) / kStagePages * kStagePages;  // usual largest
-  long long k = (long long)n * (kSizesPerBatch - 1) / top;
-  if (k > kSizesPerBatch - 1) k = kSizesPerBatch - 1;
+__device__ __forceinline__ int size_bucket(int b, int n_batches, int n, int chunk) {
+  const unsigned top = (unsigned)((chunk + kStagePages - 1) / kStagePages * kStagePages);  // usual largest
+  unsigned k = (unsigned)n * (unsigned)(kSizesPerBatch - 1) / top;  // n < 2^27: no overflow
+  if (k > (unsigned)(kSizesPerBatch - 1)) k = kSizesPerBatch - 1;
   return (n_batches - 1 - b) * kSizesPerBatch + (int)k;
+}
+
+// Reserve n consecutive slots of bucket `bucket` (< 0: none) for every lane;
+// lanes asking for the same bucket share one shared-memory atomic.  All 32
+// lanes call it.  Returns the lane's first slot, relative to the bucket.
+__device__ __forceinline__ int warp_reserve(int *slots, int bucket, int n) {
+  const int lane = threadIdx.x & 31;
+  const unsigned grp = __match_any_sync(0xffffffffu, bucket);
+  const unsigned same_n = __match_any_sync(0xffffffffu, n);
+  int excl = 0, total = 0;
+  if ((grp & same_n) == grp) {  // one count for the whole group (the usual case)
+    excl = n * __popc(grp & ((1u << lane) - 1u));
+    total = n * __popc(grp);
+  } else {
+    for (unsigned m = grp; m; m &= m - 1) {
+      const int l = __ffs(m) - 1;
+      const int v = __shfl_sync(grp, n, l);
+      if (l < lane) excl += v;
+      total += v;
+    }
+  }
+  const int leader = __ffs(grp) - 1;
+  int base = 0;
+  if (lane == leader && bucket >= 0 && total > 0) base = atomicAdd(&slots[bucket], total);
+  base = __shfl_sync(grp, base, leader);
+  return base + excl;
 }
 
 // merge entries (8-row groups) of one kv head of a split request
@@ -384,8 +415,10 @@ __global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_co
     }
   }
   const long long W = block_sum<long long>(w, red);
-  long long chunk = (W + p.target_items - 1) / p.target_items;
-  if (chunk < kMinChunkPages) chunk = kMinChunkPages;
+  long long chunk_ll = (W + p.target_items - 1) / p.target_items;
+  if (chunk_ll < kMinChunkPages) chunk_ll = kMinChunkPages;
+  if (chunk_ll > (1LL << 30)) chunk_ll = 1LL << 30;
+  const int chunk = (int)chunk_ll;
 
   // per request: split count, merge-entry, task and partial-row offsets
   // (exclusive scans), and the size histogram of its items
@@ -394,6 +427,8 @@ __global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_co
     const int gi = tid + k * kPlanThreads;
     int4 cnt = make_int4(0, 0, 0, 0);
     int nsplit = 1;
+    // splits 0 .. ns-2 have `per` pages (one bucket), the last split the rest
+    int bk_main = -1, n_main = 0, bk_last = -1, n_last = 0;
     if (gi < p.total_reqs) {
       int b;
       const ReqShape s = shape_of(k, gi, b);
@@ -404,29 +439,52 @@ __global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_co
         const int tasks = hkv * s.nrb;
         cnt = make_int4(nsplit > 1 ? hkv * merge_groups(s) : 0, tasks,
                         nsplit > 1 ? nsplit * hkv * s.rows : 0, tasks * nsplit);
-        for (int sp = 0; sp < nsplit; ++sp)
-          atomicAdd(&s_slot[size_bucket(b, p.n_batches, min(s.pages, (sp + 1) * per) - sp * per, chunk)],
-                    tasks);
+        if (nsplit > 1) {
+          bk_main = size_bucket(b, p.n_batches, per, chunk);
+          n_main = (nsplit - 1) * tasks;
+        }
+        bk_last = size_bucket(b, p.n_batches, s.pages - (nsplit - 1) * per, chunk);
+        n_last = tasks;
       }
     }
+    const int off_main = warp_reserve(s_slot, bk_main, n_main);
+    const int off_last = warp_reserve(s_slot, bk_last, n_last);
+    if (gi < p.total_reqs) p.reqslot[gi] = make_int2(off_main, off_last);
     int4 ex, tot;
     block_scan4(cnt, ex, tot, sh4);
     if (gi < p.total_reqs)
       p.reqinfo[gi] = make_int4(carry.x + ex.x, carry.y + ex.y, carry.z + ex.z, nsplit);
     carry.x += tot.x; carry.y += tot.y; carry.z += tot.z; carry.w += tot.w;
   }
+  __syncthreads();
+  if (tid < 32) {
+    // bucket start slots, largest bucket first: lane l sums buckets
+    // kSizeBuckets-1-8l .. -7 (descending), then an exclusive warp scan
+    constexpr int kPer = kSizeBuckets / 32;
+    int v[kPer], sum = 0;
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+      v[i] = s_slot[kSizeBuckets - 1 - (tid * kPer + i)];
+      sum += v[i];
+    }
+    int inc = sum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, inc, o);
+      if (tid >= o) inc += y;
+    }
+    int off = inc - sum;
+#pragma unroll
+    for (int i = 0; i < kPer; ++i) {
+      s_slot[kSizeBuckets - 1 - (tid * kPer + i)] = off;
+      off += v[i];
+    }
+  }
   if (tid == 0) {
     if (carry.w > p.item_cap || carry.y > p.task_cap || carry.z > p.prow_cap ||
         carry.x > p.merge_cap) {
       ipd_set_error(&g_attn_err, IPD_DEVERR_PLAN);
       s_fail = 1;
-    }
-    // largest bucket first
-    int off = 0;
-    for (int q = kSizeBuckets - 1; q >= 0; --q) {
-      const int n = s_slot[q];
-      s_slot[q] = off;
-      off += n;
     }
     p.ctrl[0] = s_fail ? 0 : carry.w;
     p.ctrl[1] = 0;
@@ -445,28 +503,34 @@ __global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_co
     if (s.pages == 0) continue;
     const int r = gi - p.req_base[b];
     const int4 info = p.reqinfo[gi];
-    int task = info.y, mrg = info.x;
+    const int task = info.y, mrg = info.x;
     const int ns = info.w;
     const int per = split_pages(s.pages, chunk);
-    for (int kvh = 0; kvh < p.b[b].hkv; ++kvh) {
-      for (int rb = 0; rb < s.nrb; ++rb) {
-        const int rows = min(s.rpb, s.rows - rb * s.rpb);
-        const int pbase = ns > 1 ? info.z + ns * (kvh * s.rows + rb * s.rpb) : -1;
-        for (int sp = 0; sp < ns; ++sp) {
-          Item it;
-          it.b = b; it.r = r; it.kvh = kvh; it.rb = rb;
-          it.split = sp; it.n_split = ns;
-          it.page_lo = sp * per;
-          it.page_hi = min(s.pages, (sp + 1) * per);
-          it.task = task; it.pbase = pbase; it.rows = rows;
-          it.path = s.rows < kTcMinRows ? kPathCc : (rows <= kTcSplitRows ? kPathTcSplit : kPathTcFull);
-          const int slot =
-              atomicAdd(&s_slot[size_bucket(b, p.n_batches, it.page_hi - it.page_lo, chunk)], 1);
-          p.items[slot] = it;
+    const int hkv = p.b[b].hkv;
+    const int tasks = hkv * s.nrb;
+    const int2 rs = p.reqslot[gi];
+    const int base_main = ns > 1 ? s_slot[size_bucket(b, p.n_batches, per, chunk)] + rs.x : 0;
+    const int base_last =
+        s_slot[size_bucket(b, p.n_batches, s.pages - (ns - 1) * per, chunk)] + rs.y;
+    const int path = s.rows < kTcMinRows ? kPathCc : -1;
+    for (int sp = 0; sp < ns; ++sp) {
+      const int lo = sp * per, hi = min(s.pages, (sp + 1) * per);
+      int slot = sp < ns - 1 ? base_main + sp * tasks : base_last;
+      int mrg_t = mrg;
+      int task_t = task;
+      for (int kvh = 0; kvh < hkv; ++kvh) {
+        for (int rb = 0; rb < s.nrb; ++rb) {
+          const int rows = min(s.rpb, s.rows - rb * s.rpb);
+          const int pbase = ns > 1 ? info.z + ns * (kvh * s.rows + rb * s.rpb) : -1;
+          const int pth = path >= 0 ? path : (rows <= kTcSplitRows ? kPathTcSplit : kPathTcFull);
+          int4 *dst = reinterpret_cast<int4 *>(p.items + slot);
+          dst[0] = make_int4(b, r, kvh, rb);
+          dst[1] = make_int4(sp, ns, lo, hi);
+          dst[2] = make_int4(task_t++, pbase, rows, pth);
           if (ns > 1 && sp == 0)
-            for (int g8 = 0; g8 < (rows + 7) / 8; ++g8) p.merges[mrg++] = make_int2(slot, g8);
+            for (int g8 = 0; g8 < (rows + 7) / 8; ++g8) p.merges[mrg_t++] = make_int2(slot, g8);
+          ++slot;
         }
-        ++task;
       }
     }
   }
@@ -1710,6 +1774,7 @@ int launch(const ipd_attn_batch *const *bs, int n, float scale, void *ws, size_t
   P.ctrl = reinterpret_cast<int *>(w + W.off_ctrl);
   P.reqinfo = reinterpret_cast<int4 *>(w + W.off_reqinfo);
   P.items = reinterpret_cast<Item *>(w + W.off_items);
+  P.reqslot = reinterpret_cast<int2 *>(w + W.off_reqslot);
   P.merges = reinterpret_cast<int2 *>(w + W.off_merges);
   P.merge_cap = W.merge_cap;
   P.partials = reinterpret_cast<float *>(w + W.off_partials);
