@@ -362,15 +362,34 @@ def run_gpu(args):
     t_end.record(stream)
     torch.cuda.synchronize()
     _barrier(world)
-    clocks = sampler.stop() if sampler else None
-    el_ms = t_start.elapsed_time(t_end)
+    el_direct_ms = t_start.elapsed_time(t_end)
     attn_ms = statistics.mean(e[0].elapsed_time(e[1]) for e in ev)
     score_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in ev)
     loss_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in ev)
+
+    # ---- timed region for `value`: the same K steps replayed from a CUDA graph
+    # of one step (same kernels and buffers, no per-call host work) ----
+    graph = step.capture()
+    torch.cuda.synchronize()
+    g_start = torch.cuda.Event(enable_timing=True)
+    g_end = torch.cuda.Event(enable_timing=True)
+    _barrier(world)
+    torch.cuda.synchronize()
+    g_start.record(stream)
+    for i in range(K):
+        graph.replay()
+    g_end.record(stream)
+    torch.cuda.synchronize()
+    _barrier(world)
+    clocks = sampler.stop() if sampler else None
+    if ipd.device_error() != 0:
+        raise RuntimeError("device-side check failed during the timed steps")
+    el_ms = g_start.elapsed_time(g_end)
     el_max = _max_over_ranks(el_ms, world)
     tokens_all = _sum_over_ranks(float(T_tok * K), world)
     value = tokens_all / (el_max / 1e3)
     ms_step = el_max / K
+    ms_step_direct = _max_over_ranks(el_direct_ms, world) / K
 
     # ---- end to end through host buffers ----
     e2e = run_e2e(step, w, min(K, args.e2e_steps), stream, world)
@@ -399,6 +418,9 @@ def run_gpu(args):
                      "frac_alg_of_measured": step_alg / (ms_step / 1e3) / 1e9 / peak,
                      "frac_full_of_nominal_8tbs": step_full / (ms_step / 1e3) / 1e9 / 8000.0},
         "calls_ms": {"verify_attn": attn_ms, "score_span": score_ms, "split_loss": loss_ms},
+        "ms_per_step_direct_calls": ms_step_direct,
+        "timing": "value: K steps replayed from a CUDA graph of one step; calls_ms and the "
+                  "roofline: the same K steps issued call by call with CUDA events around each call",
         "acceptance": {"coverage_rate": accept_rate, "emitted_tokens_per_step": emitted},
         "e2e": e2e, "clocks": clocks,
         "gpu_launches": LAUNCHES_PER_STEP * K,

@@ -93,6 +93,31 @@ def test_outputs_are_deterministic(lib):
     assert torch.equal(o8, step.out8)
 
 
+def test_graph_replay_equals_direct_calls(lib):
+    """A step captured with VerifyStep.capture() and replayed gives the same
+    bits as the three calls issued directly (outputs cleared in between)."""
+    spec = S.small_spec(n_req=7, ctx=(100, 2500), span=(1, 16))
+    w, step = _run(spec, 37)
+    first = {k: v.clone() for k, v in step.score.items()}
+    outs = [b.out.clone() for _, b, _, _ in step.batches]
+    o8 = step.out8.clone()
+    graph = step.capture()
+    for _ in range(2):
+        for v in step.score.values():
+            v.zero_()
+        for _, b, _, _ in step.batches:
+            b.out.zero_()
+        step.out8.zero_()
+        graph.replay()
+        torch.cuda.synchronize()
+        for k, v in step.score.items():
+            assert torch.equal(first[k].view(torch.uint8), v.view(torch.uint8)), k
+        for a, (_, b, _, _) in zip(outs, step.batches):
+            assert torch.equal(a.view(torch.int16), b.out.view(torch.int16))
+        assert torch.equal(o8, step.out8)
+    assert lib.device_error() == 0
+
+
 def test_decode_alone_equals_colaunched(lib):
     spec = S.small_spec(n_req=6, ctx=(10, 900))
     w, step = _run(spec, 41)
