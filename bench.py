@@ -369,7 +369,7 @@ def run_gpu(args):
 
     # ---- timed region for `value`: the same K steps replayed from a CUDA graph
     # of one step (same kernels and buffers, no per-call host work) ----
-    graph = step.capture()
+    graph = step.capture(overlap=True)
     torch.cuda.synchronize()
     g_start = torch.cuda.Event(enable_timing=True)
     g_end = torch.cuda.Event(enable_timing=True)
@@ -419,8 +419,9 @@ def run_gpu(args):
                      "frac_full_of_nominal_8tbs": step_full / (ms_step / 1e3) / 1e9 / 8000.0},
         "calls_ms": {"verify_attn": attn_ms, "score_span": score_ms, "split_loss": loss_ms},
         "ms_per_step_direct_calls": ms_step_direct,
-        "timing": "value: K steps replayed from a CUDA graph of one step; calls_ms and the "
-                  "roofline: the same K steps issued call by call with CUDA events around each call",
+        "timing": "value: K steps replayed from a CUDA graph of one step (the vocabulary pass "
+                  "on a forked stream, joined before the loss); calls_ms and the roofline: the "
+                  "same K steps issued call by call on one stream, CUDA events around each call",
         "acceptance": {"coverage_rate": accept_rate, "emitted_tokens_per_step": emitted},
         "e2e": e2e, "clocks": clocks,
         "gpu_launches": LAUNCHES_PER_STEP * K,

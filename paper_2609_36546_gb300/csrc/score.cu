@@ -145,7 +145,8 @@ __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
   volatile unsigned long long *vtheta = &s_theta;
   unsigned long long *buf = s_buf[warp];
 
-  float m = -INFINITY, s = 0.f;
+  float m = -INFINITY;
+  unsigned long long s2 = 0ull;     // running sum of exp(l - m), as a packed pair
   unsigned long long theta = 0ull;  // K-th best key this warp holds (0: fewer than K)
   int nb = 0;                       // keys in the warp's buffer
   int qn = 0;                       // vectors in the warp's queue
@@ -254,18 +255,24 @@ __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
     for (int u = 0; u < U; ++u) vmx[u] = bf16x8_max(raw[u]);
     const float bmax = fmaxf(fmaxf(vmx[0], vmx[1]), fmaxf(vmx[2], vmx[3]));
     if (bmax > m) {
-      s *= ex2_approx((m - bmax) * kLog2e);
+      const float f = ex2_approx((m - bmax) * kLog2e);
+      float s0, s1;
+      f2_unpack(s2, s0, s1);
+      s2 = f2_pack(s0 * f, s1 * f);
       m = bmax;
     }
     if (m != -INFINITY) {
-      const float ml = -m * kLog2e;
+      // the two halves of each bf16 pair run as one packed fp32 pair
+      const unsigned long long l2e = f2_pack(kLog2e, kLog2e);
+      const unsigned long long ml = f2_pack(-m * kLog2e, -m * kLog2e);
 #pragma unroll
       for (int u = 0; u < U; ++u) {
         const uint32_t w[4] = {raw[u].x, raw[u].y, raw[u].z, raw[u].w};
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-          s += ex2_approx(fmaf(bf16lo(w[q]), kLog2e, ml));
-          s += ex2_approx(fmaf(bf16hi(w[q]), kLog2e, ml));
+          float x0, x1;
+          f2_unpack(f2_fma(f2_pack(bf16lo(w[q]), bf16hi(w[q])), l2e, ml), x0, x1);
+          s2 = f2_add(s2, f2_pack(ex2_approx(x0), ex2_approx(x1)));
         }
       }
     }
@@ -308,6 +315,12 @@ __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
   // buffers hold distinct keys.
 
   // block merge of the log-sum-exp
+  float s;
+  {
+    float s0, s1;
+    f2_unpack(s2, s0, s1);
+    s = s0 + s1;
+  }
   float wm = warp_max(m);
   float ws = (m == -INFINITY) ? 0.f : s * exp2f((m - wm) * kLog2e);
   if (wm == -INFINITY) ws = 0.f;

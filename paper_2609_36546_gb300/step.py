@@ -121,12 +121,28 @@ class VerifyStep:
         ipd.split_loss(s["kl_rev"], s["kl_fwd"], s["source"], self.cu_span, s["n_emit"],
                        self.resp_len, self.agg_mode, self.dir_mode, self.out8, stream)
 
-    def run(self, stream=None):
-        self.run_attention(stream)
-        self.run_score(stream)
-        self.run_loss(stream)
+    def run(self, stream=None, overlap: bool = False):
+        """The step's three calls.  The vocabulary pass reads only the step's
+        inputs (logits, tokens, request metadata), not the attention outputs,
+        so with overlap=True it runs on a side stream forked from `stream`
+        and joined before the loss: its CTAs take the SMs the planner and
+        the attention kernel's last CTAs leave idle."""
+        if not overlap:
+            self.run_attention(stream)
+            self.run_score(stream)
+            self.run_loss(stream)
+            return
+        main = stream if stream is not None else torch.cuda.current_stream(self.device)
+        if getattr(self, "_side", None) is None:
+            self._side = torch.cuda.Stream(device=self.device)
+        side = self._side
+        side.wait_stream(main)
+        self.run_attention(main)
+        self.run_score(side)
+        main.wait_stream(side)
+        self.run_loss(main)
 
-    def capture(self, warmup: int = 2) -> "torch.cuda.CUDAGraph":
+    def capture(self, warmup: int = 2, overlap: bool = False) -> "torch.cuda.CUDAGraph":
         """Record one step (the three calls, six kernels) as a CUDA graph.
 
         The calls allocate nothing and never synchronise, so the whole step
@@ -137,11 +153,11 @@ class VerifyStep:
         side.wait_stream(torch.cuda.current_stream(self.device))
         with torch.cuda.stream(side):
             for _ in range(warmup):
-                self.run()
+                self.run(overlap=overlap)
         torch.cuda.current_stream(self.device).wait_stream(side)
         graph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(graph):
-            self.run()
+            self.run(overlap=overlap)
         return graph
 
     # -- bytes the step must move (algorithmic) --------------------------------

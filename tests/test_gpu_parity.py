@@ -93,15 +93,17 @@ def test_outputs_are_deterministic(lib):
     assert torch.equal(o8, step.out8)
 
 
-def test_graph_replay_equals_direct_calls(lib):
-    """A step captured with VerifyStep.capture() and replayed gives the same
-    bits as the three calls issued directly (outputs cleared in between)."""
+@pytest.mark.parametrize("overlap", [False, True])
+def test_graph_replay_equals_direct_calls(lib, overlap):
+    """A step captured with VerifyStep.capture() (vocabulary pass on the main
+    stream or on a forked side stream) and replayed gives the same bits as
+    the three calls issued directly (outputs cleared in between)."""
     spec = S.small_spec(n_req=7, ctx=(100, 2500), span=(1, 16))
     w, step = _run(spec, 37)
     first = {k: v.clone() for k, v in step.score.items()}
     outs = [b.out.clone() for _, b, _, _ in step.batches]
     o8 = step.out8.clone()
-    graph = step.capture()
+    graph = step.capture(overlap=overlap)
     for _ in range(2):
         for v in step.score.values():
             v.zero_()
