@@ -385,6 +385,15 @@ def run_gpu(args):
     if ipd.device_error() != 0:
         raise RuntimeError("device-side check failed during the timed steps")
     el_ms = g_start.elapsed_time(g_end)
+    # the same graph with every call on one stream (no overlap), for reference
+    graph1 = step.capture(overlap=False)
+    torch.cuda.synchronize()
+    g_start.record(stream)
+    for i in range(K):
+        graph1.replay()
+    g_end.record(stream)
+    torch.cuda.synchronize()
+    ms_step_one_stream = _max_over_ranks(g_start.elapsed_time(g_end), world) / K
     el_max = _max_over_ranks(el_ms, world)
     tokens_all = _sum_over_ranks(float(T_tok * K), world)
     value = tokens_all / (el_max / 1e3)
@@ -418,6 +427,7 @@ def run_gpu(args):
                      "frac_alg_of_measured": step_alg / (ms_step / 1e3) / 1e9 / peak,
                      "frac_full_of_nominal_8tbs": step_full / (ms_step / 1e3) / 1e9 / 8000.0},
         "calls_ms": {"verify_attn": attn_ms, "score_span": score_ms, "split_loss": loss_ms},
+        "ms_per_step_one_stream_graph": ms_step_one_stream,
         "ms_per_step_direct_calls": ms_step_direct,
         "timing": "value: K steps replayed from a CUDA graph of one step (the vocabulary pass "
                   "on a forked stream, joined before the loss); calls_ms and the roofline: the "

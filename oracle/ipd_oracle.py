@@ -140,25 +140,79 @@ def topk_kl(l_pi: np.ndarray, l_q: np.ndarray, K: int):
     return kl_rev, kl_fwd, S
 
 
-def score_position(l_s: np.ndarray, l_t: np.ndarray, x: int, driver: int, K: int) -> dict:
+def entropy(l: np.ndarray) -> float:
+    """Shannon entropy (nats) of softmax(l) over the whole vocabulary,
+    log Z - sum_v p_v l_v (the per-position entropy of Sec. 3.2, Fig.
+    teacher_unanchoring)."""
+    lz = log_partition(l)
+    p = np.exp(l - lz)
+    return float(lz - np.dot(p, l))
+
+
+def topk_overlap(l_pi: np.ndarray, l_q: np.ndarray, K: int) -> float:
+    """Top-K overlap ratio |S^pi intersect S^q| / K (Sec. 4.2, main results)."""
+    return len(set(topk(l_pi, K).tolist()) & set(topk(l_q, K).tolist())) / K
+
+
+def full_kl(l_pi: np.ndarray, l_q: np.ndarray):
+    """Full-vocabulary KL of Eq. (full_vocab_opd) in both directions:
+    (KL(pi || q), KL(q || pi)), each sum_v p(v) (log p(v) - log p'(v))."""
+    lp = l_pi - log_partition(l_pi)
+    lq = l_q - log_partition(l_q)
+    p, q = np.exp(lp), np.exp(lq)
+    return float(np.sum(p * (lp - lq))), float(np.sum(q * (lq - lp)))
+
+
+# Takeover / handback rules (Sec. 3.2.1: IPD admits other rules than top-K
+# coverage, possibly different for takeover and handback; an entropy threshold
+# on either model is the paper's example, and SKD is top-K takeover with a
+# fixed one-token handback).  A span proposed by the student is governed by
+# the takeover rule (its predicate true = accept), a span proposed by the
+# teacher by the handback rule (true = hand back).
+RULE_TOPK, RULE_ENTROPY_S, RULE_ENTROPY_T, RULE_ALWAYS, RULE_NEVER = 0, 1, 2, 3, 4
+
+
+def rule_predicate(rule: int, tau: float, l_s: np.ndarray, l_t: np.ndarray, x: int, driver: int,
+                   K: int):
+    """(predicate, margin) of a rule at one position.  The margin is the signed
+    distance of the decision from its threshold, >= 0 when the predicate holds
+    except for exact top-K ties, which the token-id order decides."""
+    if rule == RULE_TOPK:
+        ver = l_t if driver == 0 else l_s  # the verifier's row
+        return covered(ver, x, K), margin(ver, x, K)
+    if rule in (RULE_ENTROPY_S, RULE_ENTROPY_T):
+        h = entropy(l_s if rule == RULE_ENTROPY_S else l_t)
+        return h <= tau, tau - h
+    if rule == RULE_ALWAYS:
+        return True, np.inf
+    if rule == RULE_NEVER:
+        return False, -np.inf
+    raise ValueError(rule)
+
+
+def score_position(l_s: np.ndarray, l_t: np.ndarray, x: int, driver: int, K: int,
+                   rule: int = RULE_TOPK, tau: float = 0.0) -> dict:
     """All per-token quantities of one span position.
 
     l_s, l_t: fp64 logits of the student (pi) and teacher (q) at this position;
     x: the proposed token; driver 0 = student proposes (teacher verifies),
-    1 = teacher proposes (student verifies)."""
+    1 = teacher proposes (student verifies); rule, tau: the rule governing
+    the span (takeover rule for driver 0, handback rule for driver 1)."""
     logZ_s = log_partition(l_s)
     logZ_t = log_partition(l_t)
     logp_s = float(l_s[x] - logZ_s)
     logp_t = float(l_t[x] - logZ_t)
     kl_rev, kl_fwd, _ = topk_kl(l_s, l_t, K)
-    ver = l_t if driver == 0 else l_s
+    cov, mar = rule_predicate(rule, tau, l_s, l_t, x, driver, K)
     return dict(
         logp_s=logp_s, logp_t=logp_t,
         # token-level teacher feedback: the per-token reward -l_hat^sample =
         # log q(x) - log pi(x) (Eq. sampled_token_opd and App. B.1)
         feedback=logp_t - logp_s,
         kl_rev=kl_rev, kl_fwd=kl_fwd,
-        covered=covered(ver, x, K), margin=margin(ver, x, K))
+        covered=cov, margin=mar,
+        entropy_s=entropy(l_s), entropy_t=entropy(l_t),
+        topk_overlap=topk_overlap(l_s, l_t, K))
 
 
 def verdict(cov, tokens, driver: int, prefix_len: int, eos_id: int = -1) -> dict:
@@ -207,16 +261,20 @@ def verdict(cov, tokens, driver: int, prefix_len: int, eos_id: int = -1) -> dict
                 new_len=prefix_len + n_emit, done=done, source=source)
 
 
+POS_FIELDS = ("logp_s", "logp_t", "feedback", "kl_rev", "kl_fwd", "margin", "entropy_s",
+              "entropy_t", "topk_overlap")
+
+
 def score_span(logits_s_bits, logits_t_bits, tokens, cu_span, driver, prefix_len, K, eos_id=-1,
-               requests=None) -> dict:
+               requests=None, takeover_rule=RULE_TOPK, handback_rule=RULE_TOPK,
+               takeover_tau=0.0, handback_tau=0.0) -> dict:
     """The whole vocabulary pass + verdict for the requests in ``requests``
     (default: all).  Per-token arrays are returned in the flat span order, with
     NaN / -1 at positions of requests that were not evaluated."""
     T = int(cu_span[-1])
     R = len(cu_span) - 1
     reqs = range(R) if requests is None else requests
-    out = {name: np.full(T, np.nan) for name in
-           ("logp_s", "logp_t", "feedback", "kl_rev", "kl_fwd", "margin")}
+    out = {name: np.full(T, np.nan) for name in POS_FIELDS}
     out["covered"] = np.full(T, -1, dtype=np.int64)
     out["source"] = np.full(T, -1, dtype=np.int64)
     for name in ("first_trans", "n_emit", "next_driver", "new_len", "done"):
@@ -224,10 +282,12 @@ def score_span(logits_s_bits, logits_t_bits, tokens, cu_span, driver, prefix_len
     for r in reqs:
         t0, t1 = int(cu_span[r]), int(cu_span[r + 1])
         cov = []
+        d = int(driver[r])
+        rule, tau = (takeover_rule, takeover_tau) if d == 0 else (handback_rule, handback_tau)
         for t in range(t0, t1):
             pos = score_position(bf16_to_f64(logits_s_bits[t]), bf16_to_f64(logits_t_bits[t]),
-                                 int(tokens[t]), int(driver[r]), K)
-            for name in ("logp_s", "logp_t", "feedback", "kl_rev", "kl_fwd", "margin"):
+                                 int(tokens[t]), d, K, rule, tau)
+            for name in POS_FIELDS:
                 out[name][t] = pos[name]
             out["covered"][t] = int(pos["covered"])
             cov.append(pos["covered"])

@@ -411,3 +411,149 @@ def test_planted_mistakes_are_caught():
     a = _bf16_round(RNG.normal(size=40)); b = _bf16_round(RNG.normal(size=40) * 3)
     r, f, S = O.topk_kl(a, b, 4)
     assert abs(f - scipy.stats.entropy(scipy.special.softmax(a[S]), scipy.special.softmax(b[S]))) > 1e-6
+
+
+# ---------------------------------------------------------------------------
+# vocabulary-pass by-products: entropy, top-K overlap, full-vocabulary KL
+# ---------------------------------------------------------------------------
+def test_entropy_against_scipy_closed_forms_and_shift():
+    for V in (2, 17, 4096):
+        l = _bf16_round(RNG.normal(size=V) * 3)
+        ref = scipy.stats.entropy(scipy.special.softmax(l))  # library, natural log
+        assert abs(O.entropy(l) - ref) < 1e-10
+        assert abs(O.entropy(l + 5.0) - O.entropy(l)) < 1e-10  # shift invariance
+    # uniform row: log V exactly
+    assert abs(O.entropy(np.zeros(1000)) - math.log(1000)) < 1e-12
+    # two-point closed form: p = sigmoid(a - b), H = -p ln p - (1-p) ln(1-p)
+    a, b = 1.75, -0.5
+    p = 1.0 / (1.0 + math.exp(b - a))
+    assert abs(O.entropy(np.array([a, b])) - (-p * math.log(p) - (1 - p) * math.log(1 - p))) < 1e-12
+    # a near-one-hot row has entropy near 0
+    assert O.entropy(np.array([60.0] + [0.0] * 50)) < 1e-20
+
+
+def _brute_overlap(a, b, K):
+    sa = sorted(range(len(a)), key=lambda i: (-a[i], i))[:K]
+    sb = sorted(range(len(b)), key=lambda i: (-b[i], i))[:K]
+    return len(set(sa) & set(sb)) / K
+
+
+def test_topk_overlap_brute_force_and_extremes():
+    for K in (1, 4, 16):
+        for quantum in (0.0, 0.5):
+            a = RNG.normal(size=64) * 2; b = a + RNG.normal(size=64)
+            if quantum:
+                a = np.round(a / quantum) * quantum; b = np.round(b / quantum) * quantum
+            a, b = _bf16_round(a), _bf16_round(b)
+            assert O.topk_overlap(a, b, K) == _brute_overlap(a, b, K)
+        a = _bf16_round(RNG.normal(size=64))
+        assert O.topk_overlap(a, a, K) == 1.0
+        assert O.topk_overlap(a, -a, K) == 0.0  # reversed order: supports disjoint (2K <= 64)
+
+
+def test_full_kl_against_scipy_and_invariants():
+    for V in (3, 100, 4096):
+        a = _bf16_round(RNG.normal(size=V) * 2); b = _bf16_round(RNG.normal(size=V) * 2)
+        pa, pb = scipy.special.softmax(a), scipy.special.softmax(b)
+        rev, fwd = O.full_kl(a, b)
+        assert abs(rev - scipy.special.rel_entr(pa, pb).sum()) < 1e-10
+        assert abs(fwd - scipy.special.rel_entr(pb, pa).sum()) < 1e-10
+        assert rev >= 0 and fwd >= 0
+        assert O.full_kl(b, a) == pytest.approx((fwd, rev), abs=1e-12)
+        assert O.full_kl(a, a) == (0.0, 0.0)
+    # two-token closed form: KL of Bernoulli(p) against Bernoulli(q)
+    p = 1 / (1 + math.exp(-1.0)); q = 1 / (1 + math.exp(-(-0.5)))
+    rev, _ = O.full_kl(np.array([1.0, 0.0]), np.array([-0.5, 0.0]))
+    assert abs(rev - (p * math.log(p / q) + (1 - p) * math.log((1 - p) / (1 - q)))) < 1e-12
+    # the full-vocabulary KL equals the top-K KL when K = V (support = everything)
+    a = _bf16_round(RNG.normal(size=12)); b = _bf16_round(RNG.normal(size=12))
+    r, f, _ = O.topk_kl(a, b, 12)
+    assert O.full_kl(a, b) == pytest.approx((r, f), abs=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# takeover / handback rules
+# ---------------------------------------------------------------------------
+def _span(k, V=32, seed=0):
+    g = np.random.default_rng(seed)
+    ls = _bf16_round(g.normal(size=(k, V)) * 2)
+    lt = _bf16_round(g.normal(size=(k, V)) * 2)
+    toks = g.integers(0, V, size=k)
+    return ls, lt, toks
+
+
+def _run_rules(ls, lt, toks, driver, **kw):
+    k = len(toks)
+    to_bits = lambda x: O.f64_to_bf16(x)
+    return O.score_span(to_bits(ls), to_bits(lt), toks, np.array([0, k]), np.array([driver]),
+                        np.array([10]), 4, **kw)
+
+
+def test_always_takeover_is_a_pure_student_rollout():
+    # OPD as a special case: the student's span is accepted whole
+    ls, lt, toks = _span(9)
+    o = _run_rules(ls, lt, toks, 0, takeover_rule=O.RULE_ALWAYS)
+    assert o["n_emit"][0] == 9 and o["next_driver"][0] == 0 and o["first_trans"][0] == 9
+    assert (o["source"] == O.SRC_STUDENT).all()
+
+
+def test_skd_handback_after_one_teacher_token():
+    # SKD: top-K takeover, fixed one-token handback
+    for seed in range(5):
+        ls, lt, toks = _span(7, seed=seed)
+        o = _run_rules(ls, lt, toks, 1, handback_rule=O.RULE_ALWAYS)
+        assert o["n_emit"][0] == 1 and o["first_trans"][0] == 0 and o["next_driver"][0] == 0
+        assert o["source"][0] == O.SRC_TEACHER and (o["source"][1:] == O.SRC_DISCARDED).all()
+        # the takeover side is unchanged: student spans still follow top-K coverage
+        a = _run_rules(ls, lt, toks, 0, handback_rule=O.RULE_ALWAYS)
+        b = _run_rules(ls, lt, toks, 0)
+        assert a["n_emit"][0] == b["n_emit"][0] and (a["source"] == b["source"]).all()
+
+
+def test_never_handback_keeps_the_teacher_driving():
+    ls, lt, toks = _span(6)
+    o = _run_rules(ls, lt, toks, 1, handback_rule=O.RULE_NEVER)
+    assert o["n_emit"][0] == 6 and o["next_driver"][0] == 1 and (o["source"] == O.SRC_TEACHER).all()
+
+
+def test_entropy_rules_follow_the_threshold():
+    ls, lt, toks = _span(8, V=64, seed=3)
+    hs = [scipy.stats.entropy(scipy.special.softmax(r)) for r in ls]
+    ht = [scipy.stats.entropy(scipy.special.softmax(r)) for r in lt]
+    for tau in (-np.inf, float(np.median(hs)), np.inf):
+        o = _run_rules(ls, lt, toks, 0, takeover_rule=O.RULE_ENTROPY_S, takeover_tau=tau)
+        pred = [h <= tau for h in hs]
+        n = next((i for i, c in enumerate(pred) if not c), 8)  # first uncovered = takeover
+        assert o["n_emit"][0] == n and o["first_trans"][0] == n
+        assert (o["covered"] == np.array(pred, dtype=np.int64)).all()
+        assert np.allclose(o["margin"], tau - np.array(hs), equal_nan=True) or not np.isfinite(tau)
+    tau = float(np.median(ht))
+    o = _run_rules(ls, lt, toks, 1, handback_rule=O.RULE_ENTROPY_T, handback_tau=tau)
+    pred = [h <= tau for h in ht]
+    i = next((i for i, c in enumerate(pred) if c), None)  # first covered = handback
+    assert o["n_emit"][0] == (8 if i is None else i + 1)
+    assert o["next_driver"][0] == (1 if i is None else 0)
+    # entropy outputs are the full-vocabulary entropies of both rows
+    assert np.allclose(o["entropy_s"], hs, atol=1e-10) and np.allclose(o["entropy_t"], ht, atol=1e-10)
+
+
+def test_topk_rule_is_the_default():
+    ls, lt, toks = _span(7, seed=9)
+    a = _run_rules(ls, lt, toks, 0)
+    b = _run_rules(ls, lt, toks, 0, takeover_rule=O.RULE_TOPK, handback_rule=O.RULE_TOPK)
+    for name in ("covered", "source", "n_emit", "first_trans", "next_driver"):
+        assert (a[name] == b[name]).all()
+
+
+def test_planted_rule_mistakes_are_caught():
+    # a takeover on the teacher's entropy instead of the student's changes decisions
+    ls, lt, toks = _span(8, V=64, seed=3)
+    hs = [scipy.stats.entropy(scipy.special.softmax(r)) for r in ls]
+    tau = float(np.median(hs))
+    good = _run_rules(ls, lt, toks, 0, takeover_rule=O.RULE_ENTROPY_S, takeover_tau=tau)
+    bad = _run_rules(ls, lt, toks, 0, takeover_rule=O.RULE_ENTROPY_T, takeover_tau=tau)
+    assert (good["covered"] != bad["covered"]).any()
+    # an entropy with the wrong sign of the mean term differs from scipy
+    l = _bf16_round(RNG.normal(size=50) * 2)
+    lz = O.log_partition(l); p = np.exp(l - lz)
+    assert abs((lz + np.dot(p, l)) - scipy.stats.entropy(p)) > 1e-3
