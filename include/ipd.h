@@ -191,6 +191,59 @@ int ipd_score_span(const uint16_t *logits_student, const uint16_t *logits_teache
                    int32_t *new_len, uint8_t *done,
                    void *workspace, size_t workspace_bytes, ipd_stream_t stream);
 
+/* Takeover / handback rules (Sec. 3.2.1: top-K coverage is IPD's rule, but the
+ * framework admits others, possibly different for takeover and handback, for
+ * example a threshold on the entropy of either model; SKD is top-K takeover
+ * with a fixed one-token handback).  A rule is a per-position predicate:
+ * under the takeover rule (student-proposed spans) true = accept the student
+ * token, under the handback rule (teacher-proposed spans) true = hand back
+ * after this teacher token. */
+#define IPD_RULE_TOPK 0      /* the proposed token is in the verifier's Top_K */
+#define IPD_RULE_ENTROPY_S 1 /* H(pi_t) <= tau (student's full-vocabulary entropy, nats) */
+#define IPD_RULE_ENTROPY_T 2 /* H(q_t) <= tau (teacher's) */
+#define IPD_RULE_ALWAYS 3    /* true: OPD as a takeover rule, SKD's handback */
+#define IPD_RULE_NEVER 4     /* false: the teacher keeps driving, as a handback rule */
+
+/* Options and optional outputs of ipd_score_span_ex. */
+typedef struct {
+  int takeover_rule;   /* IPD_RULE_*: governs spans with driver 0 */
+  int handback_rule;   /* IPD_RULE_*: governs spans with driver 1 */
+  float takeover_tau;  /* threshold of the entropy rules, nats */
+  float handback_tau;
+  float *entropy_s;    /* [total_tokens] H(pi_t) over the full vocabulary, or NULL */
+  float *entropy_t;    /* [total_tokens] H(q_t), or NULL */
+  float *topk_overlap; /* [total_tokens] |Top_K(pi_t) n Top_K(q_t)| / K (Sec. 4.2), or NULL */
+} ipd_score_ext;
+
+/* ipd_score_span with selectable rules and by-products.  ext == NULL is the
+ * default (top-K coverage both ways, no extra outputs) and is exactly
+ * ipd_score_span.  With other rules, `covered` holds the governing rule's
+ * predicate and `margin` its signed distance from the threshold (tau - H for
+ * the entropy rules, +inf / -inf for ALWAYS / NEVER); the verdict applies
+ * Eq. (ipd_state_transition) with that predicate in place of coverage.
+ * Returns IPD_ERR_INVALID_ARG for an unknown rule or a NaN threshold. */
+int ipd_score_span_ex(const uint16_t *logits_student, const uint16_t *logits_teacher,
+                      const int32_t *tokens, const int32_t *cu_span, const uint8_t *driver,
+                      const int32_t *prefix_len, int num_reqs, int total_tokens, int vocab,
+                      int K, int eos_id,
+                      float *logp_s, float *logp_t, float *feedback, float *kl_rev,
+                      float *kl_fwd, uint8_t *covered, float *margin, uint8_t *source,
+                      int32_t *first_trans, int32_t *n_emit, uint8_t *next_driver,
+                      int32_t *new_len, uint8_t *done, const ipd_score_ext *ext,
+                      void *workspace, size_t workspace_bytes, ipd_stream_t stream);
+
+/* Full-vocabulary KL of Eq. (full_vocab_opd) at every span position, in both
+ * directions: kl_rev_full[t] = KL(pi_t || q_t) = sum_v pi(v) (log pi(v) -
+ * log q(v)) and kl_fwd_full[t] = KL(q_t || pi_t).  A by-product for
+ * monitoring (the quantity top-K OPD approximates, Sec. 3.1); one read of both
+ * logits rows per position.  logits_* as in ipd_score_span; outputs
+ * [total_tokens] fp32 device arrays.  No workspace.  Returns
+ * IPD_ERR_UNSUPPORTED unless vocab is a positive multiple of 8, and
+ * IPD_ERR_INVALID_ARG for NULL or misaligned (16-byte) pointers. */
+int ipd_full_kl(const uint16_t *logits_student, const uint16_t *logits_teacher,
+                int total_tokens, int vocab, float *kl_rev_full, float *kl_fwd_full,
+                ipd_stream_t stream);
+
 /* ipd_score_span for callers that cannot allocate device memory.
  *
  * No counterpart in the paper: this is a calling convention of the library.

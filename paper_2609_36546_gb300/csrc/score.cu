@@ -32,7 +32,8 @@ constexpr int kBuf = 64;     // per-warp candidate buffer: up to 32 kept keys + 
 struct RowOut {
   float m;  // maximum logit of the part (-inf if the part is empty)
   float s;  // sum over the part of exp(l - m)
-  int pad[2];
+  float u;  // sum over the part of exp(l - m) * l (entropy; 0 unless it was asked for)
+  int pad;
   unsigned long long keys[IPD_MAX_K];  // the part's best keys, best first, 0 past the end
 };
 
@@ -123,6 +124,7 @@ __device__ __forceinline__ int count_greater32(const unsigned long long *list, u
 // maximum reaches th's value go to a per-warp queue; 32 queued vectors are
 // examined at once, one per lane, and keys above th go to the warp's buffer,
 // which is cut back to its best K (by rank) whenever it fills.
+template <bool kEntropy>  // also accumulate sum exp(l - m) l (entropies / entropy rules)
 __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
     const uint16_t *__restrict__ ls, const uint16_t *__restrict__ lt, int vocab, int K,
     RowOut *__restrict__ out) {
@@ -131,7 +133,7 @@ __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
   __shared__ unsigned long long s_buf[kRowWarps][kBuf];
   __shared__ uint4 s_qraw[kRowWarps][kQueue];
   __shared__ int s_qidx[kRowWarps][kQueue];
-  __shared__ float s_m[kRowWarps], s_s[kRowWarps];
+  __shared__ float s_m[kRowWarps], s_s[kRowWarps], s_u[kRowWarps];
 
   const int row_id = blockIdx.x / kParts, part = blockIdx.x % kParts;
   const int t = row_id >> 1, model = row_id & 1;
@@ -147,6 +149,7 @@ __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
 
   float m = -INFINITY;
   unsigned long long s2 = 0ull;     // running sum of exp(l - m), as a packed pair
+  unsigned long long u2 = 0ull;     // running sum of exp(l - m) * l, as a packed pair
   unsigned long long theta = 0ull;  // K-th best key this warp holds (0: fewer than K)
   int nb = 0;                       // keys in the warp's buffer
   int qn = 0;                       // vectors in the warp's queue
@@ -256,9 +259,11 @@ __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
     const float bmax = fmaxf(fmaxf(vmx[0], vmx[1]), fmaxf(vmx[2], vmx[3]));
     if (bmax > m) {
       const float f = ex2_approx((m - bmax) * kLog2e);
-      float s0, s1;
+      float s0, s1, u0, u1;
       f2_unpack(s2, s0, s1);
+      f2_unpack(u2, u0, u1);
       s2 = f2_pack(s0 * f, s1 * f);
+      if (kEntropy) u2 = f2_pack(u0 * f, u1 * f);
       m = bmax;
     }
     if (m != -INFINITY) {
@@ -271,8 +276,11 @@ __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
           float x0, x1;
-          f2_unpack(f2_fma(f2_pack(bf16lo(w[q]), bf16hi(w[q])), l2e, ml), x0, x1);
-          s2 = f2_add(s2, f2_pack(ex2_approx(x0), ex2_approx(x1)));
+          const unsigned long long ll = f2_pack(bf16lo(w[q]), bf16hi(w[q]));
+          f2_unpack(f2_fma(ll, l2e, ml), x0, x1);
+          const unsigned long long pp = f2_pack(ex2_approx(x0), ex2_approx(x1));
+          s2 = f2_add(s2, pp);
+          if (kEntropy) u2 = f2_fma(pp, ll, u2);
         }
       }
     }
@@ -314,31 +322,36 @@ __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
   // Every logit of the part went through the filter once, so the warps'
   // buffers hold distinct keys.
 
-  // block merge of the log-sum-exp
-  float s;
+  // block merge of the log-sum-exp (and of the entropy's weighted sum)
+  float s, u;
   {
-    float s0, s1;
+    float s0, s1, u0, u1;
     f2_unpack(s2, s0, s1);
+    f2_unpack(u2, u0, u1);
     s = s0 + s1;
+    u = u0 + u1;
   }
   float wm = warp_max(m);
-  float ws = (m == -INFINITY) ? 0.f : s * exp2f((m - wm) * kLog2e);
-  if (wm == -INFINITY) ws = 0.f;
-  ws = warp_sum(ws);
+  const float wf = (m == -INFINITY || wm == -INFINITY) ? 0.f : exp2f((m - wm) * kLog2e);
+  float ws = warp_sum(s * wf);
+  float wu = warp_sum(u * wf);
   s_lists[warp][lane] = lane < nb ? buf[lane] : 0ull;
   if (lane == 0) {
     s_m[warp] = wm;
     s_s[warp] = ws;
+    s_u[warp] = wu;
   }
   __syncthreads();
   if (warp == 0) {
     float bm = lane < kRowWarps ? s_m[lane] : -INFINITY;
     const float gm = warp_max(bm);
-    float bs = (lane < kRowWarps && bm != -INFINITY) ? s_s[lane] * exp2f((bm - gm) * kLog2e) : 0.f;
-    bs = warp_sum(bs);
+    const float bf = (lane < kRowWarps && bm != -INFINITY) ? exp2f((bm - gm) * kLog2e) : 0.f;
+    const float bs = warp_sum(lane < kRowWarps ? s_s[lane] * bf : 0.f);
+    const float bu = warp_sum(lane < kRowWarps ? s_u[lane] * bf : 0.f);
     if (lane == 0) {
       out[blockIdx.x].m = gm;
       out[blockIdx.x].s = bs;
+      out[blockIdx.x].u = bu;
     }
     if (lane < IPD_MAX_K) out[blockIdx.x].keys[lane] = 0ull;
   }
@@ -354,6 +367,13 @@ __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
   }
 }
 
+// Rules and optional outputs of the epilogue (ipd_score_ext on the device).
+struct EpiOpts {
+  int take_rule, hand_rule;
+  float take_tau, hand_tau;
+  float *entropy_s, *entropy_t, *topk_overlap;
+};
+
 __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     const uint16_t *__restrict__ ls, const uint16_t *__restrict__ lt,
     const int32_t *__restrict__ tokens, const int32_t *__restrict__ cu_span,
@@ -361,7 +381,7 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     int eos_id, const RowOut *__restrict__ rows, float *logp_s, float *logp_t, float *feedback,
     float *kl_rev, float *kl_fwd, uint8_t *covered, float *margin, uint8_t *source,
     int32_t *first_trans, int32_t *n_emit, uint8_t *next_driver, int32_t *new_len, uint8_t *done,
-    int total_tokens) {
+    int total_tokens, const EpiOpts opt) {
   __shared__ uint8_t s_cov[1024];
   __shared__ unsigned long long s_pk[kEpiThreads / 32][kParts][32];  // one row's part lists
   __shared__ unsigned long long s_top[kEpiThreads / 32][2][32];      // merged top-K, S and T
@@ -383,18 +403,23 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     // each row from its parts: log Z by the log-sum-exp merge, the top-K as
     // the best K of the parts' lists (a key's rank is the number of larger
     // keys in every part list)
-    float logz[2];
+    float logz[2], ent[2];
 #pragma unroll
     for (int mdl = 0; mdl < 2; ++mdl) {
       const RowOut *pr = rows + (size_t)(2 * t + mdl) * kParts;
       float M = -INFINITY;
 #pragma unroll
       for (int q = 0; q < kParts; ++q) M = fmaxf(M, pr[q].m);
-      float S = 0.f;
+      float S = 0.f, Uw = 0.f;
 #pragma unroll
       for (int q = 0; q < kParts; ++q)
-        if (pr[q].m != -INFINITY) S += pr[q].s * expf(pr[q].m - M);
+        if (pr[q].m != -INFINITY) {
+          const float f = expf(pr[q].m - M);
+          S += pr[q].s * f;
+          Uw += pr[q].u * f;
+        }
       logz[mdl] = M + logf(S);
+      ent[mdl] = logz[mdl] - Uw / S;  // H = log Z - E[l]
 #pragma unroll
       for (int q = 0; q < kParts; ++q) s_pk[warp][q][lane] = lane < K ? pr[q].keys[lane] : 0ull;
       s_top[warp][mdl][lane] = 0ull;
@@ -465,8 +490,25 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     // coverage by the verifier's Top_K: the teacher's row when the student drives
     const unsigned long long kv = drv ? kS : kT;
     const bool hit = xok && lane < K && key_idx(kv) == (uint32_t)x;
-    const bool cov = __ballot_sync(0xffffffffu, hit) != 0;
     const unsigned long long kth = shfl_u64(kv, K - 1);
+    // the predicate of the rule governing this span (Sec. 3.2.1)
+    const int rule = drv ? opt.hand_rule : opt.take_rule;
+    const float tau = drv ? opt.hand_tau : opt.take_tau;
+    bool cov;
+    float mar;
+    if (rule == IPD_RULE_TOPK) {
+      cov = __ballot_sync(0xffffffffu, hit) != 0;
+      mar = (drv ? lxS : lxT) - key_val(kth);
+    } else if (rule == IPD_RULE_ENTROPY_S || rule == IPD_RULE_ENTROPY_T) {
+      const float h = rule == IPD_RULE_ENTROPY_S ? ent[0] : ent[1];
+      cov = h <= tau;
+      mar = tau - h;
+    } else {
+      cov = rule == IPD_RULE_ALWAYS;
+      mar = cov ? INFINITY : -INFINITY;
+    }
+    // |Top_K(pi) n Top_K(q)|: teacher keys also in the student's list
+    const int n_common = __popc(__ballot_sync(0xffffffffu, lane < K && dupT));
     if (lane == 0) {
       const float lps = lxS - logz[0], lpt = lxT - logz[1];
       logp_s[t] = lps;
@@ -475,7 +517,10 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
       kl_rev[t] = kr;
       kl_fwd[t] = kf;
       covered[t] = cov ? 1 : 0;
-      margin[t] = (drv ? lxS : lxT) - key_val(kth);
+      margin[t] = mar;
+      if (opt.entropy_s) opt.entropy_s[t] = ent[0];
+      if (opt.entropy_t) opt.entropy_t[t] = ent[1];
+      if (opt.topk_overlap) opt.topk_overlap[t] = (float)n_common / (float)K;
       if (t - t0 < 1024) s_cov[t - t0] = cov ? 1 : 0;
     }
   }
@@ -531,18 +576,35 @@ extern "C" size_t ipd_score_workspace_size(int num_reqs, int total_tokens, int v
   return (size_t)total_tokens * 2 * kParts * sizeof(RowOut) + 256;
 }
 
-extern "C" int ipd_score_span(const uint16_t *logits_student, const uint16_t *logits_teacher,
-                              const int32_t *tokens, const int32_t *cu_span,
-                              const uint8_t *driver, const int32_t *prefix_len, int num_reqs,
-                              int total_tokens, int vocab, int K, int eos_id, float *logp_s,
-                              float *logp_t, float *feedback, float *kl_rev, float *kl_fwd,
-                              uint8_t *covered, float *margin, uint8_t *source,
-                              int32_t *first_trans, int32_t *n_emit, uint8_t *next_driver,
-                              int32_t *new_len, uint8_t *done, void *workspace,
-                              size_t workspace_bytes, ipd_stream_t stream) {
+namespace {
+// host form of the options; false on an invalid rule or threshold
+bool epi_opts(const ipd_score_ext *ext, EpiOpts *o) {
+  *o = EpiOpts{IPD_RULE_TOPK, IPD_RULE_TOPK, 0.f, 0.f, nullptr, nullptr, nullptr};
+  if (!ext) return true;
+  auto ok_rule = [](int r) { return r >= IPD_RULE_TOPK && r <= IPD_RULE_NEVER; };
+  if (!ok_rule(ext->takeover_rule) || !ok_rule(ext->handback_rule)) return false;
+  if (ext->takeover_tau != ext->takeover_tau || ext->handback_tau != ext->handback_tau)
+    return false;
+  *o = EpiOpts{ext->takeover_rule, ext->handback_rule, ext->takeover_tau, ext->handback_tau,
+               ext->entropy_s, ext->entropy_t, ext->topk_overlap};
+  return true;
+}
+}  // namespace
+
+extern "C" int ipd_score_span_ex(const uint16_t *logits_student, const uint16_t *logits_teacher,
+                                 const int32_t *tokens, const int32_t *cu_span,
+                                 const uint8_t *driver, const int32_t *prefix_len, int num_reqs,
+                                 int total_tokens, int vocab, int K, int eos_id, float *logp_s,
+                                 float *logp_t, float *feedback, float *kl_rev, float *kl_fwd,
+                                 uint8_t *covered, float *margin, uint8_t *source,
+                                 int32_t *first_trans, int32_t *n_emit, uint8_t *next_driver,
+                                 int32_t *new_len, uint8_t *done, const ipd_score_ext *ext,
+                                 void *workspace, size_t workspace_bytes, ipd_stream_t stream) {
   if (num_reqs < 0 || total_tokens < 0) return IPD_ERR_INVALID_ARG;
   if (K < 1 || K > IPD_MAX_K) return IPD_ERR_UNSUPPORTED;
   if (vocab < 8 || vocab % 8 || K > vocab) return IPD_ERR_UNSUPPORTED;
+  EpiOpts opt;
+  if (!epi_opts(ext, &opt)) return IPD_ERR_INVALID_ARG;
   if (num_reqs == 0) return IPD_OK;
   if (!cu_span || !driver || !prefix_len || !first_trans || !n_emit || !next_driver || !new_len ||
       !done)
@@ -558,14 +620,173 @@ extern "C" int ipd_score_span(const uint16_t *logits_student, const uint16_t *lo
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   RowOut *rows = static_cast<RowOut *>(workspace);
   if (total_tokens > 0) {
-    score_rows_kernel<<<2 * kParts * total_tokens, kRowThreads, 0, st>>>(
-        logits_student, logits_teacher, vocab, K, rows);
+    const bool need_h = opt.entropy_s || opt.entropy_t || opt.take_rule == IPD_RULE_ENTROPY_S ||
+                        opt.take_rule == IPD_RULE_ENTROPY_T || opt.hand_rule == IPD_RULE_ENTROPY_S ||
+                        opt.hand_rule == IPD_RULE_ENTROPY_T;
+    if (need_h)
+      score_rows_kernel<true><<<2 * kParts * total_tokens, kRowThreads, 0, st>>>(
+          logits_student, logits_teacher, vocab, K, rows);
+    else
+      score_rows_kernel<false><<<2 * kParts * total_tokens, kRowThreads, 0, st>>>(
+          logits_student, logits_teacher, vocab, K, rows);
     if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   }
   score_epilogue_kernel<<<num_reqs, kEpiThreads, 0, st>>>(
       logits_student, logits_teacher, tokens, cu_span, driver, prefix_len, vocab, K, eos_id, rows,
       logp_s, logp_t, feedback, kl_rev, kl_fwd, covered, margin, source, first_trans, n_emit,
-      next_driver, new_len, done, total_tokens);
+      next_driver, new_len, done, total_tokens, opt);
+  if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
+  return IPD_OK;
+}
+
+extern "C" int ipd_score_span(const uint16_t *logits_student, const uint16_t *logits_teacher,
+                              const int32_t *tokens, const int32_t *cu_span,
+                              const uint8_t *driver, const int32_t *prefix_len, int num_reqs,
+                              int total_tokens, int vocab, int K, int eos_id, float *logp_s,
+                              float *logp_t, float *feedback, float *kl_rev, float *kl_fwd,
+                              uint8_t *covered, float *margin, uint8_t *source,
+                              int32_t *first_trans, int32_t *n_emit, uint8_t *next_driver,
+                              int32_t *new_len, uint8_t *done, void *workspace,
+                              size_t workspace_bytes, ipd_stream_t stream) {
+  return ipd_score_span_ex(logits_student, logits_teacher, tokens, cu_span, driver, prefix_len,
+                           num_reqs, total_tokens, vocab, K, eos_id, logp_s, logp_t, feedback,
+                           kl_rev, kl_fwd, covered, margin, source, first_trans, n_emit,
+                           next_driver, new_len, done, nullptr, workspace, workspace_bytes,
+                           stream);
+}
+
+// ---------------------------------------------------------------------------
+// Full-vocabulary KL (Eq. full_vocab_opd), both directions, one CTA per span
+// position reading the student's and the teacher's row together.  Per thread
+// and row: a running maximum m, s = sum exp(l - m); per thread: a = sum
+// exp(l_s - m_s) (l_s - l_t) and b = sum exp(l_t - m_t) (l_t - l_s), each
+// rescaled with its row's maximum.  Then KL(pi || q) = a / s_s - log Z_s +
+// log Z_t and KL(q || pi) = b / s_t - log Z_t + log Z_s.
+// ---------------------------------------------------------------------------
+namespace {
+constexpr int kKlThreads = 256;
+
+__global__ void __launch_bounds__(kKlThreads, 4) full_kl_kernel(
+    const uint16_t *__restrict__ ls, const uint16_t *__restrict__ lt, int vocab,
+    float *__restrict__ kl_rev, float *__restrict__ kl_fwd) {
+  __shared__ float sh[kKlThreads / 32][6];
+  const int t = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint4 *rs = reinterpret_cast<const uint4 *>(ls + (size_t)t * vocab);
+  const uint4 *rt = reinterpret_cast<const uint4 *>(lt + (size_t)t * vocab);
+  const int nvec = vocab >> 3;
+  float ms = -INFINITY, mt = -INFINITY;
+  unsigned long long ss = 0ull, st = 0ull, aa = 0ull, bb = 0ull;  // packed pairs
+  const unsigned long long l2e = f2_pack(kLog2e, kLog2e);
+  constexpr int U = 2;
+  for (int base = 0; base < nvec; base += kKlThreads * U) {
+    uint4 xs[U], xt[U];
+    bool ok[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int v = base + u * kKlThreads + (int)threadIdx.x;
+      ok[u] = v < nvec;
+      xs[u] = ok[u] ? ldg_stream(rs + v) : make_uint4(0xff80ff80u, 0xff80ff80u, 0xff80ff80u, 0xff80ff80u);
+      xt[u] = ok[u] ? ldg_stream(rt + v) : make_uint4(0xff80ff80u, 0xff80ff80u, 0xff80ff80u, 0xff80ff80u);
+    }
+    float bs = -INFINITY, bt = -INFINITY;
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      bs = fmaxf(bs, bf16x8_max(xs[u]));
+      bt = fmaxf(bt, bf16x8_max(xt[u]));
+    }
+    if (bs > ms) {  // rescale the student-weighted sums
+      const float f = ex2_approx((ms - bs) * kLog2e);
+      const unsigned long long ff = f2_pack(f, f), z = 0ull;
+      ss = f2_fma(ss, ff, z);
+      aa = f2_fma(aa, ff, z);
+      ms = bs;
+    }
+    if (bt > mt) {
+      const float f = ex2_approx((mt - bt) * kLog2e);
+      const unsigned long long ff = f2_pack(f, f), z = 0ull;
+      st = f2_fma(st, ff, z);
+      bb = f2_fma(bb, ff, z);
+      mt = bt;
+    }
+    const unsigned long long mls = f2_pack(-ms * kLog2e, -ms * kLog2e);
+    const unsigned long long mlt = f2_pack(-mt * kLog2e, -mt * kLog2e);
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (!ok[u]) continue;
+      const uint32_t ws[4] = {xs[u].x, xs[u].y, xs[u].z, xs[u].w};
+      const uint32_t wt[4] = {xt[u].x, xt[u].y, xt[u].z, xt[u].w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const unsigned long long vs = f2_pack(bf16lo(ws[q]), bf16hi(ws[q]));
+        const unsigned long long vt = f2_pack(bf16lo(wt[q]), bf16hi(wt[q]));
+        float e0, e1, g0, g1;
+        f2_unpack(f2_fma(vs, l2e, mls), e0, e1);
+        f2_unpack(f2_fma(vt, l2e, mlt), g0, g1);
+        const unsigned long long p = f2_pack(ex2_approx(e0), ex2_approx(e1));
+        const unsigned long long qq = f2_pack(ex2_approx(g0), ex2_approx(g1));
+        const unsigned long long d = f2_sub(vs, vt);  // l_s - l_t
+        ss = f2_add(ss, p);
+        st = f2_add(st, qq);
+        aa = f2_fma(p, d, aa);
+        bb = f2_fma(qq, d, bb);  // sum q (l_s - l_t) = -b
+      }
+    }
+  }
+  float v[6];  // ms, s_s, a, mt, s_t, -b (per thread)
+  {
+    float x0, x1;
+    v[0] = ms;
+    f2_unpack(ss, x0, x1); v[1] = x0 + x1;
+    f2_unpack(aa, x0, x1); v[2] = x0 + x1;
+    v[3] = mt;
+    f2_unpack(st, x0, x1); v[4] = x0 + x1;
+    f2_unpack(bb, x0, x1); v[5] = x0 + x1;
+  }
+  // warp then block merge: rescale each thread's sums to the common maxima
+#pragma unroll
+  for (int r = 0; r < 2; ++r) {
+    const float M = warp_max(v[3 * r]);
+    const float f = (v[3 * r] == -INFINITY) ? 0.f : exp2f((v[3 * r] - M) * kLog2e);
+    v[3 * r] = M;
+    v[3 * r + 1] = warp_sum(v[3 * r + 1] * f);
+    v[3 * r + 2] = warp_sum(v[3 * r + 2] * f);
+  }
+  if (lane == 0)
+#pragma unroll
+    for (int i = 0; i < 6; ++i) sh[warp][i] = v[i];
+  __syncthreads();
+  if (warp == 0) {
+    float w[6];
+#pragma unroll
+    for (int i = 0; i < 6; ++i) w[i] = lane < kKlThreads / 32 ? sh[lane][i] : (i % 3 == 0 ? -INFINITY : 0.f);
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const float M = warp_max(w[3 * r]);
+      const float f = (w[3 * r] == -INFINITY) ? 0.f : exp2f((w[3 * r] - M) * kLog2e);
+      w[3 * r] = M;
+      w[3 * r + 1] = warp_sum(w[3 * r + 1] * f);
+      w[3 * r + 2] = warp_sum(w[3 * r + 2] * f);
+    }
+    if (lane == 0) {
+      const float lzs = w[0] + logf(w[1]), lzt = w[3] + logf(w[4]);
+      kl_rev[t] = w[2] / w[1] - lzs + lzt;
+      kl_fwd[t] = -w[5] / w[4] - lzt + lzs;
+    }
+  }
+}
+}  // namespace
+
+extern "C" int ipd_full_kl(const uint16_t *logits_student, const uint16_t *logits_teacher,
+                           int total_tokens, int vocab, float *kl_rev_full, float *kl_fwd_full,
+                           ipd_stream_t stream) {
+  if (total_tokens < 0) return IPD_ERR_INVALID_ARG;
+  if (vocab < 8 || vocab % 8) return IPD_ERR_UNSUPPORTED;
+  if (total_tokens == 0) return IPD_OK;
+  if (!logits_student || !logits_teacher || !kl_rev_full || !kl_fwd_full)
+    return IPD_ERR_INVALID_ARG;
+  if (((uintptr_t)logits_student | (uintptr_t)logits_teacher) & 15) return IPD_ERR_INVALID_ARG;
+  full_kl_kernel<<<total_tokens, kKlThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+      logits_student, logits_teacher, vocab, kl_rev_full, kl_fwd_full);
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   return IPD_OK;
 }
@@ -628,14 +849,15 @@ extern "C" int ipd_score_span_static(const uint16_t *logits_student,
   // Every RowOut the epilogue reads is written by the row kernel of the same
   // call first, so nothing in the array has to start at zero.
   if (total_tokens > 0) {
-    score_rows_kernel<<<2 * kParts * total_tokens, kRowThreads, 0, s>>>(
+    score_rows_kernel<false><<<2 * kParts * total_tokens, kRowThreads, 0, s>>>(
         logits_student, logits_teacher, vocab, K, rows);
     if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   }
   score_epilogue_kernel<<<num_reqs, kEpiThreads, 0, s>>>(
       logits_student, logits_teacher, tokens, cu_span, driver, prefix_len, vocab, K, eos_id, rows,
       logp_s, logp_t, feedback, kl_rev, kl_fwd, covered, margin, source, first_trans, n_emit,
-      next_driver, new_len, done, total_tokens);
+      next_driver, new_len, done, total_tokens,
+      EpiOpts{IPD_RULE_TOPK, IPD_RULE_TOPK, 0.f, 0.f, nullptr, nullptr, nullptr});
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   return IPD_OK;
 }

@@ -31,7 +31,9 @@ LOSS_FIELDS = ("loss", "sum_on", "sum_off", "n_on", "n_off", "intervention_ratio
 EXPORTS = ("ipd_attn_workspace_size", "ipd_verify_attn", "ipd_decode_attn",
            "ipd_score_workspace_size", "ipd_score_span", "ipd_loss_workspace_size",
            "ipd_split_loss", "ipd_get_device_error", "ipd_status_string", "ipd_version",
-           "ipd_score_span_static")
+           "ipd_score_span_static", "ipd_score_span_ex", "ipd_full_kl")
+# takeover / handback rules (IPD_RULE_*)
+RULE_TOPK, RULE_ENTROPY_S, RULE_ENTROPY_T, RULE_ALWAYS, RULE_NEVER = 0, 1, 2, 3, 4
 STATIC_MAX_TOKENS = 4096  # IPD_STATIC_MAX_TOKENS
 
 
@@ -60,6 +62,12 @@ class _KVCache(ctypes.Structure):
                 ("head_dim", ctypes.c_int32)]
 
 
+class _ScoreExt(ctypes.Structure):
+    _fields_ = [("takeover_rule", ctypes.c_int32), ("handback_rule", ctypes.c_int32),
+                ("takeover_tau", ctypes.c_float), ("handback_tau", ctypes.c_float),
+                ("entropy_s", c_p), ("entropy_t", c_p), ("topk_overlap", c_p)]
+
+
 class _AttnBatch(ctypes.Structure):
     _fields_ = [("cache", ctypes.POINTER(_KVCache)), ("num_q_heads", ctypes.c_int32),
                 ("num_reqs", ctypes.c_int32), ("q", c_p), ("cu_q", c_p), ("seq_len", c_p),
@@ -79,6 +87,11 @@ _lib.ipd_score_workspace_size.restype = c_sz
 _lib.ipd_score_workspace_size.argtypes = [c_i, c_i, c_i, c_i]
 _lib.ipd_score_span.restype = c_i
 _lib.ipd_score_span.argtypes = [c_p] * 6 + [c_i] * 5 + [c_p] * 13 + [c_p, c_sz, c_p]
+_lib.ipd_score_span_ex.restype = c_i
+_lib.ipd_score_span_ex.argtypes = ([c_p] * 6 + [c_i] * 5 + [c_p] * 13 +
+                                   [ctypes.POINTER(_ScoreExt), c_p, c_sz, c_p])
+_lib.ipd_full_kl.restype = c_i
+_lib.ipd_full_kl.argtypes = [c_p, c_p, c_i, c_i, c_p, c_p, c_p]
 _lib.ipd_score_span_static.restype = c_i
 _lib.ipd_score_span_static.argtypes = [c_p] * 6 + [c_i] * 5 + [c_p] * 13 + [c_p]
 _lib.ipd_loss_workspace_size.restype = c_sz
@@ -205,6 +218,35 @@ def score_span(logits_student, logits_teacher, tokens, cu_span, driver, prefix_l
         *[_ptr(out[n]) for n, _ in SCORE_REQ_OUTPUTS],
         _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)),
         "ipd_score_span")
+
+
+def score_span_ex(logits_student, logits_teacher, tokens, cu_span, driver, prefix_len, K: int,
+                  eos_id: int, out: dict, workspace: torch.Tensor, takeover_rule: int = RULE_TOPK,
+                  handback_rule: int = RULE_TOPK, takeover_tau: float = 0.0,
+                  handback_tau: float = 0.0, entropy_s: Optional[torch.Tensor] = None,
+                  entropy_t: Optional[torch.Tensor] = None,
+                  topk_overlap: Optional[torch.Tensor] = None, stream=None):
+    """ipd_score_span with selectable takeover / handback rules and the
+    optional per-token entropies and top-K overlap ratio (fp32 [T] tensors)."""
+    R = driver.numel()
+    T, V = logits_student.shape
+    ext = _ScoreExt(takeover_rule, handback_rule, takeover_tau, handback_tau,
+                    _ptr(entropy_s), _ptr(entropy_t), _ptr(topk_overlap))
+    _check(_lib.ipd_score_span_ex(
+        _ptr(logits_student), _ptr(logits_teacher), _ptr(tokens), _ptr(cu_span), _ptr(driver),
+        _ptr(prefix_len), R, T, V, K, eos_id,
+        *[_ptr(out[n]) for n, _ in SCORE_TOKEN_OUTPUTS],
+        *[_ptr(out[n]) for n, _ in SCORE_REQ_OUTPUTS],
+        ctypes.byref(ext), _ptr(workspace), workspace.numel() * workspace.element_size(),
+        _stream(stream)), "ipd_score_span_ex")
+
+
+def full_kl(logits_student, logits_teacher, kl_rev_full: torch.Tensor, kl_fwd_full: torch.Tensor,
+            stream=None):
+    """Full-vocabulary KL in both directions at every span position."""
+    T, V = logits_student.shape
+    _check(_lib.ipd_full_kl(_ptr(logits_student), _ptr(logits_teacher), T, V, _ptr(kl_rev_full),
+                            _ptr(kl_fwd_full), _stream(stream)), "ipd_full_kl")
 
 
 def score_span_static(logits_student, logits_teacher, tokens, cu_span, driver, prefix_len,

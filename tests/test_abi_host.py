@@ -85,3 +85,19 @@ def test_score_and_loss_host_validation(ipd):
     assert L.ipd_split_loss(16, 16, 16, 16, 16, None, 3, 2, 0, 16, None, 0, None) == bad["IPD_ERR_INVALID_ARG"]
     assert L.ipd_split_loss(16, 16, 16, 16, 16, None, 3, 0, 7, 16, None, 0, None) == bad["IPD_ERR_INVALID_ARG"]
     assert L.ipd_split_loss(16, 16, 16, 16, 16, None, 3, 0, 0, None, None, 0, None) == bad["IPD_ERR_INVALID_ARG"]
+
+
+def test_score_ext_rejects_bad_rules_on_the_host():
+    import ctypes
+    from paper_2609_36546_gb300 import ipd
+    for take, hand, tt in ((7, 0, 0.0), (0, -1, 0.0), (1, 0, float("nan"))):
+        ext = ipd._ScoreExt(take, hand, tt, 0.0, None, None, None)
+        st = ipd._lib.ipd_score_span_ex(*([None] * 6), 0, 0, 4096, 16, -1, *([None] * 13),
+                                        ctypes.byref(ext), None, 0, None)
+        assert st == ipd.STATUS_CODES["IPD_ERR_INVALID_ARG"]
+    # full KL: host validation only
+    assert ipd._lib.ipd_full_kl(None, None, 0, 4096, None, None, None) == 0
+    assert ipd._lib.ipd_full_kl(None, None, 3, 4095, None, None, None) == \
+        ipd.STATUS_CODES["IPD_ERR_UNSUPPORTED"]
+    assert ipd._lib.ipd_full_kl(None, None, 3, 4096, None, None, None) == \
+        ipd.STATUS_CODES["IPD_ERR_INVALID_ARG"]
