@@ -16,5 +16,8 @@ Parity status per function (what pins it is listed in tests/test_oracle_pins.py)
   the rollback rules, exhaustive invariants).
 * ``split_loss`` -- pinned (hand-worked fixture, special cases that reduce to
   pure on-policy and pure off-policy distillation).
+* ``split_loss_grad`` -- pinned (central finite differences of ``topk_kl`` +
+  ``split_loss`` in fp64, shift invariance of every row, zero rows off the
+  emitted positions).
 """
 from .ipd_oracle import *  # noqa: F401,F403

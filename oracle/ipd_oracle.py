@@ -353,3 +353,59 @@ def split_loss(kl_rev, kl_fwd, source, cu_span, n_emit, resp_len=None, agg_mode=
 
 
 LOSS_FIELDS = ("loss", "sum_on", "sum_off", "n_on", "n_off", "intervention_ratio", "numer", "denom")
+
+
+# ----------------------------------------------------------------------------
+# gradient of the source-split objective with respect to the student's logits
+# ----------------------------------------------------------------------------
+def split_loss_grad(l_s, l_t, source, cu_span, n_emit, resp_len=None, K=16, agg_mode=0,
+                    dir_mode=DIR_IPD, grad_scale=1.0) -> np.ndarray:
+    """d(grad_scale * loss) / d l_s for the loss of ``split_loss``, as a dense
+    [T, V] fp64 array.  ``l_s`` and ``l_t`` are the two models' logits as fp64
+    rows (bf16 rows go through ``bf16_to_f64`` first).
+
+    Each emitted position t contributes its token-level KL (Eq. ipd_off_loss,
+    direction chosen per source as in ``split_loss``) with weight
+    w_t = 1 / (R' |x_r|) under the sequence-mean-token-mean of
+    Eq. (ipd_objective), or 1 / sum_r |x_r| under the global token mean.  The
+    supports S_t = Top_K(pi_t) u Top_K(q_t) are piecewise constant in the
+    logits and are held fixed.  With pi_bar the student's softmax restricted
+    to S_t (Eq. topk_normalization; its normaliser is the only place the
+    student's logits enter besides the numerator), for v in S_t:
+      d KL(pi_bar || q_bar) / d l_v = pi_bar_v (log pi_bar_v - log q_bar_v - KL(pi_bar || q_bar))
+      d KL(q_bar || pi_bar) / d l_v = pi_bar_v - q_bar_v
+    and every logit outside S_t has gradient 0."""
+    l_s = np.asarray(l_s, dtype=np.float64)
+    l_t = np.asarray(l_t, dtype=np.float64)
+    T, V = l_s.shape
+    R = len(cu_span) - 1
+    dens = [int(n_emit[r]) if resp_len is None else int(resp_len[r]) for r in range(R)]
+    if agg_mode == 0:
+        D = float(sum(1 for d in dens if d > 0))
+    else:
+        D = float(sum(d for d in dens if d > 0))
+    G = np.zeros((T, V))
+    for r in range(R):
+        if dens[r] <= 0:
+            continue
+        w = grad_scale / (D * dens[r]) if agg_mode == 0 else grad_scale / D
+        for t in range(int(cu_span[r]), int(cu_span[r + 1])):
+            if source[t] == SRC_STUDENT:
+                use_rev = dir_mode in (DIR_IPD, DIR_PURE_REV)
+            elif source[t] == SRC_TEACHER:
+                use_rev = dir_mode in (DIR_PURE_REV, DIR_INVERSE)
+            else:
+                continue
+            S = np.union1d(topk(l_s[t], K), topk(l_t[t], K))
+            log_pi_bar = l_s[t, S] - log_partition(l_s[t, S])
+            log_q_bar = l_t[t, S] - log_partition(l_t[t, S])
+            pi_bar = np.exp(log_pi_bar)
+            q_bar = np.exp(log_q_bar)
+            if use_rev:
+                d = np.where(pi_bar > 0, log_pi_bar - log_q_bar, 0.0)
+                kl = float(np.sum(pi_bar * d))
+                g = pi_bar * (d - kl)
+            else:
+                g = pi_bar - q_bar
+            G[t, S] = w * g
+    return G

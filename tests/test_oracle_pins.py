@@ -557,3 +557,82 @@ def test_planted_rule_mistakes_are_caught():
     l = _bf16_round(RNG.normal(size=50) * 2)
     lz = O.log_partition(l); p = np.exp(l - lz)
     assert abs((lz + np.dot(p, l)) - scipy.stats.entropy(p)) > 1e-3
+
+
+# ---------------------------------------------------------------------------
+# gradient of the source-split objective (finite differences of the loss)
+# ---------------------------------------------------------------------------
+def _grad_case(seed, V=40, K=4):
+    rng = np.random.default_rng(seed)
+    cu = np.array([0, 3, 3, 7, 10])            # one request with an empty span
+    T = int(cu[-1])
+    ls = rng.normal(size=(T, V)) * 2.0          # continuous: no ties, fixed supports
+    lt = rng.normal(size=(T, V)) * 2.0
+    source = np.array([0, 0, 255, 1, 1, 1, 255, 0, 0, 0])
+    n_emit = np.array([2, 0, 3, 3])
+    resp_len = np.array([5, 0, 3, 9])
+    return ls, lt, source, cu, n_emit, resp_len, K
+
+
+def _loss_of_student_logits(ls, lt, source, cu, n_emit, resp_len, K, agg, dmode):
+    T = ls.shape[0]
+    kr = np.zeros(T); kf = np.zeros(T)
+    for t in range(T):
+        kr[t], kf[t], _ = O.topk_kl(ls[t], lt[t], K)
+    return O.split_loss(kr, kf, source, cu, n_emit, resp_len, agg, dmode)["loss"]
+
+
+@pytest.mark.parametrize("agg,dmode,use_len", [(0, 0, False), (1, 0, True), (0, 1, True),
+                                                (1, 2, False), (0, 3, True)])
+def test_split_loss_grad_matches_finite_differences(agg, dmode, use_len):
+    ls, lt, source, cu, n_emit, resp_len, K = _grad_case(7 + dmode)
+    rl = resp_len if use_len else None
+    G = O.split_loss_grad(ls, lt, source, cu, n_emit, rl, K, agg, dmode, grad_scale=1.0)
+    eps = 1e-6
+    fd = np.zeros_like(G)
+    for t in range(ls.shape[0]):
+        for v in range(ls.shape[1]):
+            a = ls.copy(); a[t, v] += eps
+            b = ls.copy(); b[t, v] -= eps
+            fd[t, v] = (_loss_of_student_logits(a, lt, source, cu, n_emit, rl, K, agg, dmode)
+                        - _loss_of_student_logits(b, lt, source, cu, n_emit, rl, K, agg, dmode)) / (2 * eps)
+    assert np.abs(G - fd).max() <= 1e-8 + 1e-6 * np.abs(fd).max()
+    assert np.abs(G).max() > 1e-3                # the case is not trivially zero
+
+
+def test_split_loss_grad_rows_are_shift_invariant_and_zero_off_the_emitted_positions():
+    ls, lt, source, cu, n_emit, resp_len, K = _grad_case(3)
+    G = O.split_loss_grad(ls, lt, source, cu, n_emit, None, K, 0, 0, grad_scale=2.5)
+    # adding a constant to a student row leaves every KL unchanged
+    assert np.abs(G.sum(axis=1)).max() < 1e-14
+    for t in range(G.shape[0]):
+        S = np.union1d(O.topk(ls[t], K), O.topk(lt[t], K))
+        off = np.setdiff1d(np.arange(G.shape[1]), S)
+        assert (G[t, off] == 0).all()
+        if source[t] == O.SRC_DISCARDED:
+            assert (G[t] == 0).all()
+    # grad_scale is a plain factor
+    G1 = O.split_loss_grad(ls, lt, source, cu, n_emit, None, K, 0, 0, grad_scale=1.0)
+    assert np.allclose(G, 2.5 * G1, rtol=1e-15, atol=0)
+
+
+def test_planted_gradient_mistakes_are_caught():
+    ls, lt, source, cu, n_emit, resp_len, K = _grad_case(11)
+    G = O.split_loss_grad(ls, lt, source, cu, n_emit, None, K, 0, 0)
+    # the reverse-KL gradient without its "- KL" centring term no longer sums to 0
+    t = 0
+    S = np.union1d(O.topk(ls[t], K), O.topk(lt[t], K))
+    lp = ls[t, S] - O.log_partition(ls[t, S]); lq = lt[t, S] - O.log_partition(lt[t, S])
+    p = np.exp(lp)
+    w = G[t, S][0] / (p[0] * (lp[0] - lq[0] - np.sum(p * (lp - lq))))
+    bad = w * p * (lp - lq)
+    assert abs(bad.sum()) > 1e-6 and abs(G[t].sum()) < 1e-14
+    # the forward-KL gradient with the sign flipped disagrees with finite differences
+    eps = 1e-6
+    t = 3                                        # teacher-sourced: forward KL under IPD
+    v = int(np.union1d(O.topk(ls[t], K), O.topk(lt[t], K))[0])
+    a = ls.copy(); a[t, v] += eps
+    b = ls.copy(); b[t, v] -= eps
+    fd = (_loss_of_student_logits(a, lt, source, cu, n_emit, None, K, 0, 0)
+          - _loss_of_student_logits(b, lt, source, cu, n_emit, None, K, 0, 0)) / (2 * eps)
+    assert abs(G[t, v] - fd) < 1e-8 and abs(-G[t, v] - fd) > 1e-4
