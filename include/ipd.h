@@ -17,6 +17,11 @@
  *                    handback verdict and the new cache lengths.
  *   ipd_split_loss   the source-split objective of the step.
  *
+ * Beyond the step itself: ipd_score_span_ex (other takeover / handback rules,
+ * entropies, top-K overlap, top-K lists), ipd_full_kl (full-vocabulary KL both
+ * ways) and ipd_split_loss_grad (the objective's gradient with respect to the
+ * student's logits, sparse and dense).
+ *
  * Conventions for every call
  *   - Data pointers are DEVICE pointers owned by the caller; the library never
  *     allocates.  Scratch memory comes from a caller-provided device workspace
@@ -213,6 +218,9 @@ typedef struct {
   float *entropy_s;    /* [total_tokens] H(pi_t) over the full vocabulary, or NULL */
   float *entropy_t;    /* [total_tokens] H(q_t), or NULL */
   float *topk_overlap; /* [total_tokens] |Top_K(pi_t) n Top_K(q_t)| / K (Sec. 4.2), or NULL */
+  int32_t *topk_s;     /* [total_tokens][K] Top_K(pi_t) token ids, best first (ties: lower id
+                          first), or NULL; ipd_split_loss_grad takes these lists */
+  int32_t *topk_t;     /* [total_tokens][K] Top_K(q_t), same order, or NULL */
 } ipd_score_ext;
 
 /* ipd_score_span with selectable rules and by-products.  ext == NULL is the
@@ -302,6 +310,50 @@ int ipd_split_loss(const float *kl_rev, const float *kl_fwd, const uint8_t *sour
                    const int32_t *cu_span, const int32_t *n_emit, const int32_t *resp_len,
                    int num_reqs, int agg_mode, int dir_mode, float *out8,
                    void *workspace, size_t workspace_bytes, ipd_stream_t stream);
+
+/* Element type of the dense gradient of ipd_split_loss_grad. */
+#define IPD_DTYPE_F32 0
+#define IPD_DTYPE_BF16 1
+
+/* Workspace bytes for ipd_split_loss_grad (0: it needs none). */
+size_t ipd_loss_grad_workspace_size(int total_tokens, int K);
+
+/* Gradient of grad_scale * loss with respect to the student's logits, for the
+ * loss of ipd_split_loss (Eq. ipd_off_loss and Eq. ipd_objective; top-K
+ * renormalisation of Eq. topk_normalization).  The supports
+ * S_t = Top_K(pi_t) u Top_K(q_t) are piecewise constant in the logits and are
+ * held fixed.  Position t, when emitted, carries weight w_t = 1 / (D |x_r|)
+ * (agg_mode 0, D = number of requests with |x_r| > 0) or 1 / D (agg_mode 1,
+ * D = sum of those |x_r|); D is read from loss_out8[7], the `denom` output of
+ * ipd_split_loss, so a sharded batch passes its combined denominator.  With
+ * pi_bar, q_bar the two softmaxes restricted to S_t, for v in S_t:
+ *   reverse KL(pi_bar || q_bar): w_t pi_bar_v (log pi_bar_v - log q_bar_v - KL)
+ *   forward KL(q_bar || pi_bar): w_t (pi_bar_v - q_bar_v)
+ * (the direction per source as in ipd_split_loss's dir_mode); every other
+ * logit, and every position that was not emitted, has gradient 0.
+ *  logits_student, logits_teacher  [total_tokens][vocab] bf16 (as for ipd_score_span)
+ *  topk_s, topk_t  [total_tokens][K] int32, the lists ipd_score_span_ex writes
+ *  source, cu_span, n_emit, resp_len, num_reqs, agg_mode, dir_mode  as for ipd_split_loss
+ *  loss_out8       the 8 floats ipd_split_loss wrote (device)
+ *  grad_idx, grad_val  [total_tokens][2K] sparse gradient (required): slots
+ *      0..K-1 hold Top_K(pi_t) in order, slots K..2K-1 the entries of
+ *      Top_K(q_t) not in Top_K(pi_t); unused slots and positions with no
+ *      gradient hold id -1 and value 0
+ *  grad_dense      [total_tokens][vocab] dense gradient of dense_dtype
+ *      (IPD_DTYPE_F32 or IPD_DTYPE_BF16, round to nearest even), 16-byte
+ *      aligned, or NULL for the sparse form only
+ * Returns IPD_ERR_INVALID_ARG for a missing pointer, an unknown mode or dtype,
+ * a non-finite grad_scale or a misaligned grad_dense; IPD_ERR_UNSUPPORTED for
+ * K outside [1, IPD_MAX_K] or K > vocab.  An id outside [0, vocab) in the
+ * top-K lists is recorded as IPD_DEVERR_TOKEN and that position gets no
+ * gradient. */
+int ipd_split_loss_grad(const uint16_t *logits_student, const uint16_t *logits_teacher,
+                        const int32_t *topk_s, const int32_t *topk_t, const uint8_t *source,
+                        const int32_t *cu_span, const int32_t *n_emit, const int32_t *resp_len,
+                        const float *loss_out8, int num_reqs, int total_tokens, int vocab, int K,
+                        int agg_mode, int dir_mode, float grad_scale, int32_t *grad_idx,
+                        float *grad_val, void *grad_dense, int dense_dtype, void *workspace,
+                        size_t workspace_bytes, ipd_stream_t stream);
 
 /* Reads and clears the device error word of the current device
  * (synchronises the device).  *code receives an IPD_DEVERR_* value. */

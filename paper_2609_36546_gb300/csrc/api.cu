@@ -5,14 +5,16 @@
 
 extern "C" __attribute__((visibility("hidden"))) unsigned int ipd_internal_take_attn_error();
 extern "C" __attribute__((visibility("hidden"))) unsigned int ipd_internal_take_score_error();
+extern "C" __attribute__((visibility("hidden"))) unsigned int ipd_internal_take_loss_error();
 
 extern "C" int ipd_get_device_error(uint32_t *code) {
   if (!code) return IPD_ERR_INVALID_ARG;
   if (cudaDeviceSynchronize() != cudaSuccess) return IPD_ERR_CUDA;
   const unsigned int a = ipd_internal_take_attn_error();
   const unsigned int b = ipd_internal_take_score_error();
-  if (a == 0xffffffffu || b == 0xffffffffu) return IPD_ERR_CUDA;
-  *code = a ? a : b;
+  const unsigned int c = ipd_internal_take_loss_error();
+  if (a == 0xffffffffu || b == 0xffffffffu || c == 0xffffffffu) return IPD_ERR_CUDA;
+  *code = a ? a : (b ? b : c);
   return IPD_OK;
 }
 

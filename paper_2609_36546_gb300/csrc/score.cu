@@ -372,6 +372,7 @@ struct EpiOpts {
   int take_rule, hand_rule;
   float take_tau, hand_tau;
   float *entropy_s, *entropy_t, *topk_overlap;
+  int32_t *topk_s, *topk_t;
 };
 
 __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
@@ -507,6 +508,10 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
       cov = rule == IPD_RULE_ALWAYS;
       mar = cov ? INFINITY : -INFINITY;
     }
+    if (lane < K) {
+      if (opt.topk_s) opt.topk_s[(size_t)t * K + lane] = (int32_t)iS;
+      if (opt.topk_t) opt.topk_t[(size_t)t * K + lane] = (int32_t)iT;
+    }
     // |Top_K(pi) n Top_K(q)|: teacher keys also in the student's list
     const int n_common = __popc(__ballot_sync(0xffffffffu, lane < K && dupT));
     if (lane == 0) {
@@ -579,14 +584,15 @@ extern "C" size_t ipd_score_workspace_size(int num_reqs, int total_tokens, int v
 namespace {
 // host form of the options; false on an invalid rule or threshold
 bool epi_opts(const ipd_score_ext *ext, EpiOpts *o) {
-  *o = EpiOpts{IPD_RULE_TOPK, IPD_RULE_TOPK, 0.f, 0.f, nullptr, nullptr, nullptr};
+  *o = EpiOpts{IPD_RULE_TOPK, IPD_RULE_TOPK, 0.f, 0.f, nullptr, nullptr, nullptr, nullptr,
+               nullptr};
   if (!ext) return true;
   auto ok_rule = [](int r) { return r >= IPD_RULE_TOPK && r <= IPD_RULE_NEVER; };
   if (!ok_rule(ext->takeover_rule) || !ok_rule(ext->handback_rule)) return false;
   if (ext->takeover_tau != ext->takeover_tau || ext->handback_tau != ext->handback_tau)
     return false;
   *o = EpiOpts{ext->takeover_rule, ext->handback_rule, ext->takeover_tau, ext->handback_tau,
-               ext->entropy_s, ext->entropy_t, ext->topk_overlap};
+               ext->entropy_s, ext->entropy_t, ext->topk_overlap, ext->topk_s, ext->topk_t};
   return true;
 }
 }  // namespace

@@ -31,9 +31,12 @@ LOSS_FIELDS = ("loss", "sum_on", "sum_off", "n_on", "n_off", "intervention_ratio
 EXPORTS = ("ipd_attn_workspace_size", "ipd_verify_attn", "ipd_decode_attn",
            "ipd_score_workspace_size", "ipd_score_span", "ipd_loss_workspace_size",
            "ipd_split_loss", "ipd_get_device_error", "ipd_status_string", "ipd_version",
-           "ipd_score_span_static", "ipd_score_span_ex", "ipd_full_kl")
+           "ipd_score_span_static", "ipd_score_span_ex", "ipd_full_kl",
+           "ipd_loss_grad_workspace_size", "ipd_split_loss_grad")
 # takeover / handback rules (IPD_RULE_*)
 RULE_TOPK, RULE_ENTROPY_S, RULE_ENTROPY_T, RULE_ALWAYS, RULE_NEVER = 0, 1, 2, 3, 4
+# element type of the dense gradient (IPD_DTYPE_*)
+DTYPE_F32, DTYPE_BF16 = 0, 1
 STATIC_MAX_TOKENS = 4096  # IPD_STATIC_MAX_TOKENS
 
 
@@ -65,7 +68,8 @@ class _KVCache(ctypes.Structure):
 class _ScoreExt(ctypes.Structure):
     _fields_ = [("takeover_rule", ctypes.c_int32), ("handback_rule", ctypes.c_int32),
                 ("takeover_tau", ctypes.c_float), ("handback_tau", ctypes.c_float),
-                ("entropy_s", c_p), ("entropy_t", c_p), ("topk_overlap", c_p)]
+                ("entropy_s", c_p), ("entropy_t", c_p), ("topk_overlap", c_p),
+                ("topk_s", c_p), ("topk_t", c_p)]
 
 
 class _AttnBatch(ctypes.Structure):
@@ -98,6 +102,11 @@ _lib.ipd_loss_workspace_size.restype = c_sz
 _lib.ipd_loss_workspace_size.argtypes = [c_i]
 _lib.ipd_split_loss.restype = c_i
 _lib.ipd_split_loss.argtypes = [c_p] * 6 + [c_i, c_i, c_i, c_p, c_p, c_sz, c_p]
+_lib.ipd_loss_grad_workspace_size.restype = c_sz
+_lib.ipd_loss_grad_workspace_size.argtypes = [c_i, c_i]
+_lib.ipd_split_loss_grad.restype = c_i
+_lib.ipd_split_loss_grad.argtypes = ([c_p] * 9 + [c_i] * 6 + [ctypes.c_float, c_p, c_p, c_p, c_i,
+                                      c_p, c_sz, c_p])
 _lib.ipd_get_device_error.restype = c_i
 _lib.ipd_get_device_error.argtypes = [ctypes.POINTER(ctypes.c_uint32)]
 _lib.ipd_status_string.restype = ctypes.c_char_p
@@ -225,13 +234,17 @@ def score_span_ex(logits_student, logits_teacher, tokens, cu_span, driver, prefi
                   handback_rule: int = RULE_TOPK, takeover_tau: float = 0.0,
                   handback_tau: float = 0.0, entropy_s: Optional[torch.Tensor] = None,
                   entropy_t: Optional[torch.Tensor] = None,
-                  topk_overlap: Optional[torch.Tensor] = None, stream=None):
+                  topk_overlap: Optional[torch.Tensor] = None,
+                  topk_s: Optional[torch.Tensor] = None, topk_t: Optional[torch.Tensor] = None,
+                  stream=None):
     """ipd_score_span with selectable takeover / handback rules and the
-    optional per-token entropies and top-K overlap ratio (fp32 [T] tensors)."""
+    optional per-token entropies and top-K overlap ratio (fp32 [T] tensors)
+    and top-K id lists (int32 [T, K])."""
     R = driver.numel()
     T, V = logits_student.shape
     ext = _ScoreExt(takeover_rule, handback_rule, takeover_tau, handback_tau,
-                    _ptr(entropy_s), _ptr(entropy_t), _ptr(topk_overlap))
+                    _ptr(entropy_s), _ptr(entropy_t), _ptr(topk_overlap), _ptr(topk_s),
+                    _ptr(topk_t))
     _check(_lib.ipd_score_span_ex(
         _ptr(logits_student), _ptr(logits_teacher), _ptr(tokens), _ptr(cu_span), _ptr(driver),
         _ptr(prefix_len), R, T, V, K, eos_id,
@@ -270,6 +283,28 @@ def split_loss(kl_rev, kl_fwd, source, cu_span, n_emit, resp_len, agg_mode: int,
     _check(_lib.ipd_split_loss(_ptr(kl_rev), _ptr(kl_fwd), _ptr(source), _ptr(cu_span),
                                _ptr(n_emit), _ptr(resp_len), R, agg_mode, dir_mode, _ptr(out8),
                                None, 0, _stream(stream)), "ipd_split_loss")
+
+
+def split_loss_grad(logits_student, logits_teacher, topk_s, topk_t, source, cu_span, n_emit,
+                    resp_len, loss_out8, K: int, agg_mode: int, dir_mode: int, grad_scale: float,
+                    grad_idx: torch.Tensor, grad_val: torch.Tensor,
+                    grad_dense: Optional[torch.Tensor] = None, stream=None):
+    """Gradient of grad_scale * loss with respect to the student's logits:
+    sparse [T, 2K] ids / values, and the dense [T, V] form when ``grad_dense``
+    (fp32 or bf16) is given."""
+    R = cu_span.numel() - 1
+    T, V = logits_student.shape
+    dtype = DTYPE_F32
+    if grad_dense is not None:
+        if grad_dense.dtype == torch.bfloat16:
+            dtype = DTYPE_BF16
+        elif grad_dense.dtype != torch.float32:
+            raise IpdError(STATUS_CODES["IPD_ERR_INVALID_ARG"], "ipd_split_loss_grad: dense dtype")
+    _check(_lib.ipd_split_loss_grad(
+        _ptr(logits_student), _ptr(logits_teacher), _ptr(topk_s), _ptr(topk_t), _ptr(source),
+        _ptr(cu_span), _ptr(n_emit), _ptr(resp_len), _ptr(loss_out8), R, T, V, K, agg_mode,
+        dir_mode, grad_scale, _ptr(grad_idx), _ptr(grad_val), _ptr(grad_dense), dtype, None, 0,
+        _stream(stream)), "ipd_split_loss_grad")
 
 
 def device_error() -> int:

@@ -101,3 +101,29 @@ def test_score_ext_rejects_bad_rules_on_the_host():
         ipd.STATUS_CODES["IPD_ERR_UNSUPPORTED"]
     assert ipd._lib.ipd_full_kl(None, None, 3, 4096, None, None, None) == \
         ipd.STATUS_CODES["IPD_ERR_INVALID_ARG"]
+
+
+def test_loss_grad_host_validation():
+    from paper_2609_36546_gb300 import ipd
+    L = ipd._lib
+    bad = ipd.STATUS_CODES
+
+    def call(R=2, T=4, V=4096, K=16, agg=0, dmode=0, scale=1.0, gi=16, gv=16, dense=None,
+             dtype=0, ptr=16):
+        return L.ipd_split_loss_grad(*([ptr] * 9), R, T, V, K, agg, dmode, scale, gi, gv, dense,
+                                     dtype, None, 0, None)
+
+    assert L.ipd_loss_grad_workspace_size(100, 16) == 0
+    assert call(T=0, ptr=None, gi=None, gv=None) == 0           # nothing to do
+    assert call(K=33) == bad["IPD_ERR_UNSUPPORTED"]
+    assert call(K=0) == bad["IPD_ERR_UNSUPPORTED"]
+    assert call(V=8, K=16) == bad["IPD_ERR_UNSUPPORTED"]
+    assert call(agg=2) == bad["IPD_ERR_INVALID_ARG"]
+    assert call(dmode=4) == bad["IPD_ERR_INVALID_ARG"]
+    assert call(scale=float("nan")) == bad["IPD_ERR_INVALID_ARG"]
+    assert call(scale=float("inf")) == bad["IPD_ERR_INVALID_ARG"]
+    assert call(dense=32, dtype=2) == bad["IPD_ERR_INVALID_ARG"]
+    assert call(dense=40) == bad["IPD_ERR_INVALID_ARG"]          # not 16-byte aligned
+    assert call(gi=None) == bad["IPD_ERR_INVALID_ARG"]
+    assert call(R=0) == bad["IPD_ERR_INVALID_ARG"]                # positions without requests
+    assert call(R=-1) == bad["IPD_ERR_INVALID_ARG"]
