@@ -19,5 +19,13 @@ Parity status per function (what pins it is listed in tests/test_oracle_pins.py)
 * ``split_loss_grad`` -- pinned (central finite differences of ``topk_kl`` +
   ``split_loss`` in fp64, shift invariance of every row, zero rows off the
   emitted positions).
+* ``philox4x32_10`` -- pinned (the generator's published known-answer
+  vectors, tests/golden/philox4x32_10_kat.txt).
+* ``lg2_f32`` -- pinned (numpy log2 within 1.2e-6; exact powers of two).
+* ``sample_uniforms``, ``gumbel_scores``, ``sample_token`` -- pinned
+  (Kolmogorov-Smirnov uniformity; chi-square of 12000 draws against the
+  softmax at two temperatures; planted base and scale mistakes rejected).
+* ``next_token_after_verdict`` -- pinned (hand-worked takeover, handback,
+  no-transition and EOS cases).
 """
 from .ipd_oracle import *  # noqa: F401,F403

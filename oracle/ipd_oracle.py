@@ -409,3 +409,127 @@ def split_loss_grad(l_s, l_t, source, cu_span, n_emit, resp_len=None, K=16, agg_
                 g = pi_bar - q_bar
             G[t, S] = w * g
     return G
+
+
+# ----------------------------------------------------------------------------
+# seeded sampling: Gumbel-max over counter-based uniforms
+# ----------------------------------------------------------------------------
+# Training rollouts sample at temperature 1 with top-p 1 (App. A, training
+# configuration), i.e. from the full softmax of the logits.  A draw is defined bit-exactly so that any device
+# reproduces it:
+#   * uniform bits: Philox4x32 with 10 rounds (Salmon, Moraes, Dror and Shaw,
+#     "Parallel random numbers: as easy as 1, 2, 3", SC 2011), key = the
+#     64-bit seed (low word first), counter = (v // 4, draw low word, draw high
+#     word, 0); output word v % 4 belongs to token v;
+#   * u_v = (2 * (bits >> 9) + 1) * 2^-24, exactly representable, in (0, 1);
+#   * Gumbel-max in base 2: token = argmax_v  l_v * c - lg2(-lg2(u_v)), with
+#     c = fp32(log2 e) * inv_temperature; this is argmax_v l_v / temperature +
+#     G_v with G_v = -ln(-ln u_v) a standard Gumbel variable, rescaled by
+#     log2 e and shifted by the constant log2(ln 2), so the token is
+#     distributed as softmax(l / temperature);
+#   * lg2 is a fixed fp32 procedure (below), every operation rounded to fp32
+#     with no fused multiply-add; ties of the score go to the lower id.
+PHILOX_M0, PHILOX_M1 = 0xD2511F53, 0xCD9E8D57     # round multipliers
+PHILOX_W0, PHILOX_W1 = 0x9E3779B9, 0xBB67AE85     # key increments (Weyl sequence)
+LOG2E_F32_BITS = 0x3FB8AA3B                       # fp32 nearest to log2(e)
+# log2(1 + t) = t * P(t) on t in [sqrt(1/2) - 1, sqrt(2) - 1]; P's coefficients
+# (lowest degree first) are a least-squares fit of log2(1 + t) / t on 4000
+# Chebyshev nodes, rounded to fp32; |lg2(x) - log2(x)| <= 1.1e-6 for normal x
+LG2_POLY_BITS = (0x3FB8AA3A, 0xBF38AA93, 0x3EF63BAD, 0xBEB871A3, 0x3E92FB93, 0xBE7ECB25,
+                 0x3E6FD4B5, 0xBE15B661)
+
+
+def _f32(bits) -> np.float32:
+    return np.array([bits], dtype=np.uint32).view(np.float32)[0]
+
+
+def philox4x32_10(ctr: np.ndarray, key) -> np.ndarray:
+    """Philox4x32-10 of each counter row ctr[..., 0:4] (uint32) under the key
+    (k0, k1): ten rounds; a round multiplies words 0 and 2 by the two
+    multipliers and forms (hi(M1 c2) ^ c1 ^ k0, lo(M1 c2), hi(M0 c0) ^ c3 ^ k1,
+    lo(M0 c0)); the key is bumped by the Weyl increments between rounds."""
+    mask = np.uint64(0xFFFFFFFF)
+    c = [np.asarray(ctr[..., i], dtype=np.uint64) for i in range(4)]
+    k0, k1 = np.uint64(key[0]) & mask, np.uint64(key[1]) & mask
+    for _ in range(10):
+        p0 = np.uint64(PHILOX_M0) * c[0]
+        p1 = np.uint64(PHILOX_M1) * c[2]
+        c = [(p1 >> np.uint64(32)) ^ c[1] ^ k0, p1 & mask,
+             (p0 >> np.uint64(32)) ^ c[3] ^ k1, p0 & mask]
+        k0 = (k0 + np.uint64(PHILOX_W0)) & mask
+        k1 = (k1 + np.uint64(PHILOX_W1)) & mask
+    return np.stack(c, axis=-1).astype(np.uint32)
+
+
+def lg2_f32(x) -> np.ndarray:
+    """The fixed fp32 base-2 logarithm of the sampler, for positive normal x:
+    x = 2^e m with m in (sqrt(1/2), sqrt(2)] (exact bit operations),
+    t = m - 1 (exact), P(t) by Horner's rule, result e + t P(t); each product
+    and sum rounded to fp32."""
+    x = np.asarray(x, dtype=np.float32)
+    b = x.view(np.uint32)
+    e = ((b >> np.uint32(23)) & np.uint32(0xFF)).astype(np.int32) - 127
+    mb = (b & np.uint32(0x7FFFFF)) | np.uint32(0x3F800000)
+    big = mb > np.uint32(0x3FB504F3)                 # m > sqrt(2): halve it
+    mb = np.where(big, mb - np.uint32(0x00800000), mb).astype(np.uint32)
+    e = e + big.astype(np.int32)
+    t = mb.view(np.float32) - np.float32(1.0)
+    coef = [_f32(c) for c in LG2_POLY_BITS]
+    p = np.full(t.shape, coef[-1], dtype=np.float32)
+    for c in coef[-2::-1]:
+        p = (p * t).astype(np.float32) + c
+    return (e.astype(np.float32) + (t * p).astype(np.float32)).astype(np.float32)
+
+
+def sample_uniforms(vocab: int, seed: int, draw: int) -> np.ndarray:
+    """u_v for v in [0, vocab) of one draw (fp32)."""
+    mask = 0xFFFFFFFF
+    groups = (vocab + 3) // 4
+    ctr = np.zeros((groups, 4), dtype=np.uint32)
+    ctr[:, 0] = np.arange(groups, dtype=np.uint32)
+    ctr[:, 1] = draw & mask
+    ctr[:, 2] = (draw >> 32) & mask
+    bits = philox4x32_10(ctr, (seed & mask, (seed >> 32) & mask)).reshape(-1)[:vocab]
+    return ((bits >> np.uint32(9)).astype(np.float32) * np.float32(2.0) + np.float32(1.0)) * \
+        np.float32(2.0 ** -24)
+
+
+def gumbel_scores(l_bits, seed: int, draw: int, inv_temperature: float = 1.0) -> np.ndarray:
+    """Per-token scores l_v c - lg2(-lg2 u_v) of one draw, fp32."""
+    l = bf16_to_f64(l_bits).astype(np.float32)      # exact
+    c = _f32(LOG2E_F32_BITS) * np.float32(inv_temperature)
+    u = sample_uniforms(len(l), seed, draw)
+    e = -lg2_f32(u)
+    return (l * c).astype(np.float32) - lg2_f32(e)
+
+
+def sample_token(l_bits, seed: int, draw: int, inv_temperature: float = 1.0) -> int:
+    """One token drawn from softmax(l / temperature); ties to the lower id."""
+    return int(np.argmax(gumbel_scores(l_bits, seed, draw, inv_temperature)))
+
+
+def next_token_after_verdict(logits_s_bits, logits_t_bits, cu_span, prefix_len, verdict_out,
+                             seed: int, draw_base, inv_temperature: float = 1.0) -> np.ndarray:
+    """The first token of each request's next span when the verify step
+    already holds the logits it is drawn from.
+
+    After the verdict the accepted prefix ends at position P_r + n_r (n_r
+    emitted tokens), and the next token is drawn by the next driver from its
+    distribution at that position.  After a takeover at j (student span) the
+    teacher regenerates position j, whose distribution is the teacher's row j of
+    the span; after a handback at j (teacher span) the student continues at
+    position j + 1, its row j + 1 -- in both cases the next driver's row
+    n_r (Sec. 3.2.3, verdict stage).  With n_r = k_r (no transition) that row is not part of the step and
+    with done set the request has ended: -1.  The draw number is
+    draw_base[r] + P_r + n_r (the absolute position of the drawn token)."""
+    R = len(cu_span) - 1
+    out = np.full(R, -1, dtype=np.int64)
+    for r in range(R):
+        t0, t1 = int(cu_span[r]), int(cu_span[r + 1])
+        n = int(verdict_out["n_emit"][r])
+        if int(verdict_out["done"][r]) or n >= t1 - t0:
+            continue
+        rows = logits_t_bits if int(verdict_out["next_driver"][r]) == 1 else logits_s_bits
+        draw = (int(draw_base[r]) + int(prefix_len[r]) + n) & 0xFFFFFFFFFFFFFFFF
+        out[r] = sample_token(rows[t0 + n], seed, draw, inv_temperature)
+    return out

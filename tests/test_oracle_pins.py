@@ -636,3 +636,93 @@ def test_planted_gradient_mistakes_are_caught():
     fd = (_loss_of_student_logits(a, lt, source, cu, n_emit, None, K, 0, 0)
           - _loss_of_student_logits(b, lt, source, cu, n_emit, None, K, 0, 0)) / (2 * eps)
     assert abs(G[t, v] - fd) < 1e-8 and abs(-G[t, v] - fd) > 1e-4
+
+
+# ---------------------------------------------------------------------------
+# seeded sampler: Philox known answers, lg2 accuracy, the sampled distribution
+# ---------------------------------------------------------------------------
+def test_philox_known_answer_vectors():
+    rows = [l.split() for l in open(os.path.join(GOLDEN, "philox4x32_10_kat.txt"))
+            if l.strip() and not l.startswith("#")]
+    assert len(rows) == 3
+    for w in rows:
+        v = [int(x, 16) for x in w]
+        out = O.philox4x32_10(np.array([v[0:4]], dtype=np.uint32), (v[4], v[5]))[0]
+        assert out.tolist() == v[6:10]
+
+
+def test_lg2_against_numpy_log2():
+    xs = np.concatenate([np.exp(RNG.uniform(np.log(2.0 ** -26), np.log(32.0), 200000)),
+                         np.linspace(0.5, 2.0, 20001), [1 - 2.0 ** -24, 1 + 2.0 ** -23, 1.0,
+                                                        2.0 ** -24, 24.0, np.sqrt(2.0)]])
+    xs = xs.astype(np.float32)
+    ours = O.lg2_f32(xs).astype(np.float64)
+    ref = np.log2(xs.astype(np.float64))
+    assert np.abs(ours - ref).max() <= 1.2e-6
+    near = np.abs(xs - 1) < 0.3
+    assert (np.abs(ours - ref)[near] <= 4e-7 * np.maximum(np.abs(ref[near]), 2.0 ** -24) + 1e-12).all()
+    assert O.lg2_f32(np.float32(1.0)) == 0.0 and O.lg2_f32(np.float32(0.25)) == -2.0
+    # the sign the Gumbel transform relies on: lg2(u) < 0 for every u < 1
+    assert (O.lg2_f32(np.float32([1 - 2.0 ** -24, 0.5 + 2.0 ** -24])) < 0).all()
+
+
+def test_uniforms_are_uniform_and_open():
+    u = O.sample_uniforms(1 << 16, seed=12345, draw=7).astype(np.float64)
+    assert u.min() > 0 and u.max() < 1
+    assert scipy.stats.kstest(u, "uniform").pvalue > 1e-4
+    # distinct draws give distinct streams; the same draw repeats exactly
+    assert not np.array_equal(u, O.sample_uniforms(1 << 16, seed=12345, draw=8))
+    assert np.array_equal(u, O.sample_uniforms(1 << 16, seed=12345, draw=7))
+
+
+def _draw_counts(l_bits, n, inv_temperature=1.0, scores=None):
+    V = len(l_bits)
+    counts = np.zeros(V, dtype=np.int64)
+    for d in range(n):
+        s = O.gumbel_scores(l_bits, 99, d, inv_temperature) if scores is None else scores(d)
+        counts[int(np.argmax(s))] += 1
+    return counts
+
+
+@pytest.mark.parametrize("inv_t", [1.0, 0.5])
+def test_sampled_tokens_follow_the_softmax(inv_t):
+    l = np.array([0.0, 1.0, 2.0, -1.0, 0.5, 3.0])
+    bits = O.f64_to_bf16(l)
+    n = 12000
+    counts = _draw_counts(bits, n, inv_t)
+    p = scipy.special.softmax(l * inv_t)
+    assert scipy.stats.chisquare(counts, p * n).pvalue > 1e-4
+
+
+def test_planted_sampler_mistakes_are_caught():
+    l = np.array([0.0, 1.0, 2.0, -1.0, 0.5, 3.0])
+    bits = O.f64_to_bf16(l)
+    n = 12000
+    p = scipy.special.softmax(l) * n
+    lf = l.astype(np.float32)
+    # a natural log in the outer logarithm (base mismatch) samples a tempered softmax
+    nat = lambda d: lf * np.float32(1.4426950) - np.log(-O.lg2_f32(O.sample_uniforms(6, 99, d)))
+    assert scipy.stats.chisquare(_draw_counts(bits, n, scores=nat), p).pvalue < 1e-6
+    # dropping the log2(e) factor of the logits samples softmax(l ln 2)
+    noc = lambda d: lf - O.lg2_f32(-O.lg2_f32(O.sample_uniforms(6, 99, d)))
+    assert scipy.stats.chisquare(_draw_counts(bits, n, scores=noc), p).pvalue < 1e-6
+
+
+def test_next_token_after_verdict_picks_the_next_drivers_row():
+    V = 64
+    ls = O.f64_to_bf16(RNG.normal(size=(9, V)) * 2)
+    lt = O.f64_to_bf16(RNG.normal(size=(9, V)) * 2)
+    cu = np.array([0, 4, 7, 9])
+    prefix = np.array([10, 20, 30])
+    # request 0: student span, takeover at j = 2 -> the teacher's row 2 at position 12
+    # request 1: teacher span, handback at j = 0 -> the student's row 1 at position 21
+    # request 2: student span, everything accepted -> no row in this step
+    v = dict(n_emit=np.array([2, 1, 2]), done=np.array([0, 0, 0]),
+             next_driver=np.array([1, 0, 0]))
+    got = O.next_token_after_verdict(ls, lt, cu, prefix, v, seed=5, draw_base=np.array([100, 0, 0]))
+    assert got[0] == O.sample_token(lt[2], 5, 100 + 12)
+    assert got[1] == O.sample_token(ls[4 + 1], 5, 21)
+    assert got[2] == -1
+    # a request that ended (EOS) draws nothing
+    v["done"] = np.array([1, 0, 0])
+    assert O.next_token_after_verdict(ls, lt, cu, prefix, v, 5, np.array([100, 0, 0]))[0] == -1
