@@ -8,6 +8,8 @@ Parity status per function (what pins it is listed in tests/test_oracle_pins.py)
 
 * ``span_attention`` / ``paged_span_attention`` -- pinned (library SDPA in
   fp64, closed forms, paging invariants).
+* ``kv_append`` -- pinned (the appended paged cache attends exactly like
+  library SDPA over the concatenated sequence; unowned pages untouched).
 * ``log_softmax_row``, ``topk``, ``covered``, ``margin`` -- pinned (scipy,
   brute-force sort, rank identity).
 * ``topk_kl`` -- pinned (scipy KL on the renormalised support, K=1 closed

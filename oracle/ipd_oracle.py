@@ -60,6 +60,29 @@ def gather_pages(pages: np.ndarray, page_row: np.ndarray, L: int, page_size: int
     return cont[:L]
 
 
+def kv_append(k_pages: np.ndarray, v_pages: np.ndarray, k_new: np.ndarray, v_new: np.ndarray,
+              cu_new, seq_len, page_table, page_size: int = 16):
+    """The cache after the new tokens' K/V rows are written (Sec. 3.2.3: the
+    proposer's decode extends its own cache by one token, the verifier's
+    prefill writes the span's k tokens into its cache, each before the
+    attention that reads them).
+
+    k_pages, v_pages: [num_pages, Hkv, page_size, D]; k_new, v_new:
+    [total_new, Hkv, D].  Request r's rows cu_new[r] .. cu_new[r+1]-1 are the
+    last n_r tokens of its sequence of length seq_len[r] (the length after the
+    append): row i lands at position p = seq_len[r] - n_r + i, in page
+    page_table[r][p // page_size], slot p % page_size.  Returns new arrays."""
+    k_out, v_out = k_pages.copy(), v_pages.copy()
+    for r in range(len(cu_new) - 1):
+        n = int(cu_new[r + 1]) - int(cu_new[r])
+        for i in range(n):
+            p = int(seq_len[r]) - n + i
+            page = int(page_table[r][p // page_size])
+            k_out[page, :, p % page_size, :] = k_new[int(cu_new[r]) + i]
+            v_out[page, :, p % page_size, :] = v_new[int(cu_new[r]) + i]
+    return k_out, v_out
+
+
 def span_attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float) -> np.ndarray:
     """Causal attention of n span queries over a contiguous cache of L keys.
 

@@ -726,3 +726,44 @@ def test_next_token_after_verdict_picks_the_next_drivers_row():
     # a request that ended (EOS) draws nothing
     v["done"] = np.array([1, 0, 0])
     assert O.next_token_after_verdict(ls, lt, cu, prefix, v, 5, np.array([100, 0, 0]))[0] == -1
+
+
+# ---------------------------------------------------------------------------
+# KV append: the appended paged cache attends like the concatenated sequence
+# ---------------------------------------------------------------------------
+def test_kv_append_then_paged_attention_equals_sdpa_on_the_concatenation():
+    rng = np.random.default_rng(21)
+    Hkv, D, ps = 2, 128, 16
+    old_len = [5, 16, 30, 0]
+    n_new = [3, 1, 0, 17]                                 # span, decode, nothing, across pages
+    L = [a + b for a, b in zip(old_len, n_new)]
+    max_pages = max((x + ps - 1) // ps for x in L)
+    num_pages = sum((x + ps - 1) // ps for x in L) + 3
+    perm = rng.permutation(num_pages)
+    table = np.full((4, max_pages), -1)
+    used = 0
+    for r, x in enumerate(L):
+        for j in range((x + ps - 1) // ps):
+            table[r, j] = perm[used]; used += 1
+    kp = rng.normal(size=(num_pages, Hkv, ps, D)); vp = rng.normal(size=(num_pages, Hkv, ps, D))
+    old_k = [O.gather_pages(kp, table[r], old_len[r]) for r in range(4)]
+    old_v = [O.gather_pages(vp, table[r], old_len[r]) for r in range(4)]
+    cu = np.concatenate([[0], np.cumsum(n_new)])
+    kn = rng.normal(size=(int(cu[-1]), Hkv, D)); vn = rng.normal(size=(int(cu[-1]), Hkv, D))
+    k2, v2 = O.kv_append(kp, vp, kn, vn, cu, L, table)
+    for r in range(4):
+        if L[r] == 0:
+            continue
+        k_cat = np.concatenate([old_k[r], kn[cu[r]:cu[r + 1]]])
+        v_cat = np.concatenate([old_v[r], vn[cu[r]:cu[r + 1]]])
+        q = rng.normal(size=(max(n_new[r], 1), 4, D))
+        got = O.span_attention(q, O.gather_pages(k2, table[r], L[r]),
+                               O.gather_pages(v2, table[r], L[r]), 0.09)
+        np.testing.assert_allclose(got, _sdpa_reference(q, k_cat, v_cat, 0.09), rtol=1e-10, atol=1e-12)
+    # pages no request owns are untouched
+    free = np.setdiff1d(np.arange(num_pages), table[table >= 0])
+    assert np.array_equal(k2[free], kp[free]) and np.array_equal(v2[free], vp[free])
+    # a position off by one is caught: the appended rows no longer form the sequence
+    kb, vb = O.kv_append(kp, vp, kn, vn, cu, [x + 1 for x in L], np.pad(table, ((0, 0), (0, 1)),
+                                                                       constant_values=perm[-1]))
+    assert not np.array_equal(O.gather_pages(kb, table[0], L[0]), np.concatenate([old_k[0], kn[0:3]]))
