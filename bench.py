@@ -7,6 +7,7 @@ Inputs are synthetic, seeded, resident in HBM and larger than L2, so every
 step streams its KV pages and logits from DRAM.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--config I] [--impl reference]
+  python bench.py --next-rows [--config I] [--steps K]
 
 Prints one JSON line (rank 0).  ``--impl reference`` times the fp64 CPU
 oracle (the only reference that exists for this path) on a bounded sample of
@@ -485,6 +486,206 @@ def run_e2e(step, w, K, stream, world):
                     "host results each step, synchronised per step; KV pools resident"}
 
 
+# ---------------------------------------------------------------------------
+# --next-rows: the calls beyond the step (rules and by-products, full KL, the
+# loss gradient), each timed alone from a CUDA graph of one call, with its
+# algorithmic bytes and the oracle timed on a sample beside it
+# ---------------------------------------------------------------------------
+def _graph_ms(fn, reps: int) -> float:
+    import torch
+    cur = torch.cuda.current_stream()
+    side = torch.cuda.Stream()
+    side.wait_stream(cur)
+    with torch.cuda.stream(side):
+        for _ in range(3):
+            fn()
+    cur.wait_stream(side)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        fn()
+    for _ in range(3):
+        g.replay()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    a.record(cur)
+    for _ in range(reps):
+        g.replay()
+    b.record(cur)
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / reps
+
+
+def _oracle_ms(fn, n: int) -> float:
+    t0 = time.perf_counter()
+    fn()
+    return (time.perf_counter() - t0) * 1e3 / max(n, 1)
+
+
+def run_next_rows(args):
+    import numpy as np
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    import ipd_synth as S
+    import oracle as O
+    from paper_2609_36546_gb300 import VerifyStep, ipd
+    from tests.parity import u16
+
+    cfg = args.config
+    w = S.make_workload(cfg, seed=cfg, device="cuda")
+    st = VerifyStep.from_workload(w, device="cuda")
+    T, V, K, R = st.T, st.V, st.K, st.R
+    reps = max(5, min(args.steps, 200))
+    peak, peak_kind = _peaks()
+    dev = "cuda"
+    ent_s = torch.empty(T, device=dev)
+    ent_t = torch.empty(T, device=dev)
+    ovl = torch.empty(T, device=dev)
+    tks = torch.empty(T, K, device=dev, dtype=torch.int32)
+    tkt = torch.empty_like(tks)
+    rev = torch.empty(T, device=dev)
+    fwd = torch.empty(T, device=dev)
+    gi = torch.empty(T, 2 * K, device=dev, dtype=torch.int32)
+    gv = torch.empty(T, 2 * K, device=dev)
+    dense32 = torch.empty(T, V, device=dev, dtype=torch.float32)
+    dense16 = torch.empty(T, V, device=dev, dtype=torch.bfloat16)
+    tau = 3.0
+
+    def score_ex():
+        ipd.score_span_ex(st.logits_s, st.logits_t, st.tokens, st.cu_span, st.driver,
+                          st.prefix_len, K, st.eos_id, st.score, st.ws_score,
+                          ipd.RULE_ENTROPY_S, ipd.RULE_ALWAYS, tau, 0.0, ent_s, ent_t, ovl, tks, tkt)
+
+    nxt = torch.empty(R, device=dev, dtype=torch.int32)
+    seed = 0x5EED
+
+    def score_draw():
+        ipd.score_span_ex(st.logits_s, st.logits_t, st.tokens, st.cu_span, st.driver,
+                          st.prefix_len, K, st.eos_id, st.score, st.ws_score, next_token=nxt,
+                          sample_seed=seed)
+
+    # standalone draws: one row per request (the proposers' decode rows stand-in)
+    dec_rows = st.logits_s[:R] if T >= R else st.logits_s
+    n_dec = dec_rows.shape[0]
+    draw_ids = torch.arange(n_dec, device=dev, dtype=torch.int64)
+    dec_tok = torch.empty(n_dec, device=dev, dtype=torch.int32)
+    ws_s = torch.empty(max(8, ipd.sample_workspace_size(n_dec, V)), device=dev, dtype=torch.uint8)
+    # KV appends of the step: every batch's new rows (span rows for the verifiers,
+    # one row per request for the proposers) at the last positions of each sequence
+    appends = []
+    kv_bytes = 0
+    for name, b, idx, cname in st.batches:
+        q, cu_q, seq, ptab = b._keep[0], b._keep[1], b._keep[2], b._keep[3]
+        cache = st.cache_t if cname == "teacher" else st.cache_s
+        hkv = cache.k_pages.shape[1]
+        nrow = int(q.shape[0])
+        kn = torch.randn(nrow, hkv, 128, device=dev).to(torch.bfloat16)
+        vn = torch.randn(nrow, hkv, 128, device=dev).to(torch.bfloat16)
+        appends.append((cache, kn, vn, cu_q, seq, ptab))
+        kv_bytes += 2 * 2 * nrow * hkv * 128 * 2       # K and V rows, read and written
+
+    def kv_all():
+        for cache, kn, vn, cu_q, seq, ptab in appends:
+            ipd.kv_append(cache, kn, vn, cu_q, seq, ptab)
+
+    score_ex()
+    st.run_loss()
+    grad_args = (st.logits_s, st.logits_t, tks, tkt, st.score["source"], st.cu_span,
+                 st.score["n_emit"], st.resp_len, st.out8, K, st.agg_mode, st.dir_mode, 1.0, gi, gv)
+    sampler = ClockSampler(_smi_index(0))
+    time.sleep(0.3)
+    rows_bytes = 2 * T * V * 2
+    t_plain = _graph_ms(st.run_score, reps)
+    t_ex = _graph_ms(score_ex, reps)
+    t_kl = _graph_ms(lambda: ipd.full_kl(st.logits_s, st.logits_t, rev, fwd), reps)
+    t_gs = _graph_ms(lambda: ipd.split_loss_grad(*grad_args), reps)
+    t_g32 = _graph_ms(lambda: ipd.split_loss_grad(*grad_args, dense32), reps)
+    t_g16 = _graph_ms(lambda: ipd.split_loss_grad(*grad_args, dense16), reps)
+    t_draw = _graph_ms(score_draw, reps)
+    t_samp = _graph_ms(lambda: ipd.sample(dec_rows, seed, draw_ids, dec_tok, ws_s), reps)
+    t_kv = _graph_ms(kv_all, reps)
+    clocks = sampler.stop()
+    torch.cuda.synchronize()
+    if ipd.device_error() != 0:
+        raise RuntimeError("device-side check failed")
+    n_emitted = int((st.score["source"] != 255).sum())
+
+    # the oracle on a sample of the same inputs
+    n_s = min(4, T)
+    ls_h, lt_h = u16(st.logits_s[:n_s]), u16(st.logits_t[:n_s])
+    ls64, lt64 = O.bf16_to_f64(ls_h), O.bf16_to_f64(lt_h)
+    o_kl = _oracle_ms(lambda: [O.full_kl(ls64[i], lt64[i]) for i in range(n_s)], n_s)
+    r_s = 0
+    cu_h = st.cu_span.cpu().numpy()
+    while r_s < R and cu_h[r_s + 1] == 0:
+        r_s += 1
+    t0, t1 = int(cu_h[r_s]), int(cu_h[r_s + 1])
+    sub_cu = np.array([0, t1 - t0])
+    sub = lambda x: x[t0:t1]
+    ls_r, lt_r = u16(sub(st.logits_s)), u16(sub(st.logits_t))
+    o_ex = _oracle_ms(lambda: O.score_span(
+        ls_r, lt_r, sub(st.tokens).cpu().numpy(), sub_cu, st.driver[r_s:r_s + 1].cpu().numpy(),
+        st.prefix_len[r_s:r_s + 1].cpu().numpy(), K, st.eos_id, takeover_rule=O.RULE_ENTROPY_S,
+        handback_rule=O.RULE_ALWAYS, takeover_tau=tau), t1 - t0)
+    src_r = sub(st.score["source"]).cpu().numpy()
+    ne_r = st.score["n_emit"][r_s:r_s + 1].cpu().numpy()
+    o_g = _oracle_ms(lambda: O.split_loss_grad(O.bf16_to_f64(ls_r), O.bf16_to_f64(lt_r), src_r,
+                                               sub_cu, ne_r, None, K), t1 - t0)
+    dec_h = u16(dec_rows[:n_s])
+    o_samp = _oracle_ms(lambda: [O.sample_token(dec_h[i], seed, i) for i in range(n_s)], n_s)
+    # the oracle's append of one request's span rows, on a pool of that request's pages
+    cache0, kn0, vn0, cu0, seq0, pt0 = appends[0]
+    cu0h, seq0h, pt0h = cu0.cpu().numpy(), seq0.cpu().numpy(), pt0.cpu().numpy()
+    n0 = int(cu0h[1] - cu0h[0])
+    pg = [int(x) for x in pt0h[0, :(int(seq0h[0]) + 15) // 16]]
+    kp0 = u16(cache0.k_pages[pg]); vp0 = u16(cache0.v_pages[pg])
+    o_kv = _oracle_ms(lambda: O.kv_append(kp0, vp0, u16(kn0[:n0]), u16(vn0[:n0]), np.array([0, n0]),
+                                          seq0h[:1], np.arange(len(pg))[None, :]), n0)
+
+    def row(ms, nbytes, oracle_ms_pos, note):
+        gbs = nbytes / (ms / 1e3) / 1e9
+        return {"ms": ms, "us_per_position": ms * 1e3 / max(T, 1), "bytes": nbytes, "gbs": gbs,
+                "frac": gbs / peak, "oracle_ms_per_position": oracle_ms_pos, "note": note}
+
+    sparse_bytes = T * 2 * K * 4 * 2 + T * 2 * K * 2 * 2 + n_emitted * 2 * K * 8
+    line = {
+        "mode": "next_rows", "config": {"workload": _workload_name(cfg), "seed": cfg,
+                                         "tokens": T, "requests": R, "vocab": V, "K": K},
+        "peak": peak, "peak_kind": peak_kind, "reps": reps,
+        "timing": "each call alone, replayed from a CUDA graph of one call; CUDA events "
+                  "around the replays; inputs larger than L2",
+        "rows": {
+            "score_span (default step call, for comparison)": row(
+                t_plain, rows_bytes, None, "full rows of both models read once"),
+            "score_span_ex (entropy-S takeover, always handback, entropies, overlap, "
+            "top-K lists)": row(t_ex, rows_bytes, o_ex, "full rows of both models read once"),
+            "full_kl": row(t_kl, rows_bytes, o_kl, "full rows of both models read once"),
+            "split_loss_grad sparse": row(t_gs, sparse_bytes, o_g,
+                                          "top-K lists + 4K gathered logits + 2K (id, value)"),
+            "split_loss_grad sparse + dense fp32": row(t_g32, T * V * 4 + sparse_bytes, None,
+                                                       "dense [T, V] fp32 written"),
+            "split_loss_grad sparse + dense bf16": row(t_g16, T * V * 2 + sparse_bytes, None,
+                                                       "dense [T, V] bf16 written"),
+            "score_span_ex + next-token draw": row(
+                t_draw, rows_bytes + R * V * 2, None,
+                "score pass, then one row per request re-read for the draw"),
+            "sample (one row per request)": dict(row(
+                t_samp, n_dec * V * 2, o_samp, "ALU-bound: Philox + two lg2 per entry"),
+                rows=n_dec, us_per_row=t_samp * 1e3 / max(n_dec, 1),
+                oracle_ms_per_row=o_samp),
+            "kv_append (all span and decode rows of the step)": dict(row(
+                t_kv, kv_bytes, o_kv, "latency-bound: ~1-4 MB per step"),
+                oracle_ms_per_row=o_kv),
+        },
+        "oracle_sample": f"full_kl and sample: {n_s} rows; score_span_ex and split_loss_grad: "
+                         f"request {r_s} ({t1 - t0} positions); kv_append: one request's "
+                         f"{n0} rows; numpy, one core",
+        "clocks": clocks,
+    }
+    print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -494,9 +695,13 @@ def main():
     ap.add_argument("--impl", default="ipd", choices=["ipd", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=200)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--next-rows", action="store_true",
+                    help="time the calls beyond the step instead (one GPU)")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
-    if args.impl == "reference":
+    if args.next_rows:
+        run_next_rows(args)
+    elif args.impl == "reference":
         run_reference(args)
     else:
         run_gpu(args)

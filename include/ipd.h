@@ -18,8 +18,9 @@
  *   ipd_split_loss   the source-split objective of the step.
  *
  * Beyond the step itself: ipd_score_span_ex (other takeover / handback rules,
- * entropies, top-K overlap, top-K lists), ipd_full_kl (full-vocabulary KL both
- * ways) and ipd_split_loss_grad (the objective's gradient with respect to the
+ * entropies, top-K overlap, top-K lists, the next span's first token),
+ * ipd_full_kl (full-vocabulary KL both ways), ipd_sample (seeded sampling of
+ * rows), ipd_kv_append (new K/V rows into a paged cache) and ipd_split_loss_grad (the objective's gradient with respect to the
  * student's logits, sparse and dense).
  *
  * Conventions for every call
@@ -221,6 +222,13 @@ typedef struct {
   int32_t *topk_s;     /* [total_tokens][K] Top_K(pi_t) token ids, best first (ties: lower id
                           first), or NULL; ipd_split_loss_grad takes these lists */
   int32_t *topk_t;     /* [total_tokens][K] Top_K(q_t), same order, or NULL */
+  int32_t *next_token; /* [num_reqs] first token of each request's next span, drawn (as
+                          ipd_sample does) from the next driver's row n_emit[r] of the span
+                          with draw number draw_base[r] + prefix_len[r] + n_emit[r]; -1 when
+                          the request ended or every span token was emitted; or NULL */
+  const uint64_t *draw_base; /* [num_reqs] device, or NULL for 0 */
+  uint64_t sample_seed;
+  float inv_temperature;     /* > 0 and finite when next_token is set (1 = the paper's rollouts) */
 } ipd_score_ext;
 
 /* ipd_score_span with selectable rules and by-products.  ext == NULL is the
@@ -310,6 +318,53 @@ int ipd_split_loss(const float *kl_rev, const float *kl_fwd, const uint8_t *sour
                    const int32_t *cu_span, const int32_t *n_emit, const int32_t *resp_len,
                    int num_reqs, int agg_mode, int dir_mode, float *out8,
                    void *workspace, size_t workspace_bytes, ipd_stream_t stream);
+
+/* Writes the K/V rows of newly computed tokens into a paged cache (Sec. 3.2.3:
+ * the proposer's decode extends its own cache by one token, the verifier's
+ * prefill writes the span's k tokens into its cache; each before the
+ * attention that reads them).
+ *  k_pages, v_pages  [num_pages][num_kv_heads][16][128] bf16, written in place
+ *  k_new, v_new      [total_new][num_kv_heads][128] bf16 rows of the new tokens
+ *  cu_new            [num_reqs + 1] int32: request r owns rows cu_new[r] .. cu_new[r+1]-1
+ *  seq_len           [num_reqs] int32 sequence length AFTER the append: row i of
+ *                    request r (n_r rows) goes to position seq_len[r] - n_r + i,
+ *                    page page_table[r][pos / 16], slot pos % 16
+ *  page_table        [num_reqs][max_pages] int32, as in ipd_attn_batch
+ * All pointers 16-byte aligned.  Returns IPD_ERR_UNSUPPORTED unless
+ * page_size == 16 and head_dim == 128.  A position outside the page table or
+ * a page id outside the pool is recorded (IPD_DEVERR_SEQ_LEN /
+ * IPD_DEVERR_PAGE_ID) and that row is skipped.  Rolling a cache back after a
+ * verdict needs no kernel: the next step passes the shorter length. */
+int ipd_kv_append(uint16_t *k_pages, uint16_t *v_pages, int64_t num_pages, int num_kv_heads,
+                  int page_size, int head_dim, const uint16_t *k_new, const uint16_t *v_new,
+                  const int32_t *cu_new, const int32_t *seq_len, const int32_t *page_table,
+                  int max_pages, int num_reqs, int total_new, ipd_stream_t stream);
+
+/* Seeded sampling from softmax(l * inv_temperature) of each row (training
+ * rollouts sample at temperature 1, top-p 1: App. A).  A draw is a fixed
+ * function of (row, seed, draw number, inv_temperature), reproducible on any
+ * device:
+ *   bits_v = word v % 4 of Philox4x32-10(counter (v / 4, draw_lo, draw_hi, 0),
+ *            key (seed_lo, seed_hi))  (Salmon et al., SC 2011)
+ *   u_v    = (2 (bits_v >> 9) + 1) * 2^-24
+ *   s_v    = fl(l_v * c) - lg2(-lg2(u_v)),  c = fl(fp32(log2 e) * inv_temperature)
+ *   token  = argmax_v s_v (ties to the lower id)
+ * where every product and sum is rounded to fp32 separately and lg2(x), for
+ * x = 2^e m with m in (sqrt(1/2), sqrt(2)], is e + t P(t), t = m - 1, P by
+ * Horner's rule with the fp32 coefficients (bit patterns, lowest degree first)
+ * 3FB8AA3A BF38AA93 3EF63BAD BEB871A3 3E92FB93 BE7ECB25 3E6FD4B5 BE15B661.
+ * This is the Gumbel-max trick in base 2, so the token follows
+ * softmax(l * inv_temperature).
+ *  logits   [n_rows][vocab] bf16, 16-byte aligned, vocab a multiple of 8
+ *  draw_id  [n_rows] uint64 draw numbers (device), or NULL for all 0
+ *  tokens   [n_rows] int32 output
+ * Returns IPD_ERR_INVALID_ARG for a non-positive or non-finite
+ * inv_temperature or a missing pointer, IPD_ERR_UNSUPPORTED for vocab % 8 != 0,
+ * IPD_ERR_WORKSPACE for a workspace below ipd_sample_workspace_size. */
+size_t ipd_sample_workspace_size(int n_rows, int vocab);
+int ipd_sample(const uint16_t *logits, int n_rows, int vocab, uint64_t seed,
+               const uint64_t *draw_id, float inv_temperature, int32_t *tokens, void *workspace,
+               size_t workspace_bytes, ipd_stream_t stream);
 
 /* Element type of the dense gradient of ipd_split_loss_grad. */
 #define IPD_DTYPE_F32 0

@@ -6,6 +6,7 @@
 extern "C" __attribute__((visibility("hidden"))) unsigned int ipd_internal_take_attn_error();
 extern "C" __attribute__((visibility("hidden"))) unsigned int ipd_internal_take_score_error();
 extern "C" __attribute__((visibility("hidden"))) unsigned int ipd_internal_take_loss_error();
+extern "C" __attribute__((visibility("hidden"))) unsigned int ipd_internal_take_kv_error();
 
 extern "C" int ipd_get_device_error(uint32_t *code) {
   if (!code) return IPD_ERR_INVALID_ARG;
@@ -13,8 +14,10 @@ extern "C" int ipd_get_device_error(uint32_t *code) {
   const unsigned int a = ipd_internal_take_attn_error();
   const unsigned int b = ipd_internal_take_score_error();
   const unsigned int c = ipd_internal_take_loss_error();
-  if (a == 0xffffffffu || b == 0xffffffffu || c == 0xffffffffu) return IPD_ERR_CUDA;
-  *code = a ? a : (b ? b : c);
+  const unsigned int d = ipd_internal_take_kv_error();
+  if (a == 0xffffffffu || b == 0xffffffffu || c == 0xffffffffu || d == 0xffffffffu)
+    return IPD_ERR_CUDA;
+  *code = a ? a : (b ? b : (c ? c : d));
   return IPD_OK;
 }
 

@@ -576,9 +576,24 @@ extern "C" __attribute__((visibility("hidden"))) unsigned int ipd_internal_take_
   return v;
 }
 
+extern "C" __attribute__((visibility("hidden"))) size_t ipd_internal_sample_ws(int n_rows,
+                                                                              int vocab);
+extern "C" __attribute__((visibility("hidden"))) int ipd_internal_sample_after_verdict(
+    const uint16_t *ls, const uint16_t *lt, int num_reqs, int total_tokens, int vocab,
+    uint64_t seed, const uint64_t *draw_base, float inv_temperature, const int32_t *cu_span,
+    const int32_t *prefix_len, const int32_t *n_emit, const uint8_t *next_driver,
+    const uint8_t *done, int32_t *next_token, void *ws, cudaStream_t st);
+
+namespace {
+// workspace: the row records, then (256-byte aligned) the sampler's partials
+size_t rows_region(int total_tokens) {
+  return ((size_t)total_tokens * 2 * kParts * sizeof(RowOut) + 255) & ~(size_t)255;
+}
+}  // namespace
+
 extern "C" size_t ipd_score_workspace_size(int num_reqs, int total_tokens, int vocab, int K) {
   if (num_reqs < 0 || total_tokens < 0 || vocab < 1 || K < 1) return 0;
-  return (size_t)total_tokens * 2 * kParts * sizeof(RowOut) + 256;
+  return rows_region(total_tokens) + ipd_internal_sample_ws(num_reqs, vocab) + 256;
 }
 
 namespace {
@@ -593,6 +608,9 @@ bool epi_opts(const ipd_score_ext *ext, EpiOpts *o) {
     return false;
   *o = EpiOpts{ext->takeover_rule, ext->handback_rule, ext->takeover_tau, ext->handback_tau,
                ext->entropy_s, ext->entropy_t, ext->topk_overlap, ext->topk_s, ext->topk_t};
+  if (ext->next_token && !(ext->inv_temperature > 0.f &&
+                           ext->inv_temperature - ext->inv_temperature == 0.f))
+    return false;  // the draw needs a positive, finite inverse temperature
   return true;
 }
 }  // namespace
@@ -642,6 +660,11 @@ extern "C" int ipd_score_span_ex(const uint16_t *logits_student, const uint16_t 
       logp_s, logp_t, feedback, kl_rev, kl_fwd, covered, margin, source, first_trans, n_emit,
       next_driver, new_len, done, total_tokens, opt);
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
+  if (ext && ext->next_token)
+    return ipd_internal_sample_after_verdict(
+        logits_student, logits_teacher, num_reqs, total_tokens, vocab, ext->sample_seed,
+        ext->draw_base, ext->inv_temperature, cu_span, prefix_len, n_emit, next_driver, done,
+        ext->next_token, static_cast<char *>(workspace) + rows_region(total_tokens), st);
   return IPD_OK;
 }
 

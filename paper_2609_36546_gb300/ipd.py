@@ -32,7 +32,8 @@ EXPORTS = ("ipd_attn_workspace_size", "ipd_verify_attn", "ipd_decode_attn",
            "ipd_score_workspace_size", "ipd_score_span", "ipd_loss_workspace_size",
            "ipd_split_loss", "ipd_get_device_error", "ipd_status_string", "ipd_version",
            "ipd_score_span_static", "ipd_score_span_ex", "ipd_full_kl",
-           "ipd_loss_grad_workspace_size", "ipd_split_loss_grad")
+           "ipd_loss_grad_workspace_size", "ipd_split_loss_grad", "ipd_sample_workspace_size",
+           "ipd_sample", "ipd_kv_append")
 # takeover / handback rules (IPD_RULE_*)
 RULE_TOPK, RULE_ENTROPY_S, RULE_ENTROPY_T, RULE_ALWAYS, RULE_NEVER = 0, 1, 2, 3, 4
 # element type of the dense gradient (IPD_DTYPE_*)
@@ -69,7 +70,8 @@ class _ScoreExt(ctypes.Structure):
     _fields_ = [("takeover_rule", ctypes.c_int32), ("handback_rule", ctypes.c_int32),
                 ("takeover_tau", ctypes.c_float), ("handback_tau", ctypes.c_float),
                 ("entropy_s", c_p), ("entropy_t", c_p), ("topk_overlap", c_p),
-                ("topk_s", c_p), ("topk_t", c_p)]
+                ("topk_s", c_p), ("topk_t", c_p), ("next_token", c_p), ("draw_base", c_p),
+                ("sample_seed", ctypes.c_uint64), ("inv_temperature", ctypes.c_float)]
 
 
 class _AttnBatch(ctypes.Structure):
@@ -107,6 +109,14 @@ _lib.ipd_loss_grad_workspace_size.argtypes = [c_i, c_i]
 _lib.ipd_split_loss_grad.restype = c_i
 _lib.ipd_split_loss_grad.argtypes = ([c_p] * 9 + [c_i] * 6 + [ctypes.c_float, c_p, c_p, c_p, c_i,
                                       c_p, c_sz, c_p])
+_lib.ipd_sample_workspace_size.restype = c_sz
+_lib.ipd_sample_workspace_size.argtypes = [c_i, c_i]
+_lib.ipd_sample.restype = c_i
+_lib.ipd_sample.argtypes = [c_p, c_i, c_i, ctypes.c_uint64, c_p, ctypes.c_float, c_p, c_p, c_sz,
+                            c_p]
+_lib.ipd_kv_append.restype = c_i
+_lib.ipd_kv_append.argtypes = [c_p, c_p, ctypes.c_int64, c_i, c_i, c_i, c_p, c_p, c_p, c_p, c_p,
+                               c_i, c_i, c_i, c_p]
 _lib.ipd_get_device_error.restype = c_i
 _lib.ipd_get_device_error.argtypes = [ctypes.POINTER(ctypes.c_uint32)]
 _lib.ipd_status_string.restype = ctypes.c_char_p
@@ -236,15 +246,19 @@ def score_span_ex(logits_student, logits_teacher, tokens, cu_span, driver, prefi
                   entropy_t: Optional[torch.Tensor] = None,
                   topk_overlap: Optional[torch.Tensor] = None,
                   topk_s: Optional[torch.Tensor] = None, topk_t: Optional[torch.Tensor] = None,
-                  stream=None):
+                  next_token: Optional[torch.Tensor] = None,
+                  draw_base: Optional[torch.Tensor] = None, sample_seed: int = 0,
+                  inv_temperature: float = 1.0, stream=None):
     """ipd_score_span with selectable takeover / handback rules and the
-    optional per-token entropies and top-K overlap ratio (fp32 [T] tensors)
-    and top-K id lists (int32 [T, K])."""
+    optional per-token entropies and top-K overlap ratio (fp32 [T] tensors),
+    top-K id lists (int32 [T, K]) and the next span's first token per request
+    (int32 [R]; draw numbers from ``draw_base``, uint64 as int64 [R])."""
     R = driver.numel()
     T, V = logits_student.shape
     ext = _ScoreExt(takeover_rule, handback_rule, takeover_tau, handback_tau,
                     _ptr(entropy_s), _ptr(entropy_t), _ptr(topk_overlap), _ptr(topk_s),
-                    _ptr(topk_t))
+                    _ptr(topk_t), _ptr(next_token), _ptr(draw_base),
+                    sample_seed & 0xFFFFFFFFFFFFFFFF, inv_temperature)
     _check(_lib.ipd_score_span_ex(
         _ptr(logits_student), _ptr(logits_teacher), _ptr(tokens), _ptr(cu_span), _ptr(driver),
         _ptr(prefix_len), R, T, V, K, eos_id,
@@ -283,6 +297,33 @@ def split_loss(kl_rev, kl_fwd, source, cu_span, n_emit, resp_len, agg_mode: int,
     _check(_lib.ipd_split_loss(_ptr(kl_rev), _ptr(kl_fwd), _ptr(source), _ptr(cu_span),
                                _ptr(n_emit), _ptr(resp_len), R, agg_mode, dir_mode, _ptr(out8),
                                None, 0, _stream(stream)), "ipd_split_loss")
+
+
+def kv_append(cache: "KVCache", k_new, v_new, cu_new, seq_len, page_table, stream=None):
+    """Writes the new tokens' K/V rows ([n, Hkv, 128] bf16) into the cache's
+    pages at the last positions of each request's sequence (``seq_len`` is
+    the length after the append)."""
+    R = cu_new.numel() - 1
+    _check(_lib.ipd_kv_append(_ptr(cache.k_pages), _ptr(cache.v_pages), cache.k_pages.shape[0],
+                              cache.k_pages.shape[1], 16, 128, _ptr(k_new), _ptr(v_new),
+                              _ptr(cu_new), _ptr(seq_len), _ptr(page_table),
+                              page_table.shape[1], R, k_new.shape[0], _stream(stream)),
+           "ipd_kv_append")
+
+
+def sample_workspace_size(n_rows: int, vocab: int) -> int:
+    return int(_lib.ipd_sample_workspace_size(n_rows, vocab))
+
+
+def sample(logits, seed: int, draw_id: Optional[torch.Tensor], tokens: torch.Tensor,
+           workspace: torch.Tensor, inv_temperature: float = 1.0, stream=None):
+    """One seeded draw per row of ``logits`` ([n, V] bf16) into ``tokens``
+    (int32 [n]); ``draw_id`` holds the rows' uint64 draw numbers (as int64)."""
+    n, V = logits.shape
+    _check(_lib.ipd_sample(_ptr(logits), n, V, seed & 0xFFFFFFFFFFFFFFFF, _ptr(draw_id),
+                           inv_temperature, _ptr(tokens), _ptr(workspace),
+                           workspace.numel() * workspace.element_size(), _stream(stream)),
+           "ipd_sample")
 
 
 def split_loss_grad(logits_student, logits_teacher, topk_s, topk_t, source, cu_span, n_emit,

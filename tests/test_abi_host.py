@@ -127,3 +127,41 @@ def test_loss_grad_host_validation():
     assert call(gi=None) == bad["IPD_ERR_INVALID_ARG"]
     assert call(R=0) == bad["IPD_ERR_INVALID_ARG"]                # positions without requests
     assert call(R=-1) == bad["IPD_ERR_INVALID_ARG"]
+
+
+def test_sample_host_validation():
+    import ctypes
+    from paper_2609_36546_gb300 import ipd
+    L = ipd._lib
+    bad = ipd.STATUS_CODES
+    ws = 1 << 20
+    assert L.ipd_sample_workspace_size(4, 151936) == 4 * 19 * 8
+    assert L.ipd_sample(None, 0, 4096, 1, None, 1.0, None, None, 0, None) == 0
+    assert L.ipd_sample(16, 4, 4100, 1, None, 1.0, 16, 16, ws, None) == bad["IPD_ERR_UNSUPPORTED"]
+    for it in (0.0, -1.0, float("inf"), float("nan")):
+        assert L.ipd_sample(16, 4, 4096, 1, None, it, 16, 16, ws, None) == bad["IPD_ERR_INVALID_ARG"]
+    assert L.ipd_sample(24, 4, 4096, 1, None, 1.0, 16, 16, ws, None) == bad["IPD_ERR_INVALID_ARG"]
+    assert L.ipd_sample(16, 4, 4096, 1, None, 1.0, 16, 16, 8, None) == bad["IPD_ERR_WORKSPACE"]
+    # the draw after the verdict needs a positive, finite inverse temperature
+    ext = ipd._ScoreExt(0, 0, 0.0, 0.0, None, None, None, None, None, 16, None, 5, 0.0)
+    st = L.ipd_score_span_ex(*([None] * 6), 0, 0, 4096, 16, -1, *([None] * 13),
+                             ctypes.byref(ext), None, 0, None)
+    assert st == bad["IPD_ERR_INVALID_ARG"]
+
+
+def test_kv_append_host_validation():
+    from paper_2609_36546_gb300 import ipd
+    L = ipd._lib
+    bad = ipd.STATUS_CODES
+    p = 16
+    ok_args = lambda **kw: [kw.get("kp", p), p, kw.get("np", 100), kw.get("hkv", 4),
+                            kw.get("ps", 16), kw.get("hd", 128), kw.get("kn", p), p, p, p, p,
+                            kw.get("mp", 8), kw.get("R", 2), kw.get("n", 3), None]
+    assert L.ipd_kv_append(*ok_args(n=0)) == 0
+    assert L.ipd_kv_append(*ok_args(ps=32)) == bad["IPD_ERR_UNSUPPORTED"]
+    assert L.ipd_kv_append(*ok_args(hd=64)) == bad["IPD_ERR_UNSUPPORTED"]
+    assert L.ipd_kv_append(*ok_args(hkv=0)) == bad["IPD_ERR_INVALID_ARG"]
+    assert L.ipd_kv_append(*ok_args(R=0)) == bad["IPD_ERR_INVALID_ARG"]
+    assert L.ipd_kv_append(*ok_args(kp=None)) == bad["IPD_ERR_INVALID_ARG"]
+    assert L.ipd_kv_append(*ok_args(kn=24)) == bad["IPD_ERR_INVALID_ARG"]   # misaligned
+    assert L.ipd_kv_append(*ok_args(np=-1)) == bad["IPD_ERR_INVALID_ARG"]
