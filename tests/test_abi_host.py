@@ -135,7 +135,8 @@ def test_sample_host_validation():
     L = ipd._lib
     bad = ipd.STATUS_CODES
     ws = 1 << 20
-    assert L.ipd_sample_workspace_size(4, 151936) == 4 * 19 * 8
+    assert L.ipd_sample_workspace_size(4, 151936) == 2 * 2048 * 8
+    assert L.ipd_sample_workspace_size(3000, 4096) == 2 * 3000 * 8
     assert L.ipd_sample(None, 0, 4096, 1, None, 1.0, None, None, 0, None) == 0
     assert L.ipd_sample(16, 4, 4100, 1, None, 1.0, 16, 16, ws, None) == bad["IPD_ERR_UNSUPPORTED"]
     for it in (0.0, -1.0, float("inf"), float("nan")):
