@@ -443,39 +443,29 @@ def run_gpu(args):
 
 
 def run_e2e(step, w, K, stream, world):
-    """The same step through host buffers: the per-step inputs (queries, both
-    models' logits, tokens, request metadata) are copied from pinned host
-    memory, the step runs, and its results (per-request verdict, per-token
-    sources, loss record) are copied back; the KV pools stay resident (they
-    are the cache state, not step inputs)."""
+    """The same step through host buffers, via VerifyStep.run_from_host: the
+    per-step inputs (queries and their metadata, both models' logits, tokens,
+    request metadata) are copied from pinned host memory, the step runs, and
+    its results (per-request verdict, per-token sources, loss record) are
+    copied back and read before the next step; the KV pools stay resident
+    (they are the cache state, not step inputs).  The attention starts when
+    the queries land and the logits are scored chunk by chunk as they land,
+    so the step's time is about the host-to-device transfer."""
     import torch
-    dev_inputs = []
-    for _, b, _, _ in step.batches:
-        q, cu_q, seq, ptab, _ = b._keep
-        dev_inputs += [q, cu_q, seq, ptab]
-    dev_inputs += [step.logits_s, step.logits_t, step.tokens, step.cu_span, step.driver,
-                   step.prefix_len]
-    host_inputs = [t.cpu().pin_memory() for t in dev_inputs]
-    outs = [step.score[n] for n in ("first_trans", "n_emit", "next_driver", "new_len", "done",
-                                     "source")] + [step.out8]
-    host_outs = [torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in outs]
-    h2d = sum(t.numel() * t.element_size() for t in host_inputs)
-    d2h = sum(t.numel() * t.element_size() for t in host_outs)
+    host = step.host_inputs(n_chunks=4)
+    names = ("first_trans", "n_emit", "next_driver", "new_len", "done", "source")
+    results = {n: torch.empty(step.score[n].shape, dtype=step.score[n].dtype, pin_memory=True)
+               for n in names}
+    results["out8"] = torch.empty(8, pin_memory=True)
+    h2d = sum(t.numel() * t.element_size() for k, t in host.items() if not k.startswith("_"))
+    d2h = sum(t.numel() * t.element_size() for t in results.values())
     for _ in range(2):
-        for d, h in zip(dev_inputs, host_inputs):
-            d.copy_(h, non_blocking=True)
-        step.run(stream)
-        for h, d in zip(host_outs, outs):
-            h.copy_(d, non_blocking=True)
-        torch.cuda.synchronize()
+        step.run_from_host(host, results, stream)
+        stream.synchronize()
     _barrier(world)
     t0 = time.perf_counter()
     for _ in range(K):
-        for d, h in zip(dev_inputs, host_inputs):
-            d.copy_(h, non_blocking=True)
-        step.run(stream)
-        for h, d in zip(host_outs, outs):
-            h.copy_(d, non_blocking=True)
+        step.run_from_host(host, results, stream)
         stream.synchronize()          # the engine reads the verdict before the next step
     el = time.perf_counter() - t0
     el = _max_over_ranks(el, world)
@@ -483,7 +473,9 @@ def run_e2e(step, w, K, stream, world):
     return {"value": toks / el, "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": K,
             "note": "pinned host -> device inputs (Q, logits, tokens, metadata) and device -> "
-                    "host results each step, synchronised per step; KV pools resident"}
+                    "host results each step, synchronised per step; KV pools resident; the "
+                    "attention overlaps the logits transfer, which is scored in 4 chunks as it "
+                    "lands"}
 
 
 # ---------------------------------------------------------------------------

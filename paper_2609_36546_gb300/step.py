@@ -160,6 +160,94 @@ class VerifyStep:
             self.run(overlap=overlap)
         return graph
 
+    # -- one step end to end from host memory ---------------------------------
+    def host_inputs(self, n_chunks: int = 4) -> dict:
+        """Pinned host copies of every per-step input (each batch's queries and
+        metadata, both models' logits, tokens, request metadata), plus the
+        request-aligned chunk plan that run_from_host uses for the logits."""
+        h = {}
+        for i, (_, b, _, _) in enumerate(self.batches):
+            q, cu_q, seq, ptab, _ = b._keep
+            for name, t in (("q", q), ("cu_q", cu_q), ("seq", seq), ("ptab", ptab)):
+                h[f"{name}{i}"] = t.cpu().pin_memory()
+        for name in ("logits_s", "logits_t", "tokens", "cu_span", "driver", "prefix_len"):
+            h[name] = getattr(self, name).cpu().pin_memory()
+        # chunk c covers requests [r0, r1) and span positions [t0, t1), with
+        # about T / n_chunks positions each; its offsets are rebased to t0
+        cu = h["cu_span"].to(torch.int64)
+        bounds, r0 = [], 0
+        for c in range(1, n_chunks + 1):
+            target = self.T * c // n_chunks
+            r1 = self.R if c == n_chunks else \
+                max(r0, int(torch.searchsorted(cu, target, right=True)) - 1)
+            if r1 > r0 or c == n_chunks:
+                bounds.append((r0, r1, int(cu[r0]), int(cu[r1])))
+            r0 = r1
+        h["cu_chunk"] = torch.cat([(cu[a:b + 1] - cu[a]).to(torch.int32) for a, b, _, _ in bounds]
+                                  ).pin_memory()
+        h["_chunks"] = bounds
+        return h
+
+    def run_from_host(self, host: dict, results: dict, stream=None):
+        """One step whose inputs sit in pinned host memory (``host_inputs``)
+        and whose results (verdict per request, source per token, loss
+        record) are copied back into ``results`` (pinned, same names as the
+        score outputs plus "out8"); the caller synchronises ``stream``.
+
+        The queries and metadata go first and the attention starts as soon as
+        they land; the logits, most of the bytes, follow on a copy stream in
+        request-aligned chunks, and each chunk is scored as soon as it lands,
+        so that only the last chunk's scoring and the loss follow the
+        transfer.  Every kernel sees the same data as in run(), so the
+        results are bit-identical."""
+        main = stream if stream is not None else torch.cuda.current_stream(self.device)
+        if getattr(self, "_copy", None) is None:
+            self._copy = torch.cuda.Stream(device=self.device)
+            self._scorer = torch.cuda.Stream(device=self.device)
+            self._cu_chunk = torch.empty_like(host["cu_chunk"], device=self.device)
+        cp, sc = self._copy, self._scorer
+        if self._cu_chunk.numel() != host["cu_chunk"].numel():
+            self._cu_chunk = torch.empty_like(host["cu_chunk"], device=self.device)
+        # the previous step's kernels are done with every buffer written here
+        cp.wait_stream(main)
+        sc.wait_stream(main)
+        with torch.cuda.stream(main):
+            for i, (_, b, _, _) in enumerate(self.batches):
+                q, cu_q, seq, ptab, _ = b._keep
+                for name, t in (("q", q), ("cu_q", cu_q), ("seq", seq), ("ptab", ptab)):
+                    t.copy_(host[f"{name}{i}"], non_blocking=True)
+            for name in ("tokens", "cu_span", "driver", "prefix_len"):
+                getattr(self, name).copy_(host[name], non_blocking=True)
+            self._cu_chunk.copy_(host["cu_chunk"], non_blocking=True)
+        meta = torch.cuda.Event()
+        meta.record(main)
+        self.run_attention(main)
+        landed = []
+        with torch.cuda.stream(cp):
+            for r0, r1, t0, t1 in host["_chunks"]:
+                if t1 > t0:
+                    self.logits_s[t0:t1].copy_(host["logits_s"][t0:t1], non_blocking=True)
+                    self.logits_t[t0:t1].copy_(host["logits_t"][t0:t1], non_blocking=True)
+                ev = torch.cuda.Event()
+                ev.record(cp)
+                landed.append(ev)
+        sc.wait_event(meta)
+        off = 0
+        for (r0, r1, t0, t1), ev in zip(host["_chunks"], landed):
+            sc.wait_event(ev)
+            out = {n: self.score[n][t0:t1] for n, _ in ipd.SCORE_TOKEN_OUTPUTS}
+            out.update({n: self.score[n][r0:r1] for n, _ in ipd.SCORE_REQ_OUTPUTS})
+            ipd.score_span(self.logits_s[t0:t1], self.logits_t[t0:t1], self.tokens[t0:t1],
+                           self._cu_chunk[off:off + r1 - r0 + 1], self.driver[r0:r1],
+                           self.prefix_len[r0:r1], self.K, self.eos_id, out, self.ws_score, sc)
+            off += r1 - r0 + 1
+        main.wait_stream(sc)
+        main.wait_stream(cp)
+        self.run_loss(main)
+        with torch.cuda.stream(main):
+            for name, t in results.items():
+                t.copy_(self.out8 if name == "out8" else self.score[name], non_blocking=True)
+
     # -- bytes the step must move (algorithmic) --------------------------------
     def attn_bytes(self, ctx: torch.Tensor) -> int:
         """KV pages read (exact lengths) + Q read + O written, both caches."""

@@ -120,6 +120,43 @@ def test_graph_replay_equals_direct_calls(lib, overlap):
     assert lib.device_error() == 0
 
 
+@pytest.mark.parametrize("n_chunks", [1, 3, 5])
+def test_step_from_host_equals_direct_calls(lib, n_chunks):
+    """VerifyStep.run_from_host (queries first, logits in request-aligned
+    chunks on a copy stream, each chunk scored as it lands) gives the same
+    bits as the three calls on resident inputs."""
+    spec = S.small_spec(n_req=9, ctx=(100, 2500), span=(0, 16))
+    w, step = _run(spec, 39)
+    first = {k: v.clone() for k, v in step.score.items()}
+    outs = [b.out.clone() for _, b, _, _ in step.batches]
+    o8 = step.out8.clone()
+    host = step.host_inputs(n_chunks)
+    names = ("first_trans", "n_emit", "next_driver", "new_len", "done", "source")
+    results = {n: torch.empty(step.score[n].shape, dtype=step.score[n].dtype, pin_memory=True)
+               for n in names}
+    results["out8"] = torch.empty(8, pin_memory=True)
+    for _ in range(2):
+        for v in step.score.values():
+            v.zero_()
+        for _, b, _, _ in step.batches:
+            b.out.zero_()
+        step.logits_s.zero_()
+        step.logits_t.zero_()
+        step.out8.zero_()
+        stream = torch.cuda.current_stream()
+        step.run_from_host(host, results, stream)
+        stream.synchronize()
+        for k, v in step.score.items():
+            assert torch.equal(first[k].view(torch.uint8), v.view(torch.uint8)), k
+        for a, (_, b, _, _) in zip(outs, step.batches):
+            assert torch.equal(a.view(torch.int16), b.out.view(torch.int16))
+        assert torch.equal(o8, step.out8)
+        for n in names:
+            assert torch.equal(results[n], first[n].cpu()), n
+        assert torch.equal(results["out8"], o8.cpu())
+    assert lib.device_error() == 0
+
+
 def test_decode_alone_equals_colaunched(lib):
     spec = S.small_spec(n_req=6, ctx=(10, 900))
     w, step = _run(spec, 41)
