@@ -25,8 +25,10 @@
 //     chunk's keys) and stack the two P terms in the two 64-row halves of one
 //     operand; larger tiles keep one thread per row.  S is double-buffered,
 //     so the softmax of chunk j overlaps Q K^T of j+1 and P V of j-1.
-//   CUDA-core path (fewer rows: GQA group 2 decode): fp32 FMA, two pages of
-//     16 keys per warp and stage, two lanes per key.
+//   CUDA-core path (fewer rows: the GQA-2 decode and one-token spans, two
+//     rows): fp32 FMA, two pages of 16 keys per warp and stage, two lanes per
+//     key.  From four rows up the tensor path is faster even with most of its
+//     tile empty: at 4-6 rows the CUDA-core FMAs limit the stream.
 // Warp roles: warps 0-3 compute, warp 4 streams KV pages, warp 5 issues the
 // tensor-core instructions in a fixed order (Q K^T of chunk j, then P V of
 // chunk j-1).
@@ -62,7 +64,7 @@ constexpr int kTensorBytes = kStagePages * kPageBytes;  // 32 KB of K (or V) per
 constexpr int kStageBytes = 2 * kTensorBytes;     // 64 KB
 constexpr int kTcRows = 128;                      // TMEM lanes of a tensor-core tile (M)
 constexpr int kTcSplitRows = 64;                  // tiles up to this size split rows over two threads
-constexpr int kTcMinRows = 8;                     // tasks with at least this many rows use it
+constexpr int kTcMinRows = 4;                     // tasks with at least this many rows use it
 constexpr int kCcRows = kTcMinRows - 1;           // CUDA-core tasks have fewer rows
 constexpr int kCW = 4;                            // compute warps
 constexpr int kProducerWarp = 4;
