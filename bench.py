@@ -450,7 +450,9 @@ def run_e2e(step, w, K, stream, world):
     copied back and read before the next step; the KV pools stay resident
     (they are the cache state, not step inputs).  The attention starts when
     the queries land and the logits are scored chunk by chunk as they land,
-    so the step's time is about the host-to-device transfer."""
+    so the step's time is about the host-to-device transfer.  The step, its
+    copies included, is replayed from one CUDA graph
+    (VerifyStep.capture_from_host)."""
     import torch
     host = step.host_inputs(n_chunks=4)
     names = ("first_trans", "n_emit", "next_driver", "new_len", "done", "source")
@@ -459,13 +461,14 @@ def run_e2e(step, w, K, stream, world):
     results["out8"] = torch.empty(8, pin_memory=True)
     h2d = sum(t.numel() * t.element_size() for k, t in host.items() if not k.startswith("_"))
     d2h = sum(t.numel() * t.element_size() for t in results.values())
+    graph = step.capture_from_host(host, results)
     for _ in range(2):
-        step.run_from_host(host, results, stream)
+        graph.replay()
         stream.synchronize()
     _barrier(world)
     t0 = time.perf_counter()
     for _ in range(K):
-        step.run_from_host(host, results, stream)
+        graph.replay()                # copies in, the step, results out
         stream.synchronize()          # the engine reads the verdict before the next step
     el = time.perf_counter() - t0
     el = _max_over_ranks(el, world)
@@ -475,7 +478,7 @@ def run_e2e(step, w, K, stream, world):
             "note": "pinned host -> device inputs (Q, logits, tokens, metadata) and device -> "
                     "host results each step, synchronised per step; KV pools resident; the "
                     "attention overlaps the logits transfer, which is scored in 4 chunks as it "
-                    "lands"}
+                    "lands; the step with its copies replayed from one CUDA graph"}
 
 
 # ---------------------------------------------------------------------------

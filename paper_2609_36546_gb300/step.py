@@ -248,6 +248,22 @@ class VerifyStep:
             for name, t in results.items():
                 t.copy_(self.out8 if name == "out8" else self.score[name], non_blocking=True)
 
+    def capture_from_host(self, host: dict, results: dict, warmup: int = 2
+                          ) -> "torch.cuda.CUDAGraph":
+        """run_from_host recorded as one CUDA graph: every copy and kernel of
+        the step, with the same pinned host buffers and device buffers at
+        each replay, without the per-call host work of issuing them."""
+        side = torch.cuda.Stream(device=self.device)
+        side.wait_stream(torch.cuda.current_stream(self.device))
+        for _ in range(warmup):
+            self.run_from_host(host, results, side)
+        side.synchronize()
+        torch.cuda.current_stream(self.device).wait_stream(side)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            self.run_from_host(host, results, torch.cuda.current_stream(self.device))
+        return graph
+
     # -- bytes the step must move (algorithmic) --------------------------------
     def attn_bytes(self, ctx: torch.Tensor) -> int:
         """KV pages read (exact lengths) + Q read + O written, both caches."""

@@ -157,6 +157,37 @@ def test_step_from_host_equals_direct_calls(lib, n_chunks):
     assert lib.device_error() == 0
 
 
+def test_step_from_host_graph_equals_direct_calls(lib):
+    """capture_from_host records run_from_host as one graph; each replay
+    copies the pinned inputs in, runs the step and copies the results out."""
+    spec = S.small_spec(n_req=8, ctx=(100, 2000), span=(0, 12))
+    w, step = _run(spec, 43)
+    first = {k: v.clone() for k, v in step.score.items()}
+    o8 = step.out8.clone()
+    host = step.host_inputs(3)
+    names = ("first_trans", "n_emit", "next_driver", "new_len", "done", "source")
+    results = {n: torch.empty(step.score[n].shape, dtype=step.score[n].dtype, pin_memory=True)
+               for n in names}
+    results["out8"] = torch.empty(8, pin_memory=True)
+    graph = step.capture_from_host(host, results)
+    for _ in range(2):
+        for v in step.score.values():
+            v.zero_()
+        step.logits_s.zero_()
+        step.logits_t.zero_()
+        step.out8.zero_()
+        for r in results.values():
+            r.zero_()
+        graph.replay()
+        torch.cuda.synchronize()
+        for k, v in step.score.items():
+            assert torch.equal(first[k].view(torch.uint8), v.view(torch.uint8)), k
+        for n in names:
+            assert torch.equal(results[n], first[n].cpu()), n
+        assert torch.equal(results["out8"], o8.cpu())
+    assert lib.device_error() == 0
+
+
 def test_decode_alone_equals_colaunched(lib):
     spec = S.small_spec(n_req=6, ctx=(10, 900))
     w, step = _run(spec, 41)
