@@ -42,6 +42,12 @@ SMALL = [
     ("V-equals-K", S.small_spec(n_req=3, K=8, vocab=8, ctx=(1, 50)), 11),
     ("wide-vocab", S.small_spec(n_req=2, vocab=151936, sigma=3.0, logits="boost", span=(4, 8),
                                 ctx=(100, 400)), 12),
+    # spans past 16 tokens: teacher tasks of 264-320 rows, three 128-row tiles each
+    ("many-row-blocks", S.small_spec(n_req=3, ctx=(600, 3000), span=(33, 40), direction="S"), 13),
+    ("K32-wide-vocab", S.small_spec(n_req=2, K=32, vocab=151936, sigma=3.0, span=(2, 6),
+                                    ctx=(50, 300)), 14),
+    # student-verified spans of 1-3 tokens: 2-row (CUDA-core) and 4-6-row (tensor) tasks
+    ("short-teacher-spans", S.small_spec(n_req=9, direction="T", span=(1, 3), ctx=(30, 2000)), 15),
 ]
 
 
