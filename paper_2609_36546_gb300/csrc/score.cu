@@ -25,7 +25,8 @@ constexpr int kRowThreads = 128;  // eight row CTAs per SM: every row of a step 
 constexpr int kRowWarps = kRowThreads / 32;
 constexpr int kEpiThreads = 256;
 constexpr int kParts = 1;    // a logits row is split into this many parts, one CTA each
-constexpr int kQueue = 160;  // per-warp queue of vectors that passed the filter (32 + 4 * 32)
+constexpr int kMaxGroups = 32;    // group maxima a row thread keeps
+constexpr int kMaxGroupVecs = 8;  // vectors a lane puts on its warp's list per round
 constexpr int kBuf = 64;     // per-warp candidate buffer: up to 32 kept keys + one round of 32
 
 // One part of one logits row.
@@ -118,138 +119,65 @@ __device__ __forceinline__ int count_greater32(const unsigned long long *list, u
 //   - the part's exact top-K (K <= 32) under the order (logit desc, token id
 //     asc), a 64-bit key (bf16 order code << 32 | ~token id) making keys
 //     distinct and the order total.
-// A key at or below the current threshold th cannot be among the part's
-// top-K: th is either a key with at least K larger keys in the part (the
-// warm-up value) or the K-th best key a warp already holds.  Vectors whose
-// maximum reaches th's value go to a per-warp queue; 32 queued vectors are
-// examined at once, one per lane, and keys above th go to the warp's buffer,
-// which is cut back to its best K (by rank) whenever it fills.
+// The stream does only the log-sum-exp and, per thread, notes the largest
+// logit of every group of its vectors (two iterations, 64 logits: one
+// shared-memory store).  Afterwards tau = the K-th largest of the threads'
+// maxima: K distinct logits are >= tau, so every top-K logit is >= tau and
+// lies in a group whose maximum is >= tau -- about K groups of the part.
+// Those groups are read again (from L2), their keys >= (tau, largest id) go
+// to the warp's buffer, which is cut back to its best K (by rank) when it
+// fills, and the warps' lists are merged by rank.
 template <bool kEntropy>  // also accumulate sum exp(l - m) l (entropies / entropy rules)
 __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
     const uint16_t *__restrict__ ls, const uint16_t *__restrict__ lt, int vocab, int K,
     RowOut *__restrict__ out) {
-  __shared__ unsigned long long s_theta;
+  constexpr int U = 4;  // vectors per thread and iteration
+  __shared__ uint16_t s_gmax[kMaxGroups][kRowThreads];  // group maxima (order codes, 0: none)
+  __shared__ float s_sorted[kRowWarps][32];
+  __shared__ float s_tau;
   __shared__ unsigned long long s_lists[kRowWarps][32];
   __shared__ unsigned long long s_buf[kRowWarps][kBuf];
-  __shared__ uint4 s_qraw[kRowWarps][kQueue];
-  __shared__ int s_qidx[kRowWarps][kQueue];
+  __shared__ int s_cand[kRowWarps][32 * kMaxGroupVecs];  // a round's candidate vectors
   __shared__ float s_m[kRowWarps], s_s[kRowWarps], s_u[kRowWarps];
 
   const int row_id = blockIdx.x / kParts, part = blockIdx.x % kParts;
   const int t = row_id >> 1, model = row_id & 1;
   const uint16_t *row = (model ? lt : ls) + (size_t)t * vocab;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, tid = threadIdx.x;
   const int nvec = vocab >> 3;
   const int per = (nvec + kParts - 1) / kParts;
   const int v_lo = min(nvec, part * per), v_hi = min(nvec, v_lo + per);
-  if (threadIdx.x == 0) s_theta = 0ull;
-  __syncthreads();
-  volatile unsigned long long *vtheta = &s_theta;
+  const int n_iter = (v_hi - v_lo + kRowThreads * U - 1) / (kRowThreads * U);
+  // iterations per group: two, or more so that a thread has at most kMaxGroups
+  const int ipg = max(2, (n_iter + kMaxGroups - 1) / kMaxGroups);
+  const int n_groups = (n_iter + ipg - 1) / ipg;
   unsigned long long *buf = s_buf[warp];
 
   float m = -INFINITY;
-  unsigned long long s2 = 0ull;     // running sum of exp(l - m), as a packed pair
-  unsigned long long u2 = 0ull;     // running sum of exp(l - m) * l, as a packed pair
-  unsigned long long theta = 0ull;  // K-th best key this warp holds (0: fewer than K)
-  int nb = 0;                       // keys in the warp's buffer
-  int qn = 0;                       // vectors in the warp's queue
+  unsigned long long s2 = 0ull;  // running sum of exp(l - m), as a packed pair
+  unsigned long long u2 = 0ull;  // running sum of exp(l - m) * l, as a packed pair
 
-  // Block-wide warm-up: every thread takes the largest value among its first
-  // U vectors; with tau the (max(K,16)+1)-th largest of those values (ties
-  // counted), at least max(K,16)+1 logits of the part are >= tau, so at least
-  // that many keys lie strictly above the key (tau, largest index) =
-  // ord(tau) << 32, which starts the shared threshold.
-  constexpr int U = 4;
-  uint4 pre[U];
-  float lane_best = -INFINITY;
-#pragma unroll
-  for (int u = 0; u < U; ++u) {
-    const int v0 = v_lo + u * kRowThreads + (int)threadIdx.x;
-    pre[u] = make_uint4(0xff80ff80u, 0xff80ff80u, 0xff80ff80u, 0xff80ff80u);  // -inf
-    if (v0 < v_hi) pre[u] = ldg_stream(row + (size_t)v0 * 8);
-  }
-#pragma unroll
-  for (int u = 0; u < U; ++u) lane_best = fmaxf(lane_best, bf16x8_max(pre[u]));
-  {
-    float *sv = reinterpret_cast<float *>(s_lists);  // [8][32] floats, sorted per warp
-    sv[warp * 32 + lane] = warp_sort_desc_f(lane_best, lane);
-    __syncthreads();
-    const float c = sv[warp * 32 + lane];
-    int gt = 0, ge = 0;
-#pragma unroll 1
-    for (int w2 = 0; w2 < kRowWarps; ++w2) {
-      gt += count_above32(sv + w2 * 32, c, false);
-      ge += count_above32(sv + w2 * 32, c, true);
-    }
-    const int need = (K > 16 ? K : 16) + 1;
-    if (c != -INFINITY && gt < need && ge >= need)
-      s_theta = (unsigned long long)ord16(__float_as_uint(c) >> 16) << 32;
-    __syncthreads();
-  }
-
-  // Keep the best min(K, nb) keys of the buffer, sorted, and raise theta.
-  auto compact = [&]() {
-    __syncwarp();
-    const unsigned long long a = lane < nb ? buf[lane] : 0ull;
-    const unsigned long long b = lane + 32 < nb ? buf[lane + 32] : 0ull;
-    int ra = 0, rb = 0;
-    for (int j = 0; j < nb; ++j) {
-      const unsigned long long x = buf[j];
-      ra += x > a;
-      rb += x > b;
-    }
-    __syncwarp();
-    if (lane < nb && ra < K) buf[ra] = a;
-    if (lane + 32 < nb && rb < K) buf[rb] = b;
-    __syncwarp();
-    nb = nb < K ? nb : K;
-    if (nb == K) {
-      theta = buf[K - 1];
-      if (lane == 0 && theta > *vtheta) atomicMax(&s_theta, theta);
-    }
-  };
-  // Examine queued vectors q0 .. q0 + n - 1 (n <= 32), one per lane.
-  auto examine = [&](int q0, int n) {
-    const bool have = lane < n;
-    uint4 r = make_uint4(0, 0, 0, 0);
-    int v = 0;
-    if (have) {
-      r = s_qraw[warp][q0 + lane];
-      v = s_qidx[warp][q0 + lane];
-    }
-    __syncwarp();
-#pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      const unsigned long long sth = *vtheta;
-      const unsigned long long th = theta > sth ? theta : sth;
-      const unsigned long long key = make_key(elem_bits(r, e), (uint32_t)v * 8u + e);
-      const bool c = have && key > th;
-      const unsigned bal = __ballot_sync(0xffffffffu, c);
-      if (bal) {
-        if (nb + 32 > kBuf) compact();
-        if (c) buf[nb + __popc(bal & ((1u << lane) - 1u))] = key;
-        nb += __popc(bal);
-      }
-    }
-  };
-
+  // ---- stream: log-sum-exp and group maxima ----
   // Each iteration takes four 16-byte vectors per thread and issues the loads
   // of the next iteration's four before it works on them, so eight loads per
   // thread are in flight.  Per 8 logits: the maximum on the packed bf16
   // words, then unpack, one fused multiply-add and one hardware 2^x each for
-  // the sum.  The trip count is the same for every thread of the block
-  // (warp-wide ballots below).
+  // the sum.
   uint4 nxt[U];
 #pragma unroll
-  for (int u = 0; u < U; ++u) nxt[u] = pre[u];
-  for (int base = v_lo; base < v_hi; base += kRowThreads * U) {
+  for (int u = 0; u < U; ++u) {
+    const int v0 = v_lo + u * kRowThreads + tid;
+    nxt[u] = make_uint4(0xff80ff80u, 0xff80ff80u, 0xff80ff80u, 0xff80ff80u);  // -inf
+    if (v0 < v_hi) nxt[u] = ldg_stream(row + (size_t)v0 * 8);
+  }
+  float gmax = -INFINITY;
+  for (int it = 0; it < n_iter; ++it) {
+    const int base = v_lo + it * kRowThreads * U;
     uint4 raw[U];
-    int vv[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       raw[u] = nxt[u];
-      vv[u] = base + u * kRowThreads + (int)threadIdx.x;
-      const int vn = vv[u] + kRowThreads * U;
+      const int vn = base + (U + u) * kRowThreads + tid;
       nxt[u] = make_uint4(0xff80ff80u, 0xff80ff80u, 0xff80ff80u, 0xff80ff80u);  // -inf
       if (vn < v_hi) nxt[u] = ldg_stream(row + (size_t)vn * 8);
     }
@@ -257,6 +185,14 @@ __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
 #pragma unroll
     for (int u = 0; u < U; ++u) vmx[u] = bf16x8_max(raw[u]);
     const float bmax = fmaxf(fmaxf(vmx[0], vmx[1]), fmaxf(vmx[2], vmx[3]));
+    gmax = fmaxf(gmax, bmax);
+    if (it % ipg == ipg - 1 || it == n_iter - 1) {
+      // vectors past the part read as -inf; a group with none of the part's
+      // vectors keeps code 0 (a real logit, -inf included, has a code >= 1)
+      const bool real = v_lo + (it / ipg) * ipg * kRowThreads * U + tid < v_hi;
+      s_gmax[it / ipg][tid] = real ? (uint16_t)ord16(__float_as_uint(gmax) >> 16) : (uint16_t)0;
+      gmax = -INFINITY;
+    }
     if (bmax > m) {
       const float f = ex2_approx((m - bmax) * kLog2e);
       float s0, s1, u0, u1;
@@ -284,43 +220,115 @@ __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
         }
       }
     }
-    // vectors that may hold a key above the threshold go to the queue
-    const unsigned long long sth = *vtheta;
-    const unsigned long long th = theta > sth ? theta : sth;
-    const float thf = key_val(th);  // equal values go on to the full key test
-    uint32_t pmask = 0;
+  }
+
+  // ---- tau: the K-th largest of the threads' maxima ----
+  // A thread that read no logit of the part holds -inf and is not counted;
+  // with fewer than K counted maxima every group of the part qualifies.
+  if (tid == 0) s_tau = -INFINITY;
+  {
+    const bool real = v_lo + tid < v_hi;
+    s_sorted[warp][lane] = warp_sort_desc_f(real ? m : -INFINITY, lane);
+    __syncthreads();
+    // c is this lane's entry of its warp's sorted list; the K-th largest of
+    // all 128 has fewer than K entries above it and at least K at or above
+    // (when that is -inf -- fewer than K logits read -- tau stays -inf)
+    const float c = s_sorted[warp][lane];
+    int gt = 0, ge = 0;
+#pragma unroll 1
+    for (int w2 = 0; w2 < kRowWarps; ++w2) {
+      gt += count_above32(s_sorted[w2], c, false);
+      ge += count_above32(s_sorted[w2], c, true);
+    }
+    if (c != -INFINITY && gt < K && ge >= K) s_tau = c;
+    __syncthreads();
+  }
+  const float tau = s_tau;
+  const uint32_t g_code = tau == -INFINITY ? 1u : ord16(__float_as_uint(tau) >> 16);
+
+  // ---- examine the groups that reach tau ----
+  // Keys > (tau, largest id) are the candidates: every logit >= tau.  A lane
+  // loads four of a qualifying group's vectors at once, then the warp
+  // examines them vector by vector.
+  const unsigned long long th = tau == -INFINITY ? 0ull : (unsigned long long)g_code << 32;
+  unsigned long long theta = 0ull;  // K-th best key this warp holds (0: fewer than K)
+  int nb = 0;
+  auto compact = [&]() {
+    __syncwarp();
+    const unsigned long long a = lane < nb ? buf[lane] : 0ull;
+    const unsigned long long b = lane + 32 < nb ? buf[lane + 32] : 0ull;
+    int ra = 0, rb = 0;
+    for (int j = 0; j < nb; ++j) {
+      const unsigned long long x = buf[j];
+      ra += x > a;
+      rb += x > b;
+    }
+    __syncwarp();
+    if (lane < nb && ra < K) buf[ra] = a;
+    if (lane + 32 < nb && rb < K) buf[rb] = b;
+    __syncwarp();
+    nb = nb < K ? nb : K;
+    if (nb == K) theta = buf[K - 1];
+  };
+  // Rounds: every lane takes up to kMaxGroupVecs vectors of its next
+  // qualifying group; the warp lists them (a prefix sum over lanes) and
+  // examines the list one vector per lane, loading 32 at a time.  Usually a
+  // single round.
+  int j_next = 0, q_next = 0;  // this lane's next group, and next vector in it
+  while (true) {
+    while (j_next < n_groups && s_gmax[j_next][tid] < g_code) ++j_next;
+    const bool have = j_next < n_groups;
+    if (!__any_sync(0xffffffffu, have)) break;
+    const int it0 = j_next * ipg;
+    const int g_n = have ? (min(it0 + ipg, n_iter) - it0) * U : 0;  // the group's vectors
+    const int n_lane = min(kMaxGroupVecs, g_n - q_next);
+    int off = n_lane;  // inclusive prefix sum over lanes
 #pragma unroll
-    for (int u = 0; u < U; ++u)
-      if (vv[u] < v_hi && (th == 0ull || vmx[u] >= thf)) pmask |= 1u << u;
-    if (__any_sync(0xffffffffu, pmask != 0)) {
-      const int cnt = __popc(pmask);
-      int off = cnt;  // inclusive scan over lanes
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, off, o);
+      if (lane >= o) off += y;
+    }
+    const int total = __shfl_sync(0xffffffffu, off, 31);
+    off -= n_lane;
+    int *cand = s_cand[warp];
+    for (int q = 0; q < n_lane; ++q) {
+      const int qq = q_next + q;
+      cand[off + q] = v_lo + (it0 + qq / U) * kRowThreads * U + (qq % U) * kRowThreads + tid;
+    }
+    __syncwarp();
+    for (int b0 = 0; b0 < total; b0 += 32) {
+      const int v = b0 + lane < total ? cand[b0 + lane] : -1;
+      const bool ok = v >= 0 && v < v_hi;
+      uint4 r = make_uint4(0xff80ff80u, 0xff80ff80u, 0xff80ff80u, 0xff80ff80u);  // -inf
+      if (ok) r = __ldg(reinterpret_cast<const uint4 *>(row + (size_t)v * 8));
 #pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, off, o);
-        if (lane >= o) off += y;
-      }
-      const int total = __shfl_sync(0xffffffffu, off, 31);
-      off -= cnt;
-#pragma unroll
-      for (int u = 0; u < U; ++u)
-        if (pmask & (1u << u)) {
-          s_qraw[warp][qn + off] = raw[u];
-          s_qidx[warp][qn + off] = vv[u];
-          ++off;
+      for (int e = 0; e < 8; ++e) {
+        const uint32_t bits = elem_bits(r, e);
+        // a logit below tau's value cannot pass; the rest take the key test
+        const bool maybe = ok && ord16(bits) >= g_code;
+        if (__any_sync(0xffffffffu, maybe)) {
+          const unsigned long long th_now = theta > th ? theta : th;
+          const unsigned long long key = make_key(bits, (uint32_t)v * 8u + e);
+          const bool c = maybe && key > th_now;
+          const unsigned bal = __ballot_sync(0xffffffffu, c);
+          if (bal) {
+            if (nb + 32 > kBuf) compact();
+            if (c) buf[nb + __popc(bal & ((1u << lane) - 1u))] = key;
+            nb += __popc(bal);
+          }
         }
-      qn += total;
-      __syncwarp();
-      while (qn >= 32) {
-        examine(qn - 32, 32);
-        qn -= 32;
+      }
+    }
+    __syncwarp();
+    if (have) {
+      q_next += n_lane;
+      if (q_next >= g_n) {
+        ++j_next;
+        q_next = 0;
       }
     }
   }
-  if (qn > 0) examine(0, qn);
   if (nb > 0) compact();
-  // Every logit of the part went through the filter once, so the warps'
-  // buffers hold distinct keys.
 
   // block merge of the log-sum-exp (and of the entropy's weighted sum)
   float s, u;
