@@ -114,6 +114,30 @@ __device__ __forceinline__ int count_greater32(const unsigned long long *list, u
   return lo;
 }
 
+// Top 32 of two descending lists of 32 (one entry per lane), descending:
+// max(a[l], b[31 - l]) is a bitonic sequence holding the 32 largest entries,
+// which a bitonic merge (five compare-exchange steps) sorts.
+__device__ __forceinline__ float warp_top32_f(float a, float b, int lane) {
+  float c = fmaxf(a, __shfl_sync(0xffffffffu, b, 31 - lane));
+#pragma unroll
+  for (int j = 16; j > 0; j >>= 1) {
+    const float o = __shfl_xor_sync(0xffffffffu, c, j);
+    c = (lane & j) ? fminf(c, o) : fmaxf(c, o);
+  }
+  return c;
+}
+__device__ __forceinline__ unsigned long long warp_top32_u64(unsigned long long a,
+                                                             unsigned long long b, int lane) {
+  const unsigned long long br = shfl_u64(b, 31 - lane);
+  unsigned long long c = a > br ? a : br;
+#pragma unroll
+  for (int j = 16; j > 0; j >>= 1) {
+    const unsigned long long o = __shfl_xor_sync(0xffffffffu, c, j);
+    c = (lane & j) ? (c < o ? c : o) : (c > o ? c : o);
+  }
+  return c;
+}
+
 // Row pass over one part of one logits row (Sec. 3.1, Sec. 3.2.1):
 //   - the part's log-sum-exp as (m, s) with a per-thread online maximum;
 //   - the part's exact top-K (K <= 32) under the order (logit desc, token id
@@ -135,6 +159,7 @@ __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
   __shared__ uint16_t s_gmax[kMaxGroups][kRowThreads];  // group maxima (order codes, 0: none)
   __shared__ float s_sorted[kRowWarps][32];
   __shared__ float s_tau;
+  static_assert(IPD_MAX_K == 32, "one key per lane");
   __shared__ unsigned long long s_lists[kRowWarps][32];
   __shared__ unsigned long long s_buf[kRowWarps][kBuf];
   __shared__ int s_cand[kRowWarps][32 * kMaxGroupVecs];  // a round's candidate vectors
@@ -225,22 +250,17 @@ __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
   // ---- tau: the K-th largest of the threads' maxima ----
   // A thread that read no logit of the part holds -inf and is not counted;
   // with fewer than K counted maxima every group of the part qualifies.
-  if (tid == 0) s_tau = -INFINITY;
   {
     const bool real = v_lo + tid < v_hi;
     s_sorted[warp][lane] = warp_sort_desc_f(real ? m : -INFINITY, lane);
     __syncthreads();
-    // c is this lane's entry of its warp's sorted list; the K-th largest of
-    // all 128 has fewer than K entries above it and at least K at or above
-    // (when that is -inf -- fewer than K logits read -- tau stays -inf)
-    const float c = s_sorted[warp][lane];
-    int gt = 0, ge = 0;
-#pragma unroll 1
-    for (int w2 = 0; w2 < kRowWarps; ++w2) {
-      gt += count_above32(s_sorted[w2], c, false);
-      ge += count_above32(s_sorted[w2], c, true);
+    if (warp == 0) {  // the top 32 of the four sorted lists, then its K-th entry
+      static_assert(kRowWarps == 4, "two rounds of pairwise merges");
+      const float a = warp_top32_f(s_sorted[0][lane], s_sorted[1][lane], lane);
+      const float b = warp_top32_f(s_sorted[2][lane], s_sorted[3][lane], lane);
+      const float c = warp_top32_f(a, b, lane);
+      if (lane == K - 1) s_tau = c;  // -inf when fewer than K logits were read
     }
-    if (c != -INFINITY && gt < K && ge >= K) s_tau = c;
     __syncthreads();
   }
   const float tau = s_tau;
@@ -361,17 +381,11 @@ __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
       out[blockIdx.x].s = bs;
       out[blockIdx.x].u = bu;
     }
-    if (lane < IPD_MAX_K) out[blockIdx.x].keys[lane] = 0ull;
-  }
-  __syncthreads();
-  // merge of the warp lists: a key's rank in the union is the number of
-  // larger keys in every list (each thread ranks one key)
-  {
-    const unsigned long long c = s_lists[warp][lane];
-    int rank = 0;
-#pragma unroll 1
-    for (int w2 = 0; w2 < kRowWarps; ++w2) rank += count_greater32(s_lists[w2], c);
-    if (c != 0ull && rank < K) out[blockIdx.x].keys[rank] = c;
+    // the warps' lists (each sorted, 0 past its end) merged to the part's top K
+    const unsigned long long a = warp_top32_u64(s_lists[0][lane], s_lists[1][lane], lane);
+    const unsigned long long b = warp_top32_u64(s_lists[2][lane], s_lists[3][lane], lane);
+    const unsigned long long c = warp_top32_u64(a, b, lane);
+    out[blockIdx.x].keys[lane] = lane < K ? c : 0ull;
   }
 }
 
