@@ -12,14 +12,26 @@ IPD_DECLARE_ERROR_WORD(g_loss_err);
 
 namespace {
 
-constexpr int kLossThreads = 512;
+constexpr int kLossThreads = 256;
+constexpr int kLossWarps = kLossThreads / 32;
 
+// Fixed-shape butterfly sum over a warp (the same order on every run).
+__device__ __forceinline__ float warp_tree_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Eight warps; thread i reduces requests i, i + 256, ... in position order,
+// each warp sums its lanes by a fixed butterfly, and warp 0 adds the eight
+// warp sums in warp order.  192 bytes of shared memory, so the kernel fits
+// beside a running attention CTA.
 __global__ void __launch_bounds__(kLossThreads) split_loss_kernel(
     const float *__restrict__ kl_rev, const float *__restrict__ kl_fwd,
     const uint8_t *__restrict__ source, const int32_t *__restrict__ cu_span,
     const int32_t *__restrict__ n_emit, const int32_t *__restrict__ resp_len, int num_reqs,
     int agg_mode, int dir_mode, float *__restrict__ out8) {
-  __shared__ float sh[6][kLossThreads];
+  __shared__ float sh[6][kLossWarps];
   const bool on_rev = dir_mode == IPD_DIR_SPLIT || dir_mode == IPD_DIR_REVERSE;
   const bool off_fwd = dir_mode == IPD_DIR_SPLIT || dir_mode == IPD_DIR_FORWARD;
   float sum_on = 0.f, sum_off = 0.f, numer = 0.f, denom = 0.f;
@@ -51,31 +63,31 @@ __global__ void __launch_bounds__(kLossThreads) split_loss_kernel(
       }
     }
   }
-  const int tid = threadIdx.x;
-  sh[0][tid] = sum_on;
-  sh[1][tid] = sum_off;
-  sh[2][tid] = (float)n_on;
-  sh[3][tid] = (float)n_off;
-  sh[4][tid] = numer;
-  sh[5][tid] = denom;
-  __syncthreads();
-  for (int stride = kLossThreads / 2; stride > 0; stride >>= 1) {
-    if (tid < stride) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const float v[6] = {sum_on, sum_off, (float)n_on, (float)n_off, numer, denom};
 #pragma unroll
-      for (int q = 0; q < 6; ++q) sh[q][tid] += sh[q][tid + stride];
-    }
-    __syncthreads();
+  for (int q = 0; q < 6; ++q) {
+    const float w = warp_tree_sum(v[q]);
+    if (lane == 0) sh[q][warp] = w;
   }
-  if (tid == 0) {
-    const float nt = sh[2][0] + sh[3][0];
-    out8[0] = sh[5][0] > 0.f ? sh[4][0] / sh[5][0] : 0.f;
-    out8[1] = sh[0][0];
-    out8[2] = sh[1][0];
-    out8[3] = sh[2][0];
-    out8[4] = sh[3][0];
-    out8[5] = nt > 0.f ? sh[3][0] / nt : 0.f;
-    out8[6] = sh[4][0];
-    out8[7] = sh[5][0];
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float a[6];
+#pragma unroll
+    for (int q = 0; q < 6; ++q) {
+      a[q] = 0.f;
+#pragma unroll
+      for (int w = 0; w < kLossWarps; ++w) a[q] += sh[q][w];
+    }
+    const float nt = a[2] + a[3];
+    out8[0] = a[5] > 0.f ? a[4] / a[5] : 0.f;
+    out8[1] = a[0];
+    out8[2] = a[1];
+    out8[3] = a[2];
+    out8[4] = a[3];
+    out8[5] = nt > 0.f ? a[3] / nt : 0.f;
+    out8[6] = a[4];
+    out8[7] = a[5];
   }
 }
 

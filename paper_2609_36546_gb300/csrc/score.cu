@@ -405,9 +405,10 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     float *kl_rev, float *kl_fwd, uint8_t *covered, float *margin, uint8_t *source,
     int32_t *first_trans, int32_t *n_emit, uint8_t *next_driver, int32_t *new_len, uint8_t *done,
     int total_tokens, const EpiOpts opt) {
-  __shared__ uint8_t s_cov[1024];
-  __shared__ unsigned long long s_pk[kEpiThreads / 32][kParts][32];  // one row's part lists
-  __shared__ unsigned long long s_top[kEpiThreads / 32][2][32];      // merged top-K, S and T
+  // No shared memory: the kernel fits beside a running attention CTA, so a
+  // step that forks the vocabulary pass onto its own stream keeps this
+  // kernel off the attention's critical path.
+  static_assert(kParts == 1, "one record per row: its keys are the row's sorted top-K");
   const int r = blockIdx.x;
   const int t0 = cu_span[r], t1 = cu_span[r + 1];
   const int drv = driver[r] ? 1 : 0;
@@ -423,41 +424,17 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     const bool xok = x >= 0 && x < vocab;
     if (!xok && lane == 0) ipd_set_error(&g_score_err, IPD_DEVERR_TOKEN);
     const uint16_t *rowS = ls + (size_t)t * vocab, *rowT = lt + (size_t)t * vocab;
-    // each row from its parts: log Z by the log-sum-exp merge, the top-K as
-    // the best K of the parts' lists (a key's rank is the number of larger
-    // keys in every part list)
+    // each row's record: log Z = m + log s, the entropy log Z - u / s, and
+    // its top-K keys, best first (lane j holds the j-th)
     float logz[2], ent[2];
+    unsigned long long key2[2];
 #pragma unroll
     for (int mdl = 0; mdl < 2; ++mdl) {
-      const RowOut *pr = rows + (size_t)(2 * t + mdl) * kParts;
-      float M = -INFINITY;
-#pragma unroll
-      for (int q = 0; q < kParts; ++q) M = fmaxf(M, pr[q].m);
-      float S = 0.f, Uw = 0.f;
-#pragma unroll
-      for (int q = 0; q < kParts; ++q)
-        if (pr[q].m != -INFINITY) {
-          const float f = expf(pr[q].m - M);
-          S += pr[q].s * f;
-          Uw += pr[q].u * f;
-        }
+      const RowOut *pr = rows + (size_t)(2 * t + mdl);
+      const float M = pr->m, S = pr->s, Uw = pr->u;
       logz[mdl] = M + logf(S);
       ent[mdl] = logz[mdl] - Uw / S;  // H = log Z - E[l]
-#pragma unroll
-      for (int q = 0; q < kParts; ++q) s_pk[warp][q][lane] = lane < K ? pr[q].keys[lane] : 0ull;
-      s_top[warp][mdl][lane] = 0ull;
-      __syncwarp();
-#pragma unroll
-      for (int q = 0; q < kParts; ++q) {
-        const unsigned long long c = s_pk[warp][q][lane];
-        if (c != 0ull) {
-          int rank = 0;
-#pragma unroll
-          for (int q2 = 0; q2 < kParts; ++q2) rank += count_greater32(s_pk[warp][q2], c);
-          if (rank < K) s_top[warp][mdl][rank] = c;
-        }
-      }
-      __syncwarp();
+      key2[mdl] = lane < K ? pr->keys[lane] : 0ull;
     }
     const float nan = __int_as_float(0x7fc00000);
     const float lxS = xok ? bf16f(rowS[x]) : nan, lxT = xok ? bf16f(rowT[x]) : nan;
@@ -465,8 +442,8 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     unsigned long long kS = 0ull, kT = 0ull;
     uint32_t iS = 0, iT = 0;
     if (lane < K) {
-      kS = s_top[warp][0][lane];
-      kT = s_top[warp][1][lane];
+      kS = key2[0];
+      kT = key2[1];
       iS = key_idx(kS);
       iT = key_idx(kT);
       if (iS >= (uint32_t)vocab) iS = 0;  // never taken: K <= vocab fills every slot
@@ -548,16 +525,15 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
       if (opt.entropy_s) opt.entropy_s[t] = ent[0];
       if (opt.entropy_t) opt.entropy_t[t] = ent[1];
       if (opt.topk_overlap) opt.topk_overlap[t] = (float)n_common / (float)K;
-      if (t - t0 < 1024) s_cov[t - t0] = cov ? 1 : 0;
     }
   }
-  __syncthreads();
+  __syncthreads();  // the block's writes of `covered` are visible to thread 0
   if (threadIdx.x == 0) {
     // Eq. (ipd_state_transition) applied position by position until the first
     // state change or an accepted EOS; rollback rules of the verdict stage.
     int n = 0, ft = k, nd = drv, dn = 0;
     for (int i = 0; i < k; ++i) {
-      const int c = (i < 1024) ? s_cov[i] : covered[t0 + i];
+      const int c = covered[t0 + i];
       const bool eos = eos_id >= 0 && tokens[t0 + i] == eos_id;
       if (drv == 0) {
         if (!c) {  // takeover: the student token is rejected, not emitted

@@ -122,11 +122,12 @@ class VerifyStep:
                        self.resp_len, self.agg_mode, self.dir_mode, self.out8, stream)
 
     def run(self, stream=None, overlap: bool = False):
-        """The step's three calls.  The vocabulary pass reads only the step's
-        inputs (logits, tokens, request metadata), not the attention outputs,
-        so with overlap=True it runs on a side stream forked from `stream`
-        and joined before the loss: its CTAs take the SMs the planner and
-        the attention kernel's last CTAs leave idle."""
+        """The step's three calls.  The vocabulary pass and the loss read only
+        the step's inputs (logits, tokens, request metadata) and each other,
+        never the attention outputs, so with overlap=True they run on a side
+        stream forked from `stream` and joined at the end: the row pass takes
+        the SMs before the attention's CTAs do, and the epilogue and the
+        loss, whose CTAs fit beside a running attention CTA, run under it."""
         if not overlap:
             self.run_attention(stream)
             self.run_score(stream)
@@ -139,8 +140,8 @@ class VerifyStep:
         side.wait_stream(main)
         self.run_attention(main)
         self.run_score(side)
+        self.run_loss(side)
         main.wait_stream(side)
-        self.run_loss(main)
 
     def capture(self, warmup: int = 2, overlap: bool = False) -> "torch.cuda.CUDAGraph":
         """Record one step (the three calls, six kernels) as a CUDA graph.
