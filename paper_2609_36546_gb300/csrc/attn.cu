@@ -10,8 +10,8 @@
 //   task  = (batch, request, kv head, row block); a row is one (span query,
 //           query head) pair, row = i * G + j for query i and head kvh*G + j.
 //   item  = (task, KV chunk); tasks longer than about a quarter of an SM's
-//           share are split, items are claimed longest first, and a small
-//           follow-up kernel merges the partials of split tasks.
+//           share are split, items are claimed longest first, and the CTA
+//           that finishes a split task's last item merges its partials.
 // KV pages stream through a 3-stage ring of 128-key stages (64 KB), one
 // 4 KB 4-D TMA box per page and tensor.
 // Two compute paths, chosen per task by its row count:
@@ -117,6 +117,7 @@ struct AttnParams {
   int4 *reqinfo;   // per flattened request: merge-entry offset, task offset, partial offset, n_split
   Item *items;
   int2 *merges;    // merge entries: (work-list slot of a split task's first item, 8-row group)
+  int *split_done; // per task: split items finished (the planner zeroes those of split tasks)
   int2 *reqslot;   // per flattened request: slot offsets of its full-size and last splits
   float *partials;
   int item_cap, task_cap, merge_cap;
@@ -139,7 +140,7 @@ struct StageMeta {
 // host-side sizes
 // --------------------------------------------------------------------------
 struct WsLayout {
-  size_t off_ctrl, off_reqinfo, off_reqslot, off_items, off_merges, off_partials, total;
+  size_t off_ctrl, off_reqinfo, off_reqslot, off_items, off_merges, off_done, off_partials, total;
   int item_cap, task_cap, merge_cap, total_reqs;
   long long prow_cap;
 };
@@ -225,6 +226,8 @@ WsLayout layout(const ipd_attn_batch *const *bs, int n) {
   L.merge_cap = (int)std::min<long long>(prow_cap / 2 + 1, (long long)kMaxTargetItems * (kTcRows / 8));
   L.off_merges = off;
   off = align_up(off + (size_t)L.merge_cap * sizeof(int2), 256);
+  L.off_done = off;
+  off = align_up(off + (size_t)L.task_cap * sizeof(int), 256);
   L.off_partials = off;
   off = align_up(off + (size_t)prow_cap * kPStride * sizeof(float), 256);
   L.total = off;
@@ -505,7 +508,7 @@ __global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_co
     if (s.pages == 0) continue;
     const int r = gi - p.req_base[b];
     const int4 info = p.reqinfo[gi];
-    const int task = info.y, mrg = info.x;
+    const int task = info.y;
     const int ns = info.w;
     const int per = split_pages(s.pages, chunk);
     const int hkv = p.b[b].hkv;
@@ -518,7 +521,6 @@ __global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_co
     for (int sp = 0; sp < ns; ++sp) {
       const int lo = sp * per, hi = min(s.pages, (sp + 1) * per);
       int slot = sp < ns - 1 ? base_main + sp * tasks : base_last;
-      int mrg_t = mrg;
       int task_t = task;
       for (int kvh = 0; kvh < hkv; ++kvh) {
         for (int rb = 0; rb < s.nrb; ++rb) {
@@ -528,9 +530,8 @@ __global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_co
           int4 *dst = reinterpret_cast<int4 *>(p.items + slot);
           dst[0] = make_int4(b, r, kvh, rb);
           dst[1] = make_int4(sp, ns, lo, hi);
+          if (ns > 1 && sp == 0) p.split_done[task_t] = 0;
           dst[2] = make_int4(task_t++, pbase, rows, pth);
-          if (ns > 1 && sp == 0)
-            for (int g8 = 0; g8 < (rows + 7) / 8; ++g8) p.merges[mrg_t++] = make_int2(slot, g8);
           ++slot;
         }
       }
@@ -538,53 +539,45 @@ __global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_co
   }
 }
 
-// Split-KV merge: each task split over several items combines its splits'
-// partial rows (unnormalised O, maximum m, sum l, all in log2 units) into the
-// output rows.  The planner lists one entry per (split task, group of 8
-// rows); warp = row, lane = 4 dims, every split's loads in flight at once.
-__global__ void __launch_bounds__(256) attn_merge_kernel(const __grid_constant__ AttnParams p) {
-  const int n_entries = p.ctrl[4];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int e = blockIdx.x; e < n_entries; e += gridDim.x) {
-    const int2 me = p.merges[e];
-    const Item I = p.items[me.x];
-    const int r = me.y * 8 + warp;
-    if (r >= I.rows) continue;
-    const BatchDev &Bt = p.b[I.b];
-    const int q0 = Bt.cu_q[I.r], G = Bt.group;
-    const int rpb = I.path != kPathCc ? kTcRows : kCcRows;
-    const int ns = I.n_split;
-    const size_t sstr = (size_t)I.rows * kPStride;
-    const float *base = p.partials + (size_t)(I.pbase + r) * kPStride;
-    const float mv = lane < ns ? __ldcg(base + lane * sstr + 128) : -INFINITY;
-    const float lv = lane < ns ? __ldcg(base + lane * sstr + 129) : 0.f;
-    float4 ov[kSplitMax];
+// Split-KV merge of one output row of a task split over several items: the
+// splits' partial rows (unnormalised O, maximum m, sum l, all in log2 units)
+// combine into the output row; lane = 4 dims, every split's loads in flight
+// at once.
+__device__ void merge_split_row(const AttnParams &p, const Item &I, int r, int lane) {
+  const BatchDev &Bt = p.b[I.b];
+  const int q0 = Bt.cu_q[I.r], G = Bt.group;
+  const int rpb = I.path != kPathCc ? kTcRows : kCcRows;
+  const int ns = I.n_split;
+  const size_t sstr = (size_t)I.rows * kPStride;
+  const float *base = p.partials + (size_t)(I.pbase + r) * kPStride;
+  const float mv = lane < ns ? __ldcg(base + lane * sstr + 128) : -INFINITY;
+  const float lv = lane < ns ? __ldcg(base + lane * sstr + 129) : 0.f;
+  float4 ov[kSplitMax];
 #pragma unroll
-    for (int sp = 0; sp < kSplitMax; ++sp)
-      if (sp < ns) ov[sp] = __ldcg(reinterpret_cast<const float4 *>(base + sp * sstr) + lane);
-    const float Mx = warp_max(mv);
-    const float f = mv == -INFINITY ? 0.f : ex2_approx(mv - Mx);
-    const float Ls = warp_sum(lv * f);
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int sp = 0; sp < kSplitMax; ++sp)
+    if (sp < ns) ov[sp] = __ldcg(reinterpret_cast<const float4 *>(base + sp * sstr) + lane);
+  const float Mx = warp_max(mv);
+  const float f = mv == -INFINITY ? 0.f : ex2_approx(mv - Mx);
+  const float Ls = warp_sum(lv * f);
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-    for (int sp = 0; sp < kSplitMax; ++sp) {
-      if (sp < ns) {
-        const float fs = __shfl_sync(0xffffffffu, f, sp);
-        acc.x = fmaf(ov[sp].x, fs, acc.x);
-        acc.y = fmaf(ov[sp].y, fs, acc.y);
-        acc.z = fmaf(ov[sp].z, fs, acc.z);
-        acc.w = fmaf(ov[sp].w, fs, acc.w);
-      }
+  for (int sp = 0; sp < kSplitMax; ++sp) {
+    if (sp < ns) {
+      const float fs = __shfl_sync(0xffffffffu, f, sp);
+      acc.x = fmaf(ov[sp].x, fs, acc.x);
+      acc.y = fmaf(ov[sp].y, fs, acc.y);
+      acc.z = fmaf(ov[sp].z, fs, acc.z);
+      acc.w = fmaf(ov[sp].w, fs, acc.w);
     }
-    const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
-    const int grow = I.rb * rpb + r;
-    const int qi = grow / G, j = grow % G;
-    uint2 pk;
-    pk.x = pack_bf16x2(acc.x * inv, acc.y * inv);
-    pk.y = pack_bf16x2(acc.z * inv, acc.w * inv);
-    *reinterpret_cast<uint2 *>(Bt.out + ((size_t)(q0 + qi) * Bt.hq + I.kvh * G + j) * kD +
-                               lane * 4) = pk;
   }
+  const float inv = Ls > 0.f ? 1.f / Ls : 0.f;
+  const int grow = I.rb * rpb + r;
+  const int qi = grow / G, j = grow % G;
+  uint2 pk;
+  pk.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+  pk.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+  *reinterpret_cast<uint2 *>(Bt.out + ((size_t)(q0 + qi) * Bt.hq + I.kvh * G + j) * kD +
+                             lane * 4) = pk;
 }
 
 // --------------------------------------------------------------------------
@@ -1669,6 +1662,22 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
       else ok = cc_item<kCcRows>(p, X, I, it);
     }
     if (!ok) break;
+    if (I.n_split > 1) {
+      // The last of a split task's items to finish merges the task's
+      // partials.  Every thread's partial rows are made visible device-wide
+      // before one thread counts the item; the CTA that completes the count
+      // reads every split's rows (its own and other CTAs') from L2.
+      __threadfence();
+      named_bar_sync(1, kCW * 32);
+      if (threadIdx.x == 0)
+        misc[2] = atomicAdd(&p.split_done[I.task], 1) == I.n_split - 1 ? 1u : 0u;
+      named_bar_sync(1, kCW * 32);
+      if (*(volatile uint32_t *)&misc[2]) {
+        __threadfence();
+        for (int r = warp; r < I.rows; r += kCW) merge_split_row(p, I, r, lane);
+      }
+      named_bar_sync(1, kCW * 32);  // misc[2] is read before the next split item rewrites it
+    }
   }
   named_bar_sync(2, (kCW + 1) * 32);
 }
@@ -1778,6 +1787,7 @@ int launch(const ipd_attn_batch *const *bs, int n, float scale, void *ws, size_t
   P.items = reinterpret_cast<Item *>(w + W.off_items);
   P.reqslot = reinterpret_cast<int2 *>(w + W.off_reqslot);
   P.merges = reinterpret_cast<int2 *>(w + W.off_merges);
+  P.split_done = reinterpret_cast<int *>(w + W.off_done);
   P.merge_cap = W.merge_cap;
   P.partials = reinterpret_cast<float *>(w + W.off_partials);
   P.item_cap = W.item_cap;
@@ -1790,8 +1800,6 @@ int launch(const ipd_attn_batch *const *bs, int n, float scale, void *ws, size_t
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   const int grid = std::max(1, std::min(D.sms, W.item_cap));
   attn_kernel<<<grid, kThreads, Smem::total, stream>>>(P);
-  if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
-  attn_merge_kernel<<<4 * D.sms, 256, 0, stream>>>(P);
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   return IPD_OK;
 }

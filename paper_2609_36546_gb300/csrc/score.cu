@@ -92,28 +92,6 @@ __device__ __forceinline__ float warp_sort_desc_f(float k, int lane) {
   return k;
 }
 
-// number of values above c (or at least c) in a descending list of 32
-__device__ __forceinline__ int count_above32(const float *list, float c, bool or_equal) {
-  int lo = 0, hi = 32;
-  while (lo < hi) {
-    const int mid = (lo + hi) >> 1;
-    if (list[mid] > c || (or_equal && list[mid] == c)) lo = mid + 1;
-    else hi = mid;
-  }
-  return lo;
-}
-
-// number of keys greater than c in a descending list of 32 (binary search)
-__device__ __forceinline__ int count_greater32(const unsigned long long *list, unsigned long long c) {
-  int lo = 0, hi = 32;
-  while (lo < hi) {
-    const int mid = (lo + hi) >> 1;
-    if (list[mid] > c) lo = mid + 1;
-    else hi = mid;
-  }
-  return lo;
-}
-
 // Top 32 of two descending lists of 32 (one entry per lane), descending:
 // max(a[l], b[31 - l]) is a bitonic sequence holding the 32 largest entries,
 // which a bitonic merge (five compare-exchange steps) sorts.
