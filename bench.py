@@ -28,9 +28,10 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-# kernels one step launches: ipd_verify_attn (planner, attention, split merge),
-# ipd_score_span (row pass, epilogue), ipd_split_loss (one)
-LAUNCHES_PER_STEP = 6
+# kernels one step launches: ipd_verify_attn (planner, attention; split tasks
+# are merged inside the attention kernel), ipd_score_span (row pass,
+# epilogue), ipd_split_loss (one)
+LAUNCHES_PER_STEP = 5
 METRIC = "verified tokens/s on 1 GB300; achieved HBM GB/s as % of peak"
 UNIT = "tokens/s"
 HBM_FALLBACK_GBS = 6800.0
@@ -420,7 +421,7 @@ def run_gpu(args):
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
-                     "kernel": "ipd_verify_attn (planner, attention and split-merge launches)",
+                     "kernel": "ipd_verify_attn (planner and attention launches; split merge inside)",
                      "bytes_per_launch": attn_bytes, "ms_per_launch": attn_ms},
         "step_hbm": {"bytes_alg": step_alg, "bytes_full": step_full,
                      "gbs_alg": step_alg / (ms_step / 1e3) / 1e9,
