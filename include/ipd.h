@@ -410,6 +410,15 @@ int ipd_split_loss_grad(const uint16_t *logits_student, const uint16_t *logits_t
                         float *grad_val, void *grad_dense, int dense_dtype, void *workspace,
                         size_t workspace_bytes, ipd_stream_t stream);
 
+/* Measurement aid.  While on, every ipd_verify_attn / ipd_decode_attn call
+ * records CUDA events on its stream around its attention kernel alone (not
+ * the planner), for up to 4096 calls; ipd_attn_kernel_time synchronises on
+ * them, returns the summed kernel time and the number of timed launches, and
+ * starts a new record.  Not for use while capturing a CUDA graph, nor from
+ * several host threads at once. */
+int ipd_set_attn_kernel_timing(int on);
+int ipd_attn_kernel_time(double *total_ms, int *launches);
+
 /* Reads and clears the device error word of the current device
  * (synchronises the device).  *code receives an IPD_DEVERR_* value. */
 int ipd_get_device_error(uint32_t *code);

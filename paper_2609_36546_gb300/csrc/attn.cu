@@ -1721,6 +1721,15 @@ int encode_pool(CUtensorMap *m, const void *base, long long rows) {
   return r == CUDA_SUCCESS ? IPD_OK : IPD_ERR_CUDA;
 }
 
+// Optional timing of the attention kernel alone (a measurement aid): CUDA
+// events recorded on the call's stream around each attn_kernel launch.
+struct KernelTiming {
+  bool on = false;
+  int n = 0;
+  cudaEvent_t ev[2 * 4096] = {};
+};
+KernelTiming g_timing;
+
 int launch(const ipd_attn_batch *const *bs, int n, float scale, void *ws, size_t ws_bytes,
            cudaStream_t stream) {
   if (!(scale > 0.f) || scale != scale) return IPD_ERR_INVALID_ARG;
@@ -1799,7 +1808,20 @@ int launch(const ipd_attn_batch *const *bs, int n, float scale, void *ws, size_t
   attn_plan_kernel<<<1, kPlanThreads, 0, stream>>>(P);
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   const int grid = std::max(1, std::min(D.sms, W.item_cap));
+  const bool timed = g_timing.on && g_timing.n < 4096;
+  if (timed) {
+    cudaEvent_t *e = &g_timing.ev[2 * g_timing.n];
+    if ((!e[0] && cudaEventCreate(&e[0]) != cudaSuccess) ||
+        (!e[1] && cudaEventCreate(&e[1]) != cudaSuccess) ||
+        cudaEventRecord(e[0], stream) != cudaSuccess)
+      return IPD_ERR_CUDA;
+  }
   attn_kernel<<<grid, kThreads, Smem::total, stream>>>(P);
+  if (timed) {
+    if (cudaEventRecord(g_timing.ev[2 * g_timing.n + 1], stream) != cudaSuccess)
+      return IPD_ERR_CUDA;
+    ++g_timing.n;
+  }
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   return IPD_OK;
 }
@@ -1834,4 +1856,26 @@ extern "C" int ipd_decode_attn(const ipd_attn_batch *decode, int n_decode, float
                                void *workspace, size_t workspace_bytes, ipd_stream_t stream) {
   return ipd_verify_attn(nullptr, 0, decode, n_decode, softmax_scale, workspace, workspace_bytes,
                          stream);
+}
+
+extern "C" int ipd_set_attn_kernel_timing(int on) {
+  g_timing.on = on != 0;
+  g_timing.n = 0;
+  return IPD_OK;
+}
+
+extern "C" int ipd_attn_kernel_time(double *total_ms, int *launches) {
+  if (!total_ms || !launches) return IPD_ERR_INVALID_ARG;
+  double sum = 0.0;
+  for (int i = 0; i < g_timing.n; ++i) {
+    float ms = 0.f;
+    if (cudaEventSynchronize(g_timing.ev[2 * i + 1]) != cudaSuccess ||
+        cudaEventElapsedTime(&ms, g_timing.ev[2 * i], g_timing.ev[2 * i + 1]) != cudaSuccess)
+      return IPD_ERR_CUDA;
+    sum += ms;
+  }
+  *total_ms = sum;
+  *launches = g_timing.n;
+  g_timing.n = 0;
+  return IPD_OK;
 }

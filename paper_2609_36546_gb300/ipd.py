@@ -33,7 +33,7 @@ EXPORTS = ("ipd_attn_workspace_size", "ipd_verify_attn", "ipd_decode_attn",
            "ipd_split_loss", "ipd_get_device_error", "ipd_status_string", "ipd_version",
            "ipd_score_span_static", "ipd_score_span_ex", "ipd_full_kl",
            "ipd_loss_grad_workspace_size", "ipd_split_loss_grad", "ipd_sample_workspace_size",
-           "ipd_sample", "ipd_kv_append")
+           "ipd_sample", "ipd_kv_append", "ipd_set_attn_kernel_timing", "ipd_attn_kernel_time")
 # takeover / handback rules (IPD_RULE_*)
 RULE_TOPK, RULE_ENTROPY_S, RULE_ENTROPY_T, RULE_ALWAYS, RULE_NEVER = 0, 1, 2, 3, 4
 # element type of the dense gradient (IPD_DTYPE_*)
@@ -117,6 +117,10 @@ _lib.ipd_sample.argtypes = [c_p, c_i, c_i, ctypes.c_uint64, c_p, ctypes.c_float,
 _lib.ipd_kv_append.restype = c_i
 _lib.ipd_kv_append.argtypes = [c_p, c_p, ctypes.c_int64, c_i, c_i, c_i, c_p, c_p, c_p, c_p, c_p,
                                c_i, c_i, c_i, c_p]
+_lib.ipd_set_attn_kernel_timing.restype = c_i
+_lib.ipd_set_attn_kernel_timing.argtypes = [c_i]
+_lib.ipd_attn_kernel_time.restype = c_i
+_lib.ipd_attn_kernel_time.argtypes = [ctypes.POINTER(ctypes.c_double), ctypes.POINTER(c_i)]
 _lib.ipd_get_device_error.restype = c_i
 _lib.ipd_get_device_error.argtypes = [ctypes.POINTER(ctypes.c_uint32)]
 _lib.ipd_status_string.restype = ctypes.c_char_p
@@ -346,6 +350,19 @@ def split_loss_grad(logits_student, logits_teacher, topk_s, topk_t, source, cu_s
         _ptr(cu_span), _ptr(n_emit), _ptr(resp_len), _ptr(loss_out8), R, T, V, K, agg_mode,
         dir_mode, grad_scale, _ptr(grad_idx), _ptr(grad_val), _ptr(grad_dense), dtype, None, 0,
         _stream(stream)), "ipd_split_loss_grad")
+
+
+def set_attn_kernel_timing(on: bool):
+    _check(_lib.ipd_set_attn_kernel_timing(1 if on else 0), "ipd_set_attn_kernel_timing")
+
+
+def attn_kernel_time():
+    """(summed ms, launches) of the attention kernels timed since timing was
+    switched on or last read (synchronises)."""
+    ms = ctypes.c_double(0.0)
+    n = c_i(0)
+    _check(_lib.ipd_attn_kernel_time(ctypes.byref(ms), ctypes.byref(n)), "ipd_attn_kernel_time")
+    return float(ms.value), int(n.value)
 
 
 def device_error() -> int:
