@@ -166,3 +166,15 @@ def test_kv_append_host_validation():
     assert L.ipd_kv_append(*ok_args(kp=None)) == bad["IPD_ERR_INVALID_ARG"]
     assert L.ipd_kv_append(*ok_args(kn=24)) == bad["IPD_ERR_INVALID_ARG"]   # misaligned
     assert L.ipd_kv_append(*ok_args(np=-1)) == bad["IPD_ERR_INVALID_ARG"]
+
+
+def test_attn_kernel_timing_host_side():
+    import ctypes
+    from paper_2609_36546_gb300 import ipd
+    L = ipd._lib
+    assert L.ipd_attn_kernel_time(None, None) == ipd.STATUS_CODES["IPD_ERR_INVALID_ARG"]
+    assert L.ipd_set_attn_kernel_timing(1) == 0
+    ms, n = ctypes.c_double(-1.0), ctypes.c_int(-1)
+    assert L.ipd_attn_kernel_time(ctypes.byref(ms), ctypes.byref(n)) == 0
+    assert n.value == 0 and ms.value == 0.0          # nothing launched: nothing recorded
+    assert L.ipd_set_attn_kernel_timing(0) == 0
