@@ -112,15 +112,13 @@ struct AttnParams {
   int n_batches;
   int total_reqs;
   float scale_log2;
-  int *ctrl;       // [0] n_items, [1] dynamic item counter, [2] n_tasks, [3] partial rows,
-                   // [4] merge entries
-  int4 *reqinfo;   // per flattened request: merge-entry offset, task offset, partial offset, n_split
+  int *ctrl;       // [0] n_items, [1] dynamic item counter, [2] n_tasks, [3] partial rows
+  int4 *reqinfo;   // per flattened request: (unused), task offset, partial offset, n_split
   Item *items;
-  int2 *merges;    // merge entries: (work-list slot of a split task's first item, 8-row group)
   int *split_done; // per task: split items finished (the planner zeroes those of split tasks)
   int2 *reqslot;   // per flattened request: slot offsets of its full-size and last splits
   float *partials;
-  int item_cap, task_cap, merge_cap;
+  int item_cap, task_cap;
   long long prow_cap;
   int target_items;  // work-list size the planner aims for (a multiple of the SM count)
   int n_sms;
@@ -140,8 +138,8 @@ struct StageMeta {
 // host-side sizes
 // --------------------------------------------------------------------------
 struct WsLayout {
-  size_t off_ctrl, off_reqinfo, off_reqslot, off_items, off_merges, off_done, off_partials, total;
-  int item_cap, task_cap, merge_cap, total_reqs;
+  size_t off_ctrl, off_reqinfo, off_reqslot, off_items, off_done, off_partials, total;
+  int item_cap, task_cap, total_reqs;
   long long prow_cap;
 };
 
@@ -220,12 +218,6 @@ WsLayout layout(const ipd_attn_batch *const *bs, int n) {
   off = align_up(off + (size_t)reqs * sizeof(int2), 256);
   L.off_items = off;
   off = align_up(off + (size_t)L.item_cap * sizeof(Item), 256);
-  // a split task has more pages than the chunk, and the chunk is at least
-  // 1 / kMaxTargetItems of all pages, so fewer than kMaxTargetItems tasks are
-  // split; each has at most kTcRows / 8 row groups
-  L.merge_cap = (int)std::min<long long>(prow_cap / 2 + 1, (long long)kMaxTargetItems * (kTcRows / 8));
-  L.off_merges = off;
-  off = align_up(off + (size_t)L.merge_cap * sizeof(int2), 256);
   L.off_done = off;
   off = align_up(off + (size_t)L.task_cap * sizeof(int), 256);
   L.off_partials = off;
@@ -362,13 +354,6 @@ __device__ __forceinline__ int warp_reserve(int *slots, int bucket, int n) {
   return base + excl;
 }
 
-// merge entries (8-row groups) of one kv head of a split request
-__device__ __forceinline__ int merge_groups(const ReqShape &s) {
-  int n = 0;
-  for (int rb = 0; rb < s.nrb; ++rb) n += (min(s.rpb, s.rows - rb * s.rpb) + 7) / 8;
-  return n;
-}
-
 // One block of 1024 threads.  Each thread owns requests tid, tid + 1024, ...;
 // the first kPlanCache of them keep their shape (two loads each) in
 // registers across the three passes: total work, per-request counts with
@@ -425,9 +410,9 @@ __global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_co
   if (chunk_ll > (1LL << 30)) chunk_ll = 1LL << 30;
   const int chunk = (int)chunk_ll;
 
-  // per request: split count, merge-entry, task and partial-row offsets
-  // (exclusive scans), and the size histogram of its items
-  int4 carry = make_int4(0, 0, 0, 0);  // merge entries, tasks, partial rows, items
+  // per request: split count, task and partial-row offsets (exclusive
+  // scans), and the size histogram of its items
+  int4 carry = make_int4(0, 0, 0, 0);  // (unused), tasks, partial rows, items
   for (int k = 0; k < n_rounds; ++k) {
     const int gi = tid + k * kPlanThreads;
     int4 cnt = make_int4(0, 0, 0, 0);
@@ -442,8 +427,7 @@ __global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_co
         const int per = split_pages(s.pages, chunk);
         const int hkv = p.b[b].hkv;
         const int tasks = hkv * s.nrb;
-        cnt = make_int4(nsplit > 1 ? hkv * merge_groups(s) : 0, tasks,
-                        nsplit > 1 ? nsplit * hkv * s.rows : 0, tasks * nsplit);
+        cnt = make_int4(0, tasks, nsplit > 1 ? nsplit * hkv * s.rows : 0, tasks * nsplit);
         if (nsplit > 1) {
           bk_main = size_bucket(b, p.n_batches, per, chunk);
           n_main = (nsplit - 1) * tasks;
@@ -486,8 +470,7 @@ __global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_co
     }
   }
   if (tid == 0) {
-    if (carry.w > p.item_cap || carry.y > p.task_cap || carry.z > p.prow_cap ||
-        carry.x > p.merge_cap) {
+    if (carry.w > p.item_cap || carry.y > p.task_cap || carry.z > p.prow_cap) {
       ipd_set_error(&g_attn_err, IPD_DEVERR_PLAN);
       s_fail = 1;
     }
@@ -495,7 +478,6 @@ __global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_co
     p.ctrl[1] = 0;
     p.ctrl[2] = carry.y;
     p.ctrl[3] = carry.z;
-    p.ctrl[4] = s_fail ? 0 : carry.x;
   }
   __syncthreads();
   if (s_fail) return;
@@ -1795,9 +1777,7 @@ int launch(const ipd_attn_batch *const *bs, int n, float scale, void *ws, size_t
   P.reqinfo = reinterpret_cast<int4 *>(w + W.off_reqinfo);
   P.items = reinterpret_cast<Item *>(w + W.off_items);
   P.reqslot = reinterpret_cast<int2 *>(w + W.off_reqslot);
-  P.merges = reinterpret_cast<int2 *>(w + W.off_merges);
   P.split_done = reinterpret_cast<int *>(w + W.off_done);
-  P.merge_cap = W.merge_cap;
   P.partials = reinterpret_cast<float *>(w + W.off_partials);
   P.item_cap = W.item_cap;
   P.task_cap = W.task_cap;
