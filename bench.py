@@ -63,7 +63,7 @@ def _committed_traffic(cfg: int):
 def _workload_name(cfg: int) -> str:
     import ipd_synth as S
     s = S.CONFIGS[cfg]
-    return (f"configs[{cfg}] {s.name}: {s.n_req} requests, ctx {s.ctx}, span {s.span}, "
+    return (f"{s.name}: {s.n_req} requests, ctx {s.ctx}, span {s.span}, "
             f"direction {s.direction}, teacher 32Q/4KV + student 16Q/8KV heads, head_dim 128, "
             f"page 16, vocab {s.vocab}, logits '{s.logits}', K={s.K}, one attention layer per model")
 
