@@ -144,7 +144,7 @@ class VerifyStep:
         main.wait_stream(side)
 
     def capture(self, warmup: int = 2, overlap: bool = False) -> "torch.cuda.CUDAGraph":
-        """Record one step (the three calls, six kernels) as a CUDA graph.
+        """Record one step (the three calls, five kernels) as a CUDA graph.
 
         The calls allocate nothing and never synchronise, so the whole step
         captures; each replay re-runs the step on the current contents of
