@@ -24,8 +24,7 @@ __device__ __forceinline__ float warp_tree_sum(float v) {
 
 // Eight warps; thread i reduces requests i, i + 256, ... in position order,
 // each warp sums its lanes by a fixed butterfly, and warp 0 adds the eight
-// warp sums in warp order.  192 bytes of shared memory, so the kernel fits
-// beside a running attention CTA.
+// warp sums in warp order.  192 bytes of shared memory.
 __global__ void __launch_bounds__(kLossThreads) split_loss_kernel(
     const float *__restrict__ kl_rev, const float *__restrict__ kl_fwd,
     const uint8_t *__restrict__ source, const int32_t *__restrict__ cu_span,

@@ -383,9 +383,9 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     float *kl_rev, float *kl_fwd, uint8_t *covered, float *margin, uint8_t *source,
     int32_t *first_trans, int32_t *n_emit, uint8_t *next_driver, int32_t *new_len, uint8_t *done,
     int total_tokens, const EpiOpts opt) {
-  // No shared memory: the kernel fits beside a running attention CTA, so a
-  // step that forks the vocabulary pass onto its own stream keeps this
-  // kernel off the attention's critical path.
+  // No shared memory.  In a step that forks the vocabulary pass onto its
+  // own stream, this kernel's CTAs take the SMs that the first attention
+  // CTAs to finish leave free, so it runs inside the attention's tail.
   static_assert(kParts == 1, "one record per row: its keys are the row's sorted top-K");
   const int r = blockIdx.x;
   const int t0 = cu_span[r], t1 = cu_span[r + 1];

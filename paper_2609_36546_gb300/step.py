@@ -126,8 +126,9 @@ class VerifyStep:
         the step's inputs (logits, tokens, request metadata) and each other,
         never the attention outputs, so with overlap=True they run on a side
         stream forked from `stream` and joined at the end: the row pass takes
-        the SMs before the attention's CTAs do, and the epilogue and the
-        loss, whose CTAs fit beside a running attention CTA, run under it."""
+        the SMs while the attention's planner runs, and the epilogue and the
+        loss take the SMs that the first attention CTAs to finish leave
+        free, inside the attention's tail."""
         if not overlap:
             self.run_attention(stream)
             self.run_score(stream)
