@@ -112,7 +112,8 @@ struct AttnParams {
   int n_batches;
   int total_reqs;
   float scale_log2;
-  int *ctrl;       // [0] n_items, [1] dynamic item counter, [2] n_tasks, [3] partial rows
+  int *ctrl;       // [0] n_items, [1] dynamic item counter, [2] n_tasks, [3] partial rows,
+                   // [4] 1 if some task is split (claim the next item late)
   int4 *reqinfo;   // per flattened request: (unused), task offset, partial offset, n_split
   Item *items;
   int *split_done; // per task: split items finished (the planner zeroes those of split tasks)
@@ -500,6 +501,7 @@ __global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_co
     p.ctrl[1] = 0;
     p.ctrl[2] = carry.y;
     p.ctrl[3] = carry.z;
+    p.ctrl[4] = chunk < P_max ? 1 : 0;
   }
   __syncthreads();
   if (s_fail) return;
@@ -1444,6 +1446,11 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
     // Page ids are read 32 at a time (one coalesced load per warp), one batch
     // ahead of use, and the next item's descriptor is fetched while the
     // current one streams, so no TMA issue waits on a global load.
+    // When the planner split tasks into chunks of about equal size, the next
+    // item is claimed four stages before the current one ends, so that the
+    // CTA that frees up first takes it (2 % off a launch whose tasks split).
+    // With whole tasks of very different sizes, claiming it as the current
+    // one starts measured as good or better.
     const uint64_t policy = l2_policy_evict_first();
     uint32_t it = 0;
     bool aborted = false;
@@ -1466,10 +1473,10 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
       I = p.items[idx];
       ids = load_ids(I, 0);
     }
+    const bool late_claim = p.ctrl[4] != 0;
     while (idx < n_items) {
-      const int nxt = claim();
+      int nxt = n_items;
       Item In = I;
-      if (nxt < n_items) In = p.items[nxt];  // consumed at the next item
       const BatchDev &Bt = p.b[I.b];
       const void *tk = &p.tmap[2 * Bt.cache];
       const void *tv = &p.tmap[2 * Bt.cache + 1];
@@ -1478,8 +1485,13 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
       const int nst = (npages + kStagePages - 1) / kStagePages;
       int ids_next = (npages > 32) ? load_ids(I, 1) : -1;
       int ids_item_next = -1;
+      const int st_claim = late_claim ? max(0, nst - 4) : 0;
       for (int st = 0; st < nst; ++st) {
-        if (st == max(0, nst - 2) && nxt < n_items) ids_item_next = load_ids(In, 0);
+        if (st == st_claim) {
+          nxt = claim();
+          if (nxt < n_items) In = p.items[nxt];  // consumed at the next item
+        }
+        if (st == max(st_claim, nst - 2) && nxt < n_items) ids_item_next = load_ids(In, 0);
         const int rel = st * kStagePages;  // first page of the stage, relative to page_lo
         if (rel > 0 && (rel & 31) == 0) {   // move to the next batch of 32 ids
           ids = ids_next;
@@ -1520,6 +1532,13 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
           tma_load_4d(stage_v(smem, s) + lane * kPageBytes, tv, 0, 0, 0, w, &B.full[s], policy);
         }
         ++it;
+      }
+      if (nst == 0 && !aborted) {  // (the planner emits no empty item)
+        nxt = claim();
+        if (nxt < n_items) {
+          In = p.items[nxt];
+          ids_item_next = load_ids(In, 0);
+        }
       }
       if (aborted) break;
       idx = nxt;
