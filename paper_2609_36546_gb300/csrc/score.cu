@@ -10,6 +10,7 @@
 // Kernel 2 (epilogue), one CTA per request: each row's log Z and top-K from
 // its parts, union support, renormalised KL in both directions, log-probs
 // and feedback, coverage and margin, then the verdict of the request's span.
+#include <algorithm>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -24,7 +25,8 @@ namespace {
 constexpr int kRowThreads = 128;  // eight row CTAs per SM: every row of a step in flight at once
 constexpr int kRowWarps = kRowThreads / 32;
 constexpr int kEpiThreads = 256;
-constexpr int kParts = 1;    // a logits row is split into this many parts, one CTA each
+constexpr int kMaxParts = 4;  // a logits row is split into up to this many parts, one CTA each
+constexpr int kRowCtasPerSm = 8;  // resident row CTAs per SM (the kernel's launch bounds)
 constexpr int kMaxGroups = 32;    // group maxima a row thread keeps
 constexpr int kMaxGroupVecs = 8;  // vectors a lane puts on its warp's list per round
 constexpr int kBuf = 64;     // per-warp candidate buffer: up to 32 kept keys + one round of 32
@@ -130,8 +132,8 @@ __device__ __forceinline__ unsigned long long warp_top32_u64(unsigned long long 
 // to the warp's buffer, which is cut back to its best K (by rank) when it
 // fills, and the warps' lists are merged by rank.
 template <bool kEntropy>  // also accumulate sum exp(l - m) l (entropies / entropy rules)
-__global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
-    const uint16_t *__restrict__ ls, const uint16_t *__restrict__ lt, int vocab, int K,
+__global__ void __launch_bounds__(kRowThreads, kRowCtasPerSm) score_rows_kernel(
+    const uint16_t *__restrict__ ls, const uint16_t *__restrict__ lt, int vocab, int K, int parts,
     RowOut *__restrict__ out) {
   constexpr int U = 4;  // vectors per thread and iteration
   __shared__ uint16_t s_gmax[kMaxGroups][kRowThreads];  // group maxima (order codes, 0: none)
@@ -143,12 +145,12 @@ __global__ void __launch_bounds__(kRowThreads, 8) score_rows_kernel(
   __shared__ int s_cand[kRowWarps][32 * kMaxGroupVecs];  // a round's candidate vectors
   __shared__ float s_m[kRowWarps], s_s[kRowWarps], s_u[kRowWarps];
 
-  const int row_id = blockIdx.x / kParts, part = blockIdx.x % kParts;
+  const int row_id = blockIdx.x / parts, part = blockIdx.x % parts;
   const int t = row_id >> 1, model = row_id & 1;
   const uint16_t *row = (model ? lt : ls) + (size_t)t * vocab;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, tid = threadIdx.x;
   const int nvec = vocab >> 3;
-  const int per = (nvec + kParts - 1) / kParts;
+  const int per = (nvec + parts - 1) / parts;
   const int v_lo = min(nvec, part * per), v_hi = min(nvec, v_lo + per);
   const int n_iter = (v_hi - v_lo + kRowThreads * U - 1) / (kRowThreads * U);
   // iterations per group: two, or more so that a thread has at most kMaxGroups
@@ -379,14 +381,14 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     const uint16_t *__restrict__ ls, const uint16_t *__restrict__ lt,
     const int32_t *__restrict__ tokens, const int32_t *__restrict__ cu_span,
     const uint8_t *__restrict__ driver, const int32_t *__restrict__ prefix_len, int vocab, int K,
-    int eos_id, const RowOut *__restrict__ rows, float *logp_s, float *logp_t, float *feedback,
+    int eos_id, const RowOut *__restrict__ rows, int parts, float *logp_s, float *logp_t,
+    float *feedback,
     float *kl_rev, float *kl_fwd, uint8_t *covered, float *margin, uint8_t *source,
     int32_t *first_trans, int32_t *n_emit, uint8_t *next_driver, int32_t *new_len, uint8_t *done,
     int total_tokens, const EpiOpts opt) {
   // No shared memory.  In a step that forks the vocabulary pass onto its
   // own stream, this kernel's CTAs take the SMs that the first attention
   // CTAs to finish leave free, so it runs inside the attention's tail.
-  static_assert(kParts == 1, "one record per row: its keys are the row's sorted top-K");
   const int r = blockIdx.x;
   const int t0 = cu_span[r], t1 = cu_span[r + 1];
   const int drv = driver[r] ? 1 : 0;
@@ -402,17 +404,33 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     const bool xok = x >= 0 && x < vocab;
     if (!xok && lane == 0) ipd_set_error(&g_score_err, IPD_DEVERR_TOKEN);
     const uint16_t *rowS = ls + (size_t)t * vocab, *rowT = lt + (size_t)t * vocab;
-    // each row's record: log Z = m + log s, the entropy log Z - u / s, and
-    // its top-K keys, best first (lane j holds the j-th)
+    // each row's records, one per part: log Z = m + log s, the entropy
+    // log Z - u / s, and the top-K keys, best first (lane j holds the j-th).
+    // The parts' sums combine against their common maximum, and their
+    // sorted key lists merge into the row's (the top K of the union of the
+    // parts' top K is the row's top K).
     float logz[2], ent[2];
     unsigned long long key2[2];
 #pragma unroll
     for (int mdl = 0; mdl < 2; ++mdl) {
-      const RowOut *pr = rows + (size_t)(2 * t + mdl);
-      const float M = pr->m, S = pr->s, Uw = pr->u;
+      const RowOut *pr = rows + (size_t)(2 * t + mdl) * parts;
+      float M = pr->m, S = pr->s, Uw = pr->u;
+      unsigned long long kk = pr->keys[lane];  // 0 past the part's K keys
+      for (int q = 1; q < parts; ++q) {
+        const float mq = pr[q].m, sq = pr[q].s, uq = pr[q].u;
+        const float mn = fmaxf(M, mq);
+        if (mn != -INFINITY) {
+          const float a = M == -INFINITY ? 0.f : exp2f((M - mn) * kLog2e);
+          const float b = mq == -INFINITY ? 0.f : exp2f((mq - mn) * kLog2e);
+          S = S * a + sq * b;
+          Uw = Uw * a + uq * b;
+          M = mn;
+        }
+        kk = warp_top32_u64(kk, pr[q].keys[lane], lane);
+      }
       logz[mdl] = M + logf(S);
       ent[mdl] = logz[mdl] - Uw / S;  // H = log Z - E[l]
-      key2[mdl] = lane < K ? pr->keys[lane] : 0ull;
+      key2[mdl] = lane < K ? kk : 0ull;
     }
     const float nan = __int_as_float(0x7fc00000);
     const float lxS = xok ? bf16f(rowS[x]) : nan, lxT = xok ? bf16f(rowT[x]) : nan;
@@ -561,9 +579,27 @@ extern "C" __attribute__((visibility("hidden"))) int ipd_internal_sample_after_v
     const uint8_t *done, int32_t *next_token, void *ws, cudaStream_t st);
 
 namespace {
-// workspace: the row records, then (256-byte aligned) the sampler's partials
+// workspace: the row records (room for kMaxParts per row), then (256-byte
+// aligned) the sampler's partials
 size_t rows_region(int total_tokens) {
-  return ((size_t)total_tokens * 2 * kParts * sizeof(RowOut) + 255) & ~(size_t)255;
+  return ((size_t)total_tokens * 2 * kMaxParts * sizeof(RowOut) + 255) & ~(size_t)255;
+}
+
+int g_sms[64] = {};  // SM count per device, read once
+
+// Parts per logits row: as many (up to kMaxParts) as keep every row CTA of
+// the call in one wave, so a pass over few rows is not held to one CTA's
+// streaming rate per row.  A part keeps at least four loads per thread.
+int row_parts(int total_tokens, int vocab, int max_parts) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+  if (!g_sms[dev] &&
+      cudaDeviceGetAttribute(&g_sms[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return 1;
+  const long long slots = (long long)kRowCtasPerSm * g_sms[dev];
+  for (int q = max_parts; q > 1; q >>= 1)
+    if (2LL * total_tokens * q <= slots && vocab / 8 / q >= kRowThreads * 4) return q;
+  return 1;
 }
 }  // namespace
 
@@ -619,22 +655,23 @@ extern "C" int ipd_score_span_ex(const uint16_t *logits_student, const uint16_t 
     return IPD_ERR_WORKSPACE;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   RowOut *rows = static_cast<RowOut *>(workspace);
+  const int parts = row_parts(total_tokens, vocab, kMaxParts);
   if (total_tokens > 0) {
     const bool need_h = opt.entropy_s || opt.entropy_t || opt.take_rule == IPD_RULE_ENTROPY_S ||
                         opt.take_rule == IPD_RULE_ENTROPY_T || opt.hand_rule == IPD_RULE_ENTROPY_S ||
                         opt.hand_rule == IPD_RULE_ENTROPY_T;
     if (need_h)
-      score_rows_kernel<true><<<2 * kParts * total_tokens, kRowThreads, 0, st>>>(
-          logits_student, logits_teacher, vocab, K, rows);
+      score_rows_kernel<true><<<2 * parts * total_tokens, kRowThreads, 0, st>>>(
+          logits_student, logits_teacher, vocab, K, parts, rows);
     else
-      score_rows_kernel<false><<<2 * kParts * total_tokens, kRowThreads, 0, st>>>(
-          logits_student, logits_teacher, vocab, K, rows);
+      score_rows_kernel<false><<<2 * parts * total_tokens, kRowThreads, 0, st>>>(
+          logits_student, logits_teacher, vocab, K, parts, rows);
     if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   }
   score_epilogue_kernel<<<num_reqs, kEpiThreads, 0, st>>>(
       logits_student, logits_teacher, tokens, cu_span, driver, prefix_len, vocab, K, eos_id, rows,
-      logp_s, logp_t, feedback, kl_rev, kl_fwd, covered, margin, source, first_trans, n_emit,
-      next_driver, new_len, done, total_tokens, opt);
+      parts, logp_s, logp_t, feedback, kl_rev, kl_fwd, covered, margin, source, first_trans,
+      n_emit, next_driver, new_len, done, total_tokens, opt);
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   if (ext && ext->next_token)
     return ipd_internal_sample_after_verdict(
@@ -803,7 +840,7 @@ extern "C" int ipd_full_kl(const uint16_t *logits_student, const uint16_t *logit
 // IPD_STATIC_MAX_TOKENS span positions.  Every GPU that loads the library
 // holds this array (about 2.1 MiB) until the process exits.
 // ---------------------------------------------------------------------------
-static __device__ __align__(256) RowOut g_static_rows[2 * kParts * IPD_STATIC_MAX_TOKENS];
+static __device__ __align__(256) RowOut g_static_rows[2 * IPD_STATIC_MAX_TOKENS];
 
 namespace {
 std::mutex g_static_mu;
@@ -852,16 +889,20 @@ extern "C" int ipd_score_span_static(const uint16_t *logits_student,
   if (st != IPD_OK) return st;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   // Every RowOut the epilogue reads is written by the row kernel of the same
-  // call first, so nothing in the array has to start at zero.
+  // call first, so nothing in the array has to start at zero.  The array
+  // holds 2 IPD_STATIC_MAX_TOKENS records: parts * total_tokens stays within.
+  const int parts = row_parts(
+      total_tokens, vocab,
+      total_tokens > 0 ? std::min(kMaxParts, IPD_STATIC_MAX_TOKENS / total_tokens) : 1);
   if (total_tokens > 0) {
-    score_rows_kernel<false><<<2 * kParts * total_tokens, kRowThreads, 0, s>>>(
-        logits_student, logits_teacher, vocab, K, rows);
+    score_rows_kernel<false><<<2 * parts * total_tokens, kRowThreads, 0, s>>>(
+        logits_student, logits_teacher, vocab, K, parts, rows);
     if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   }
   score_epilogue_kernel<<<num_reqs, kEpiThreads, 0, s>>>(
       logits_student, logits_teacher, tokens, cu_span, driver, prefix_len, vocab, K, eos_id, rows,
-      logp_s, logp_t, feedback, kl_rev, kl_fwd, covered, margin, source, first_trans, n_emit,
-      next_driver, new_len, done, total_tokens,
+      parts, logp_s, logp_t, feedback, kl_rev, kl_fwd, covered, margin, source, first_trans,
+      n_emit, next_driver, new_len, done, total_tokens,
       EpiOpts{IPD_RULE_TOPK, IPD_RULE_TOPK, 0.f, 0.f, nullptr, nullptr, nullptr});
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   return IPD_OK;
