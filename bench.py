@@ -470,12 +470,11 @@ def run_e2e(step, w, K, stream, world):
     (VerifyStep.capture_from_host)."""
     import torch
     host = step.host_inputs(n_chunks=4)
-    names = ("first_trans", "n_emit", "next_driver", "new_len", "done", "source")
-    results = {n: torch.empty(step.score[n].shape, dtype=step.score[n].dtype, pin_memory=True)
-               for n in names}
-    results["out8"] = torch.empty(8, pin_memory=True)
-    h2d = sum(t.numel() * t.element_size() for k, t in host.items() if not k.startswith("_"))
-    d2h = sum(t.numel() * t.element_size() for t in results.values())
+    results = step.host_results()
+    # bytes copied per step: the packed inputs, both models' logits, the packed results
+    h2d = host["_arena"].numel() + sum(host[k].numel() * host[k].element_size()
+                                       for k in ("logits_s", "logits_t"))
+    d2h = results["_arena"].numel()
     graph = step.capture_from_host(host, results)
     for _ in range(2):
         graph.replay()
@@ -490,10 +489,11 @@ def run_e2e(step, w, K, stream, world):
     toks = _sum_over_ranks(float(step.T * K), world)
     return {"value": toks / el, "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": K,
-            "note": "pinned host -> device inputs (Q, logits, tokens, metadata) and device -> "
-                    "host results each step, synchronised per step; KV pools resident; the "
-                    "attention overlaps the logits transfer, which is scored in 4 chunks as it "
-                    "lands; the step with its copies replayed from one CUDA graph"}
+            "note": "pinned host -> device inputs (Q, tokens and metadata in one copy, the "
+                    "logits in 4 chunks) and device -> host results (one copy) each step, "
+                    "synchronised per step; KV pools resident; the attention overlaps the logits "
+                    "transfer, and each chunk is scored as it lands; the step with its copies "
+                    "replayed from one CUDA graph"}
 
 
 # ---------------------------------------------------------------------------

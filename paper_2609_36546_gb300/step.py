@@ -28,6 +28,39 @@ def _cu(lengths: torch.Tensor) -> torch.Tensor:
     return out
 
 
+# Names of the score outputs a host-fed step copies back, besides "out8".
+RESULT_NAMES = ("first_trans", "n_emit", "next_driver", "new_len", "done", "source")
+
+
+class _Packed:
+    """Named tensors laid out in one byte buffer (256-byte aligned slots), so
+    that a host<->device transfer of all of them is one copy: many small
+    copies each pay a fixed cost that dwarfs their bytes."""
+
+    def __init__(self, named, device, pin: bool = False):
+        self.layout, off = [], 0
+        for name, t in named:
+            nb = t.numel() * t.element_size()
+            self.layout.append((name, off, nb, t.dtype, tuple(t.shape)))
+            off = (off + nb + 255) // 256 * 256
+        self.buf = torch.empty(max(off, 256), dtype=torch.uint8, device=device, pin_memory=pin)
+        self.views = {name: self._view(o, nb, dt, sh) for name, o, nb, dt, sh in self.layout}
+        for name, t in named:
+            self.views[name].copy_(t)
+
+    def _view(self, off, nb, dtype, shape):
+        return self.buf[off:off + nb].view(dtype).view(shape)
+
+    def mirror(self, device, pin: bool = False) -> "_Packed":
+        """The same layout in a new buffer, holding a copy of this one."""
+        m = _Packed.__new__(_Packed)
+        m.layout = self.layout
+        m.buf = torch.empty(self.buf.numel(), dtype=torch.uint8, device=device, pin_memory=pin)
+        m.buf.copy_(self.buf)
+        m.views = {name: m._view(o, nb, dt, sh) for name, o, nb, dt, sh in self.layout}
+        return m
+
+
 class VerifyStep:
     """Device buffers and calls of one verify step.
 
@@ -58,42 +91,51 @@ class VerifyStep:
         idx_t = torch.nonzero(driver == 1).flatten()
         self.idx_s, self.idx_t = idx_s, idx_t
 
-        def mk(cache, q, idx, q_len, pt):
-            if idx.numel() == 0:
-                return None
-            cu_q = _cu(q_len).to(dev)
-            seq = ctx[idx].contiguous().to(dev)
-            ptab = pt[idx].contiguous().to(dev)
-            out = torch.empty_like(q)
-            return ipd.AttnBatch(cache, q, cu_q, seq, ptab, out, int(q_len.max()),
-                                 int(ctx[idx].max()))
-
         one = lambda idx: torch.ones(idx.numel(), dtype=torch.int32)
+        # (name, cache, queries, request indices, query lengths, page table, cache name)
+        subs = [s for s in (
+            ("verify_teacher", self.cache_t, q_verify_t, idx_s, span[idx_s], pt_teacher, "teacher"),
+            ("verify_student", self.cache_s, q_verify_s, idx_t, span[idx_t], pt_student, "student"),
+            ("decode_student", self.cache_s, q_decode_s, idx_s, one(idx_s), pt_student, "student"),
+            ("decode_teacher", self.cache_t, q_decode_t, idx_t, one(idx_t), pt_teacher, "teacher"))
+            if s[3].numel() > 0]
+        # Every per-step input but the logits (queries, query offsets, lengths,
+        # page tables, tokens, request metadata, and room for the chunk
+        # offsets of a host-fed step) lives in one device buffer.
+        named = []
+        for n, _, q, idx, q_len, pt, _ in subs:
+            named += [(n + ".q", q), (n + ".cu_q", _cu(q_len)), (n + ".seq", ctx[idx].contiguous()),
+                      (n + ".ptab", pt[idx].contiguous())]
+        named += [("tokens", tokens), ("cu_span", _cu(span)), ("driver", driver),
+                  ("prefix_len", (ctx - span).to(torch.int32)),
+                  ("cu_chunk", torch.zeros(2 * self.R + 2, dtype=torch.int32))]
+        self._in = _Packed(named, dev)
+        v = self._in.views
         # (name, batch, request indices, cache name) for every non-empty sub-batch
-        self.batches = [(n, b, idx, c) for n, b, idx, c in (
-            ("verify_teacher", mk(self.cache_t, q_verify_t, idx_s, span[idx_s], pt_teacher),
-             idx_s, "teacher"),
-            ("verify_student", mk(self.cache_s, q_verify_s, idx_t, span[idx_t], pt_student),
-             idx_t, "student"),
-            ("decode_student", mk(self.cache_s, q_decode_s, idx_s, one(idx_s), pt_student),
-             idx_s, "student"),
-            ("decode_teacher", mk(self.cache_t, q_decode_t, idx_t, one(idx_t), pt_teacher),
-             idx_t, "teacher")) if b is not None]
+        self.batches = []
+        for n, cache, _, idx, q_len, _, cname in subs:
+            q = v[n + ".q"]
+            b = ipd.AttnBatch(cache, q, v[n + ".cu_q"], v[n + ".seq"], v[n + ".ptab"],
+                              torch.empty_like(q), int(q_len.max()), int(ctx[idx].max()))
+            self.batches.append((n, b, idx, cname))
         self.verify = [b for n, b, _, _ in self.batches if n.startswith("verify")]
         self.decode = [b for n, b, _, _ in self.batches if n.startswith("decode")]
         self.ws_attn = torch.empty(max(256, ipd.attn_workspace_size(self.verify, self.decode)),
                                    dtype=torch.uint8, device=dev)
         # scoring
-        self.logits_s, self.logits_t, self.tokens = logits_s, logits_t, tokens
+        self.logits_s, self.logits_t = logits_s, logits_t
+        self.tokens, self.cu_span, self.driver, self.prefix_len = (
+            v["tokens"], v["cu_span"], v["driver"], v["prefix_len"])
         self.V = int(logits_s.shape[1])
-        self.cu_span = _cu(span).to(dev)
-        self.driver = driver.to(dev)
-        self.prefix_len = (ctx - span).to(torch.int32).to(dev)
         self.resp_len = None if resp_len is None else resp_len.to(torch.int32).to(dev)
         self.score = ipd.alloc_score_outputs(self.R, self.T, dev)
+        # the results a host-fed step reads back, in one buffer as well
+        self._res = _Packed([(n, self.score[n]) for n in RESULT_NAMES] +
+                            [("out8", torch.zeros(8, dtype=torch.float32))], dev)
+        self.score.update({n: self._res.views[n] for n in RESULT_NAMES})
+        self.out8 = self._res.views["out8"]
         self.ws_score = torch.empty(max(256, ipd.score_workspace_size(self.R, self.T, self.V, K)),
                                     dtype=torch.uint8, device=dev)
-        self.out8 = torch.zeros(8, dtype=torch.float32, device=dev)
 
     @classmethod
     def from_workload(cls, w, device="cuda", **kw):
@@ -165,15 +207,15 @@ class VerifyStep:
     # -- one step end to end from host memory ---------------------------------
     def host_inputs(self, n_chunks: int = 4) -> dict:
         """Pinned host copies of every per-step input (each batch's queries and
-        metadata, both models' logits, tokens, request metadata), plus the
-        request-aligned chunk plan that run_from_host uses for the logits."""
-        h = {}
-        for i, (_, b, _, _) in enumerate(self.batches):
-            q, cu_q, seq, ptab, _ = b._keep
-            for name, t in (("q", q), ("cu_q", cu_q), ("seq", seq), ("ptab", ptab)):
-                h[f"{name}{i}"] = t.cpu().pin_memory()
-        for name in ("logits_s", "logits_t", "tokens", "cu_span", "driver", "prefix_len"):
-            h[name] = getattr(self, name).cpu().pin_memory()
+        metadata, tokens, request metadata, both models' logits), plus the
+        request-aligned chunk plan that run_from_host uses for the logits.
+        Everything but the logits sits in one pinned buffer ("_arena") laid out
+        like the step's device buffer; the other keys are views into it."""
+        arena = self._in.mirror("cpu", pin=True)
+        h = dict(arena.views)
+        h["_arena"] = arena.buf
+        h["logits_s"] = self.logits_s.cpu().pin_memory()
+        h["logits_t"] = self.logits_t.cpu().pin_memory()
         # chunk c covers requests [r0, r1) and span positions [t0, t1), with
         # about T / n_chunks positions each; its offsets are rebased to t0
         cu = h["cu_span"].to(torch.int64)
@@ -185,42 +227,43 @@ class VerifyStep:
             if r1 > r0 or c == n_chunks:
                 bounds.append((r0, r1, int(cu[r0]), int(cu[r1])))
             r0 = r1
-        h["cu_chunk"] = torch.cat([(cu[a:b + 1] - cu[a]).to(torch.int32) for a, b, _, _ in bounds]
-                                  ).pin_memory()
+        cu_chunk = torch.cat([(cu[a:b + 1] - cu[a]).to(torch.int32) for a, b, _, _ in bounds])
+        h["cu_chunk"][:cu_chunk.numel()] = cu_chunk  # at most 2R + 1 entries
         h["_chunks"] = bounds
         return h
+
+    def host_results(self) -> dict:
+        """Pinned host buffers for the results of a host-fed step: the names of
+        RESULT_NAMES plus "out8", views into one pinned buffer ("_arena") that
+        run_from_host fills with one copy."""
+        arena = self._res.mirror("cpu", pin=True)
+        out = dict(arena.views)
+        out["_arena"] = arena.buf
+        return out
 
     def run_from_host(self, host: dict, results: dict, stream=None):
         """One step whose inputs sit in pinned host memory (``host_inputs``)
         and whose results (verdict per request, source per token, loss
-        record) are copied back into ``results`` (pinned, same names as the
-        score outputs plus "out8"); the caller synchronises ``stream``.
+        record) are copied back into ``results``: ``host_results()``, read
+        back with one copy, or any dict of pinned tensors named like the
+        score outputs plus "out8".  The caller synchronises ``stream``.
 
-        The queries and metadata go first and the attention starts as soon as
-        they land; the logits, most of the bytes, follow on a copy stream in
-        request-aligned chunks, and each chunk is scored as soon as it lands,
-        so that only the last chunk's scoring and the loss follow the
-        transfer.  Every kernel sees the same data as in run(), so the
-        results are bit-identical."""
+        The queries and metadata go first, in one copy, and the attention
+        starts as soon as they land; the logits, most of the bytes, follow on
+        a copy stream in request-aligned chunks, and each chunk is scored as
+        soon as it lands, so that only the last chunk's scoring and the loss
+        follow the transfer.  Every kernel sees the same data as in run(), so
+        the results are bit-identical."""
         main = stream if stream is not None else torch.cuda.current_stream(self.device)
         if getattr(self, "_copy", None) is None:
             self._copy = torch.cuda.Stream(device=self.device)
             self._scorer = torch.cuda.Stream(device=self.device)
-            self._cu_chunk = torch.empty_like(host["cu_chunk"], device=self.device)
         cp, sc = self._copy, self._scorer
-        if self._cu_chunk.numel() != host["cu_chunk"].numel():
-            self._cu_chunk = torch.empty_like(host["cu_chunk"], device=self.device)
         # the previous step's kernels are done with every buffer written here
         cp.wait_stream(main)
         sc.wait_stream(main)
         with torch.cuda.stream(main):
-            for i, (_, b, _, _) in enumerate(self.batches):
-                q, cu_q, seq, ptab, _ = b._keep
-                for name, t in (("q", q), ("cu_q", cu_q), ("seq", seq), ("ptab", ptab)):
-                    t.copy_(host[f"{name}{i}"], non_blocking=True)
-            for name in ("tokens", "cu_span", "driver", "prefix_len"):
-                getattr(self, name).copy_(host[name], non_blocking=True)
-            self._cu_chunk.copy_(host["cu_chunk"], non_blocking=True)
+            self._in.buf.copy_(host["_arena"], non_blocking=True)
         meta = torch.cuda.Event()
         meta.record(main)
         self.run_attention(main)
@@ -234,21 +277,25 @@ class VerifyStep:
                 ev.record(cp)
                 landed.append(ev)
         sc.wait_event(meta)
+        cu_chunk = self._in.views["cu_chunk"]
         off = 0
         for (r0, r1, t0, t1), ev in zip(host["_chunks"], landed):
             sc.wait_event(ev)
             out = {n: self.score[n][t0:t1] for n, _ in ipd.SCORE_TOKEN_OUTPUTS}
             out.update({n: self.score[n][r0:r1] for n, _ in ipd.SCORE_REQ_OUTPUTS})
             ipd.score_span(self.logits_s[t0:t1], self.logits_t[t0:t1], self.tokens[t0:t1],
-                           self._cu_chunk[off:off + r1 - r0 + 1], self.driver[r0:r1],
+                           cu_chunk[off:off + r1 - r0 + 1], self.driver[r0:r1],
                            self.prefix_len[r0:r1], self.K, self.eos_id, out, self.ws_score, sc)
             off += r1 - r0 + 1
         main.wait_stream(sc)
         main.wait_stream(cp)
         self.run_loss(main)
         with torch.cuda.stream(main):
-            for name, t in results.items():
-                t.copy_(self.out8 if name == "out8" else self.score[name], non_blocking=True)
+            if "_arena" in results:
+                results["_arena"].copy_(self._res.buf, non_blocking=True)
+            else:
+                for name, t in results.items():
+                    t.copy_(self.out8 if name == "out8" else self.score[name], non_blocking=True)
 
     def capture_from_host(self, host: dict, results: dict, warmup: int = 2
                           ) -> "torch.cuda.CUDAGraph":

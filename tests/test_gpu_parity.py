@@ -138,9 +138,12 @@ def test_step_from_host_equals_direct_calls(lib, n_chunks):
     o8 = step.out8.clone()
     host = step.host_inputs(n_chunks)
     names = ("first_trans", "n_emit", "next_driver", "new_len", "done", "source")
-    results = {n: torch.empty(step.score[n].shape, dtype=step.score[n].dtype, pin_memory=True)
-               for n in names}
-    results["out8"] = torch.empty(8, pin_memory=True)
+    if n_chunks == 1:  # any dict of pinned tensors, one copy per result
+        results = {n: torch.empty(step.score[n].shape, dtype=step.score[n].dtype,
+                                  pin_memory=True) for n in names}
+        results["out8"] = torch.empty(8, pin_memory=True)
+    else:  # the packed results, one copy
+        results = step.host_results()
     for _ in range(2):
         for v in step.score.values():
             v.zero_()
@@ -149,6 +152,7 @@ def test_step_from_host_equals_direct_calls(lib, n_chunks):
         step.logits_s.zero_()
         step.logits_t.zero_()
         step.out8.zero_()
+        step._in.buf.zero_()  # queries, page tables and metadata come from the host copy
         stream = torch.cuda.current_stream()
         step.run_from_host(host, results, stream)
         stream.synchronize()
@@ -172,9 +176,7 @@ def test_step_from_host_graph_equals_direct_calls(lib):
     o8 = step.out8.clone()
     host = step.host_inputs(3)
     names = ("first_trans", "n_emit", "next_driver", "new_len", "done", "source")
-    results = {n: torch.empty(step.score[n].shape, dtype=step.score[n].dtype, pin_memory=True)
-               for n in names}
-    results["out8"] = torch.empty(8, pin_memory=True)
+    results = step.host_results()
     graph = step.capture_from_host(host, results)
     for _ in range(2):
         for v in step.score.values():
@@ -182,6 +184,7 @@ def test_step_from_host_graph_equals_direct_calls(lib):
         step.logits_s.zero_()
         step.logits_t.zero_()
         step.out8.zero_()
+        step._in.buf.zero_()
         for r in results.values():
             r.zero_()
         graph.replay()
