@@ -48,6 +48,12 @@ SMALL = [
                                     ctx=(50, 300)), 14),
     # student-verified spans of 1-3 tokens: 2-row (CUDA-core) and 4-6-row (tensor) tasks
     ("short-teacher-spans", S.small_spec(n_req=9, direction="T", span=(1, 3), ctx=(30, 2000)), 15),
+    # few rows of a wide vocabulary: each row is scored in four parts, whose sums and
+    # key lists the epilogue merges; quantised logits put equal values in every part
+    ("ties-across-parts", S.small_spec(n_req=6, vocab=32768, sigma=3.0, tie_quantum=0.5,
+                                       span=(2, 6)), 16),
+    ("K32-ties-across-parts", S.small_spec(n_req=4, K=32, vocab=16384, sigma=2.0,
+                                           tie_quantum=0.25, span=(1, 5)), 17),
 ]
 
 
