@@ -69,6 +69,12 @@ class VerifyStep:
     [R, max_pages] for the teacher and the student cache.  Device inputs:
     the four paged pools, the span queries for each verifier, the decode
     queries for each proposer, the proposed tokens and both models' logits.
+
+    The pools and the logits are used in place.  The queries, tokens and
+    request metadata are copied, at construction, into one device buffer
+    owned by the step (attributes ``tokens``, ``cu_span``, ``driver``,
+    ``prefix_len`` and each batch's tensors are views into it), so that a
+    host-fed step moves them with one copy.
     """
 
     def __init__(self, teacher_k, teacher_v, student_k, student_v, ctx, span, driver,
