@@ -11,6 +11,7 @@
 // its parts, union support, renormalised KL in both directions, log-probs
 // and feedback, coverage and margin, then the verdict of the request's span.
 #include <algorithm>
+#include <cooperative_groups.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -698,29 +699,39 @@ extern "C" int ipd_score_span(const uint16_t *logits_student, const uint16_t *lo
 }
 
 // ---------------------------------------------------------------------------
-// Full-vocabulary KL (Eq. full_vocab_opd), both directions, one CTA per span
-// position reading the student's and the teacher's row together.  Per thread
+// Full-vocabulary KL (Eq. full_vocab_opd), both directions, reading the
+// student's and the teacher's row of a span position together.  Per thread
 // and row: a running maximum m, s = sum exp(l - m); per thread: a = sum
 // exp(l_s - m_s) (l_s - l_t) and b = sum exp(l_t - m_t) (l_t - l_s), each
 // rescaled with its row's maximum.  Then KL(pi || q) = a / s_s - log Z_s +
 // log Z_t and KL(q || pi) = b / s_t - log Z_t + log Z_s.
+// A position is one cluster of P CTAs (P = 1, 2 or 4), CTA r taking part r
+// of both rows; the parts' six sums meet in CTA 0's shared memory (the
+// cluster's distributed shared memory), so a call over few positions still
+// fills the GPU in one wave without a scratch buffer or a second launch.
 // ---------------------------------------------------------------------------
 namespace {
 constexpr int kKlThreads = 256;
+constexpr int kKlCtasPerSm = 4;  // the kernel's launch bounds
 
-__global__ void __launch_bounds__(kKlThreads, 4) full_kl_kernel(
+template <int P>
+__global__ void __launch_bounds__(kKlThreads, kKlCtasPerSm) full_kl_kernel(
     const uint16_t *__restrict__ ls, const uint16_t *__restrict__ lt, int vocab,
     float *__restrict__ kl_rev, float *__restrict__ kl_fwd) {
   __shared__ float sh[kKlThreads / 32][6];
-  const int t = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  __shared__ float s_part[6];  // this CTA's part: ms, s_s, a, mt, s_t, -b
+  const int t = blockIdx.x / P, part = blockIdx.x % P;  // part = rank in the cluster
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const uint4 *rs = reinterpret_cast<const uint4 *>(ls + (size_t)t * vocab);
   const uint4 *rt = reinterpret_cast<const uint4 *>(lt + (size_t)t * vocab);
-  const int nvec = vocab >> 3;
+  const int nvec_all = vocab >> 3;
+  const int per = (nvec_all + P - 1) / P;
+  const int v_lo = min(nvec_all, part * per), nvec = min(nvec_all, v_lo + per);
   float ms = -INFINITY, mt = -INFINITY;
   unsigned long long ss = 0ull, st = 0ull, aa = 0ull, bb = 0ull;  // packed pairs
   const unsigned long long l2e = f2_pack(kLog2e, kLog2e);
   constexpr int U = 2;
-  for (int base = 0; base < nvec; base += kKlThreads * U) {
+  for (int base = v_lo; base < nvec; base += kKlThreads * U) {
     uint4 xs[U], xt[U];
     bool ok[U];
 #pragma unroll
@@ -809,12 +820,66 @@ __global__ void __launch_bounds__(kKlThreads, 4) full_kl_kernel(
       w[3 * r + 1] = warp_sum(w[3 * r + 1] * f);
       w[3 * r + 2] = warp_sum(w[3 * r + 2] * f);
     }
-    if (lane == 0) {
-      const float lzs = w[0] + logf(w[1]), lzt = w[3] + logf(w[4]);
-      kl_rev[t] = w[2] / w[1] - lzs + lzt;
-      kl_fwd[t] = -w[5] / w[4] - lzt + lzs;
+    if (P == 1) {
+      if (lane == 0) {
+        const float lzs = w[0] + logf(w[1]), lzt = w[3] + logf(w[4]);
+        kl_rev[t] = w[2] / w[1] - lzs + lzt;
+        kl_fwd[t] = -w[5] / w[4] - lzt + lzs;
+      }
+    } else if (lane == 0) {
+#pragma unroll
+      for (int i = 0; i < 6; ++i) s_part[i] = w[i];
     }
   }
+  if constexpr (P > 1) {
+    namespace cg = cooperative_groups;
+    cg::cluster_group cluster = cg::this_cluster();
+    cluster.sync();  // every part's sums are in its CTA's shared memory
+    if (part == 0 && warp == 0) {
+      // lane q < P holds part q's sums; then the same max-rescaled merge
+      float w[6];
+      const float *src = lane < P ? cluster.map_shared_rank(s_part, lane) : nullptr;
+#pragma unroll
+      for (int i = 0; i < 6; ++i) w[i] = src ? src[i] : (i % 3 == 0 ? -INFINITY : 0.f);
+#pragma unroll
+      for (int r = 0; r < 2; ++r) {
+        const float M = warp_max(w[3 * r]);
+        const float f = (w[3 * r] == -INFINITY) ? 0.f : exp2f((w[3 * r] - M) * kLog2e);
+        w[3 * r] = M;
+        w[3 * r + 1] = warp_sum(w[3 * r + 1] * f);
+        w[3 * r + 2] = warp_sum(w[3 * r + 2] * f);
+      }
+      if (lane == 0) {
+        const float lzs = w[0] + logf(w[1]), lzt = w[3] + logf(w[4]);
+        kl_rev[t] = w[2] / w[1] - lzs + lzt;
+        kl_fwd[t] = -w[5] / w[4] - lzt + lzs;
+      }
+    }
+    cluster.sync();  // CTA 0 has read every part before any CTA exits
+  }
+}
+
+int g_kl_sms[64] = {};  // SM count per device, read once
+
+template <int P>
+cudaError_t launch_full_kl(const uint16_t *ls, const uint16_t *lt, int T, int vocab, float *rev,
+                           float *fwd, cudaStream_t st) {
+  if (P == 1) {
+    full_kl_kernel<1><<<T, kKlThreads, 0, st>>>(ls, lt, vocab, rev, fwd);
+    return cudaGetLastError();
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)T * P);
+  cfg.blockDim = dim3(kKlThreads);
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = P;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, full_kl_kernel<P>, ls, lt, vocab, rev, fwd);
 }
 }  // namespace
 
@@ -827,9 +892,29 @@ extern "C" int ipd_full_kl(const uint16_t *logits_student, const uint16_t *logit
   if (!logits_student || !logits_teacher || !kl_rev_full || !kl_fwd_full)
     return IPD_ERR_INVALID_ARG;
   if (((uintptr_t)logits_student | (uintptr_t)logits_teacher) & 15) return IPD_ERR_INVALID_ARG;
-  full_kl_kernel<<<total_tokens, kKlThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
-      logits_student, logits_teacher, vocab, kl_rev_full, kl_fwd_full);
-  if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
+  // parts per position: as many as keep every CTA of the call in one wave,
+  // with at least two loads per thread and row in a part
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return IPD_ERR_CUDA;
+  if (!g_kl_sms[dev] &&
+      cudaDeviceGetAttribute(&g_kl_sms[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return IPD_ERR_CUDA;
+  const long long slots = (long long)kKlCtasPerSm * g_kl_sms[dev];
+  int P = 1;
+  for (int q = 4; q > 1; q >>= 1)
+    if ((long long)total_tokens * q <= slots && vocab / 8 / q >= kKlThreads * 2) {
+      P = q;
+      break;
+    }
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const cudaError_t e =
+      P == 4 ? launch_full_kl<4>(logits_student, logits_teacher, total_tokens, vocab, kl_rev_full,
+                                 kl_fwd_full, st)
+      : P == 2 ? launch_full_kl<2>(logits_student, logits_teacher, total_tokens, vocab,
+                                   kl_rev_full, kl_fwd_full, st)
+               : launch_full_kl<1>(logits_student, logits_teacher, total_tokens, vocab,
+                                   kl_rev_full, kl_fwd_full, st);
+  if (e != cudaSuccess || cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   return IPD_OK;
 }
 

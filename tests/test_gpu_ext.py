@@ -115,7 +115,8 @@ def test_default_ext_equals_plain_score_span(lib):
         assert np.array_equal(v.cpu().numpy().view(np.uint8), g[k].view(np.uint8)), k
 
 
-@pytest.mark.parametrize("V,T", [(4096, 9), (151936, 4)])
+# positions split over clusters of 4 and 2 CTAs, and one CTA per position
+@pytest.mark.parametrize("V,T", [(151936, 4), (151936, 200), (4096, 9), (4096, 700)])
 def test_full_kl_matches_oracle(lib, V, T):
     g = torch.Generator().manual_seed(V + T)
     a = (torch.randn(T, V, generator=g) * 2.5).to(torch.bfloat16)
