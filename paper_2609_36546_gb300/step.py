@@ -32,6 +32,26 @@ def _cu(lengths: torch.Tensor) -> torch.Tensor:
 RESULT_NAMES = ("first_trans", "n_emit", "next_driver", "new_len", "done", "source")
 
 
+def chunk_plan(cu_span: torch.Tensor, n_chunks: int):
+    """Request-aligned chunks of a step's span positions for a host-fed step.
+
+    Chunk c covers requests [r0, r1) and positions [t0, t1) = [cu[r0], cu[r1]),
+    about T / n_chunks positions each (a chunk may hold no request, except
+    the last).  Returns the list of (r0, r1, t0, t1) and the chunks' span
+    offsets, each rebased to its t0 and concatenated (R + #chunks entries)."""
+    cu = cu_span.to(torch.int64).cpu()
+    R, T = cu.numel() - 1, int(cu[-1])
+    bounds, r0 = [], 0
+    for c in range(1, n_chunks + 1):
+        target = T * c // n_chunks
+        r1 = R if c == n_chunks else max(r0, int(torch.searchsorted(cu, target, right=True)) - 1)
+        if r1 > r0 or c == n_chunks:
+            bounds.append((r0, r1, int(cu[r0]), int(cu[r1])))
+        r0 = r1
+    cu_chunk = torch.cat([(cu[a:b + 1] - cu[a]).to(torch.int32) for a, b, _, _ in bounds])
+    return bounds, cu_chunk
+
+
 class _Packed:
     """Named tensors laid out in one byte buffer (256-byte aligned slots), so
     that a host<->device transfer of all of them is one copy: many small
@@ -222,18 +242,7 @@ class VerifyStep:
         h["_arena"] = arena.buf
         h["logits_s"] = self.logits_s.cpu().pin_memory()
         h["logits_t"] = self.logits_t.cpu().pin_memory()
-        # chunk c covers requests [r0, r1) and span positions [t0, t1), with
-        # about T / n_chunks positions each; its offsets are rebased to t0
-        cu = h["cu_span"].to(torch.int64)
-        bounds, r0 = [], 0
-        for c in range(1, n_chunks + 1):
-            target = self.T * c // n_chunks
-            r1 = self.R if c == n_chunks else \
-                max(r0, int(torch.searchsorted(cu, target, right=True)) - 1)
-            if r1 > r0 or c == n_chunks:
-                bounds.append((r0, r1, int(cu[r0]), int(cu[r1])))
-            r0 = r1
-        cu_chunk = torch.cat([(cu[a:b + 1] - cu[a]).to(torch.int32) for a, b, _, _ in bounds])
+        bounds, cu_chunk = chunk_plan(h["cu_span"], n_chunks)
         h["cu_chunk"][:cu_chunk.numel()] = cu_chunk  # at most 2R + 1 entries
         h["_chunks"] = bounds
         return h

@@ -36,3 +36,34 @@ def test_packed_views_alignment_and_mirror():
     m.views["cu"][1] = 42
     p.buf.copy_(m.buf)
     assert int(p.views["cu"][1]) == 42
+
+
+@pytest.mark.parametrize("n_chunks", [1, 2, 3, 4, 5, 9])
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_chunk_plan_covers_the_step(n_chunks, seed):
+    g = torch.Generator().manual_seed(seed)
+    R = 11
+    span = torch.randint(0, 17, (R,), generator=g, dtype=torch.int32)
+    span[seed] = 0                       # empty spans are allowed
+    cu = torch.zeros(R + 1, dtype=torch.int32)
+    cu[1:] = torch.cumsum(span, 0)
+    T = int(cu[-1])
+    bounds, cu_chunk = step_mod.chunk_plan(cu, n_chunks)
+    # contiguous, request-aligned, covering every request and position once
+    assert bounds[0][0] == 0 and bounds[-1][1] == R
+    for (a0, a1, s0, s1), (b0, b1, u0, u1) in zip(bounds, bounds[1:]):
+        assert a1 == b0 and s1 == u0
+    for r0, r1, t0, t1 in bounds:
+        assert r0 <= r1 and t0 == int(cu[r0]) and t1 == int(cu[r1])
+    assert len(bounds) <= n_chunks
+    # each chunk's offsets are the step's, rebased to its first position
+    off = 0
+    for r0, r1, t0, t1 in bounds:
+        part = cu_chunk[off:off + r1 - r0 + 1]
+        assert torch.equal(part, cu[r0:r1 + 1] - cu[r0])
+        off += r1 - r0 + 1
+    assert off == cu_chunk.numel() <= 2 * R + 1
+    # every chunk but the last ends at or before the end of its share of T
+    shares = [T * c // n_chunks for c in range(1, n_chunks + 1)]
+    for r0, r1, t0, t1 in bounds[:-1]:
+        assert any(t1 <= sh for sh in shares[:-1])
