@@ -595,7 +595,10 @@ def run_next_rows(args):
         appends.append((cache, kn, vn, cu_q, seq, ptab))
         kv_bytes += 2 * 2 * nrow * hkv * 128 * 2       # K and V rows, read and written
 
-    def kv_all():
+    def kv_all():  # the step's appends in one launch
+        ipd.kv_append_many(appends)
+
+    def kv_each():  # one call (one launch) per append
         for cache, kn, vn, cu_q, seq, ptab in appends:
             ipd.kv_append(cache, kn, vn, cu_q, seq, ptab)
 
@@ -615,6 +618,7 @@ def run_next_rows(args):
     t_draw = _graph_ms(score_draw, reps)
     t_samp = _graph_ms(lambda: ipd.sample(dec_rows, seed, draw_ids, dec_tok, ws_s), reps)
     t_kv = _graph_ms(kv_all, reps)
+    t_kv_each = _graph_ms(kv_each, reps)
     clocks = sampler.stop()
     torch.cuda.synchronize()
     if ipd.device_error() != 0:
@@ -686,7 +690,8 @@ def run_next_rows(args):
                 oracle_ms_per_row=o_samp),
             "kv_append (all span and decode rows of the step)": dict(row(
                 t_kv, kv_bytes, o_kv, "latency-bound: ~1-4 MB per step"),
-                oracle_ms_per_row=o_kv),
+                oracle_ms_per_row=o_kv, appends=len(appends), launches=1,
+                ms_one_call_per_append=t_kv_each),
         },
         "oracle_sample": f"full_kl and sample: {n_s} rows; score_span_ex and split_loss_grad: "
                          f"request {r_s} ({t1 - t0} positions); kv_append: one request's "

@@ -20,7 +20,8 @@
  * Beyond the step itself: ipd_score_span_ex (other takeover / handback rules,
  * entropies, top-K overlap, top-K lists, the next span's first token),
  * ipd_full_kl (full-vocabulary KL both ways), ipd_sample (seeded sampling of
- * rows), ipd_kv_append (new K/V rows into a paged cache) and ipd_split_loss_grad (the objective's gradient with respect to the
+ * rows), ipd_kv_append / ipd_kv_append_many (new K/V rows into paged caches)
+ * and ipd_split_loss_grad (the objective's gradient with respect to the
  * student's logits, sparse and dense).
  *
  * Conventions for every call
@@ -339,6 +340,24 @@ int ipd_kv_append(uint16_t *k_pages, uint16_t *v_pages, int64_t num_pages, int n
                   int page_size, int head_dim, const uint16_t *k_new, const uint16_t *v_new,
                   const int32_t *cu_new, const int32_t *seq_len, const int32_t *page_table,
                   int max_pages, int num_reqs, int total_new, ipd_stream_t stream);
+
+/* One append of ipd_kv_append_many: the arguments of ipd_kv_append. */
+typedef struct {
+  uint16_t *k_pages, *v_pages;
+  int64_t num_pages;
+  int num_kv_heads, page_size, head_dim;
+  const uint16_t *k_new, *v_new;
+  const int32_t *cu_new, *seq_len, *page_table;
+  int max_pages, num_reqs, total_new;
+} ipd_kv_append_desc;
+
+/* Several appends (a step's span rows into each verifier's cache and decode
+ * rows into each proposer's cache) in one launch: appends[0 .. n-1], n <=
+ * IPD_MAX_BATCHES, each with the meaning, checks and device error behaviour
+ * of ipd_kv_append.  The descriptor array is host memory, read during the
+ * call.  Any invalid descriptor returns its error and launches nothing.  Two
+ * appends must not write the same page slot. */
+int ipd_kv_append_many(const ipd_kv_append_desc *appends, int n, ipd_stream_t stream);
 
 /* Seeded sampling from softmax(l * inv_temperature) of each row (training
  * rollouts sample at temperature 1, top-p 1: App. A).  A draw is a fixed

@@ -33,7 +33,8 @@ EXPORTS = ("ipd_attn_workspace_size", "ipd_verify_attn", "ipd_decode_attn",
            "ipd_split_loss", "ipd_get_device_error", "ipd_status_string", "ipd_version",
            "ipd_score_span_static", "ipd_score_span_ex", "ipd_full_kl",
            "ipd_loss_grad_workspace_size", "ipd_split_loss_grad", "ipd_sample_workspace_size",
-           "ipd_sample", "ipd_kv_append", "ipd_set_attn_kernel_timing", "ipd_attn_kernel_time")
+           "ipd_sample", "ipd_kv_append", "ipd_kv_append_many", "ipd_set_attn_kernel_timing",
+           "ipd_attn_kernel_time")
 # takeover / handback rules (IPD_RULE_*)
 RULE_TOPK, RULE_ENTROPY_S, RULE_ENTROPY_T, RULE_ALWAYS, RULE_NEVER = 0, 1, 2, 3, 4
 # element type of the dense gradient (IPD_DTYPE_*)
@@ -72,6 +73,14 @@ class _ScoreExt(ctypes.Structure):
                 ("entropy_s", c_p), ("entropy_t", c_p), ("topk_overlap", c_p),
                 ("topk_s", c_p), ("topk_t", c_p), ("next_token", c_p), ("draw_base", c_p),
                 ("sample_seed", ctypes.c_uint64), ("inv_temperature", ctypes.c_float)]
+
+
+class _KvAppendDesc(ctypes.Structure):
+    _fields_ = [("k_pages", c_p), ("v_pages", c_p), ("num_pages", ctypes.c_int64),
+                ("num_kv_heads", ctypes.c_int32), ("page_size", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("k_new", c_p), ("v_new", c_p), ("cu_new", c_p),
+                ("seq_len", c_p), ("page_table", c_p), ("max_pages", ctypes.c_int32),
+                ("num_reqs", ctypes.c_int32), ("total_new", ctypes.c_int32)]
 
 
 class _AttnBatch(ctypes.Structure):
@@ -117,6 +126,8 @@ _lib.ipd_sample.argtypes = [c_p, c_i, c_i, ctypes.c_uint64, c_p, ctypes.c_float,
 _lib.ipd_kv_append.restype = c_i
 _lib.ipd_kv_append.argtypes = [c_p, c_p, ctypes.c_int64, c_i, c_i, c_i, c_p, c_p, c_p, c_p, c_p,
                                c_i, c_i, c_i, c_p]
+_lib.ipd_kv_append_many.restype = c_i
+_lib.ipd_kv_append_many.argtypes = [ctypes.POINTER(_KvAppendDesc), c_i, c_p]
 _lib.ipd_set_attn_kernel_timing.restype = c_i
 _lib.ipd_set_attn_kernel_timing.argtypes = [c_i]
 _lib.ipd_attn_kernel_time.restype = c_i
@@ -313,6 +324,19 @@ def kv_append(cache: "KVCache", k_new, v_new, cu_new, seq_len, page_table, strea
                               _ptr(cu_new), _ptr(seq_len), _ptr(page_table),
                               page_table.shape[1], R, k_new.shape[0], _stream(stream)),
            "ipd_kv_append")
+
+
+def kv_append_many(appends, stream=None):
+    """Several appends in one launch: ``appends`` is a sequence of (cache,
+    k_new, v_new, cu_new, seq_len, page_table) tuples, each as in kv_append."""
+    n = len(appends)
+    arr = (_KvAppendDesc * max(n, 1))()
+    for i, (cache, k_new, v_new, cu_new, seq_len, page_table) in enumerate(appends):
+        arr[i] = _KvAppendDesc(_ptr(cache.k_pages), _ptr(cache.v_pages), cache.k_pages.shape[0],
+                               cache.k_pages.shape[1], 16, 128, _ptr(k_new), _ptr(v_new),
+                               _ptr(cu_new), _ptr(seq_len), _ptr(page_table),
+                               page_table.shape[1], cu_new.numel() - 1, k_new.shape[0])
+    _check(_lib.ipd_kv_append_many(arr, n, _stream(stream)), "ipd_kv_append_many")
 
 
 def sample_workspace_size(n_rows: int, vocab: int) -> int:

@@ -168,6 +168,53 @@ def test_kv_append_host_validation():
     assert L.ipd_kv_append(*ok_args(np=-1)) == bad["IPD_ERR_INVALID_ARG"]
 
 
+def test_kv_append_many_host_validation():
+    """Every descriptor is checked before anything launches (no GPU: every
+    case returns before a launch)."""
+    import ctypes
+    from paper_2609_36546_gb300 import ipd
+    L = ipd._lib
+    bad = ipd.STATUS_CODES
+    D = ipd._KvAppendDesc
+    p = 16
+
+    def desc(**kw):
+        return D(kw.get("kp", p), p, kw.get("np", 100), kw.get("hkv", 4), kw.get("ps", 16),
+                 kw.get("hd", 128), p, p, p, p, p, kw.get("mp", 8), kw.get("R", 2),
+                 kw.get("n", 3))
+
+    def call(*ds, n=None):
+        arr = (D * max(len(ds), 1))(*ds)
+        return L.ipd_kv_append_many(arr, len(ds) if n is None else n, None)
+
+    assert call() == 0                                     # nothing to append
+    assert call(desc(n=0), desc(n=0)) == 0                 # only empty appends: no launch
+    assert L.ipd_kv_append_many(None, 0, None) == 0
+    assert L.ipd_kv_append_many(None, 1, None) == bad["IPD_ERR_INVALID_ARG"]
+    assert call(desc(n=0), n=-1) == bad["IPD_ERR_INVALID_ARG"]
+    assert call(*[desc(n=0)] * 9) == bad["IPD_ERR_INVALID_ARG"]   # more than IPD_MAX_BATCHES
+    # one bad descriptor among good ones fails the call, whatever its place
+    assert call(desc(n=0), desc(ps=32)) == bad["IPD_ERR_UNSUPPORTED"]
+    assert call(desc(hd=64), desc(n=0)) == bad["IPD_ERR_UNSUPPORTED"]
+    assert call(desc(n=0), desc(kp=None)) == bad["IPD_ERR_INVALID_ARG"]
+    assert call(desc(n=0), desc(R=0)) == bad["IPD_ERR_INVALID_ARG"]
+    assert call(desc(np=-1)) == bad["IPD_ERR_INVALID_ARG"]
+    # the binding's struct has the C layout (plain C compile of the header)
+    import os, shutil, subprocess, tempfile
+    if shutil.which("gcc"):
+        inc = os.path.join(ROOT, "include")
+        src = ('#include <stdio.h>\n#include <stddef.h>\n#include "ipd.h"\n'
+               'int main(void) { printf("%zu %zu %zu", sizeof(ipd_kv_append_desc), '
+               'offsetof(ipd_kv_append_desc, k_new), offsetof(ipd_kv_append_desc, total_new)); '
+               'return 0; }\n')
+        with tempfile.TemporaryDirectory() as d:
+            c, exe = os.path.join(d, "l.c"), os.path.join(d, "l")
+            open(c, "w").write(src)
+            subprocess.check_call(["gcc", "-std=c99", "-I", inc, c, "-o", exe])
+            got = [int(x) for x in subprocess.check_output([exe]).split()]
+        assert got == [ctypes.sizeof(D), D.k_new.offset, D.total_new.offset]
+
+
 def test_attn_kernel_timing_host_side():
     import ctypes
     from paper_2609_36546_gb300 import ipd

@@ -76,3 +76,34 @@ def test_kv_append_bad_page_is_recorded_and_skipped(lib):
     # request 0 is appended; request 1's rows that map to the bad page are skipped
     exp_k, exp_v = O.kv_append(kp, vp, kn[:2], vn[:2], cu[:2], L[:1], table[:1])
     assert np.array_equal(got_k, exp_k) and np.array_equal(got_v, exp_v)
+
+
+def test_kv_append_many_equals_one_by_one_and_oracle(lib):
+    """The appends of one step (span rows into two caches of different head
+    counts, decode rows into both) in one launch: every pool bit-identical
+    to the oracle and to the appends made one call at a time."""
+    from paper_2609_36546_gb300.ipd import KVCache
+    cases = [_case(11, 4, [100, 7, 0, 31], [8, 8, 8, 1]),     # teacher cache, span rows
+             _case(12, 8, [1000, 15, 16, 300], [1, 1, 1, 1]),  # student cache, decode rows
+             _case(13, 2, [3, 50, 0], [0, 17, 33])]            # an empty request, multi-page
+    def devs():
+        out = []
+        for kp, vp, kn, vn, cu, L, table in cases:
+            cache = KVCache(_t(kp).view(torch.bfloat16), _t(vp).view(torch.bfloat16))
+            out.append((cache, _t(kn).view(torch.bfloat16), _t(vn).view(torch.bfloat16), _t(cu),
+                        _t(L), _t(table)))
+        return out
+    many = devs()
+    lib.kv_append_many(many)
+    single = devs()
+    for a in single:
+        lib.kv_append(*a)
+    torch.cuda.synchronize()
+    assert lib.device_error() == 0
+    for (kp, vp, kn, vn, cu, L, table), m, o in zip(cases, many, single):
+        exp_k, exp_v = O.kv_append(kp, vp, kn, vn, cu, L, table)
+        got_k = m[0].k_pages.view(torch.int16).cpu().numpy().view(np.uint16)
+        got_v = m[0].v_pages.view(torch.int16).cpu().numpy().view(np.uint16)
+        assert np.array_equal(got_k, exp_k) and np.array_equal(got_v, exp_v)
+        assert torch.equal(m[0].k_pages.view(torch.int16), o[0].k_pages.view(torch.int16))
+        assert torch.equal(m[0].v_pages.view(torch.int16), o[0].v_pages.view(torch.int16))
