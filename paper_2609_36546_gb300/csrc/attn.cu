@@ -369,27 +369,31 @@ __device__ __forceinline__ int warp_reserve(int *slots, int bucket, int n) {
   return base + excl;
 }
 
-// One block of 1024 threads.  Each thread owns requests tid, tid + 1024, ...;
-// the first kPlanCache of them keep their shape (two loads each) in
-// registers across the three passes: total work, per-request counts with
-// their block scan, and the items.
-constexpr int kPlanThreads = 1024;
+// One block of kT threads (256 for up to 1024 requests, else 1024).  Each
+// thread owns requests tid, tid + kT, ...; the first kPlanCache of them keep
+// their shape (two loads each) in registers across the three passes: total
+// work, per-request counts with their block scan, and the items.  The
+// 256-thread block needs a quarter of an SM's registers, so it starts beside
+// row-pass CTAs already resident there; a 1024-thread block needs a whole
+// SM's registers and would wait for the row pass to drain an SM.
+constexpr int kPlanThreads = 1024;  // the planner block for more than 256 * kPlanCache requests
 constexpr int kPlanCache = 4;
 
-__global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_constant__ AttnParams p) {
+template <int kT>
+__global__ void __launch_bounds__(kT) attn_plan_kernel(const __grid_constant__ AttnParams p) {
   __shared__ long long red[32];
   __shared__ int4 sh4[32];
   __shared__ int s_fail;
   __shared__ int s_slot[kSizeBuckets];  // items per size bucket, then each bucket's next slot
   const int tid = threadIdx.x;
   if (tid == 0) s_fail = 0;
-  for (int i = tid; i < kSizeBuckets; i += kPlanThreads) s_slot[i] = 0;
+  for (int i = tid; i < kSizeBuckets; i += kT) s_slot[i] = 0;
 
   ReqShape cs[kPlanCache];
   int cbat[kPlanCache];
 #pragma unroll
   for (int k = 0; k < kPlanCache; ++k) {
-    const int gi = tid + k * kPlanThreads;
+    const int gi = tid + k * kT;
     cbat[k] = 0;
     cs[k] = ReqShape{};
     if (gi < p.total_reqs) {
@@ -408,12 +412,12 @@ __global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_co
     b = find_batch(p, gi);
     return req_shape(p, b, gi - p.req_base[b]);
   };
-  const int n_rounds = (p.total_reqs + kPlanThreads - 1) / kPlanThreads;
+  const int n_rounds = (p.total_reqs + kT - 1) / kT;
 
   long long w = 0;
   int pmax = 0;
   for (int k = 0; k < n_rounds; ++k) {
-    const int gi = tid + k * kPlanThreads;
+    const int gi = tid + k * kT;
     if (gi < p.total_reqs) {
       int b;
       const ReqShape s = shape_of(k, gi, b);
@@ -437,7 +441,7 @@ __global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_co
   // scans), and the size histogram of its items
   int4 carry = make_int4(0, 0, 0, 0);  // (unused), tasks, partial rows, items
   for (int k = 0; k < n_rounds; ++k) {
-    const int gi = tid + k * kPlanThreads;
+    const int gi = tid + k * kT;
     int4 cnt = make_int4(0, 0, 0, 0);
     int nsplit = 1;
     // splits 0 .. ns-2 have `per` pages (one bucket), the last split the rest
@@ -507,7 +511,7 @@ __global__ void __launch_bounds__(kPlanThreads) attn_plan_kernel(const __grid_co
   if (s_fail) return;
 
   for (int k = 0; k < n_rounds; ++k) {
-    const int gi = tid + k * kPlanThreads;
+    const int gi = tid + k * kT;
     if (gi >= p.total_reqs) continue;
     int b;
     const ReqShape s = shape_of(k, gi, b);
@@ -1826,7 +1830,12 @@ int launch(const ipd_attn_batch *const *bs, int n, float scale, void *ws, size_t
   P.target_items = std::min(kMaxTargetItems, kTargetItemsPerSm * D.sms);
   P.n_sms = D.sms;
 
-  attn_plan_kernel<<<1, kPlanThreads, 0, stream>>>(P);
+  // a small planner block fits beside row-pass CTAs already on an SM, so a
+  // step that runs both at once does not hold the attention back
+  if (W.total_reqs <= 256 * kPlanCache)
+    attn_plan_kernel<256><<<1, 256, 0, stream>>>(P);
+  else
+    attn_plan_kernel<kPlanThreads><<<1, kPlanThreads, 0, stream>>>(P);
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   const int grid = std::max(1, std::min(D.sms, W.item_cap));
   const bool timed = g_timing.on && g_timing.n < 4096;
