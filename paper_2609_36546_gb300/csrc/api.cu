@@ -30,6 +30,7 @@ extern "C" const char *ipd_status_string(int status) {
     case IPD_ERR_CUDA: return "IPD_ERR_CUDA";
     case IPD_ERR_TIMEOUT: return "IPD_ERR_TIMEOUT";
     case IPD_ERR_DEVICE: return "IPD_ERR_DEVICE";
+    case IPD_ERR_CAPACITY: return "IPD_ERR_CAPACITY";
     default: return "IPD_ERR_UNKNOWN";
   }
 }

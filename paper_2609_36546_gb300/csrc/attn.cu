@@ -15,23 +15,29 @@
 // KV pages stream through a 3-stage ring of 128-key stages (64 KB), one
 // 4 KB 4-D TMA box per page and tensor.
 // Two compute paths, chosen per task by its row count:
-//   tensor path (rows >= kTcMinRows): a 128-lane tile.  S = Q K^T (Q read
-//     from TMEM, K from shared memory, N = 128 keys) and O += P V run on
-//     tcgen05 with fp32 accumulators in TMEM.  O stays in TMEM for the whole
-//     item and is rescaled only when a row maximum grows by more than 2^8.
-//     P is passed as two bf16 terms (its upper 16 bits and the truncated
-//     residual), so the P V product keeps about 16 bits of each probability.
-//     Tiles of at most 64 rows give each row two threads (one per half of the
-//     chunk's keys) and stack the two P terms in the two 64-row halves of one
-//     operand; larger tiles keep one thread per row.  S is double-buffered,
-//     so the softmax of chunk j overlaps Q K^T of j+1 and P V of j-1.
+//   tensor path (rows >= kTcMinRows): a 128-lane tile.  S = Q K^T (Q and K
+//     from shared memory, N = 128 keys) and P V run on tcgen05 with fp32
+//     accumulators in TMEM.  P is passed as three bf16 terms (its upper 16
+//     bits, the truncated residual and what is left of it, rounded), A
+//     operands read from TMEM, so P V sees each probability to within 2^-25
+//     of itself.  Each chunk's P V starts a fresh accumulator, and the chunks
+//     are summed in fp32 registers with round-to-nearest adds: the tensor
+//     core's own accumulation does not round to nearest, and summed over a
+//     whole long context its error reaches several bf16 ulp of the result.
+//     All eight compute warps work on a tile, two threads per TMEM lane, each
+//     taking half of a chunk's keys and half of the output dimensions; tiles
+//     of at most 64 rows repeat their rows in lanes 64..127, which carry the
+//     third term of P.  S is double-buffered, so the softmax of chunk j
+//     overlaps Q K^T of j+1 and P V of j-1.
 //   CUDA-core path (fewer rows: the GQA-2 decode and one-token spans, two
-//     rows): fp32 FMA, two pages of 16 keys per warp and stage, two lanes per
-//     key.  From four rows up the tensor path is faster even with most of its
-//     tile empty: at 4-6 rows the CUDA-core FMAs limit the stream.
-// Warp roles: warps 0-3 compute, warp 4 streams KV pages, warp 5 issues the
+//     rows): fp32 FMA on the first four compute warps, two pages of 16 keys
+//     per warp and stage, two lanes per key.  From four rows up the tensor
+//     path is faster even with most of its tile empty: at 4-6 rows the
+//     CUDA-core FMAs limit the stream.
+// Warp roles: warps 0-7 compute, warp 8 streams KV pages, warp 9 issues the
 // tensor-core instructions in a fixed order (Q K^T of chunk j, then P V of
-// chunk j-1).
+// chunk j-1); warps 10 and 11 only complete the third warpgroup, whose
+// registers go to the compute warps.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
@@ -66,10 +72,18 @@ constexpr int kTcRows = 128;                      // TMEM lanes of a tensor-core
 constexpr int kTcSplitRows = 64;                  // tiles up to this size split rows over two threads
 constexpr int kTcMinRows = 4;                     // tasks with at least this many rows use it
 constexpr int kCcRows = kTcMinRows - 1;           // CUDA-core tasks have fewer rows
-constexpr int kCW = 4;                            // compute warps
-constexpr int kProducerWarp = 4;
-constexpr int kMmaWarp = 5;
-constexpr int kThreads = 6 * 32;
+constexpr int kCW = 8;                            // compute warps (two per TMEM lane block)
+constexpr int kCcW = 4;                           // of them, the CUDA-core path's warps
+constexpr int kProducerWarp = kCW;
+constexpr int kMmaWarp = kCW + 1;
+constexpr int kThreads = (kCW + 4) * 32;           // three warpgroups; warps 10 and 11 exit early
+// Register split: the block is launched with 168 registers a thread (three
+// warps share each SM sub-partition's 16K registers); the third warpgroup
+// (producer, MMA issuer and two idle warps) gives registers back so that the
+// compute warpgroups can hold their per-lane output sums.
+constexpr int kRegsLaunch = 168, kRegsAux = 56, kRegsCompute = 224;
+static_assert(2 * 128 * kRegsCompute + 128 * kRegsAux <= kThreads * kRegsLaunch,
+              "the register split must fit the registers the block was launched with");
 constexpr int kTargetItemsPerSm = 4;               // items of about a quarter of an SM's share
 constexpr int kSizesPerBatch = 32;                // claim order: batch by batch, and within a
 constexpr int kSizeBuckets = IPD_MAX_BATCHES * kSizesPerBatch;  // batch the longest items first
@@ -79,12 +93,25 @@ constexpr int kMinChunkPages = 16;
 constexpr int kSplitMax = 16;
 constexpr int kPStride = 132;                     // floats per partial row: o[128], m, l, pad
 constexpr uint32_t kTmemCols = 512;
-// TMEM columns: the S double buffer at 0 and 128 (fp32, one column per key;
-// 128-row tiles later overwrite a consumed buffer with their P residual),
-// the O accumulator at 256, the Q tile at 384 (64 columns of bf16 pairs).
+// TMEM columns: the S double buffer at 0 and 128 (fp32, one column per key),
+// the O product of one chunk at 256, and at 384 + 64 b the third term of P
+// for S buffer b.  A consumed S buffer is overwritten with two terms of P as
+// bf16 pairs: for keys 16kk .. 16kk + 15, columns 16kk .. 16kk + 7 hold the
+// first and 16kk + 8 .. 16kk + 15 the second (p_col), in place of the S
+// values of the same keys, so that each thread writes only columns it has
+// itself just read.
 __device__ __forceinline__ uint32_t col_s(uint32_t b) { return b * 128u; }
 constexpr uint32_t kColO = 256;
-constexpr uint32_t kColQ = 384;
+constexpr uint32_t kColT3 = 384;
+// column (relative to an S buffer) of keys 16 kk .. 16 kk + 15 of term 1 or
+// term 2 of P
+__host__ __device__ constexpr uint32_t p_col(int kk, int term) {
+  return 16u * (uint32_t)kk + 8u * (uint32_t)(term - 1);
+}
+// column of keys 16 kk .. 16 kk + 15 of the third term of P for S buffer b
+__host__ __device__ constexpr uint32_t t3_col(uint32_t b, int kk) {
+  return kColT3 + 64u * b + 8u * (uint32_t)kk;
+}
 // item paths
 constexpr int kPathCc = 0, kPathTcSplit = 1, kPathTcFull = 2;
 
@@ -595,21 +622,25 @@ __device__ void merge_split_row(const AttnParams &p, const Item &I, int r, int l
 // --------------------------------------------------------------------------
 struct Smem {
   static constexpr int off_stage = 0;                              // 3 x 64 KB, 1024-aligned
-  static constexpr int off_p = off_stage + kStages * kStageBytes;  // P: two blocks of 128 rows x 64 keys
-  static constexpr int kPBlock = kTcRows * 128;                    // 16 KB
-  static constexpr int off_x = off_p + 2 * kPBlock;                // row-max exchange [2][128], l [128]
-  static constexpr int off_meta = off_x + 3 * kTcRows * 4;
+  // the Q tile of a tensor item: two 64-dim halves of 128 rows x 128 B,
+  // 128-byte swizzled (a K-major operand); also the finalize's exchange area
+  // and the CUDA-core path's scratch
+  static constexpr int off_q = off_stage + kStages * kStageBytes;
+  static constexpr int kQHalf = kTcRows * 128;                     // 16 KB
+  static constexpr int off_x = off_q + 2 * kQHalf;                 // row-max / row-sum exchange [2][256]
+  static constexpr int off_meta = off_x + 2 * 256 * 4;
   static constexpr int off_bar = off_meta + kStages * (int)sizeof(StageMeta);
   static constexpr int n_bars = 2 * kStages + 5;
   static constexpr int off_misc = off_bar + n_bars * 8;
   static constexpr int total = off_misc + 64;
-  // CUDA-core path scratch (inside the P region, unused by that path)
-  static constexpr int off_ccq = off_p;                              // fp32 [7][128]
+  // CUDA-core path scratch (inside the Q region, unused by that path)
+  static constexpr int off_ccq = off_q;                              // fp32 [7][128]
   static constexpr int off_merge = off_ccq + kCcRows * kD * 4;       // fp32 [4][8][132]
-  static constexpr int off_ps = off_merge + kCW * 8 * kPStride * 4;  // fp32 [4][8][16] / [4][32][2]
+  static constexpr int off_ps = off_merge + kCcW * 8 * kPStride * 4;  // fp32 [4][8][16] / [4][32][2]
 };
-static_assert(Smem::off_ps + kCW * 8 * 16 * 4 <= Smem::off_x, "CUDA-core scratch overflow");
-static_assert(kTcSplitRows * kD * 4 <= 2 * Smem::kPBlock, "O exchange overflow");
+static_assert(Smem::off_ps + kCcW * 8 * 16 * 4 <= Smem::off_x, "CUDA-core scratch overflow");
+static_assert(kTcSplitRows * kD * 4 <= 2 * Smem::kQHalf, "O exchange overflow");
+static_assert(Smem::off_q % 1024 == 0, "swizzle atoms of the Q tile");
 static_assert(Smem::off_bar % 8 == 0, "mbarrier alignment");
 static_assert(Smem::total <= 227 * 1024, "shared memory");
 
@@ -705,78 +736,132 @@ __device__ __forceinline__ const uint16_t *q_row(const ItemGeom &g, const Item &
 
 // Zero the V rows of stage s at or past the end of the sequence: unwritten
 // cache slots may hold non-finite bits, and a zero probability times NaN is NaN.
-__device__ __forceinline__ void zero_tail(const CompCtx &X, int s, int page0, int L) {
+__device__ __forceinline__ void zero_tail(const CompCtx &X, int s, int page0, int L, int nthreads,
+                                          int bar) {
   const int tail0 = max(L - page0 * kPage, 0);  // first key slot at or past L
   if (tail0 >= kStageKeys) return;
   uint8_t *vb = stage_v(X.smem, s);
-  for (int e = X.ctid; e < (kStageKeys - tail0) * 16; e += kCW * 32) {
+  for (int e = X.ctid; e < (kStageKeys - tail0) * 16; e += nthreads) {
     const int row = tail0 + e / 16, cpart = e % 16;
     *reinterpret_cast<uint4 *>(const_cast<uint8_t *>(kv_row(vb, row, cpart >> 3)) + (cpart & 7) * 16) =
         make_uint4(0, 0, 0, 0);
   }
   fence_proxy_async_smem();
-  named_bar_sync(1, kCW * 32);
+  named_bar_sync(bar, nthreads);
 }
 
 // ============================ tensor-core path ============================
-// One 128-lane tile over the item's KV chunks of 128 keys.
-//   kSplit (at most 64 rows): TMEM lanes 64..127 repeat rows 0..63 (the Q
-//     tile is written twice), and thread t takes row t mod 64 and keys
-//     [64 h, 64 h + 64) of every chunk, h = t / 64, so the exponentials are
-//     spread over all four warps; the two threads of a row agree on the
-//     chunk maximum through shared memory.  P goes to shared memory with its
-//     upper bf16 term in rows 0..63 and its residual in rows 64..127 of one
-//     128-row operand: one MMA per 16 keys leaves P_hi V in O rows 0..63 and
-//     P_lo V in O rows 64..127, which the finalize adds.
-//   otherwise (65..128 rows): thread t takes row t and all 128 keys.  The
-//     upper term of P goes to shared memory, the residual to the TMEM columns
-//     of the chunk's own (already consumed) S buffer, and P V takes two MMAs
-//     per 16 keys.
+// One 128-lane tile over the item's KV chunks of 128 keys, worked on by all
+// eight compute warps.  Warps w and w + 4 reach the same TMEM lanes
+// 32 (w % 4) .. 32 (w % 4) + 31, so every lane has two threads.
+// A tile of at most 128 / F rows (F = 4, 2 or 1) is repeated F times over the
+// lanes: lane t holds row t mod (128 / F) and owns keys [128 k / F,
+// 128 (k + 1) / F) of every chunk, k = t / (128 / F), which its two threads
+// split.  Every SM sub-partition thus has work however few rows the tile
+// has, and a thread's share of a chunk is 64 / F keys.
+// P reaches the tensor cores as three bf16 terms (its upper 16 bits, the
+// truncated residual and what is left of it, rounded), so P V sees each
+// probability to within 2^-25 of itself.  The terms are A operands in TMEM:
+// the first two overwrite the chunk's own S columns, the third goes to the
+// columns of the S buffer's parity at 384.  A lane's A row holds the terms of
+// its own keys and zeros for the other copies' keys, so P V (three MMAs per 16
+// keys, one per term) leaves in O row t the product over lane t's keys, and
+// the finalize adds the copies of a row.
+// Every chunk's P V lands in a fresh O (its first MMA overwrites O), and each
+// thread adds its 64 output dimensions of it into fp32 registers with
+// round-to-nearest adds.  The tensor core's accumulator does not round to
+// nearest, and its error grows with the number of products summed into one
+// accumulator (measured: 6 to 25 bf16 ulp of the tolerance floor after 8K to
+// 32K keys); within one 128-key chunk it stays far below the floor.
+// The row maximum is exchanged among the row's threads through shared memory
+// and rescales the register sums only when it grows by more than 2^8.
 // Returns false on a wait time-out.  `it` (stage counter) and `c` (chunk
 // counter) advance.
-template <bool kSplit>
+template <int F>
 __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, const Item &I,
                                         uint32_t &it, uint32_t &c) {
+  constexpr int kRep = kTcRows / F;                 // rows of one copy (>= 32: a copy is warp-uniform)
+  constexpr int kKT = 64 / F;                       // keys of a chunk per thread
+  constexpr int kSteps = kKT / 16;                  // 16-key steps per thread
   const ItemGeom g = item_geom(p, I);
   const Bars &B = X.B;
-  const int t = X.ctid;                                   // TMEM lane
-  const int row = kSplit ? (t & (kTcSplitRows - 1)) : t;  // tile row
-  const int h = kSplit ? (t >> 6) : 0;                    // key half (split rows)
+  const int lb = X.warp & 3;                        // lane block of this warp
+  const int second = X.warp >> 2;                   // which of the lane's two threads
+  const int t = lb * 32 + X.lane;                   // TMEM lane (and operand row)
+  const int copy = t / kRep;
+  const int row = t % kRep;                         // tile row
+  const int kown = copy * (kStageKeys / F);         // first key the lane owns
+  const int k0 = kown + second * kKT;               // first key of this thread
+  const int kk_lo = kown / 16, kk_hi = kk_lo + 8 / F;  // the lane's 16-key steps
   const bool real = row < I.rows;
-  const uint32_t tl = X.tmem + ((uint32_t)(X.warp * 32) << 16);
+  const uint32_t tl = X.tmem + ((uint32_t)(lb * 32) << 16);
   const int lim = g.L - g.ql + (I.rb * kTcRows + row) / g.G;  // last key this row sees
   const int lim_all = g.L - g.ql;                             // every row sees up to here
   const float sl2 = p.scale_log2;
-  float *xbuf = reinterpret_cast<float *>(X.smem + Smem::off_x);
+  float *xbuf = reinterpret_cast<float *>(X.smem + Smem::off_x);  // [2][2][128]
+  uint8_t *qs = X.smem + Smem::off_q;
   float m_used = -INFINITY;  // maximum the exponentials are taken against (log2 units)
   float l_run = 0.f;         // this thread's share of the row sum
+  float acc[64];             // output dims 64 second .. of this lane's O, summed over chunks
+#pragma unroll
+  for (int e = 0; e < 64; ++e) acc[e] = 0.f;
   // "P V of chunk k has landed in O" is completion k of p_free.  Chunk k waits
-  // for completion k - 1 before it writes P, so the barrier is never more than
-  // one phase behind a wait and the parity cannot alias.
+  // for completion k - 1 before its threads arrive on p_full, so the barrier
+  // is never more than one phase behind a wait and the parity cannot alias.
   auto wait_pv_done = [&](uint32_t k) -> bool { return wait_or_abort(X, B.p_free, k & 1); };
+  // acc = (acc + this thread's dims of O) * alpha
+  auto take_o = [&](float alpha) {
+    const bool scaled = __any_sync(0xffffffffu, alpha != 1.f);
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      uint32_t r[32];
+      tc_ld_32x32b_x32(tl + kColO + 64 * second + 32 * q, r);
+      tc_wait_ld();
+      if (scaled) {
+#pragma unroll
+        for (int e = 0; e < 32; ++e)
+          acc[32 * q + e] = (acc[32 * q + e] + __uint_as_float(r[e])) * alpha;
+      } else {
+#pragma unroll
+        for (int e = 0; e < 32; ++e) acc[32 * q + e] += __uint_as_float(r[e]);
+      }
+    }
+  };
+  // zeros in n TMEM columns from `col` of this lane (n a multiple of 8)
+  auto zero_cols = [&](uint32_t col, int n) {
+    const uint32_t z32[32] = {};
+    const uint32_t z16[16] = {};
+    const uint32_t z8[8] = {};
+    for (; n >= 32; n -= 32, col += 32) tc_st_32x32b_x32(tl + col, z32);
+    if (n >= 16) {
+      tc_st_32x32b_x16(tl + col, z16);
+      n -= 16;
+      col += 16;
+    }
+    if (n >= 8) tc_st_32x32b_x8(tl + col, z8);
+  };
 
   for (bool first = true;; first = false) {
     const int s = it % kStages;
     if (!wait_or_abort(X, &B.full[s], (it / kStages) & 1)) return false;
     const StageMeta M = X.meta[s];
-    zero_tail(X, s, M.page0, g.L);
+    zero_tail(X, s, M.page0, g.L, kCW * 32, 1);
     if (first) {
-      // Q: lane t <- tile row `row` as 64 columns of bf16 pairs (zeros past the rows)
-      uint32_t qw[2][32];
-      const uint4 *src = reinterpret_cast<const uint4 *>(q_row(g, I, I.rb * kTcRows + row));
+      // The Q region is the CUDA-core path's scratch: after a CUDA-core item,
+      // warps kCcW.. get here while the first warps may still be using it.
+      named_bar_sync(1, kCW * 32);
+      // Q: this thread's half of the lane's row (dims 64 second ..) into
+      // operand row t of the swizzled Q tile (zeros past the rows)
+      const uint4 *src =
+          reinterpret_cast<const uint4 *>(q_row(g, I, I.rb * kTcRows + row) + 64 * second);
+      uint8_t *qh = qs + second * Smem::kQHalf;
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
+      for (int j = 0; j < 8; ++j) {
         uint4 v = make_uint4(0, 0, 0, 0);
         if (real) v = __ldg(src + j);
-        qw[j >> 3][(j & 7) * 4 + 0] = v.x;
-        qw[j >> 3][(j & 7) * 4 + 1] = v.y;
-        qw[j >> 3][(j & 7) * 4 + 2] = v.z;
-        qw[j >> 3][(j & 7) * 4 + 3] = v.w;
+        *reinterpret_cast<uint4 *>(qh + sw128(t, j)) = v;
       }
-      tc_st_32x32b_x32(tl + kColQ, qw[0]);
-      tc_st_32x32b_x32(tl + kColQ + 32, qw[1]);
-      tc_wait_st();
-      tc_fence_before();
+      fence_proxy_async_smem();
       __syncwarp();
       if (X.lane == 0) mbar_arrive(B.q_ready);
     }
@@ -790,10 +875,10 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
     const bool full_vis =
         M.npages == kStagePages && M.invalid == 0 && kp0 + kStageKeys - 1 <= lim_all;
     // -inf for the keys of the stage this row does not see
-    auto mask32 = [&](uint32_t (&v)[32], int col0) {
+    auto mask = [&](auto &v, int col0) {
       if (!full_vis) {
 #pragma unroll
-        for (int e = 0; e < 32; ++e) {
+        for (int e = 0; e < (int)(sizeof(v) / sizeof(v[0])); ++e) {
           const int col = col0 + e;
           const bool vis = (col >> 4) < M.npages && !((M.invalid >> (col >> 4)) & 1u) &&
                            kp0 + col <= lim;
@@ -801,142 +886,98 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
         }
       }
     };
-    auto max32 = [](const uint32_t (&v)[32], float m) {
+    // the chunk maximum over this thread's keys, then over the row's threads
+    float mc = -INFINITY;
 #pragma unroll
-      for (int e = 0; e < 32; ++e) m = fmaxf(m, __uint_as_float(v[e]));
-      return m;
-    };
+    for (int q = 0; q < kSteps; ++q) {
+      uint32_t sr[16];
+      tc_ld_32x32b_x16(tl + col_s(b) + k0 + 16 * q, sr);
+      tc_wait_ld();
+      mask(sr, k0 + 16 * q);
+#pragma unroll
+      for (int e = 0; e < 16; ++e) mc = fmaxf(mc, __uint_as_float(sr[e]));
+    }
+    float *xm = xbuf + (c & 1) * (2 * kTcRows);
+    xm[second * kTcRows + t] = mc;
+    // zeros for the other copies' keys: the first thread of the lane takes
+    // the steps below the lane's, the second those above (no thread of this
+    // lane reads those S columns)
+    if (second == 0) {
+      zero_cols(col_s(b), 16 * kk_lo);
+      zero_cols(t3_col(b, 0), 8 * kk_lo);
+    } else {
+      zero_cols(col_s(b) + 16 * kk_hi, 16 * (8 - kk_hi));
+      zero_cols(t3_col(b, kk_hi), 8 * (8 - kk_hi));
+    }
+    named_bar_sync(1, kCW * 32);
+#pragma unroll
+    for (int j = 0; j < F; ++j)
+      mc = fmaxf(mc, fmaxf(xm[row + j * kRep], xm[kTcRows + row + j * kRep]));
     // the lazy rescale: keep the old maximum unless the chunk's is 2^8 larger
-    auto rescale = [&](float mc) -> bool {
+    float alpha = 1.f;
+    {
       const float mcs = mc * sl2;
-      float alpha = 1.f;
-      bool resc = false;
       if (real && mcs != -INFINITY) {
         if (m_used == -INFINITY) {
           m_used = mcs;
         } else if (mcs > m_used + 8.f) {
           alpha = ex2_approx(m_used - mcs);
           m_used = mcs;
-          resc = true;
-        }
-      }
-      if (__any_sync(0xffffffffu, resc)) {
-        // O holds the P V products of earlier chunks of this item: let them land
-        if (!wait_pv_done(c - 1)) return false;
-        tc_fence_after();
-#pragma unroll
-        for (int q4 = 0; q4 < kD / 32; ++q4) {
-          uint32_t r[32];
-          tc_ld_32x32b_x32(tl + kColO + q4 * 32, r);
-          tc_wait_ld();
-#pragma unroll
-          for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
-          tc_st_32x32b_x32(tl + kColO + q4 * 32, r);
-        }
-        tc_wait_st();
-      }
-      l_run *= alpha;
-      return true;
-    };
-    // p = 2^(s*scale - m) as a truncated bf16 pair and the truncated residual;
-    // the scaling, residual and row sum run on packed fp32 pairs
-    unsigned long long lsum2 = 0ull;  // {0.f, 0.f}
-    auto exp_pairs = [&](const uint32_t (&v)[32], float moff, uint32_t *hi, uint32_t *lo) {
-      const unsigned long long sl2x2 = f2_pack(sl2, sl2), moffx2 = f2_pack(moff, moff);
-#pragma unroll
-      for (int e = 0; e < 32; e += 2) {
-        float x0, x1;
-        f2_unpack(f2_fma(f2_pack(__uint_as_float(v[e]), __uint_as_float(v[e + 1])), sl2x2, moffx2),
-                  x0, x1);
-        const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
-        const unsigned long long pp = f2_pack(p0, p1);
-        const unsigned long long hh =
-            f2_pack(__uint_as_float(__float_as_uint(p0) & 0xffff0000u),
-                    __uint_as_float(__float_as_uint(p1) & 0xffff0000u));
-        float l0, l1;
-        f2_unpack(f2_sub(pp, hh), l0, l1);
-        hi[e >> 1] = pack_bf16x2_trunc(p0, p1);
-        lo[e >> 1] = pack_bf16x2_trunc(l0, l1);
-        lsum2 = f2_add(lsum2, pp);
-      }
-    };
-
-    if constexpr (kSplit) {
-      uint32_t sr[2][32];
-      tc_ld_32x32b_x32(tl + col_s(b) + 64 * h, sr[0]);
-      tc_ld_32x32b_x32(tl + col_s(b) + 64 * h + 32, sr[1]);
-      tc_wait_ld();
-      mask32(sr[0], 64 * h);
-      mask32(sr[1], 64 * h + 32);
-      float mc = max32(sr[1], max32(sr[0], -INFINITY));
-      // the partner thread (other key half of the same row) holds the rest
-      float *xm = xbuf + (c & 1) * kTcRows;
-      xm[t] = mc;
-      named_bar_sync(1, kCW * 32);
-      mc = fmaxf(mc, xm[t ^ kTcSplitRows]);
-      if (!rescale(mc)) return false;
-      const float moff = (!real || m_used == -INFINITY) ? -INFINITY : -m_used;  // -inf: p = 0
-      uint32_t ph[32], pl[32];
-      exp_pairs(sr[0], moff, ph, pl);
-      exp_pairs(sr[1], moff, ph + 16, pl + 16);
-      // the P buffer is free once the previous chunk's P V product is done
-      if (!wait_pv_done(c - 1)) return false;
-      uint8_t *pb = X.smem + Smem::off_p + h * Smem::kPBlock;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        *reinterpret_cast<uint4 *>(pb + sw128(row, j)) =
-            make_uint4(ph[4 * j], ph[4 * j + 1], ph[4 * j + 2], ph[4 * j + 3]);
-        *reinterpret_cast<uint4 *>(pb + sw128(row + kTcSplitRows, j)) =
-            make_uint4(pl[4 * j], pl[4 * j + 1], pl[4 * j + 2], pl[4 * j + 3]);
-      }
-    } else {
-      float mc = -INFINITY;
-#pragma unroll
-      for (int q2 = 0; q2 < kStageKeys / 64; ++q2) {
-        uint32_t sr[2][32];
-        tc_ld_32x32b_x32(tl + col_s(b) + 64 * q2, sr[0]);
-        tc_ld_32x32b_x32(tl + col_s(b) + 64 * q2 + 32, sr[1]);
-        tc_wait_ld();
-        mask32(sr[0], 64 * q2);
-        mask32(sr[1], 64 * q2 + 32);
-        mc = max32(sr[1], max32(sr[0], mc));
-      }
-      if (!rescale(mc)) return false;
-      const float moff = (!real || m_used == -INFINITY) ? -INFINITY : -m_used;
-      // four groups of 32 keys; the TMEM load of group g+1 is in flight while
-      // group g is worked on
-      uint32_t ph[64];
-      uint32_t sr[2][32];
-      tc_ld_32x32b_x32(tl + col_s(b), sr[0]);
-      tc_wait_ld();
-#pragma unroll
-      for (int q4 = 0; q4 < kStageKeys / 32; ++q4) {
-        if (q4 + 1 < kStageKeys / 32) tc_ld_32x32b_x32(tl + col_s(b) + 32 * (q4 + 1), sr[(q4 + 1) & 1]);
-        uint32_t pl[16];
-        mask32(sr[q4 & 1], 32 * q4);
-        exp_pairs(sr[q4 & 1], moff, ph + 16 * q4, pl);
-        // the residual overwrites S columns 16 q4 .. that this thread has already read
-        tc_st_32x32b_x16(tl + col_s(b) + 16 * q4, pl);
-        if (q4 + 1 < kStageKeys / 32) tc_wait_ld();
-      }
-      tc_wait_st();
-      if (!wait_pv_done(c - 1)) return false;
-#pragma unroll
-      for (int blk = 0; blk < 2; ++blk) {
-        uint8_t *pb = X.smem + Smem::off_p + blk * Smem::kPBlock;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const uint32_t *w = ph + 32 * blk + 4 * j;
-          *reinterpret_cast<uint4 *>(pb + sw128(row, j)) = make_uint4(w[0], w[1], w[2], w[3]);
         }
       }
     }
+    const float moff = (!real || m_used == -INFINITY) ? -INFINITY : -m_used;  // -inf: p = 0
+
+    // p = 2^(s*scale - m) as three bf16 terms: hi = p truncated to bf16, lo =
+    // the residual p - hi truncated, lo2 = the rest rounded to nearest.  Both
+    // subtractions are exact, so |p - hi - lo - lo2| <= 2^-25 p.  The scaling,
+    // residuals and row sum run on packed fp32 pairs.
+    unsigned long long lsum2 = 0ull;  // {0.f, 0.f}
+    {
+      const unsigned long long sl2x2 = f2_pack(sl2, sl2), moffx2 = f2_pack(moff, moff);
+      auto upper = [](float x) { return __uint_as_float(__float_as_uint(x) & 0xffff0000u); };
+#pragma unroll
+      for (int q = 0; q < kSteps; ++q) {
+        uint32_t sr[16];
+        tc_ld_32x32b_x16(tl + col_s(b) + k0 + 16 * q, sr);
+        tc_wait_ld();
+        mask(sr, k0 + 16 * q);
+        uint32_t hi[8], lo[8], lo2[8];
+#pragma unroll
+        for (int e = 0; e < 16; e += 2) {
+          float x0, x1;
+          f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[e]), __uint_as_float(sr[e + 1])), sl2x2,
+                           moffx2),
+                    x0, x1);
+          const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+          const unsigned long long pp = f2_pack(p0, p1);
+          float l0, l1, t0, t1;
+          f2_unpack(f2_sub(pp, f2_pack(upper(p0), upper(p1))), l0, l1);
+          f2_unpack(f2_sub(f2_pack(l0, l1), f2_pack(upper(l0), upper(l1))), t0, t1);
+          hi[e >> 1] = pack_bf16x2_trunc(p0, p1);
+          lo[e >> 1] = pack_bf16x2_trunc(l0, l1);
+          lo2[e >> 1] = pack_bf16x2(t0, t1);
+          lsum2 = f2_add(lsum2, pp);
+        }
+        // the first two terms overwrite the S columns of these 16 keys, which
+        // this thread has just read (and no other thread reads)
+        const int kk = (k0 >> 4) + q;
+        tc_st_32x32b_x8(tl + col_s(b) + p_col(kk, 1), hi);
+        tc_st_32x32b_x8(tl + col_s(b) + p_col(kk, 2), lo);
+        tc_st_32x32b_x8(tl + t3_col(b, kk), lo2);
+      }
+    }
+    // the previous chunk's product into the registers (before this chunk's
+    // product overwrites O)
+    if (!wait_pv_done(c - 1)) return false;
+    tc_fence_after();
+    if (!first) take_o(alpha);
     {
       float a0, a1;
       f2_unpack(lsum2, a0, a1);
-      if (real) l_run += a0 + a1;
+      if (real) l_run = l_run * alpha + (a0 + a1);
     }
-    fence_proxy_async_smem();
+    tc_wait_st();
     tc_fence_before();
     __syncwarp();
     if (X.lane == 0) mbar_arrive(B.p_full);
@@ -945,80 +986,69 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
     if (M.flags & 2) break;
   }
 
-  // ---- the tile is done once the last P V product has landed in O ----
+  // ---- the last chunk's product, then the copies' sums into the first copy ----
   if (!wait_pv_done(c - 1)) return false;
   tc_fence_after();
-  float *ox = reinterpret_cast<float *>(X.smem + Smem::off_p);  // [64][128] fp32, O exchange
-  float *xl = xbuf + 2 * kTcRows;
-  // 16-byte chunk j of exchange row r sits at chunk j ^ (r & 7) (conflict-free)
+  take_o(1.f);
+  // the other parity of the maximum exchange: its last readers (chunk c - 2)
+  // have all passed chunk c - 1's barrier
+  float *xl = xbuf + (c & 1) * (2 * kTcRows);
+  xl[second * kTcRows + t] = l_run;
+  // O sums travel through the Q region (free: the item's last Q K^T has
+  // completed); 16-byte chunk j of exchange row r sits at chunk j ^ (r & 7)
+  float *ox = reinterpret_cast<float *>(qs);  // [64][128] fp32
   auto ox_at = [&](int r, int j) { return reinterpret_cast<float4 *>(ox + r * kD) + (j ^ (r & 7)); };
-  if constexpr (kSplit) {
-    if (h == 1) {
 #pragma unroll
-      for (int q4 = 0; q4 < kD / 32; ++q4) {
-        uint32_t r[32];
-        tc_ld_32x32b_x32(tl + kColO + q4 * 32, r);
-        tc_wait_ld();
+  for (int step = kTcRows / 2; step >= kRep; step >>= 1) {
+    if (t >= step && t < 2 * step) {
 #pragma unroll
-        for (int c4 = 0; c4 < 8; ++c4)
-          *ox_at(row, q4 * 8 + c4) =
-              make_float4(__uint_as_float(r[4 * c4]), __uint_as_float(r[4 * c4 + 1]),
-                          __uint_as_float(r[4 * c4 + 2]), __uint_as_float(r[4 * c4 + 3]));
+      for (int c4 = 0; c4 < 16; ++c4)
+        *ox_at(t - step, 16 * second + c4) =
+            make_float4(acc[4 * c4], acc[4 * c4 + 1], acc[4 * c4 + 2], acc[4 * c4 + 3]);
+    }
+    named_bar_sync(1, kCW * 32);
+    if (t < step) {
+#pragma unroll
+      for (int c4 = 0; c4 < 16; ++c4) {
+        const float4 v = *ox_at(t, 16 * second + c4);
+        acc[4 * c4] += v.x;
+        acc[4 * c4 + 1] += v.y;
+        acc[4 * c4 + 2] += v.z;
+        acc[4 * c4 + 3] += v.w;
       }
-      xl[row] = l_run;
     }
     named_bar_sync(1, kCW * 32);
   }
-  if (h == 0) {
-    const float l_tot = kSplit ? l_run + xl[row] : l_run;
-    const float inv = l_tot > 0.f ? 1.f / l_tot : 0.f;
-    uint16_t *orow = real ? out_row(g, I, I.rb * kTcRows + row) : nullptr;
-    float *prow = (real && I.n_split > 1)
-                      ? p.partials + ((size_t)I.pbase + (size_t)I.split * I.rows + row) * kPStride
-                      : nullptr;
+  if (F == 1) named_bar_sync(1, kCW * 32);  // the row sums are visible
+  if (t < kRep && real) {
+    float l_tot = 0.f;
 #pragma unroll
-    for (int q4 = 0; q4 < kD / 32; ++q4) {
-      uint32_t r[32];
-      tc_ld_32x32b_x32(tl + kColO + q4 * 32, r);
-      tc_wait_ld();
-      float o[32];
+    for (int j = 0; j < F; ++j) l_tot += xl[row + j * kRep] + xl[kTcRows + row + j * kRep];
+    if (I.n_split == 1) {
+      const float inv = l_tot > 0.f ? 1.f / l_tot : 0.f;
+      uint4 *orow = reinterpret_cast<uint4 *>(out_row(g, I, I.rb * kTcRows + row) + 64 * second);
 #pragma unroll
-      for (int e = 0; e < 32; ++e) o[e] = __uint_as_float(r[e]);
-      if (kSplit) {
-#pragma unroll
-        for (int c4 = 0; c4 < 8; ++c4) {
-          const float4 v = *ox_at(row, q4 * 8 + c4);
-          o[4 * c4] += v.x;
-          o[4 * c4 + 1] += v.y;
-          o[4 * c4 + 2] += v.z;
-          o[4 * c4 + 3] += v.w;
-        }
+      for (int c8 = 0; c8 < 8; ++c8) {
+        uint4 v;
+        v.x = pack_bf16x2(acc[8 * c8 + 0] * inv, acc[8 * c8 + 1] * inv);
+        v.y = pack_bf16x2(acc[8 * c8 + 2] * inv, acc[8 * c8 + 3] * inv);
+        v.z = pack_bf16x2(acc[8 * c8 + 4] * inv, acc[8 * c8 + 5] * inv);
+        v.w = pack_bf16x2(acc[8 * c8 + 6] * inv, acc[8 * c8 + 7] * inv);
+        orow[c8] = v;
       }
-      if (real) {
-        if (I.n_split == 1) {
+    } else {
+      float *prow = p.partials + ((size_t)I.pbase + (size_t)I.split * I.rows + row) * kPStride;
 #pragma unroll
-          for (int c8 = 0; c8 < 4; ++c8) {
-            uint4 v;
-            v.x = pack_bf16x2(o[8 * c8 + 0] * inv, o[8 * c8 + 1] * inv);
-            v.y = pack_bf16x2(o[8 * c8 + 2] * inv, o[8 * c8 + 3] * inv);
-            v.z = pack_bf16x2(o[8 * c8 + 4] * inv, o[8 * c8 + 5] * inv);
-            v.w = pack_bf16x2(o[8 * c8 + 6] * inv, o[8 * c8 + 7] * inv);
-            reinterpret_cast<uint4 *>(orow + q4 * 32)[c8] = v;
-          }
-        } else {
-#pragma unroll
-          for (int c4 = 0; c4 < 8; ++c4)
-            __stcg(reinterpret_cast<float4 *>(prow + q4 * 32) + c4,
-                   make_float4(o[4 * c4], o[4 * c4 + 1], o[4 * c4 + 2], o[4 * c4 + 3]));
-        }
+      for (int c4 = 0; c4 < 16; ++c4)
+        __stcg(reinterpret_cast<float4 *>(prow + 64 * second) + c4,
+               make_float4(acc[4 * c4], acc[4 * c4 + 1], acc[4 * c4 + 2], acc[4 * c4 + 3]));
+      if (second == 0) {
+        __stcg(prow + 128, m_used);
+        __stcg(prow + 129, l_tot);
       }
-    }
-    if (real && I.n_split > 1) {
-      __stcg(prow + 128, m_used);
-      __stcg(prow + 129, l_tot);
     }
   }
-  // TMEM O and the exchange area are free again once every thread is here
+  // TMEM O and the exchange areas are free again once every thread is here
   tc_fence_before();
   named_bar_sync(1, kCW * 32);
   return true;
@@ -1044,9 +1074,9 @@ __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, c
     const int s = it % kStages;
     if (!wait_or_abort(X, &B.full[s], (it / kStages) & 1)) return false;
     const StageMeta M = X.meta[s];
-    zero_tail(X, s, M.page0, g.L);
+    zero_tail(X, s, M.page0, g.L, kCcW * 32, 3);
     if (first) {
-      for (int e = X.ctid; e < nrow * (kD / 8); e += kCW * 32) {
+      for (int e = X.ctid; e < nrow * (kD / 8); e += kCcW * 32) {
         const int rho = e / (kD / 8), c8 = e % (kD / 8);
         const int grow = I.rb * kCcRows + rho;
         const int qi = grow / g.G, j = grow % g.G;
@@ -1069,11 +1099,11 @@ __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, c
         cl[r] = 0.f;
         co[r][0] = co[r][1] = co[r][2] = co[r][3] = 0.f;
       }
-      named_bar_sync(1, kCW * 32);
+      named_bar_sync(3, kCcW * 32);
     }
 #pragma unroll 1
-    for (int jp = 0; jp < kStagePages / kCW; ++jp) {
-      const int pg = warp + kCW * jp;  // pages warp, warp + 4 of the stage
+    for (int jp = 0; jp < kStagePages / kCcW; ++jp) {
+      const int pg = warp + kCcW * jp;  // pages warp, warp + 4 of the stage
       if (pg < M.npages) {
         const int key = lane >> 1, half = lane & 1;
         const int R = pg * kPage + key;  // key row within the stage
@@ -1175,15 +1205,15 @@ __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, c
       }
     }
   }
-  named_bar_sync(1, kCW * 32);
+  named_bar_sync(3, kCcW * 32);
   if (warp == 0) {
 #pragma unroll
     for (int r = 0; r < NR; ++r) {
       if (r < nrow) {
         float Mx = -INFINITY;
-        for (int w2 = 0; w2 < kCW; ++w2) Mx = fmaxf(Mx, mg[(w2 * 8 + r) * kPStride + 128]);
+        for (int w2 = 0; w2 < kCcW; ++w2) Mx = fmaxf(Mx, mg[(w2 * 8 + r) * kPStride + 128]);
         float Ls = 0.f, O0 = 0.f, O1 = 0.f, O2 = 0.f, O3 = 0.f;
-        for (int w2 = 0; w2 < kCW; ++w2) {
+        for (int w2 = 0; w2 < kCcW; ++w2) {
           const float *src = mg + (w2 * 8 + r) * kPStride;
           const float sc = (src[128] == -INFINITY) ? 0.f : exp2f(src[128] - Mx);
           const float4 ov = *reinterpret_cast<const float4 *>(src + lane * 4);
@@ -1213,7 +1243,7 @@ __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, c
       }
     }
   }
-  named_bar_sync(1, kCW * 32);
+  named_bar_sync(3, kCcW * 32);
   return true;
 }
 
@@ -1269,14 +1299,14 @@ __device__ __forceinline__ bool cc2_item(const AttnParams &p, const CompCtx &X, 
     const int s = it % kStages;
     if (!wait_or_abort(X, &B.full[s], (it / kStages) & 1)) return false;
     const StageMeta M = X.meta[s];
-    zero_tail(X, s, M.page0, g.L);
+    zero_tail(X, s, M.page0, g.L, kCcW * 32, 3);
     const uint8_t *kst = stage_k(X.smem, s);
     const uint8_t *vb = stage_v(X.smem, s);
     // ---- partial dot products of this lane's quarter for keys g * 8 + k ----
     float part[4][NR];
 #pragma unroll
     for (int gg = 0; gg < 4; ++gg) {
-      const int R = (warp + kCW * (gg >> 1)) * kPage + (gg & 1) * 8 + kq;
+      const int R = (warp + kCcW * (gg >> 1)) * kPage + (gg & 1) * 8 + kq;
       const uint8_t *kb = kv_row(kst, R, qq >> 1);
       uint4 kr[4];
 #pragma unroll
@@ -1311,7 +1341,7 @@ __device__ __forceinline__ bool cc2_item(const AttnParams &p, const CompCtx &X, 
         half_sum[i][r] = keep + __shfl_xor_sync(0xffffffffu, send, 1);
       }
     float sc[NR];
-    const int pg = warp + kCW * up;
+    const int pg = warp + kCcW * up;
     const int kpos = (M.page0 + pg) * kPage + (int)odd * 8 + kq;
     const bool page_ok = pg < M.npages && !((M.invalid >> pg) & 1u);
 #pragma unroll
@@ -1340,7 +1370,7 @@ __device__ __forceinline__ bool cc2_item(const AttnParams &p, const CompCtx &X, 
     // ---- P V: 32 keys into this lane's 4 dims of both rows ----
 #pragma unroll 8
     for (int key = 0; key < 32; ++key) {
-      const int R = (warp + kCW * (key >> 4)) * kPage + (key & 15);
+      const int R = (warp + kCcW * (key >> 4)) * kPage + (key & 15);
       const uint2 vv = *reinterpret_cast<const uint2 *>(kv_row(vb, R, vhalf) +
                                                         ((vc ^ (R & 7)) << 4) + vsub);
       const float2 pk = *reinterpret_cast<const float2 *>(pw + key * NR);
@@ -1372,15 +1402,15 @@ __device__ __forceinline__ bool cc2_item(const AttnParams &p, const CompCtx &X, 
       dst[129] = cl[r];
     }
   }
-  named_bar_sync(1, kCW * 32);
+  named_bar_sync(3, kCcW * 32);
   if (warp < NR) {  // warp r merges row r
     const int r = warp;
     float Mx = -INFINITY;
 #pragma unroll
-    for (int w2 = 0; w2 < kCW; ++w2) Mx = fmaxf(Mx, mg[(w2 * 8 + r) * kPStride + 128]);
+    for (int w2 = 0; w2 < kCcW; ++w2) Mx = fmaxf(Mx, mg[(w2 * 8 + r) * kPStride + 128]);
     float Ls = 0.f, O0 = 0.f, O1 = 0.f, O2 = 0.f, O3 = 0.f;
 #pragma unroll
-    for (int w2 = 0; w2 < kCW; ++w2) {
+    for (int w2 = 0; w2 < kCcW; ++w2) {
       const float *src = mg + (w2 * 8 + r) * kPStride;
       const float sc = (src[128] == -INFINITY) ? 0.f : ex2_approx(src[128] - Mx);
       const float4 ov = *reinterpret_cast<const float4 *>(src + lane * 4);
@@ -1406,8 +1436,22 @@ __device__ __forceinline__ bool cc2_item(const AttnParams &p, const CompCtx &X, 
       }
     }
   }
-  named_bar_sync(1, kCW * 32);
+  named_bar_sync(3, kCcW * 32);
   return true;
+}
+
+// A CUDA-core item runs on the first kCcW compute warps; the others release
+// each of its stages (the stage's empty barrier counts every compute warp).
+__device__ __forceinline__ bool pass_item(const CompCtx &X, uint32_t &it) {
+  for (;;) {
+    const int s = it % kStages;
+    if (!wait_or_abort(X, &X.B.full[s], (it / kStages) & 1)) return false;
+    const int flags = X.meta[s].flags;
+    __syncwarp();
+    if (X.lane == 0) mbar_arrive(&X.B.empty[s]);
+    ++it;
+    if (flags & 2) return true;
+  }
 }
 
 __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant__ AttnParams p) {
@@ -1445,6 +1489,10 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
   const uint32_t tmem = misc[0];
   const int n_items = p.ctrl[0];
 
+  if (warp >= kCW) {
+  // the third warpgroup: producer, MMA issuer, and two warps that only take
+  // part in the register split
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(kRegsAux));
   if (warp == kProducerWarp) {
     // ------------------------------ producer ------------------------------
     // Page ids are read 32 at a time (one coalesced load per warp), one batch
@@ -1580,17 +1628,18 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
     // issues its own P V, so no product waits on the next item's stages.
     constexpr uint32_t idesc_s = idesc_bf16_f32(kTcRows, kStageKeys, 0);
     constexpr uint32_t idesc_o = idesc_bf16_f32(kTcRows, kD, 1);
-    const uint32_t pa = smem_u32(smem + Smem::off_p);
+    const uint32_t qa = smem_u32(smem + Smem::off_q);
     uint32_t it = 0, c = 0, nq = 0;
     bool ok = true, pend = false;
     uint32_t pc = 0;  // pending chunk
-    int pstage = 0, pfirst = 0, ppath = 0;
+    int pstage = 0;
     auto mwait = [&](uint64_t *bar, uint32_t par) -> bool {
       if (mbar_wait_bounded(bar, par)) return true;
       ok = false;
       return false;
     };
-    // O (+)= P V of the pending chunk; the first chunk of an item overwrites O
+    // O = P V of the pending chunk (every chunk's product starts a fresh O;
+    // the compute warps sum the chunks in registers)
     auto issue_pv = [&]() -> bool {
       if (!mwait(B.p_full, pc & 1)) return false;
       tc_fence_after();
@@ -1600,10 +1649,12 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
         for (int kk = 0; kk < kStageKeys / 16; ++kk) {
           // V keys 16kk.. as an MN-major operand: 64-dim halves 1 KB apart, 8-key groups 2 KB
           const uint64_t bd = sdesc_sw128(va + kk * 2 * kGroupBytes, kAtomBytes, kGroupBytes);
-          const uint64_t ad = sdesc_sw128(pa + (kk >> 2) * Smem::kPBlock + (kk & 3) * 32, 16, 1024);
-          tc_mma_bf16(tmem + kColO, ad, bd, idesc_o, (pfirst && kk == 0) ? 0u : 1u);
-          if (ppath == kPathTcFull)  // residual of P, from the chunk's S buffer
-            tc_mma_bf16_ta(tmem + kColO, tmem + col_s(pc & 1) + 8 * kk, bd, idesc_o, 1u);
+          // the three terms of P: the chunk's S buffer and the third term's
+          // columns of that buffer's parity
+          const uint32_t pt = tmem + col_s(pc & 1);
+          tc_mma_bf16_ta(tmem + kColO, pt + p_col(kk, 1), bd, idesc_o, kk == 0 ? 0u : 1u);
+          tc_mma_bf16_ta(tmem + kColO, pt + p_col(kk, 2), bd, idesc_o, 1u);
+          tc_mma_bf16_ta(tmem + kColO, tmem + t3_col(pc & 1, kk), bd, idesc_o, 1u);
         }
         tc_commit(B.p_free);
         tc_commit(&B.empty[pstage]);
@@ -1631,7 +1682,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
         ++it;
         continue;
       }
-      if (flags & 1) {  // a new tensor item: its Q tile must be in TMEM
+      if (flags & 1) {  // a new tensor item: its Q tile must be in shared memory
         if (!mwait(B.q_ready, nq & 1)) break;
         ++nq;
       }
@@ -1640,9 +1691,11 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
         const uint32_t ka = smem_u32(stage_k(smem, s));
 #pragma unroll
         for (int kk = 0; kk < kD / 16; ++kk) {
+          // Q dims 16kk.. (K-major: 64-dim halves 16 KB apart, 8-row groups 1 KB)
+          const uint64_t ad = sdesc_sw128(qa + (kk >> 2) * Smem::kQHalf + (kk & 3) * 32, 16, 1024);
           const uint64_t bd =
               sdesc_sw128(ka + (kk >> 2) * kAtomBytes + (kk & 3) * 32, 16, kGroupBytes);
-          tc_mma_bf16_ta(tmem + col_s(c & 1), tmem + kColQ + 8 * kk, bd, idesc_s, kk > 0);
+          tc_mma_bf16(tmem + col_s(c & 1), ad, bd, idesc_s, kk > 0);
         }
         tc_commit(&B.s_full[c & 1]);
       }
@@ -1651,8 +1704,6 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
       pend = true;
       pc = c;
       pstage = s;
-      pfirst = flags & 1;
-      ppath = path;
       ++c;
       ++it;
       if ((flags & 2) && !issue_pv()) break;
@@ -1668,7 +1719,11 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
     return;
   }
 
+  return;
+  }
+
   // -------------------------------- compute warps --------------------------------
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(kRegsCompute));
   const CompCtx X{smem, B, meta, misc, tmem, warp, lane, (int)threadIdx.x};
   uint32_t it = 0, c = 0;
   for (;;) {
@@ -1678,15 +1733,18 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
     if (M.item < 0 || *(volatile uint32_t *)&misc[1]) break;
     const Item I = p.items[M.item];
     bool ok;
-    if (I.path == kPathTcSplit) {
-      ok = tc_item<true>(p, X, I, it, c);
-    } else if (I.path == kPathTcFull) {
-      ok = tc_item<false>(p, X, I, it, c);
-    } else {
+    if (I.path != kPathCc) {
+      // copies of the tile's rows over the 128 lanes: 4 (<= 32 rows), 2 (<= 64) or 1
+      if (I.rows <= kTcRows / 4) ok = tc_item<4>(p, X, I, it, c);
+      else if (I.rows <= kTcRows / 2) ok = tc_item<2>(p, X, I, it, c);
+      else ok = tc_item<1>(p, X, I, it, c);
+    } else if (warp < kCcW) {
       // GQA-2 decode (two rows) has its own layout; other sizes take the
       // guarded loop
       if (I.rows == 2) ok = cc2_item(p, X, I, it);
       else ok = cc_item<kCcRows>(p, X, I, it);
+    } else {
+      ok = pass_item(X, it);  // the other warps only release the item's stages
     }
     if (!ok) break;
     if (I.n_split > 1) {

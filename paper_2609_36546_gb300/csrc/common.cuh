@@ -238,6 +238,18 @@ IPD_DEVINL void tc_ld_32x32b_x32(uint32_t taddr, uint32_t (&r)[32]) {
       : "memory");
 }
 
+// Each lane of the warp reads 16 consecutive 32-bit TMEM columns of its lane.
+IPD_DEVINL void tc_ld_32x32b_x16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+      "%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr)
+      : "memory");
+}
+
 // Shared-memory matrix descriptor, 128-byte swizzle (tcgen05 format: start
 // address, leading and stride byte offsets in 16-byte units, version 1 at
 // bit 46, layout type 2 = SWIZZLE_128B at bits 61-63).  The swizzle atoms
@@ -287,6 +299,14 @@ IPD_DEVINL void tc_st_32x32b_x16(uint32_t taddr, const uint32_t (&r)[16]) {
       "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
       "r"(r[15])
       : "memory");
+}
+
+// Each lane of the warp writes 8 consecutive 32-bit TMEM columns of its lane.
+IPD_DEVINL void tc_st_32x32b_x8(uint32_t taddr, const uint32_t (&r)[8]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr),
+               "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]),
+               "r"(r[7])
+               : "memory");
 }
 
 // Two floats truncated to their upper 16 bits (bf16 rounded toward zero) and

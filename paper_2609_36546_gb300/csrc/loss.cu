@@ -92,7 +92,8 @@ __global__ void __launch_bounds__(kLossThreads) split_loss_kernel(
 
 }  // namespace
 
-extern "C" size_t ipd_loss_workspace_size(int num_reqs) { return num_reqs < 0 ? 0 : 0; }
+// The loss needs no scratch: one CTA reduces the step in shared memory.
+extern "C" size_t ipd_loss_workspace_size(int /*num_reqs*/) { return 0; }
 
 extern "C" int ipd_split_loss(const float *kl_rev, const float *kl_fwd, const uint8_t *source,
                               const int32_t *cu_span, const int32_t *n_emit,

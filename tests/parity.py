@@ -3,11 +3,15 @@ by __graft_entry__.smoke()).
 
 Tolerances (stated once here):
 * attention: every output within 2 bf16 ulp of the fp64 oracle rounded to
-  bf16, the ulp taken at max(|ref|, rowmax/8) where rowmax is the largest
-  magnitude of that (query, head) output vector; the strict ulp at |ref| is
-  reported alongside.  (Reading of "2 bf16 ulp" for near-zero components: an
-  fp32-accumulated average of bf16 values carries an absolute error tied to
-  the scale of the vector, not of one tiny component.)
+  bf16, the ulp taken at max(|ref|, ATTN_FLOOR * a), where a = sum_j w_j |v_jd|
+  is the softmax-weighted mean magnitude of the values that output averages
+  (the oracle's attention over |V|).  An fp32 evaluation of the weighted sum
+  has an absolute error of a few fp32 roundings of a, whatever the size of the
+  result, so a component that cancels to nearly zero cannot be held to 2 ulp
+  of itself.  ATTN_FLOOR = 2^-16 is the smallest power of two under which a
+  plain IEEE-fp32 evaluation (tests/attn_fp32_model.py) passes every small
+  case (tests/test_attn_tolerance.py).  The strict ulp at |ref| is reported
+  beside it, and at least ATTN_STRICT_FRAC of all elements must meet it.
 * log-probs within 1e-3 absolute; feedback within 2e-3 (difference of two).
 * KL terms within 2e-4 + 1e-4 |ref| (fp32 sums of <= 64 terms of size <= ~40).
 * margin: exact (difference of two bf16 values is exact in fp32).
@@ -26,21 +30,30 @@ ATOL_LOGP = 1e-3
 ATOL_FEEDBACK = 2e-3
 KL_ATOL, KL_RTOL = 2e-4, 1e-4
 LOSS_RTOL = 1e-4
+ATTN_FLOOR = 2.0 ** -16
+ATTN_STRICT_FRAC = 0.9999
 
 
 def u16(t: torch.Tensor) -> np.ndarray:
     return t.detach().contiguous().cpu().view(torch.int16).numpy().view(np.uint16)
 
 
-def attn_ulp_errors(got_bits: np.ndarray, ref: np.ndarray):
-    """(floored-ulp error, strict-ulp error) arrays, in bf16 ulps."""
+def attn_ulp_errors(got_bits: np.ndarray, ref: np.ndarray, ref_abs: np.ndarray):
+    """(error under the floor, strict error) arrays, in bf16 ulps.
+
+    ref: the fp64 oracle output; ref_abs: the oracle's attention over |V|
+    (the weighted mean magnitude a of the averaged values), same shape."""
     got = O.bf16_to_f64(got_bits)
     ref_b = O.bf16_to_f64(O.f64_to_bf16(ref))
-    rowmax = np.abs(ref).max(axis=-1, keepdims=True)
-    ulp_floor = O.bf16_ulp(np.maximum(np.abs(ref), rowmax / 8.0))
-    ulp_strict = O.bf16_ulp(np.maximum(np.abs(ref_b), 1e-30))
     err = np.abs(got - ref_b)
+    ulp_floor = O.bf16_ulp(np.maximum(np.abs(ref_b), ATTN_FLOOR * np.abs(ref_abs)))
+    ulp_strict = O.bf16_ulp(np.maximum(np.abs(ref_b), 1e-30))
     return err / ulp_floor, err / ulp_strict
+
+
+def abs_bits(bits: np.ndarray) -> np.ndarray:
+    """|x| of bf16 bit patterns (the sign bit cleared: exact)."""
+    return (np.asarray(bits, np.uint16) & np.uint16(0x7FFF)).astype(np.uint16)
 
 
 def check_attention(step, requests=None, max_reqs_per_batch=None, rng=None):
@@ -70,8 +83,9 @@ def check_attention(step, requests=None, max_reqs_per_batch=None, rng=None):
             vp = u16(pool_v.index_select(0, pages))
             qb = u16(q[cu[j]:cu[j + 1]])
             ref = O.paged_span_attention(qb, kp, vp, np.arange(npg), L, step.scale)
+            ref_abs = O.paged_span_attention(qb, kp, abs_bits(vp), np.arange(npg), L, step.scale)
             got = u16(out[cu[j]:cu[j + 1]])
-            e_floor, e_strict = attn_ulp_errors(got, ref)
+            e_floor, e_strict = attn_ulp_errors(got, ref, ref_abs)
             stats["attn_rows"] += ref.shape[0] * ref.shape[1]
             stats["attn_max_ulp"] = max(stats["attn_max_ulp"], float(e_floor.max()))
             stats["attn_max_ulp_strict"] = max(stats["attn_max_ulp_strict"], float(e_strict.max()))
@@ -80,7 +94,7 @@ def check_attention(step, requests=None, max_reqs_per_batch=None, rng=None):
             n_all += e_strict.size
     if n_all:
         stats["attn_frac_strict_le2"] = n_strict_ok / n_all
-    stats["attn_ok"] = stats["attn_bad"] == 0
+    stats["attn_ok"] = stats["attn_bad"] == 0 and stats["attn_frac_strict_le2"] >= ATTN_STRICT_FRAC
     return stats
 
 

@@ -9,6 +9,7 @@ import pytest
 import torch
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "ipd.h")
 
 
 @pytest.fixture(scope="module")
@@ -34,9 +35,16 @@ def test_library_exports_every_declared_function(ipd):
 
 
 def test_status_strings_and_version(ipd):
-    assert ipd.lib().ipd_status_string(0) == b"IPD_OK"
-    assert ipd.lib().ipd_status_string(3) == b"IPD_ERR_WORKSPACE"
+    """Every status code the header defines has its own name."""
+    with open(HEADER) as f:
+        codes = dict((n, int(v)) for n, v in
+                     re.findall(r"#define\s+(IPD_OK|IPD_ERR_[A-Z_]+)\s+(\d+)", f.read()))
+    assert len(codes) >= 8 and codes["IPD_ERR_CAPACITY"] == 7
+    for name, v in codes.items():
+        assert ipd.lib().ipd_status_string(v) == name.encode(), name
+        assert ipd.STATUS_CODES[name] == v
     assert ipd.lib().ipd_status_string(99) == b"IPD_ERR_UNKNOWN"
+    assert ipd.lib().ipd_status_string(-1) == b"IPD_ERR_UNKNOWN"
     assert ipd.lib().ipd_version() == 100
 
 

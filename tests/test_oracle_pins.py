@@ -40,6 +40,28 @@ def test_bf16_conversions_match_torch():
                           .to(torch.float64).numpy())
 
 
+def test_bf16_ulp_is_the_spacing_of_neighbouring_bf16_values():
+    """bf16_ulp sets every attention tolerance, so it is pinned to the spacing
+    of adjacent bf16 numbers for every finite normal bit pattern of either
+    sign: value(b + 1) - value(b) in magnitude, both values taken through
+    torch's own bf16 -> fp64 conversion.  An exponent off by one anywhere
+    would double or halve the spacing and fail here."""
+    mags = np.arange(0x0080, 0x7f7f, dtype=np.int32)          # normal, next one still finite
+    for sign in (0, 0x8000):
+        b = (mags | sign).astype(np.uint16)
+        nb = (mags + 1 | sign).astype(np.uint16)
+        val = lambda u: torch.from_numpy(u.view(np.int16)).view(torch.bfloat16).to(
+            torch.float64).numpy()
+        x, xn = val(b), val(nb)
+        assert np.all(np.isfinite(xn))
+        assert np.array_equal(O.bf16_ulp(x), np.abs(xn - x))
+    # between two bf16 values the spacing is that of the binade holding x
+    assert O.bf16_ulp(1.5) == 2.0 ** -7 and O.bf16_ulp(1.999) == 2.0 ** -7
+    assert O.bf16_ulp(0.75) == 2.0 ** -8 and O.bf16_ulp(-3.0e-3) == 2.0 ** -16
+    assert O.bf16_ulp(float(torch.finfo(torch.bfloat16).max)) == 2.0 ** 120
+    assert O.bf16_ulp(1.0) == float(torch.finfo(torch.bfloat16).eps)
+
+
 # ---------------------------------------------------------------------------
 # attention
 # ---------------------------------------------------------------------------
