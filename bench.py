@@ -9,6 +9,10 @@ step streams its KV pages and logits from DRAM.
   python bench.py [--gpus N] [--steps K] [--warmup W] [--config I] [--impl reference]
   python bench.py --next-rows [--config I] [--steps K]
 
+The headline workload is the full rollout-step mix (1024 requests, lognormal
+contexts up to 32K, spans of 1-16 tokens, both directions, 120 GB of KV
+pools), the largest that fits one GPU; the other full-size workloads follow
+in a `per_config` record (device-timed the same way, fewer steps).
 Prints one JSON line (rank 0).  ``--impl reference`` times the fp64 CPU
 oracle (the only reference that exists for this path) on a bounded sample of
 the same workload.
@@ -315,23 +319,19 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
-def run_gpu(args):
+def measure_config(cfg, K, W, world, rank, stream, sampler=None):
+    """Device-timed steps of one workload: per-call events, the attention
+    kernel's own events, and the step replayed from CUDA graphs.  Returns the
+    step, the workload and a dict of figures (max over ranks)."""
     import torch
-    world, rank, local = _init_dist(args)
-    torch.cuda.set_device(local)
-    import __graft_entry__
-    __graft_entry__.build()
     import ipd_synth as S
     from paper_2609_36546_gb300 import VerifyStep, ipd
 
-    cfg = args.config
     w = S.make_workload(cfg, seed=cfg + 1000 * rank, device="cuda")
     step = VerifyStep.from_workload(w, device="cuda")
-    stream = torch.cuda.current_stream()
     T_tok = step.T
-
     # warm-up (also yields the verdict used for the algorithmic byte count)
-    for _ in range(max(3, args.warmup)):
+    for _ in range(W):
         step.run(stream)
     torch.cuda.synchronize()
     if ipd.device_error() != 0:
@@ -342,13 +342,10 @@ def run_gpu(args):
     accept_rate = float(step.score["covered"].float().mean()) if T_tok else 0.0
     emitted = int(step.score["n_emit"].sum())
 
-    # ---- timed region: K steps, per-call events on the launching stream ----
-    K = args.steps
+    # ---- K steps call by call, per-call events on the launching stream ----
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(K)]
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
-    sampler = ClockSampler(_smi_index(local)) if rank == 0 else None
-    time.sleep(0.3 if sampler else 0.0)
     _barrier(world)
     torch.cuda.synchronize()
     # the library also records events around the attention kernel alone
@@ -375,8 +372,8 @@ def run_gpu(args):
     score_ms = statistics.mean(e[1].elapsed_time(e[2]) for e in ev)
     loss_ms = statistics.mean(e[2].elapsed_time(e[3]) for e in ev)
 
-    # ---- timed region for `value`: the same K steps replayed from a CUDA graph
-    # of one step (same kernels and buffers, no per-call host work) ----
+    # ---- the same K steps replayed from a CUDA graph of one step (same
+    # kernels and buffers, no per-call host work): the step time ----
     graph = step.capture(overlap=True)
     torch.cuda.synchronize()
     g_start = torch.cuda.Event(enable_timing=True)
@@ -401,33 +398,22 @@ def run_gpu(args):
         graph1.replay()
     g_end.record(stream)
     torch.cuda.synchronize()
+    del graph, graph1
     ms_step_one_stream = _max_over_ranks(g_start.elapsed_time(g_end), world) / K
     el_max = _max_over_ranks(el_ms, world)
     tokens_all = _sum_over_ranks(float(T_tok * K), world)
-    value = tokens_all / (el_max / 1e3)
     ms_step = el_max / K
-    ms_step_direct = _max_over_ranks(el_direct_ms, world) / K
-
-    # ---- end to end through host buffers ----
-    e2e = run_e2e(step, w, min(K, args.e2e_steps), stream, world)
-
     peak, peak_kind = _peaks()
-    if rank != 0:
-        return
     achieved = attn_bytes / (attn_kernel_ms / 1e3) / 1e9
     achieved_call = attn_bytes / (attn_ms / 1e3) / 1e9
-    traffic = _committed_traffic(cfg)
     step_alg = attn_bytes + logits_alg
     step_full = attn_bytes + logits_full
-    line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
-        "warmup": max(3, args.warmup), "ms_per_step": ms_step, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": _workload_name(cfg), "seed": cfg, "tokens_per_step": T_tok,
-                   "requests": step.R, "l2": "inputs larger than L2 (no flush needed)",
-                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+    fig = {
+        "value": tokens_all / (el_max / 1e3), "ms_per_step": ms_step, "tokens_per_step": T_tok,
+        "requests": step.R, "clocks": clocks,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
+                     "frac": achieved / peak, "traffic": _committed_traffic(cfg),
+                     "peak_kind": peak_kind,
                      "kernel": "attn_kernel (the attention launch of ipd_verify_attn; split "
                                "tasks merge inside it)",
                      "bytes_per_launch": attn_bytes, "ms_per_launch": attn_kernel_ms,
@@ -442,18 +428,80 @@ def run_gpu(args):
                      "frac_full_of_nominal_8tbs": step_full / (ms_step / 1e3) / 1e9 / 8000.0},
         "calls_ms": {"verify_attn": attn_ms, "score_span": score_ms, "split_loss": loss_ms},
         "ms_per_step_one_stream_graph": ms_step_one_stream,
-        "ms_per_step_direct_calls": ms_step_direct,
+        "ms_per_step_direct_calls": _max_over_ranks(el_direct_ms, world) / K,
+        "acceptance": {"coverage_rate": accept_rate, "emitted_tokens_per_step": emitted},
+    }
+    return step, w, fig
+
+
+def run_gpu(args):
+    import torch
+    world, rank, local = _init_dist(args)
+    torch.cuda.set_device(local)
+    import __graft_entry__
+    __graft_entry__.build()
+
+    cfg = args.config
+    stream = torch.cuda.current_stream()
+    K = args.steps
+    sampler = ClockSampler(_smi_index(local)) if rank == 0 else None
+    time.sleep(0.3 if sampler else 0.0)
+    step, w, fig = measure_config(cfg, K, max(3, args.warmup), world, rank, stream, sampler)
+
+    # ---- end to end through host buffers ----
+    e2e = run_e2e(step, w, min(K, args.e2e_steps), stream, world)
+    cpu = cpu_baseline(step, w) if (world == 1 and rank == 0 and not args.no_cpu_baseline) \
+        else None
+    del step, w
+    torch.cuda.empty_cache()
+
+    # ---- the other full-size workloads, device-timed the same way (fewer
+    # steps, no end-to-end leg), one at a time ----
+    per_config = {}
+    if world == 1 and not args.no_per_config:
+        import ipd_synth as S
+        for c in range(1, len(S.CONFIGS)):
+            if c == cfg:
+                continue
+            st, wc, f = measure_config(c, min(K, args.per_config_steps), max(3, args.warmup),
+                                       world, rank, stream)
+            per_config[S.CONFIGS[c].name] = {
+                "workload": _workload_name(c), "value": f["value"], "unit": UNIT,
+                "ms_per_step": f["ms_per_step"],
+                "roofline_frac": f["roofline"]["frac"],
+                "attn_kernel_ms": f["roofline"]["ms_per_launch"],
+                "attn_call_frac": f["roofline"]["call"]["frac"],
+                "step_hbm_frac_alg_of_measured": f["step_hbm"]["frac_alg_of_measured"],
+                "traffic": f["roofline"]["traffic"]}
+            del st, wc
+            torch.cuda.empty_cache()
+    if rank != 0:
+        return
+    line = {
+        "metric": METRIC, "value": fig["value"], "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": max(3, args.warmup), "ms_per_step": fig["ms_per_step"],
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic",
+        "config": {"workload": _workload_name(cfg), "seed": cfg,
+                   "tokens_per_step": fig["tokens_per_step"], "requests": fig["requests"],
+                   "l2": "inputs larger than L2 (no flush needed)",
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
+        "roofline": fig["roofline"], "step_hbm": fig["step_hbm"], "calls_ms": fig["calls_ms"],
+        "ms_per_step_one_stream_graph": fig["ms_per_step_one_stream_graph"],
+        "ms_per_step_direct_calls": fig["ms_per_step_direct_calls"],
         "timing": "value: K steps replayed from a CUDA graph of one step (the vocabulary pass "
                   "and the loss on a forked stream, joined at the end); calls_ms and the "
                   "roofline: the same K steps issued call by call on one stream, CUDA events "
                   "around each call, and around each attention kernel launch (recorded by the "
                   "library on the call's stream)",
-        "acceptance": {"coverage_rate": accept_rate, "emitted_tokens_per_step": emitted},
-        "e2e": e2e, "clocks": clocks,
+        "acceptance": fig["acceptance"],
+        "e2e": e2e, "clocks": fig["clocks"],
         "gpu_launches": LAUNCHES_PER_STEP * K,
     }
-    if world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(step, w)
+    if cpu is not None:
+        line["cpu_baseline"] = cpu
+    if per_config:
+        line["per_config"] = per_config
     print(json.dumps(line), flush=True)
 
 
@@ -704,12 +752,16 @@ def run_next_rows(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
-    ap.add_argument("--config", type=int, default=1)
+    # the largest single-GPU workload: the full rollout-step mix
+    ap.add_argument("--config", type=int, default=4)
     ap.add_argument("--impl", default="ipd", choices=["ipd", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=200)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-per-config", action="store_true",
+                    help="skip the device-timed figures of the other workloads")
+    ap.add_argument("--per-config-steps", type=int, default=100)
     ap.add_argument("--next-rows", action="store_true",
                     help="time the calls beyond the step instead (one GPU)")
     args = ap.parse_args()

@@ -15,20 +15,24 @@
 // KV pages stream through a 3-stage ring of 128-key stages (64 KB), one
 // 4 KB 4-D TMA box per page and tensor.
 // Two compute paths, chosen per task by its row count:
-//   tensor path (rows >= kTcMinRows): a 128-lane tile.  S = Q K^T (Q and K
-//     from shared memory, N = 128 keys) and P V run on tcgen05 with fp32
-//     accumulators in TMEM.  P is passed as three bf16 terms (its upper 16
-//     bits, the truncated residual and what is left of it, rounded), A
-//     operands read from TMEM, so P V sees each probability to within 2^-25
-//     of itself.  Each chunk's P V starts a fresh accumulator, and the chunks
-//     are summed in fp32 registers with round-to-nearest adds: the tensor
-//     core's own accumulation does not round to nearest, and summed over a
-//     whole long context its error reaches several bf16 ulp of the result.
+//   tensor path (rows >= kTcMinRows): a 128-lane tile.  S = Q K^T (Q from
+//     TMEM, K from shared memory, N = 128 keys) and P V run on tcgen05 with
+//     fp32 accumulators in TMEM.  P is passed as three bf16 terms (its upper
+//     16 bits, the truncated residual and what is left of it, rounded), so
+//     P V sees each probability to within 2^-25 of itself.  Each chunk's P V
+//     starts a fresh accumulator, and the chunks are summed in fp32
+//     registers with round-to-nearest adds: the tensor core's own
+//     accumulation does not round to nearest, and summed over a whole long
+//     context its error reaches several bf16 ulp of the result.
 //     All eight compute warps work on a tile, two threads per TMEM lane, each
-//     taking half of a chunk's keys and half of the output dimensions; tiles
-//     of at most 64 rows repeat their rows in lanes 64..127, which carry the
-//     third term of P.  S is double-buffered, so the softmax of chunk j
-//     overlaps Q K^T of j+1 and P V of j-1.
+//     taking part of a chunk's keys and half of the output dimensions.  A
+//     tile of at most 32 (64) rows is repeated 4 (2) times over the lanes,
+//     the copies splitting each chunk's keys, and its P terms are stacked in
+//     the 128 rows of one shared-memory operand (three terms of 32 rows, or
+//     two of 64 with the third in TMEM), so P V costs 8 (16) MMAs per chunk
+//     instead of 24: those tiles would otherwise be bound by the tensor pipe.
+//     S is double-buffered, so the softmax of chunk j overlaps Q K^T of j+1
+//     and P V of j-1.
 //   CUDA-core path (fewer rows: the GQA-2 decode and one-token spans, two
 //     rows): fp32 FMA on the first four compute warps, two pages of 16 keys
 //     per warp and stage, two lanes per key.  From four rows up the tensor
@@ -69,7 +73,6 @@ constexpr int kAtomBytes = 1024;                  // 8 keys, one 64-dim half
 constexpr int kTensorBytes = kStagePages * kPageBytes;  // 32 KB of K (or V) per stage
 constexpr int kStageBytes = 2 * kTensorBytes;     // 64 KB
 constexpr int kTcRows = 128;                      // TMEM lanes of a tensor-core tile (M)
-constexpr int kTcSplitRows = 64;                  // tiles up to this size split rows over two threads
 constexpr int kTcMinRows = 4;                     // tasks with at least this many rows use it
 constexpr int kCcRows = kTcMinRows - 1;           // CUDA-core tasks have fewer rows
 constexpr int kCW = 8;                            // compute warps (two per TMEM lane block)
@@ -93,27 +96,38 @@ constexpr int kMinChunkPages = 16;
 constexpr int kSplitMax = 16;
 constexpr int kPStride = 132;                     // floats per partial row: o[128], m, l, pad
 constexpr uint32_t kTmemCols = 512;
-// TMEM columns: the S double buffer at 0 and 128 (fp32, one column per key),
-// the O product of one chunk at 256, and at 384 + 64 b the third term of P
-// for S buffer b.  A consumed S buffer is overwritten with two terms of P as
-// bf16 pairs: for keys 16kk .. 16kk + 15, columns 16kk .. 16kk + 7 hold the
-// first and 16kk + 8 .. 16kk + 15 the second (p_col), in place of the S
-// values of the same keys, so that each thread writes only columns it has
-// itself just read.
+// TMEM columns: the S double buffer at 0 and 128 (fp32, one column per key)
+// and the O product of one chunk at 256.  Columns 384..511 hold, for tiles of
+// up to 64 rows, the Q tile at 384 (64 columns of bf16 pairs) and the third
+// term of P at 448 (64 columns of bf16 pairs; one buffer, written only after
+// the previous chunk's P V has completed); for 128-row tiles, whose Q tile
+// sits in shared memory, the third term of P at 384 + 64 b for S buffer b.
+// In 128-row tiles a consumed S buffer is overwritten with the first two
+// terms of P as bf16 pairs: for keys 16kk .. 16kk + 15, columns 16kk ..
+// 16kk + 7 hold the first and 16kk + 8 .. 16kk + 15 the second (p_col), in
+// place of the S values of the same keys, so that each thread writes only
+// columns it has itself just read.
 __device__ __forceinline__ uint32_t col_s(uint32_t b) { return b * 128u; }
 constexpr uint32_t kColO = 256;
-constexpr uint32_t kColT3 = 384;
+constexpr uint32_t kColQ = 384;
+constexpr uint32_t kColT3 = 448;
 // column (relative to an S buffer) of keys 16 kk .. 16 kk + 15 of term 1 or
 // term 2 of P
 __host__ __device__ constexpr uint32_t p_col(int kk, int term) {
   return 16u * (uint32_t)kk + 8u * (uint32_t)(term - 1);
 }
-// column of keys 16 kk .. 16 kk + 15 of the third term of P for S buffer b
-__host__ __device__ constexpr uint32_t t3_col(uint32_t b, int kk) {
-  return kColT3 + 64u * b + 8u * (uint32_t)kk;
+// column of keys 16 kk .. 16 kk + 15 of the third term of P (tiles of up to
+// 64 rows), and for S buffer b of a 128-row tile
+__host__ __device__ constexpr uint32_t t3_col(int kk) { return kColT3 + 8u * (uint32_t)kk; }
+__host__ __device__ constexpr uint32_t t3_col_full(uint32_t b, int kk) {
+  return kColQ + 64u * b + 8u * (uint32_t)kk;
 }
-// item paths
-constexpr int kPathCc = 0, kPathTcSplit = 1, kPathTcFull = 2;
+// item paths: CUDA cores, or a tensor tile repeated 4, 2 or 1 times over the
+// 128 TMEM lanes (at most 32, at most 64, or up to 128 rows)
+constexpr int kPathCc = 0, kPathTc4 = 1, kPathTc2 = 2, kPathTc1 = 3;
+__host__ __device__ constexpr int tc_path(int rows) {
+  return rows <= kTcRows / 4 ? kPathTc4 : rows <= kTcRows / 2 ? kPathTc2 : kPathTc1;
+}
 
 struct BatchDev {
   const uint16_t *q;
@@ -128,7 +142,7 @@ struct BatchDev {
 struct __align__(16) Item {
   int b, r, kvh, rb;
   int split, n_split, page_lo, page_hi;
-  int task, pbase, rows, path;  // path: kPathCc, kPathTcSplit or kPathTcFull
+  int task, pbase, rows, path;  // path: kPathCc or kPathTc4 / 2 / 1
 };
 static_assert(sizeof(Item) == 48, "items are written as three 16-byte vectors");
 
@@ -563,7 +577,7 @@ __global__ void __launch_bounds__(kT) attn_plan_kernel(const __grid_constant__ A
         for (int rb = 0; rb < s.nrb; ++rb) {
           const int rows = min(s.rpb, s.rows - rb * s.rpb);
           const int pbase = ns > 1 ? info.z + ns * (kvh * s.rows + rb * s.rpb) : -1;
-          const int pth = path >= 0 ? path : (rows <= kTcSplitRows ? kPathTcSplit : kPathTcFull);
+          const int pth = path >= 0 ? path : tc_path(rows);
           int4 *dst = reinterpret_cast<int4 *>(p.items + slot);
           dst[0] = make_int4(b, r, kvh, rb);
           dst[1] = make_int4(sp, ns, lo, hi);
@@ -622,25 +636,26 @@ __device__ void merge_split_row(const AttnParams &p, const Item &I, int r, int l
 // --------------------------------------------------------------------------
 struct Smem {
   static constexpr int off_stage = 0;                              // 3 x 64 KB, 1024-aligned
-  // the Q tile of a tensor item: two 64-dim halves of 128 rows x 128 B,
-  // 128-byte swizzled (a K-major operand); also the finalize's exchange area
-  // and the CUDA-core path's scratch
-  static constexpr int off_q = off_stage + kStages * kStageBytes;
-  static constexpr int kQHalf = kTcRows * 128;                     // 16 KB
-  static constexpr int off_x = off_q + 2 * kQHalf;                 // row-max / row-sum exchange [2][256]
+  // the P operand of a stacked tile, or the Q tile of a 128-row tile: two
+  // halves (64 keys, or 64 dims) of 128 rows x 128 B, 128-byte swizzled (a
+  // K-major A operand); also the finalize's exchange area and the CUDA-core
+  // path's scratch
+  static constexpr int off_p = off_stage + kStages * kStageBytes;
+  static constexpr int kPHalf = kTcRows * 128;                     // 16 KB
+  static constexpr int off_x = off_p + 2 * kPHalf;                 // row-max / row-sum exchange [2][256]
   static constexpr int off_meta = off_x + 2 * 256 * 4;
   static constexpr int off_bar = off_meta + kStages * (int)sizeof(StageMeta);
   static constexpr int n_bars = 2 * kStages + 5;
   static constexpr int off_misc = off_bar + n_bars * 8;
   static constexpr int total = off_misc + 64;
-  // CUDA-core path scratch (inside the Q region, unused by that path)
-  static constexpr int off_ccq = off_q;                              // fp32 [7][128]
+  // CUDA-core path scratch (inside the P region, unused by that path)
+  static constexpr int off_ccq = off_p;                              // fp32 [7][128]
   static constexpr int off_merge = off_ccq + kCcRows * kD * 4;       // fp32 [4][8][132]
   static constexpr int off_ps = off_merge + kCcW * 8 * kPStride * 4;  // fp32 [4][8][16] / [4][32][2]
 };
 static_assert(Smem::off_ps + kCcW * 8 * 16 * 4 <= Smem::off_x, "CUDA-core scratch overflow");
-static_assert(kTcSplitRows * kD * 4 <= 2 * Smem::kQHalf, "O exchange overflow");
-static_assert(Smem::off_q % 1024 == 0, "swizzle atoms of the Q tile");
+static_assert(kTcRows / 2 * kD * 4 <= 2 * Smem::kPHalf, "O exchange overflow");
+static_assert(Smem::off_p % 1024 == 0, "swizzle atoms of the P tile");
 static_assert(Smem::off_bar % 8 == 0, "mbarrier alignment");
 static_assert(Smem::total <= 227 * 1024, "shared memory");
 
@@ -755,18 +770,26 @@ __device__ __forceinline__ void zero_tail(const CompCtx &X, int s, int page0, in
 // eight compute warps.  Warps w and w + 4 reach the same TMEM lanes
 // 32 (w % 4) .. 32 (w % 4) + 31, so every lane has two threads.
 // A tile of at most 128 / F rows (F = 4, 2 or 1) is repeated F times over the
-// lanes: lane t holds row t mod (128 / F) and owns keys [128 k / F,
-// 128 (k + 1) / F) of every chunk, k = t / (128 / F), which its two threads
-// split.  Every SM sub-partition thus has work however few rows the tile
-// has, and a thread's share of a chunk is 64 / F keys.
+// lanes (its Q is written F times): lane t holds row t mod (128 / F) and owns
+// keys [128 k / F, 128 (k + 1) / F) of every chunk, k = t / (128 / F), which
+// its two threads split.  Every SM sub-partition thus has softmax work
+// however few rows the tile has, and a thread's share of a chunk is 64 / F
+// keys.
 // P reaches the tensor cores as three bf16 terms (its upper 16 bits, the
 // truncated residual and what is left of it, rounded), so P V sees each
-// probability to within 2^-25 of itself.  The terms are A operands in TMEM:
-// the first two overwrite the chunk's own S columns, the third goes to the
-// columns of the S buffer's parity at 384.  A lane's A row holds the terms of
-// its own keys and zeros for the other copies' keys, so P V (three MMAs per 16
-// keys, one per term) leaves in O row t the product over lane t's keys, and
-// the finalize adds the copies of a row.
+// probability to within 2^-25 of itself.  Where the terms go:
+//   F = 4: all three to the shared-memory P operand, term j of row r in
+//     operand row 32 j + r (rows 96..127 are not used): one MMA per 16 keys
+//     leaves the three terms' products in O lanes r, 32 + r and 64 + r;
+//   F = 2: terms 1 and 2 to operand rows r and 64 + r, the third to the
+//     lane's TMEM columns at kColT3 (the other copy's keys there are zeros,
+//     written once per item): two MMAs per 16 keys, O lanes r and 64 + r;
+//   F = 1: terms 1 and 2 overwrite the chunk's own S columns, the third goes
+//     to the columns of the S buffer's parity at 384: three MMAs per 16 keys,
+//     every A operand read from TMEM.  Its Q tile is in shared memory.
+// Terms bound for the P operand or kColT3 are written only once the previous
+// chunk's P V, their last reader, has completed: the first 16-key step's
+// terms wait in registers for it, later steps are stored as they are made.
 // Every chunk's P V lands in a fresh O (its first MMA overwrites O), and each
 // thread adds its 64 output dimensions of it into fp32 registers with
 // round-to-nearest adds.  The tensor core's accumulator does not round to
@@ -787,19 +810,21 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
   const Bars &B = X.B;
   const int lb = X.warp & 3;                        // lane block of this warp
   const int second = X.warp >> 2;                   // which of the lane's two threads
-  const int t = lb * 32 + X.lane;                   // TMEM lane (and operand row)
+  const int t = lb * 32 + X.lane;                   // TMEM lane
   const int copy = t / kRep;
   const int row = t % kRep;                         // tile row
   const int kown = copy * (kStageKeys / F);         // first key the lane owns
   const int k0 = kown + second * kKT;               // first key of this thread
-  const int kk_lo = kown / 16, kk_hi = kk_lo + 8 / F;  // the lane's 16-key steps
   const bool real = row < I.rows;
+  // F = 4 leaves O lanes 96..127 unused (the P operand's rows 96..127 are
+  // not written); their threads take no O.
+  const bool takes_o = F != 4 || t < 3 * kRep;
   const uint32_t tl = X.tmem + ((uint32_t)(lb * 32) << 16);
   const int lim = g.L - g.ql + (I.rb * kTcRows + row) / g.G;  // last key this row sees
   const int lim_all = g.L - g.ql;                             // every row sees up to here
   const float sl2 = p.scale_log2;
   float *xbuf = reinterpret_cast<float *>(X.smem + Smem::off_x);  // [2][2][128]
-  uint8_t *qs = X.smem + Smem::off_q;
+  uint8_t *ps = X.smem + Smem::off_p;
   float m_used = -INFINITY;  // maximum the exponentials are taken against (log2 units)
   float l_run = 0.f;         // this thread's share of the row sum
   float acc[64];             // output dims 64 second .. of this lane's O, summed over chunks
@@ -811,34 +836,26 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
   auto wait_pv_done = [&](uint32_t k) -> bool { return wait_or_abort(X, B.p_free, k & 1); };
   // acc = (acc + this thread's dims of O) * alpha
   auto take_o = [&](float alpha) {
+    if (!takes_o) return;
     const bool scaled = __any_sync(0xffffffffu, alpha != 1.f);
+    uint32_t r[2][32];
+    tc_ld_32x32b_x32(tl + kColO + 64 * second, r[0]);
+    tc_ld_32x32b_x32(tl + kColO + 64 * second + 32, r[1]);
+    tc_wait_ld();
+    if (scaled) {
 #pragma unroll
-    for (int q = 0; q < 2; ++q) {
-      uint32_t r[32];
-      tc_ld_32x32b_x32(tl + kColO + 64 * second + 32 * q, r);
-      tc_wait_ld();
-      if (scaled) {
+      for (int e = 0; e < 64; ++e) acc[e] = (acc[e] + __uint_as_float(r[e >> 5][e & 31])) * alpha;
+    } else {
 #pragma unroll
-        for (int e = 0; e < 32; ++e)
-          acc[32 * q + e] = (acc[32 * q + e] + __uint_as_float(r[e])) * alpha;
-      } else {
-#pragma unroll
-        for (int e = 0; e < 32; ++e) acc[32 * q + e] += __uint_as_float(r[e]);
-      }
+      for (int e = 0; e < 64; ++e) acc[e] += __uint_as_float(r[e >> 5][e & 31]);
     }
   };
-  // zeros in n TMEM columns from `col` of this lane (n a multiple of 8)
-  auto zero_cols = [&](uint32_t col, int n) {
-    const uint32_t z32[32] = {};
-    const uint32_t z16[16] = {};
-    const uint32_t z8[8] = {};
-    for (; n >= 32; n -= 32, col += 32) tc_st_32x32b_x32(tl + col, z32);
-    if (n >= 16) {
-      tc_st_32x32b_x16(tl + col, z16);
-      n -= 16;
-      col += 16;
-    }
-    if (n >= 8) tc_st_32x32b_x8(tl + col, z8);
+  // 16 keys (8 bf16 pairs) of one term into P operand row `ar`, from key kb
+  auto store_p = [&](int ar, int kb, const uint32_t (&v)[8]) {
+    uint8_t *h = ps + (kb >> 6) * Smem::kPHalf;
+    const int j = (kb & 63) >> 3;
+    *reinterpret_cast<uint4 *>(h + sw128(ar, j)) = make_uint4(v[0], v[1], v[2], v[3]);
+    *reinterpret_cast<uint4 *>(h + sw128(ar, j + 1)) = make_uint4(v[4], v[5], v[6], v[7]);
   };
 
   for (bool first = true;; first = false) {
@@ -847,21 +864,42 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
     const StageMeta M = X.meta[s];
     zero_tail(X, s, M.page0, g.L, kCW * 32, 1);
     if (first) {
-      // The Q region is the CUDA-core path's scratch: after a CUDA-core item,
-      // warps kCcW.. get here while the first warps may still be using it.
-      named_bar_sync(1, kCW * 32);
-      // Q: this thread's half of the lane's row (dims 64 second ..) into
-      // operand row t of the swizzled Q tile (zeros past the rows)
       const uint4 *src =
           reinterpret_cast<const uint4 *>(q_row(g, I, I.rb * kTcRows + row) + 64 * second);
-      uint8_t *qh = qs + second * Smem::kQHalf;
+      if (F == 1) {
+        // The shared-memory region is the CUDA-core path's scratch: after a
+        // CUDA-core item, warps kCcW.. get here while the first warps may
+        // still be using it.
+        named_bar_sync(1, kCW * 32);
+        // Q: this thread's half of the lane's row (dims 64 second ..) into
+        // operand row t of the swizzled Q tile
+        uint8_t *qh = ps + second * Smem::kPHalf;
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        uint4 v = make_uint4(0, 0, 0, 0);
-        if (real) v = __ldg(src + j);
-        *reinterpret_cast<uint4 *>(qh + sw128(t, j)) = v;
+        for (int j = 0; j < 8; ++j)
+          *reinterpret_cast<uint4 *>(qh + sw128(t, j)) = real ? __ldg(src + j) : make_uint4(0, 0, 0, 0);
+        fence_proxy_async_smem();
+      } else {
+        // Q: this thread's half of the lane's row (dims 64 second ..) as 32
+        // TMEM columns of bf16 pairs (zeros past the rows)
+        uint32_t qw[32];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          uint4 v = make_uint4(0, 0, 0, 0);
+          if (real) v = __ldg(src + j);
+          qw[4 * j + 0] = v.x;
+          qw[4 * j + 1] = v.y;
+          qw[4 * j + 2] = v.z;
+          qw[4 * j + 3] = v.w;
+        }
+        tc_st_32x32b_x32(tl + kColQ + 32 * second, qw);
+        if (F == 2 && second == 0) {
+          // zeros in the third-term columns of the other copy's keys
+          const uint32_t z[32] = {};
+          tc_st_32x32b_x32(tl + t3_col(copy == 0 ? 4 : 0), z);
+        }
+        tc_wait_st();
+        tc_fence_before();
       }
-      fence_proxy_async_smem();
       __syncwarp();
       if (X.lane == 0) mbar_arrive(B.q_ready);
     }
@@ -886,29 +924,31 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
         }
       }
     };
-    // the chunk maximum over this thread's keys, then over the row's threads
+    // this thread's S values, then the chunk maximum over its keys and over
+    // the row's threads.  Tiles repeated over the lanes keep their (16 or 32)
+    // values in registers, loaded at once; 128-row tiles read their 64 again
+    // for the exponentials, 16 at a time.
+    constexpr int kKeep = F == 1 ? 1 : kSteps;
+    uint32_t sv[kKeep][16];
     float mc = -INFINITY;
+    if (F != 1) {
+#pragma unroll
+      for (int q = 0; q < kKeep; ++q) tc_ld_32x32b_x16(tl + col_s(b) + k0 + 16 * q, sv[q]);
+      tc_wait_ld();
+    }
 #pragma unroll
     for (int q = 0; q < kSteps; ++q) {
-      uint32_t sr[16];
-      tc_ld_32x32b_x16(tl + col_s(b) + k0 + 16 * q, sr);
-      tc_wait_ld();
+      uint32_t(&sr)[16] = sv[F == 1 ? 0 : q];
+      if (F == 1) {
+        tc_ld_32x32b_x16(tl + col_s(b) + k0 + 16 * q, sr);
+        tc_wait_ld();
+      }
       mask(sr, k0 + 16 * q);
 #pragma unroll
       for (int e = 0; e < 16; ++e) mc = fmaxf(mc, __uint_as_float(sr[e]));
     }
     float *xm = xbuf + (c & 1) * (2 * kTcRows);
     xm[second * kTcRows + t] = mc;
-    // zeros for the other copies' keys: the first thread of the lane takes
-    // the steps below the lane's, the second those above (no thread of this
-    // lane reads those S columns)
-    if (second == 0) {
-      zero_cols(col_s(b), 16 * kk_lo);
-      zero_cols(t3_col(b, 0), 8 * kk_lo);
-    } else {
-      zero_cols(col_s(b) + 16 * kk_hi, 16 * (8 - kk_hi));
-      zero_cols(t3_col(b, kk_hi), 8 * (8 - kk_hi));
-    }
     named_bar_sync(1, kCW * 32);
 #pragma unroll
     for (int j = 0; j < F; ++j)
@@ -933,16 +973,25 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
     // subtractions are exact, so |p - hi - lo - lo2| <= 2^-25 p.  The scaling,
     // residuals and row sum run on packed fp32 pairs.
     unsigned long long lsum2 = 0ull;  // {0.f, 0.f}
+    // the previous chunk's P V has read the P operand and the third-term
+    // columns once this returns
+    auto wait_prev = [&]() -> bool {
+      if (!wait_pv_done(c - 1)) return false;
+      tc_fence_after();
+      return true;
+    };
     {
       const unsigned long long sl2x2 = f2_pack(sl2, sl2), moffx2 = f2_pack(moff, moff);
       auto upper = [](float x) { return __uint_as_float(__float_as_uint(x) & 0xffff0000u); };
 #pragma unroll
       for (int q = 0; q < kSteps; ++q) {
-        uint32_t sr[16];
-        tc_ld_32x32b_x16(tl + col_s(b) + k0 + 16 * q, sr);
-        tc_wait_ld();
-        mask(sr, k0 + 16 * q);
-        uint32_t hi[8], lo[8], lo2[8];
+        uint32_t(&sr)[16] = sv[F == 1 ? 0 : q];
+        if (F == 1) {
+          tc_ld_32x32b_x16(tl + col_s(b) + k0 + 16 * q, sr);
+          tc_wait_ld();
+          mask(sr, k0 + 16 * q);
+        }
+        uint32_t th[8], tlo[8], t3[8];
 #pragma unroll
         for (int e = 0; e < 16; e += 2) {
           float x0, x1;
@@ -951,26 +1000,36 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
                     x0, x1);
           const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
           const unsigned long long pp = f2_pack(p0, p1);
-          float l0, l1, t0, t1;
+          float l0, l1, r0, r1;
           f2_unpack(f2_sub(pp, f2_pack(upper(p0), upper(p1))), l0, l1);
-          f2_unpack(f2_sub(f2_pack(l0, l1), f2_pack(upper(l0), upper(l1))), t0, t1);
-          hi[e >> 1] = pack_bf16x2_trunc(p0, p1);
-          lo[e >> 1] = pack_bf16x2_trunc(l0, l1);
-          lo2[e >> 1] = pack_bf16x2(t0, t1);
+          f2_unpack(f2_sub(f2_pack(l0, l1), f2_pack(upper(l0), upper(l1))), r0, r1);
+          th[e >> 1] = pack_bf16x2_trunc(p0, p1);
+          tlo[e >> 1] = pack_bf16x2_trunc(l0, l1);
+          t3[e >> 1] = pack_bf16x2(r0, r1);
           lsum2 = f2_add(lsum2, pp);
         }
-        // the first two terms overwrite the S columns of these 16 keys, which
-        // this thread has just read (and no other thread reads)
-        const int kk = (k0 >> 4) + q;
-        tc_st_32x32b_x8(tl + col_s(b) + p_col(kk, 1), hi);
-        tc_st_32x32b_x8(tl + col_s(b) + p_col(kk, 2), lo);
-        tc_st_32x32b_x8(tl + t3_col(b, kk), lo2);
+        const int kb = k0 + 16 * q;
+        if (F == 1) {
+          // the first two terms overwrite the S columns of these 16 keys,
+          // which this thread has just read (and no other thread reads); the
+          // third goes to the columns of this S buffer's parity, last read
+          // by the P V of chunk c - 2
+          tc_st_32x32b_x8(tl + col_s(b) + p_col(kb >> 4, 1), th);
+          tc_st_32x32b_x8(tl + col_s(b) + p_col(kb >> 4, 2), tlo);
+          tc_st_32x32b_x8(tl + t3_col_full(b, kb >> 4), t3);
+        } else {
+          if (q == 0 && !wait_prev()) return false;
+          store_p(row, kb, th);
+          store_p(kRep + row, kb, tlo);
+          if (F == 4) store_p(2 * kRep + row, kb, t3);
+          else tc_st_32x32b_x8(tl + t3_col(kb >> 4), t3);
+        }
       }
     }
-    // the previous chunk's product into the registers (before this chunk's
-    // product overwrites O)
-    if (!wait_pv_done(c - 1)) return false;
-    tc_fence_after();
+    // then the previous chunk's product into the registers (before this
+    // chunk's product overwrites O)
+    if (F == 1 && !wait_prev()) return false;
+    if (F != 1) fence_proxy_async_smem();
     if (!first) take_o(alpha);
     {
       float a0, a1;
@@ -994,9 +1053,9 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
   // have all passed chunk c - 1's barrier
   float *xl = xbuf + (c & 1) * (2 * kTcRows);
   xl[second * kTcRows + t] = l_run;
-  // O sums travel through the Q region (free: the item's last Q K^T has
+  // O sums travel through the P region (free: the item's last P V has
   // completed); 16-byte chunk j of exchange row r sits at chunk j ^ (r & 7)
-  float *ox = reinterpret_cast<float *>(qs);  // [64][128] fp32
+  float *ox = reinterpret_cast<float *>(ps);  // [64][128] fp32
   auto ox_at = [&](int r, int j) { return reinterpret_cast<float4 *>(ox + r * kD) + (j ^ (r & 7)); };
 #pragma unroll
   for (int step = kTcRows / 2; step >= kRep; step >>= 1) {
@@ -1624,15 +1683,16 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
   if (warp == kMmaWarp) {
     // ------------------------------ MMA issuer -----------------------------
     // Fixed order per tensor chunk j: Q K^T of j into S buffer j & 1, then
-    // P V of chunk j-1 (once its P is written); an item's last chunk also
-    // issues its own P V, so no product waits on the next item's stages.
+    // P V of chunk j-1 (once its P is written): the softmax of j, which waits
+    // for Q K^T, is the longer path.  An item's last chunk also issues its own
+    // P V, so no product waits on the next item's stages.
     constexpr uint32_t idesc_s = idesc_bf16_f32(kTcRows, kStageKeys, 0);
     constexpr uint32_t idesc_o = idesc_bf16_f32(kTcRows, kD, 1);
-    const uint32_t qa = smem_u32(smem + Smem::off_q);
+    const uint32_t pa = smem_u32(smem + Smem::off_p);
     uint32_t it = 0, c = 0, nq = 0;
     bool ok = true, pend = false;
     uint32_t pc = 0;  // pending chunk
-    int pstage = 0;
+    int pstage = 0, ppath = 0;
     auto mwait = [&](uint64_t *bar, uint32_t par) -> bool {
       if (mbar_wait_bounded(bar, par)) return true;
       ok = false;
@@ -1644,17 +1704,33 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
       if (!mwait(B.p_full, pc & 1)) return false;
       tc_fence_after();
       if (lane == 0) {
-        const uint32_t va = smem_u32(stage_v(smem, pstage));
+        // V keys 16kk.. as an MN-major operand: 64-dim halves 1 KB apart,
+        // 8-key groups 2 KB; the descriptor of step kk + 1 is that of kk with
+        // its start address 4 KB further
+        uint64_t bd = sdesc_sw128(smem_u32(stage_v(smem, pstage)), kAtomBytes, kGroupBytes);
+        constexpr uint64_t kVStep = (2 * kGroupBytes) >> 4;
+        if (ppath == kPathTc1) {
+          // the three terms of P: two in the chunk's S buffer, the third in
+          // the columns of its parity
+          const uint32_t pt = tmem + col_s(pc & 1), p3 = tmem + t3_col_full(pc & 1, 0);
 #pragma unroll
-        for (int kk = 0; kk < kStageKeys / 16; ++kk) {
-          // V keys 16kk.. as an MN-major operand: 64-dim halves 1 KB apart, 8-key groups 2 KB
-          const uint64_t bd = sdesc_sw128(va + kk * 2 * kGroupBytes, kAtomBytes, kGroupBytes);
-          // the three terms of P: the chunk's S buffer and the third term's
-          // columns of that buffer's parity
-          const uint32_t pt = tmem + col_s(pc & 1);
-          tc_mma_bf16_ta(tmem + kColO, pt + p_col(kk, 1), bd, idesc_o, kk == 0 ? 0u : 1u);
-          tc_mma_bf16_ta(tmem + kColO, pt + p_col(kk, 2), bd, idesc_o, 1u);
-          tc_mma_bf16_ta(tmem + kColO, tmem + t3_col(pc & 1, kk), bd, idesc_o, 1u);
+          for (int kk = 0; kk < kStageKeys / 16; ++kk, bd += kVStep) {
+            tc_mma_bf16_ta(tmem + kColO, pt + p_col(kk, 1), bd, idesc_o, kk == 0 ? 0u : 1u);
+            tc_mma_bf16_ta(tmem + kColO, pt + p_col(kk, 2), bd, idesc_o, 1u);
+            tc_mma_bf16_ta(tmem + kColO, p3 + 8 * kk, bd, idesc_o, 1u);
+          }
+        } else {
+          // the stacked terms in the shared-memory P operand (K-major:
+          // 64-key halves 16 KB apart, 8-row groups 1 KB), and for tiles of
+          // up to 64 rows the third term from TMEM
+          const uint64_t ad0 = sdesc_sw128(pa, 16, 1024);
+          const bool t3 = ppath == kPathTc2;
+#pragma unroll
+          for (int kk = 0; kk < kStageKeys / 16; ++kk, bd += kVStep) {
+            const uint64_t ad = sdesc_advance(ad0, (kk >> 2) * Smem::kPHalf + (kk & 3) * 32);
+            tc_mma_bf16(tmem + kColO, ad, bd, idesc_o, kk == 0 ? 0u : 1u);
+            if (t3) tc_mma_bf16_ta(tmem + kColO, tmem + t3_col(kk), bd, idesc_o, 1u);
+          }
         }
         tc_commit(B.p_free);
         tc_commit(&B.empty[pstage]);
@@ -1682,20 +1758,32 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
         ++it;
         continue;
       }
-      if (flags & 1) {  // a new tensor item: its Q tile must be in shared memory
+      if (flags & 1) {  // a new tensor item: its Q tile must be written
         if (!mwait(B.q_ready, nq & 1)) break;
         ++nq;
       }
       tc_fence_after();
       if (lane == 0) {
-        const uint32_t ka = smem_u32(stage_k(smem, s));
+        // K dims 16kk.. (K-major: 64-dim halves 1 KB apart, 8-key groups 2 KB)
+        const uint64_t bd0 = sdesc_sw128(smem_u32(stage_k(smem, s)), 16, kGroupBytes);
+        const uint32_t sd = tmem + col_s(c & 1);
+        if (path == kPathTc1) {
+          // Q dims 16kk.. in shared memory (K-major: 64-dim halves 16 KB
+          // apart, 8-row groups 1 KB)
+          const uint64_t ad0 = sdesc_sw128(pa, 16, 1024);
 #pragma unroll
-        for (int kk = 0; kk < kD / 16; ++kk) {
-          // Q dims 16kk.. (K-major: 64-dim halves 16 KB apart, 8-row groups 1 KB)
-          const uint64_t ad = sdesc_sw128(qa + (kk >> 2) * Smem::kQHalf + (kk & 3) * 32, 16, 1024);
-          const uint64_t bd =
-              sdesc_sw128(ka + (kk >> 2) * kAtomBytes + (kk & 3) * 32, 16, kGroupBytes);
-          tc_mma_bf16(tmem + col_s(c & 1), ad, bd, idesc_s, kk > 0);
+          for (int kk = 0; kk < kD / 16; ++kk) {
+            const uint64_t bd = bd0 + (uint64_t)(((kk >> 2) * kAtomBytes + (kk & 3) * 32) >> 4);
+            const uint64_t ad = sdesc_advance(ad0, (kk >> 2) * Smem::kPHalf + (kk & 3) * 32);
+            tc_mma_bf16(sd, ad, bd, idesc_s, kk > 0);
+          }
+        } else {
+          // Q dims 16kk.. are TMEM columns 8kk.. of the Q tile
+#pragma unroll
+          for (int kk = 0; kk < kD / 16; ++kk) {
+            const uint64_t bd = bd0 + (uint64_t)(((kk >> 2) * kAtomBytes + (kk & 3) * 32) >> 4);
+            tc_mma_bf16_ta(sd, tmem + kColQ + 8 * kk, bd, idesc_s, kk > 0);
+          }
         }
         tc_commit(&B.s_full[c & 1]);
       }
@@ -1704,6 +1792,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
       pend = true;
       pc = c;
       pstage = s;
+      ppath = path;
       ++c;
       ++it;
       if ((flags & 2) && !issue_pv()) break;
@@ -1735,8 +1824,8 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
     bool ok;
     if (I.path != kPathCc) {
       // copies of the tile's rows over the 128 lanes: 4 (<= 32 rows), 2 (<= 64) or 1
-      if (I.rows <= kTcRows / 4) ok = tc_item<4>(p, X, I, it, c);
-      else if (I.rows <= kTcRows / 2) ok = tc_item<2>(p, X, I, it, c);
+      if (I.path == kPathTc4) ok = tc_item<4>(p, X, I, it, c);
+      else if (I.path == kPathTc2) ok = tc_item<2>(p, X, I, it, c);
       else ok = tc_item<1>(p, X, I, it, c);
     } else if (warp < kCcW) {
       // GQA-2 decode (two rows) has its own layout; other sizes take the

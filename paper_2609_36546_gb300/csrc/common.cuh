@@ -264,6 +264,16 @@ IPD_DEVINL uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo_bytes, uint32_t sbo
   return d;
 }
 
+// A shared-memory descriptor `off_bytes` further on (start address field
+// only; no carry leaves it for addresses inside shared memory).  An opaque
+// add, so that the compiler recomputes it where it is used instead of keeping
+// every step's descriptor of a fixed buffer live in registers.
+IPD_DEVINL uint64_t sdesc_advance(uint64_t d, uint32_t off_bytes) {
+  uint64_t r;
+  asm volatile("add.u64 %0, %1, %2;" : "=l"(r) : "l"(d), "l"((uint64_t)(off_bytes >> 4)));
+  return r;
+}
+
 // Instruction descriptor of tcgen05.mma kind::f16: bf16 A and B, fp32 D,
 // A K-major, B K-major (b_mn_major = 0) or MN-major (1), shape M x N.
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, int b_mn_major) {
