@@ -38,10 +38,11 @@
 //     per warp and stage, two lanes per key.  From four rows up the tensor
 //     path is faster even with most of its tile empty: at 4-6 rows the
 //     CUDA-core FMAs limit the stream.
-// Warp roles: warps 0-7 compute, warp 8 streams KV pages, warp 9 issues the
-// tensor-core instructions in a fixed order (Q K^T of chunk j, then P V of
-// chunk j-1); warps 10 and 11 only complete the third warpgroup, whose
-// registers go to the compute warps.
+// Warp roles: warps 0-7 compute, warp 8 streams KV pages, warp 9 issues Q K^T
+// and warp 10 P V; warp 11 only completes the third warpgroup, whose
+// registers go to the compute warps.  One thread issuing a burst of MMAs
+// stalls about 100 cycles per instruction, more than an MMA takes to run, so
+// the two products of a chunk are issued by two warps.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
@@ -78,7 +79,8 @@ constexpr int kCcRows = kTcMinRows - 1;           // CUDA-core tasks have fewer 
 constexpr int kCW = 8;                            // compute warps (two per TMEM lane block)
 constexpr int kCcW = 4;                           // of them, the CUDA-core path's warps
 constexpr int kProducerWarp = kCW;
-constexpr int kMmaWarp = kCW + 1;
+constexpr int kMmaWarp = kCW + 1;                 // issues Q K^T (and owns the TMEM allocation)
+constexpr int kPvWarp = kCW + 2;                  // issues P V
 constexpr int kThreads = (kCW + 4) * 32;           // three warpgroups; warps 10 and 11 exit early
 // Register split: the block is launched with 168 registers a thread (three
 // warps share each SM sub-partition's 16K registers); the third warpgroup
@@ -645,7 +647,7 @@ struct Smem {
   static constexpr int off_x = off_p + 2 * kPHalf;                 // row-max / row-sum exchange [2][256]
   static constexpr int off_meta = off_x + 2 * 256 * 4;
   static constexpr int off_bar = off_meta + kStages * (int)sizeof(StageMeta);
-  static constexpr int n_bars = 2 * kStages + 5;
+  static constexpr int n_bars = 2 * kStages + 7;
   static constexpr int off_misc = off_bar + n_bars * 8;
   static constexpr int total = off_misc + 64;
   // CUDA-core path scratch (inside the P region, unused by that path)
@@ -665,6 +667,7 @@ struct Bars {
   uint64_t *s_full;        // S = Q K^T landed, per S buffer (one phase per use)
   uint64_t *p_full;        // P of a chunk written (one phase per chunk)
   uint64_t *p_free;        // P V product of a chunk done: P read, O written (one phase per chunk)
+  uint64_t *s_free;        // P V of a chunk done, per S buffer: the buffer may take the next Q K^T
 };
 
 __device__ __forceinline__ Bars bars(uint8_t *smem) {
@@ -676,6 +679,7 @@ __device__ __forceinline__ Bars bars(uint8_t *smem) {
   r.s_full = r.q_ready + 1;
   r.p_full = r.s_full + 2;
   r.p_free = r.p_full + 1;
+  r.s_free = r.p_free + 1;
   return r;
 }
 
@@ -1529,12 +1533,13 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&B.full[s], 1);
-      mbar_init(&B.empty[s], 1 + kCW);  // the MMA warp and every compute warp
+      mbar_init(&B.empty[s], 1 + kCW);  // the P V issuer and every compute warp
     }
     mbar_init(B.q_ready, kCW);
     for (int i = 0; i < 2; ++i) mbar_init(&B.s_full[i], 1);
     mbar_init(B.p_full, kCW);
     mbar_init(B.p_free, 1);
+    for (int i = 0; i < 2; ++i) mbar_init(&B.s_free[i], 1);
     misc[1] = 0;
     fence_mbar_init();
   }
@@ -1680,64 +1685,22 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
     return;
   }
 
-  if (warp == kMmaWarp) {
-    // ------------------------------ MMA issuer -----------------------------
-    // Fixed order per tensor chunk j: Q K^T of j into S buffer j & 1, then
-    // P V of chunk j-1 (once its P is written): the softmax of j, which waits
-    // for Q K^T, is the longer path.  An item's last chunk also issues its own
-    // P V, so no product waits on the next item's stages.
+  if (warp == kMmaWarp || warp == kPvWarp) {
+    // ----------------------------- MMA issuers ------------------------------
+    // Both issuers walk the same stages.  Warp kMmaWarp issues Q K^T of
+    // tensor chunk j into S buffer j & 1 as soon as its stage has landed (and
+    // the buffer's previous chunk, j - 2, has had its P V); warp kPvWarp
+    // issues P V of chunk j once its P is written, and releases the stage.
     constexpr uint32_t idesc_s = idesc_bf16_f32(kTcRows, kStageKeys, 0);
     constexpr uint32_t idesc_o = idesc_bf16_f32(kTcRows, kD, 1);
     const uint32_t pa = smem_u32(smem + Smem::off_p);
+    const bool is_qk = warp == kMmaWarp;
     uint32_t it = 0, c = 0, nq = 0;
-    bool ok = true, pend = false;
-    uint32_t pc = 0;  // pending chunk
-    int pstage = 0, ppath = 0;
+    bool ok = true;
     auto mwait = [&](uint64_t *bar, uint32_t par) -> bool {
       if (mbar_wait_bounded(bar, par)) return true;
       ok = false;
       return false;
-    };
-    // O = P V of the pending chunk (every chunk's product starts a fresh O;
-    // the compute warps sum the chunks in registers)
-    auto issue_pv = [&]() -> bool {
-      if (!mwait(B.p_full, pc & 1)) return false;
-      tc_fence_after();
-      if (lane == 0) {
-        // V keys 16kk.. as an MN-major operand: 64-dim halves 1 KB apart,
-        // 8-key groups 2 KB; the descriptor of step kk + 1 is that of kk with
-        // its start address 4 KB further
-        uint64_t bd = sdesc_sw128(smem_u32(stage_v(smem, pstage)), kAtomBytes, kGroupBytes);
-        constexpr uint64_t kVStep = (2 * kGroupBytes) >> 4;
-        if (ppath == kPathTc1) {
-          // the three terms of P: two in the chunk's S buffer, the third in
-          // the columns of its parity
-          const uint32_t pt = tmem + col_s(pc & 1), p3 = tmem + t3_col_full(pc & 1, 0);
-#pragma unroll
-          for (int kk = 0; kk < kStageKeys / 16; ++kk, bd += kVStep) {
-            tc_mma_bf16_ta(tmem + kColO, pt + p_col(kk, 1), bd, idesc_o, kk == 0 ? 0u : 1u);
-            tc_mma_bf16_ta(tmem + kColO, pt + p_col(kk, 2), bd, idesc_o, 1u);
-            tc_mma_bf16_ta(tmem + kColO, p3 + 8 * kk, bd, idesc_o, 1u);
-          }
-        } else {
-          // the stacked terms in the shared-memory P operand (K-major:
-          // 64-key halves 16 KB apart, 8-row groups 1 KB), and for tiles of
-          // up to 64 rows the third term from TMEM
-          const uint64_t ad0 = sdesc_sw128(pa, 16, 1024);
-          const bool t3 = ppath == kPathTc2;
-#pragma unroll
-          for (int kk = 0; kk < kStageKeys / 16; ++kk, bd += kVStep) {
-            const uint64_t ad = sdesc_advance(ad0, (kk >> 2) * Smem::kPHalf + (kk & 3) * 32);
-            tc_mma_bf16(tmem + kColO, ad, bd, idesc_o, kk == 0 ? 0u : 1u);
-            if (t3) tc_mma_bf16_ta(tmem + kColO, tmem + t3_col(kk), bd, idesc_o, 1u);
-          }
-        }
-        tc_commit(B.p_free);
-        tc_commit(&B.empty[pstage]);
-      }
-      __syncwarp();
-      pend = false;
-      return true;
     };
     for (;;) {
       const int s = it % kStages;
@@ -1753,58 +1716,95 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
       path = __shfl_sync(0xffffffffu, path, 0);
       if (item < 0 || *(volatile uint32_t *)&misc[1]) break;
       if (path == kPathCc) {
-        if (lane == 0) mbar_arrive(&B.empty[s]);
+        if (!is_qk && lane == 0) mbar_arrive(&B.empty[s]);
         __syncwarp();
         ++it;
         continue;
       }
-      if (flags & 1) {  // a new tensor item: its Q tile must be written
-        if (!mwait(B.q_ready, nq & 1)) break;
-        ++nq;
-      }
-      tc_fence_after();
-      if (lane == 0) {
-        // K dims 16kk.. (K-major: 64-dim halves 1 KB apart, 8-key groups 2 KB)
-        const uint64_t bd0 = sdesc_sw128(smem_u32(stage_k(smem, s)), 16, kGroupBytes);
-        const uint32_t sd = tmem + col_s(c & 1);
-        if (path == kPathTc1) {
-          // Q dims 16kk.. in shared memory (K-major: 64-dim halves 16 KB
-          // apart, 8-row groups 1 KB)
-          const uint64_t ad0 = sdesc_sw128(pa, 16, 1024);
-#pragma unroll
-          for (int kk = 0; kk < kD / 16; ++kk) {
-            const uint64_t bd = bd0 + (uint64_t)(((kk >> 2) * kAtomBytes + (kk & 3) * 32) >> 4);
-            const uint64_t ad = sdesc_advance(ad0, (kk >> 2) * Smem::kPHalf + (kk & 3) * 32);
-            tc_mma_bf16(sd, ad, bd, idesc_s, kk > 0);
-          }
-        } else {
-          // Q dims 16kk.. are TMEM columns 8kk.. of the Q tile
-#pragma unroll
-          for (int kk = 0; kk < kD / 16; ++kk) {
-            const uint64_t bd = bd0 + (uint64_t)(((kk >> 2) * kAtomBytes + (kk & 3) * 32) >> 4);
-            tc_mma_bf16_ta(sd, tmem + kColQ + 8 * kk, bd, idesc_s, kk > 0);
-          }
+      if (is_qk) {
+        if (flags & 1) {  // a new tensor item: its Q tile must be written
+          if (!mwait(B.q_ready, nq & 1)) break;
+          ++nq;
         }
-        tc_commit(&B.s_full[c & 1]);
+        // the S buffer's previous chunk has had its P V (which for 128-row
+        // tiles reads two terms of P from it)
+        if (c >= 2 && !mwait(&B.s_free[c & 1], ((c >> 1) - 1) & 1)) break;
+        tc_fence_after();
+        if (lane == 0) {
+          // K dims 16kk.. (K-major: 64-dim halves 1 KB apart, 8-key groups 2 KB)
+          const uint64_t bd0 = sdesc_sw128(smem_u32(stage_k(smem, s)), 16, kGroupBytes);
+          const uint32_t sd = tmem + col_s(c & 1);
+          if (path == kPathTc1) {
+            // Q dims 16kk.. in shared memory (K-major: 64-dim halves 16 KB
+            // apart, 8-row groups 1 KB)
+            const uint64_t ad0 = sdesc_sw128(pa, 16, 1024);
+#pragma unroll
+            for (int kk = 0; kk < kD / 16; ++kk) {
+              const uint64_t bd = bd0 + (uint64_t)(((kk >> 2) * kAtomBytes + (kk & 3) * 32) >> 4);
+              const uint64_t ad = sdesc_advance(ad0, (kk >> 2) * Smem::kPHalf + (kk & 3) * 32);
+              tc_mma_bf16(sd, ad, bd, idesc_s, kk > 0);
+            }
+          } else {
+            // Q dims 16kk.. are TMEM columns 8kk.. of the Q tile
+#pragma unroll
+            for (int kk = 0; kk < kD / 16; ++kk) {
+              const uint64_t bd = bd0 + (uint64_t)(((kk >> 2) * kAtomBytes + (kk & 3) * 32) >> 4);
+              tc_mma_bf16_ta(sd, tmem + kColQ + 8 * kk, bd, idesc_s, kk > 0);
+            }
+          }
+          tc_commit(&B.s_full[c & 1]);
+        }
+        __syncwarp();
+      } else {
+        if (!mwait(B.p_full, c & 1)) break;
+        tc_fence_after();
+        if (lane == 0) {
+          // V keys 16kk.. as an MN-major operand: 64-dim halves 1 KB apart,
+          // 8-key groups 2 KB; the descriptor of step kk + 1 is that of kk with
+          // its start address 4 KB further
+          uint64_t bd = sdesc_sw128(smem_u32(stage_v(smem, s)), kAtomBytes, kGroupBytes);
+          constexpr uint64_t kVStep = (2 * kGroupBytes) >> 4;
+          if (path == kPathTc1) {
+            // the three terms of P: two in the chunk's S buffer, the third in
+            // the columns of its parity
+            const uint32_t pt = tmem + col_s(c & 1), p3 = tmem + t3_col_full(c & 1, 0);
+#pragma unroll
+            for (int kk = 0; kk < kStageKeys / 16; ++kk, bd += kVStep) {
+              tc_mma_bf16_ta(tmem + kColO, pt + p_col(kk, 1), bd, idesc_o, kk == 0 ? 0u : 1u);
+              tc_mma_bf16_ta(tmem + kColO, pt + p_col(kk, 2), bd, idesc_o, 1u);
+              tc_mma_bf16_ta(tmem + kColO, p3 + 8 * kk, bd, idesc_o, 1u);
+            }
+          } else {
+            // the stacked terms in the shared-memory P operand (K-major:
+            // 64-key halves 16 KB apart, 8-row groups 1 KB), and for tiles of
+            // up to 64 rows the third term from TMEM
+            const uint64_t ad0 = sdesc_sw128(pa, 16, 1024);
+            const bool t3 = path == kPathTc2;
+#pragma unroll
+            for (int kk = 0; kk < kStageKeys / 16; ++kk, bd += kVStep) {
+              const uint64_t ad = sdesc_advance(ad0, (kk >> 2) * Smem::kPHalf + (kk & 3) * 32);
+              tc_mma_bf16(tmem + kColO, ad, bd, idesc_o, kk == 0 ? 0u : 1u);
+              if (t3) tc_mma_bf16_ta(tmem + kColO, tmem + t3_col(kk), bd, idesc_o, 1u);
+            }
+          }
+          tc_commit(B.p_free);
+          tc_commit(&B.s_free[c & 1]);
+          tc_commit(&B.empty[s]);
+        }
+        __syncwarp();
       }
-      __syncwarp();
-      if (pend && !issue_pv()) break;
-      pend = true;
-      pc = c;
-      pstage = s;
-      ppath = path;
       ++c;
       ++it;
-      if ((flags & 2) && !issue_pv()) break;
     }
     if (!ok) {
       ipd_set_error(&g_attn_err, IPD_DEVERR_WAIT);
       atomicExch(&misc[1], 1u);
     }
     // every tensor-core op and TMEM access is finished before TMEM is released
-    named_bar_sync(2, (kCW + 1) * 32);
+    tc_fence_before();
+    named_bar_sync(2, (kCW + 2) * 32);
     tc_fence_after();
-    tc_dealloc(tmem, kTmemCols);
+    if (is_qk) tc_dealloc(tmem, kTmemCols);
     return;
   }
 
@@ -1853,7 +1853,8 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
       named_bar_sync(1, kCW * 32);  // misc[2] is read before the next split item rewrites it
     }
   }
-  named_bar_sync(2, (kCW + 1) * 32);
+  tc_fence_before();
+  named_bar_sync(2, (kCW + 2) * 32);
 }
 
 // --------------------------------------------------------------------------
