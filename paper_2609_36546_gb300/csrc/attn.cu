@@ -38,11 +38,12 @@
 //     per warp and stage, two lanes per key.  From four rows up the tensor
 //     path is faster even with most of its tile empty: at 4-6 rows the
 //     CUDA-core FMAs limit the stream.
-// Warp roles: warps 0-7 compute, warp 8 streams KV pages, warp 9 issues Q K^T
-// and warp 10 P V; warp 11 only completes the third warpgroup, whose
-// registers go to the compute warps.  One thread issuing a burst of MMAs
-// stalls about 100 cycles per instruction, more than an MMA takes to run, so
-// the two products of a chunk are issued by two warps.
+// Warp roles: warps 0-7 compute, warp 8 streams the K pages of each stage and
+// warp 11 its V pages, warp 9 issues Q K^T and warp 10 P V.  One thread issuing
+// a burst of MMAs stalls about 100 cycles per instruction, more than an MMA
+// takes to run, so the two products of a chunk are issued by two warps; a
+// warp issuing a stage's 16 TMA boxes took about 2000 cycles, two thirds of
+// the stage's time at the HBM rate, so K and V boxes come from two warps.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
@@ -81,6 +82,7 @@ constexpr int kCcW = 4;                           // of them, the CUDA-core path
 constexpr int kProducerWarp = kCW;
 constexpr int kMmaWarp = kCW + 1;                 // issues Q K^T (and owns the TMEM allocation)
 constexpr int kPvWarp = kCW + 2;                  // issues P V
+constexpr int kVLoadWarp = kCW + 3;               // issues the V boxes of each stage
 constexpr int kThreads = (kCW + 4) * 32;           // three warpgroups; warps 10 and 11 exit early
 // Register split: the block is launched with 168 registers a thread (three
 // warps share each SM sub-partition's 16K registers); the third warpgroup
@@ -647,9 +649,12 @@ struct Smem {
   static constexpr int off_x = off_p + 2 * kPHalf;                 // row-max / row-sum exchange [2][256]
   static constexpr int off_meta = off_x + 2 * 256 * 4;
   static constexpr int off_bar = off_meta + kStages * (int)sizeof(StageMeta);
-  static constexpr int n_bars = 2 * kStages + 7;
+  static constexpr int n_bars = 3 * kStages + 7;
   static constexpr int off_misc = off_bar + n_bars * 8;
-  static constexpr int total = off_misc + 64;
+  // per stage, the V boxes' coordinates for the second producer warp: eight
+  // page slots and the V tensor map's index (-1: stop)
+  static constexpr int off_vjob = off_misc + 64;
+  static constexpr int total = off_vjob + kStages * 16 * 4;
   // CUDA-core path scratch (inside the P region, unused by that path)
   static constexpr int off_ccq = off_p;                              // fp32 [7][128]
   static constexpr int off_merge = off_ccq + kCcRows * kD * 4;       // fp32 [4][8][132]
@@ -668,6 +673,7 @@ struct Bars {
   uint64_t *p_full;        // P of a chunk written (one phase per chunk)
   uint64_t *p_free;        // P V product of a chunk done: P read, O written (one phase per chunk)
   uint64_t *s_free;        // P V of a chunk done, per S buffer: the buffer may take the next Q K^T
+  uint64_t *v_go;          // per stage: its V boxes may be issued (one phase per stage use)
 };
 
 __device__ __forceinline__ Bars bars(uint8_t *smem) {
@@ -680,6 +686,7 @@ __device__ __forceinline__ Bars bars(uint8_t *smem) {
   r.p_full = r.s_full + 2;
   r.p_free = r.p_full + 1;
   r.s_free = r.p_free + 1;
+  r.v_go = r.s_free + 2;
   return r;
 }
 
@@ -1540,6 +1547,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
     mbar_init(B.p_full, kCW);
     mbar_init(B.p_free, 1);
     for (int i = 0; i < 2; ++i) mbar_init(&B.s_free[i], 1);
+    for (int s = 0; s < kStages; ++s) mbar_init(&B.v_go[s], 1);
     misc[1] = 0;
     fence_mbar_init();
   }
@@ -1570,10 +1578,24 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
     const uint64_t policy = l2_policy_evict_first();
     uint32_t it = 0;
     bool aborted = false;
+    int *vjob = reinterpret_cast<int *>(smem + Smem::off_vjob);  // [kStages][16]
+    // the next item's index: the atomic is issued at one stage and its value
+    // taken at a later one, so that the producer does not wait for it
+    int claim_v = 0;
+    auto claim_issue = [&]() {
+      if (lane == 0) claim_v = atomicAdd(&p.ctrl[1], 1);
+    };
+    auto claim_take = [&]() -> int { return __shfl_sync(0xffffffffu, claim_v, 0); };
     auto claim = [&]() -> int {
-      int v = 0;
-      if (lane == 0) v = atomicAdd(&p.ctrl[1], 1);
-      return __shfl_sync(0xffffffffu, v, 0);
+      claim_issue();
+      return claim_take();
+    };
+    // hands stage s's V boxes (or a stop, tm < 0) to the V producer warp
+    auto post_v = [&](int s, int w, int tm) {
+      if (lane < kStagePages) vjob[16 * s + lane] = w;
+      if (lane == 0) vjob[16 * s + 8] = tm;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&B.v_go[s]);
     };
     // page id of page `page_lo + 32 * batch + lane`, or -1 past the item
     auto load_ids = [&](const Item &I, int batch) -> int {
@@ -1595,19 +1617,20 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
       Item In = I;
       const BatchDev &Bt = p.b[I.b];
       const void *tk = &p.tmap[2 * Bt.cache];
-      const void *tv = &p.tmap[2 * Bt.cache + 1];
       const int oob_w = (int)(Bt.num_pages * Bt.hkv * 2);  // a box here reads zeros
       const int npages = I.page_hi - I.page_lo;
       const int nst = (npages + kStagePages - 1) / kStagePages;
       int ids_next = (npages > 32) ? load_ids(I, 1) : -1;
       int ids_item_next = -1;
       const int st_claim = late_claim ? max(0, nst - 4) : 0;
+      const int st_take = min(nst - 1, st_claim + 1);
       for (int st = 0; st < nst; ++st) {
-        if (st == st_claim) {
-          nxt = claim();
+        if (st == st_claim) claim_issue();
+        if (st == st_take) {
+          nxt = claim_take();
           if (nxt < n_items) In = p.items[nxt];  // consumed at the next item
         }
-        if (st == max(st_claim, nst - 2) && nxt < n_items) ids_item_next = load_ids(In, 0);
+        if (st == max(st_take, nst - 2) && nxt < n_items) ids_item_next = load_ids(In, 0);
         const int rel = st * kStagePages;  // first page of the stage, relative to page_lo
         if (rel > 0 && (rel & 31) == 0) {   // move to the next batch of 32 ids
           ids = ids_next;
@@ -1640,13 +1663,12 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
           m.invalid = (~okmask) & ((1u << np) - 1u);
           m.path = I.path;
           meta[s] = m;
+          // both tensors' bytes, before either warp's copies can land
           mbar_arrive_expect_tx(&B.full[s], kStageBytes);
         }
-        __syncwarp();
-        if (lane < kStagePages) {  // every page slot is written (zeros past the item)
+        post_v(s, w, 2 * Bt.cache + 1);
+        if (lane < kStagePages)  // every page slot is written (zeros past the item)
           tma_load_4d(stage_k(smem, s) + lane * kPageBytes, tk, 0, 0, 0, w, &B.full[s], policy);
-          tma_load_4d(stage_v(smem, s) + lane * kPageBytes, tv, 0, 0, 0, w, &B.full[s], policy);
-        }
         ++it;
       }
       if (nst == 0 && !aborted) {  // (the planner emits no empty item)
@@ -1667,6 +1689,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
       const int s = it % kStages;
       const uint32_t ph = (it / kStages) & 1;
       if (mbar_wait_bounded(&B.empty[s], ph ^ 1)) {
+        post_v(s, 0, -1);
         if (lane == 0) {
           meta[s].item = -1;
           mbar_arrive(&B.full[s]);
@@ -1676,11 +1699,36 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
         aborted = true;
       }
     }
+    // (stage `it` has not been handed over: its v_go phase is free)
+    if (aborted) post_v(it % kStages, 0, -1);
     if (aborted) {
       // the consumers stopped: let this CTA's copies land before exiting
       if (lane == 0) atomicExch(&misc[1], 1u);
       for (uint32_t k = (it > (uint32_t)kStages ? it - kStages : 0); k < it; ++k)
         (void)mbar_wait_bounded(&B.full[k % kStages], (k / kStages) & 1);
+    }
+    return;
+  }
+
+  if (warp == kVLoadWarp) {
+    // ---------------------------- V producer -------------------------------
+    // Issues each stage's V boxes as the K producer hands them over (the K
+    // producer has already waited for the stage to be free and registered
+    // both tensors' bytes on its barrier).
+    const uint64_t policy = l2_policy_evict_first();
+    const int *vjob = reinterpret_cast<const int *>(smem + Smem::off_vjob);
+    for (uint32_t it = 0;; ++it) {
+      const int s = it % kStages;
+      if (!mbar_wait_bounded(&B.v_go[s], (it / kStages) & 1)) {
+        ipd_set_error(&g_attn_err, IPD_DEVERR_WAIT);
+        atomicExch(&misc[1], 1u);
+        break;
+      }
+      const int tm = vjob[16 * s + 8];
+      if (tm < 0) break;
+      if (lane < kStagePages)
+        tma_load_4d(stage_v(smem, s) + lane * kPageBytes, &p.tmap[tm], 0, 0, 0,
+                    vjob[16 * s + lane], &B.full[s], policy);
     }
     return;
   }
