@@ -8,6 +8,7 @@ step streams its KV pages and logits from DRAM.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--config I] [--impl reference]
   python bench.py --next-rows [--config I] [--steps K]
+  python bench.py --attn-only [--config I] [--requests R] [--direction S|T] [--span LO HI]
 
 The headline workload is the full rollout-step mix (1024 requests, lognormal
 contexts up to 32K, spans of 1-16 tokens, both directions, 120 GB of KV
@@ -50,16 +51,20 @@ def _peaks():
         return HBM_FALLBACK_GBS, "fallback"
 
 
-def _committed_traffic(cfg: int):
-    """DRAM bytes per attention launch from the committed ncu capture, or None
-    when the kernel source has changed since that capture."""
+def _committed_traffic(cfg: int, attn_bytes: int):
+    """DRAM bytes per attention launch from the committed ncu record of this
+    workload, or None when the kernel source has changed since it was taken.
+    The record is a capture of a smaller case of the same shape; its ratio of
+    DRAM bytes to algorithmic bytes scales to this launch's bytes."""
     import hashlib
     path = os.path.join(ROOT, "profiles", f"attn_traffic_cfg{cfg}.json")
     src = os.path.join(ROOT, "paper_2609_36546_gb300", "csrc", "attn.cu")
     try:
         rec = json.load(open(path))
         h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-        return rec["traffic_bytes_per_launch"] if rec.get("source_sha256_16") == h else None
+        if rec.get("source_sha256_16") != h:
+            return None
+        return int(round(rec["traffic_over_algorithmic"] * attn_bytes))
     except Exception:
         return None
 
@@ -412,7 +417,7 @@ def measure_config(cfg, K, W, world, rank, stream, sampler=None):
         "value": tokens_all / (el_max / 1e3), "ms_per_step": ms_step, "tokens_per_step": T_tok,
         "requests": step.R, "clocks": clocks,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": _committed_traffic(cfg),
+                     "frac": achieved / peak, "traffic": _committed_traffic(cfg, attn_bytes),
                      "peak_kind": peak_kind,
                      "kernel": "attn_kernel (the attention launch of ipd_verify_attn; split "
                                "tasks merge inside it)",
@@ -749,6 +754,53 @@ def run_next_rows(args):
     print(json.dumps(line), flush=True)
 
 
+def run_attn_only(args):
+    """--attn-only: only the attention call (planner + attention launch) of a
+    workload shaped like configuration --config, optionally with fewer
+    requests (--requests; pools then hold only the pages used), one direction
+    (--direction S|T) or other span lengths (--span LO HI).  A small case of
+    this kind is what an ncu capture runs; it prints one JSON line with the
+    algorithmic bytes and the mean time of the attention launch."""
+    import dataclasses
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    import ipd_synth as S
+    from paper_2609_36546_gb300 import VerifyStep, ipd
+    spec = S.CONFIGS[args.config]
+    changes = {}
+    if args.requests:
+        changes.update(n_req=args.requests, pool_bytes=None)
+    if args.direction:
+        changes.update(direction=args.direction)
+    if args.span:
+        changes.update(span=("uniform", args.span[0], args.span[1]))
+    if changes:
+        spec = dataclasses.replace(spec, name=spec.name + " (shape kept, " +
+                                   ", ".join(f"{k}={v}" for k, v in changes.items()) + ")",
+                                   **changes)
+    w = S.make_workload(spec, seed=args.config, device="cuda")
+    step = VerifyStep.from_workload(w, device="cuda")
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        step.run_attention(stream)
+    torch.cuda.synchronize()
+    ipd.set_attn_kernel_timing(True)
+    for _ in range(args.steps):
+        step.run_attention(stream)
+    ms, n = ipd.attn_kernel_time()
+    ipd.set_attn_kernel_timing(False)
+    if ipd.device_error() != 0:
+        raise RuntimeError("device-side check failed")
+    nbytes = step.attn_bytes(w.ctx)
+    ms /= max(n, 1)
+    peak, kind = _peaks()
+    print(json.dumps({"workload": spec.name, "requests": spec.n_req, "launches": n,
+                      "bytes_per_launch": nbytes, "ms_per_launch": ms,
+                      "gbs": nbytes / ms / 1e6, "frac": nbytes / ms / 1e6 / peak,
+                      "peak_kind": kind}), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -764,10 +816,20 @@ def main():
     ap.add_argument("--per-config-steps", type=int, default=100)
     ap.add_argument("--next-rows", action="store_true",
                     help="time the calls beyond the step instead (one GPU)")
+    ap.add_argument("--attn-only", action="store_true",
+                    help="time only the attention call (profiling cases; one GPU)")
+    ap.add_argument("--requests", type=int, default=0,
+                    help="--attn-only: requests of the workload (pools sized to them)")
+    ap.add_argument("--direction", choices=["S", "T", "half", "bernoulli"], default=None,
+                    help="--attn-only: which model proposes")
+    ap.add_argument("--span", type=int, nargs=2, default=None,
+                    help="--attn-only: span lengths drawn uniformly in [LO, HI]")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     if args.next_rows:
         run_next_rows(args)
+    elif args.attn_only:
+        run_attn_only(args)
     elif args.impl == "reference":
         run_reference(args)
     else:

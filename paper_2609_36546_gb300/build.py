@@ -29,12 +29,23 @@ def sources():
     return sorted(os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".cu"))
 
 
+def _defines():
+    """Build-time switches from the environment.  IPD_TC_MIN_ROWS (default 4)
+    moves the row count from which attention tasks use the tensor cores; it
+    exists to measure the crossover between the two paths."""
+    v = os.environ.get("IPD_TC_MIN_ROWS")
+    return [f"-DIPD_TC_MIN_ROWS={int(v)}"] if v else []
+
+
 def build(verbose: bool = False, force: bool = False) -> str:
     os.makedirs(OUT_DIR, exist_ok=True)
     srcs = sources()
     deps = srcs + [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".cuh")] + \
         [os.path.join(HERE, "..", "include", "ipd.h")]
-    if not force and os.path.exists(LIB):
+    defines = _defines()
+    stamp = os.path.join(OUT_DIR, "defines.txt")
+    same_defines = os.path.exists(stamp) and open(stamp).read() == " ".join(defines)
+    if not force and same_defines and os.path.exists(LIB):
         t = os.path.getmtime(LIB)
         if all(os.path.getmtime(d) <= t for d in deps):
             return LIB
@@ -43,7 +54,7 @@ def build(verbose: bool = False, force: bool = False) -> str:
 
     def compile_one(src):
         obj = os.path.join(OUT_DIR, os.path.basename(src)[:-3] + ".o")
-        cmd = [nvcc, *ARCH, *FLAGS, "-c", src, "-o", obj]
+        cmd = [nvcc, *ARCH, *FLAGS, *defines, "-c", src, "-o", obj]
         if verbose:
             cmd.insert(1, "-Xptxas=-v")
         r = subprocess.run(cmd, capture_output=True, text=True)
@@ -60,6 +71,8 @@ def build(verbose: bool = False, force: bool = False) -> str:
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
     os.replace(tmp, LIB)
+    with open(stamp, "w") as f:
+        f.write(" ".join(defines))
     return LIB
 
 

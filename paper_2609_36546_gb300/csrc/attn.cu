@@ -75,7 +75,14 @@ constexpr int kAtomBytes = 1024;                  // 8 keys, one 64-dim half
 constexpr int kTensorBytes = kStagePages * kPageBytes;  // 32 KB of K (or V) per stage
 constexpr int kStageBytes = 2 * kTensorBytes;     // 64 KB
 constexpr int kTcRows = 128;                      // TMEM lanes of a tensor-core tile (M)
-constexpr int kTcMinRows = 4;                     // tasks with at least this many rows use it
+// Tasks with at least this many rows use the tensor path.  The library is
+// built with 4; the build accepts another value (IPD_TC_MIN_ROWS) only to
+// measure the crossover between the two paths.
+#ifndef IPD_TC_MIN_ROWS
+#define IPD_TC_MIN_ROWS 4
+#endif
+constexpr int kTcMinRows = IPD_TC_MIN_ROWS;
+static_assert(kTcMinRows >= 3 && kTcMinRows <= 8, "CUDA-core tasks have 2 to 7 rows");
 constexpr int kCcRows = kTcMinRows - 1;           // CUDA-core tasks have fewer rows
 constexpr int kCW = 8;                            // compute warps (two per TMEM lane block)
 constexpr int kCcW = 4;                           // of them, the CUDA-core path's warps
