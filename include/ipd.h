@@ -67,7 +67,7 @@ typedef struct CUstream_st *ipd_stream_t; /* same handle as cudaStream_t */
 #define IPD_DEVERR_TOKEN 3u      /* proposed token id outside [0, vocab)     */
 #define IPD_DEVERR_PLAN 4u       /* work list larger than the workspace     */
 #define IPD_DEVERR_WAIT 5u       /* a bounded pipeline wait ran out         */
-#define IPD_DEVERR_SPAN 6u       /* cu_span / cu_q not non-decreasing       */
+#define IPD_DEVERR_SPAN 6u       /* cu_span / cu_q / cu_new not non-decreasing, or rows past them */
 
 #define IPD_MAX_BATCHES 8
 #define IPD_MAX_K 32
@@ -332,9 +332,10 @@ int ipd_split_loss(const float *kl_rev, const float *kl_fwd, const uint8_t *sour
  *                    page page_table[r][pos / 16], slot pos % 16
  *  page_table        [num_reqs][max_pages] int32, as in ipd_attn_batch
  * All pointers 16-byte aligned.  Returns IPD_ERR_UNSUPPORTED unless
- * page_size == 16 and head_dim == 128.  A position outside the page table or
- * a page id outside the pool is recorded (IPD_DEVERR_SEQ_LEN /
- * IPD_DEVERR_PAGE_ID) and that row is skipped.  Rolling a cache back after a
+ * page_size == 16 and head_dim == 128.  A row outside cu_new[0] ..
+ * cu_new[num_reqs] - 1 (IPD_DEVERR_SPAN), a position outside the page table
+ * or at or past seq_len (IPD_DEVERR_SEQ_LEN) and a page id outside the pool
+ * (IPD_DEVERR_PAGE_ID) are recorded and that row is skipped.  Rolling a cache back after a
  * verdict needs no kernel: the next step passes the shorter length. */
 int ipd_kv_append(uint16_t *k_pages, uint16_t *v_pages, int64_t num_pages, int num_kv_heads,
                   int page_size, int head_dim, const uint16_t *k_new, const uint16_t *v_new,

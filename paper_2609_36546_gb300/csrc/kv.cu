@@ -7,8 +7,8 @@
 // pieces): consecutive threads cover one head row, then the next head, then
 // the next token, so both the reads of the new rows and the writes into a
 // page slot are contiguous 256-byte runs.  Every write is bounds-checked
-// against the page table and the pool; a bad entry is recorded in the device
-// error word and skipped.  One launch takes up to IPD_MAX_BATCHES appends
+// against the request offsets, the sequence length, the page table and the
+// pool; a bad entry is recorded in the device error word and skipped.  One launch takes up to IPD_MAX_BATCHES appends
 // (caches and request batches), so a step's appends cost one launch.
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -54,6 +54,11 @@ __global__ void __launch_bounds__(kAppendThreads) kv_append_kernel(
     const int tok = (int)(w / per_tok);
     const int rem = (int)(w % per_tok);
     const int h = rem / kPieces, c = rem % kPieces;
+    // a row that no request's offsets cover is not written
+    if (tok < D.cu_new[0] || tok >= D.cu_new[D.num_reqs]) {
+      ipd_set_error(&g_kv_err, IPD_DEVERR_SPAN);
+      continue;
+    }
     // the request holding new row `tok`: the last r with cu_new[r] <= tok
     int lo = 0, hi = D.num_reqs - 1;
     while (lo < hi) {
@@ -63,7 +68,7 @@ __global__ void __launch_bounds__(kAppendThreads) kv_append_kernel(
     }
     const int n = D.cu_new[lo + 1] - D.cu_new[lo];
     const int p = D.seq_len[lo] - n + (tok - D.cu_new[lo]);  // absolute position of the row
-    if (p < 0 || (p >> 4) >= D.max_pages) {
+    if (p < 0 || p >= D.seq_len[lo] || (p >> 4) >= D.max_pages) {
       ipd_set_error(&g_kv_err, IPD_DEVERR_SEQ_LEN);
       continue;
     }

@@ -78,6 +78,18 @@ def test_kv_append_bad_page_is_recorded_and_skipped(lib):
     assert np.array_equal(got_k, exp_k) and np.array_equal(got_v, exp_v)
 
 
+def test_kv_append_rows_past_the_offsets_are_skipped(lib):
+    """total_new counts five rows but cu_new ends at three: rows 3 and 4
+    belong to no request and must not be written anywhere (recorded as
+    IPD_DEVERR_SPAN); rows 0-2 land where the offsets place them."""
+    kp, vp, kn, vn, cu, L, table = _case(5, 4, [20, 40], [2, 3])
+    short = np.array([0, 2, 3], dtype=np.int32)     # request 1 owns only row 2
+    got_k, got_v = _run(lib, kp, vp, kn, vn, short, L, table)
+    assert lib.device_error() == 6                   # IPD_DEVERR_SPAN
+    exp_k, exp_v = O.kv_append(kp, vp, kn[:3], vn[:3], short, L, table)
+    assert np.array_equal(got_k, exp_k) and np.array_equal(got_v, exp_v)
+
+
 def test_kv_append_many_equals_one_by_one_and_oracle(lib):
     """The appends of one step (span rows into two caches of different head
     counts, decode rows into both) in one launch: every pool bit-identical
