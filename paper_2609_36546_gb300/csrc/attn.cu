@@ -986,10 +986,12 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
     }
     const float moff = (!real || m_used == -INFINITY) ? -INFINITY : -m_used;  // -inf: p = 0
 
-    // p = 2^(s*scale - m) as three bf16 terms: hi = p truncated to bf16, lo =
-    // the residual p - hi truncated, lo2 = the rest rounded to nearest.  Both
-    // subtractions are exact, so |p - hi - lo - lo2| <= 2^-25 p.  The scaling,
-    // residuals and row sum run on packed fp32 pairs.
+    // p = 2^(s*scale - m) as three bf16 terms, each the residual of the ones
+    // before rounded to nearest: hi = bf16(p), lo = bf16(p - hi), lo2 =
+    // bf16(p - hi - lo).  Both subtractions are exact (a residual has at most
+    // 16 significant bits), so |p - hi - lo - lo2| <= 2^-27 p.  One conversion
+    // packs a pair of keys' terms; the scaling, residuals and row sum run on
+    // packed fp32 pairs.
     unsigned long long lsum2 = 0ull;  // {0.f, 0.f}
     // the previous chunk's P V has read the P operand and the third-term
     // columns once this returns
@@ -1000,7 +1002,9 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
     };
     {
       const unsigned long long sl2x2 = f2_pack(sl2, sl2), moffx2 = f2_pack(moff, moff);
-      auto upper = [](float x) { return __uint_as_float(__float_as_uint(x) & 0xffff0000u); };
+      // the two bf16 halves of a packed pair as fp32 values
+      auto lo_f = [](uint32_t w) { return __uint_as_float(w << 16); };
+      auto hi_f = [](uint32_t w) { return __uint_as_float(w & 0xffff0000u); };
 #pragma unroll
       for (int q = 0; q < kSteps; ++q) {
         uint32_t(&sr)[16] = sv[F == 1 ? 0 : q];
@@ -1018,11 +1022,14 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
                     x0, x1);
           const float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
           const unsigned long long pp = f2_pack(p0, p1);
+          const uint32_t w1 = pack_bf16x2(p0, p1);
+          const unsigned long long l2 = f2_sub(pp, f2_pack(lo_f(w1), hi_f(w1)));
           float l0, l1, r0, r1;
-          f2_unpack(f2_sub(pp, f2_pack(upper(p0), upper(p1))), l0, l1);
-          f2_unpack(f2_sub(f2_pack(l0, l1), f2_pack(upper(l0), upper(l1))), r0, r1);
-          th[e >> 1] = pack_bf16x2_trunc(p0, p1);
-          tlo[e >> 1] = pack_bf16x2_trunc(l0, l1);
+          f2_unpack(l2, l0, l1);
+          const uint32_t w2 = pack_bf16x2(l0, l1);
+          f2_unpack(f2_sub(l2, f2_pack(lo_f(w2), hi_f(w2))), r0, r1);
+          th[e >> 1] = w1;
+          tlo[e >> 1] = w2;
           t3[e >> 1] = pack_bf16x2(r0, r1);
           lsum2 = f2_add(lsum2, pp);
         }
