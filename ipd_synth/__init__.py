@@ -86,6 +86,9 @@ class Spec:
     eos_prob: float = 0.0
     tie_quantum: float = 0.0
     force: str = ""       # "" | "accept" | "reject" | "mixed"
+    # K rows at absolute position p are scaled by 1 + key_growth * p / 128, so
+    # that attention scores grow along the sequence (test workloads only)
+    key_growth: float = 0.0
 
 
 GB = 1 << 30
@@ -266,6 +269,8 @@ def make_workload(spec_or_index, seed: Optional[int] = None, device="cpu",
             v = torch.zeros_like(k) if device.type == "cpu" else torch.empty_like(k)
         _fill_pages(k, used, gd)
         _fill_pages(v, used, gd)
+        if spec.key_growth:
+            _grow_keys(k, pt, n_pages, spec.key_growth)
         caches[name] = Cache(shape, k, v, pt)
 
     T = int(span.sum())
@@ -282,6 +287,17 @@ def make_workload(spec_or_index, seed: Optional[int] = None, device="cpu",
     return Workload(spec, seed, ctx.to(torch.int32), span.to(torch.int32), driver,
                     caches["teacher"], caches["student"], q_verify_t, q_verify_s,
                     q_decode_s, q_decode_t, tokens, ls, lt)
+
+
+def _grow_keys(k, page_table, n_pages, growth: float):
+    """Scales the K row at absolute position p of every request by
+    1 + growth * p / 128 (rounded to bf16)."""
+    pos = torch.arange(PAGE_SIZE, dtype=torch.float32)
+    for r in range(page_table.shape[0]):
+        for j in range(int(n_pages[r])):
+            f = (1.0 + growth * (16 * j + pos) / 128.0).to(k.device)
+            page = int(page_table[r, j])
+            k[page] = (k[page].float() * f[None, :, None]).to(torch.bfloat16)
 
 
 def _make_logits(spec: Spec, span, driver, gh, gd, device, row_chunk):

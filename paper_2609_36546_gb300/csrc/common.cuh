@@ -352,6 +352,14 @@ IPD_DEVINL unsigned long long f2_sub(unsigned long long a, unsigned long long b)
   return d;
 }
 
+// max(a, b, c) in one instruction (sm_100 and later); like fmaxf, a NaN
+// operand is ignored.
+IPD_DEVINL float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
 // 2^x on the special-function unit (hardware approximation, about 2 ulp).
 IPD_DEVINL float ex2_approx(float x) {
   float y;
