@@ -844,7 +844,8 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
   float *xbuf = reinterpret_cast<float *>(X.smem + Smem::off_x);  // [2][2][128]
   uint8_t *ps = X.smem + Smem::off_p;
   float m_used = -INFINITY;  // maximum the exponentials are taken against (log2 units)
-  float l_run = 0.f;         // this thread's share of the row sum
+  float l_run = 0.f;         // this thread's share of the row sum (in the scale of m_used)
+  float alpha_pend = 1.f;    // rescale still owed by the product in O (see below)
   float acc[64];             // output dims 64 second .. of this lane's O, summed over chunks
 #pragma unroll
   for (int e = 0; e < 64; ++e) acc[e] = 0.f;
@@ -942,54 +943,59 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
         }
       }
     };
-    // this thread's S values, then the chunk maximum over its keys and over
-    // the row's threads.  Tiles repeated over the lanes keep their (16 or 32)
-    // values in registers, loaded at once; 128-row tiles read their 64 again
-    // for the exponentials, 16 at a time.
+    // This thread's S values: tiles repeated over the lanes keep theirs (16
+    // or 32) in registers, loaded at once; 128-row tiles read theirs 16 at a
+    // time from TMEM.
     constexpr int kKeep = F == 1 ? 1 : kSteps;
     uint32_t sv[kKeep][16];
-    float mc = -INFINITY;
     if (F != 1) {
 #pragma unroll
       for (int q = 0; q < kKeep; ++q) tc_ld_32x32b_x16(tl + col_s(b) + k0 + 16 * q, sv[q]);
       tc_wait_ld();
-    }
 #pragma unroll
-    for (int q = 0; q < kSteps; ++q) {
-      uint32_t(&sr)[16] = sv[F == 1 ? 0 : q];
-      if (F == 1) {
-        tc_ld_32x32b_x16(tl + col_s(b) + k0 + 16 * q, sr);
-        tc_wait_ld();
-      }
-      mask(sr, k0 + 16 * q);
-      // three-operand maxima: 8 instructions for 16 values
+      for (int q = 0; q < kKeep; ++q) mask(sv[q], k0 + 16 * q);
+    }
+    // the maximum of 16 values (three-operand maxima: 8 instructions)
+    auto max16 = [](const uint32_t (&v)[16], float m) {
       float m5[5];
 #pragma unroll
       for (int e = 0; e < 5; ++e)
-        m5[e] = fmax3(__uint_as_float(sr[3 * e]), __uint_as_float(sr[3 * e + 1]),
-                      __uint_as_float(sr[3 * e + 2]));
-      mc = fmax3(mc, fmax3(m5[0], m5[1], m5[2]), fmax3(m5[3], m5[4], __uint_as_float(sr[15])));
-    }
-    float *xm = xbuf + (c & 1) * (2 * kTcRows);
-    xm[second * kTcRows + t] = mc;
-    named_bar_sync(1, kCW * 32);
+        m5[e] = fmax3(__uint_as_float(v[3 * e]), __uint_as_float(v[3 * e + 1]),
+                      __uint_as_float(v[3 * e + 2]));
+      return fmax3(m, fmax3(m5[0], m5[1], m5[2]), fmax3(m5[3], m5[4], __uint_as_float(v[15])));
+    };
+    // a 128-row tile's S values of keys k0 + 16 q .. on CUDA cores, from its Q
+    // tile in shared memory and the stage's K (only after a jump of the
+    // maximum has made the tensor core's values unusable: see below)
+    auto recompute_s = [&](int q, uint32_t (&v)[16]) {
+      const uint8_t *kst = stage_k(X.smem, s);
+      float a[16];
 #pragma unroll
-    for (int j = 0; j < F; ++j)
-      mc = fmaxf(mc, fmaxf(xm[row + j * kRep], xm[kTcRows + row + j * kRep]));
-    // the lazy rescale: keep the old maximum unless the chunk's is 2^8 larger
-    float alpha = 1.f;
-    {
-      const float mcs = mc * sl2;
-      if (real && mcs != -INFINITY) {
-        if (m_used == -INFINITY) {
-          m_used = mcs;
-        } else if (mcs > m_used + 8.f) {
-          alpha = ex2_approx(m_used - mcs);
-          m_used = mcs;
+      for (int e = 0; e < 16; ++e) a[e] = 0.f;
+      for (int h = 0; h < 2; ++h) {
+        for (int j = 0; j < 8; ++j) {
+          const uint4 qv = *reinterpret_cast<const uint4 *>(ps + h * Smem::kPHalf + sw128(t, j));
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            const int R = k0 + 16 * q + e;
+            const uint4 kv =
+                *reinterpret_cast<const uint4 *>(kv_row(kst, R, h) + ((j ^ (R & 7)) << 4));
+            float x = a[e];
+            x = fmaf(bf16lo(qv.x), bf16lo(kv.x), x);
+            x = fmaf(bf16hi(qv.x), bf16hi(kv.x), x);
+            x = fmaf(bf16lo(qv.y), bf16lo(kv.y), x);
+            x = fmaf(bf16hi(qv.y), bf16hi(kv.y), x);
+            x = fmaf(bf16lo(qv.z), bf16lo(kv.z), x);
+            x = fmaf(bf16hi(qv.z), bf16hi(kv.z), x);
+            x = fmaf(bf16lo(qv.w), bf16lo(kv.w), x);
+            a[e] = fmaf(bf16hi(qv.w), bf16hi(kv.w), x);
+          }
         }
       }
-    }
-    const float moff = (!real || m_used == -INFINITY) ? -INFINITY : -m_used;  // -inf: p = 0
+#pragma unroll
+      for (int e = 0; e < 16; ++e) v[e] = __float_as_uint(a[e]);
+      mask(v, k0 + 16 * q);
+    };
 
     // p = 2^(s*scale - m) as three bf16 terms, each the residual of the ones
     // before rounded to nearest: hi = bf16(p), lo = bf16(p - hi), lo2 =
@@ -997,7 +1003,6 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
     // 16 significant bits), so |p - hi - lo - lo2| <= 2^-27 p.  One conversion
     // packs a pair of keys' terms; the scaling, residuals and row sum run on
     // packed fp32 pairs.
-    unsigned long long lsum2 = 0ull;  // {0.f, 0.f}
     // the previous chunk's P V has read the P operand and the third-term
     // columns once this returns
     auto wait_prev = [&]() -> bool {
@@ -1005,7 +1010,10 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
       tc_fence_after();
       return true;
     };
-    {
+    // source 0: S from registers (repeated tiles) or TMEM (128-row tiles);
+    // source 1: recomputed on CUDA cores (128-row tiles).  Adds the thread's
+    // chunk maximum into *lm when given.
+    auto exp_pass = [&](float moff, int source, unsigned long long &lsum2, float *lm) -> bool {
       const unsigned long long sl2x2 = f2_pack(sl2, sl2), moffx2 = f2_pack(moff, moff);
       // the two bf16 halves of a packed pair as fp32 values
       auto lo_f = [](uint32_t w) { return __uint_as_float(w << 16); };
@@ -1014,10 +1022,15 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
       for (int q = 0; q < kSteps; ++q) {
         uint32_t(&sr)[16] = sv[F == 1 ? 0 : q];
         if (F == 1) {
-          tc_ld_32x32b_x16(tl + col_s(b) + k0 + 16 * q, sr);
-          tc_wait_ld();
-          mask(sr, k0 + 16 * q);
+          if (source == 0) {
+            tc_ld_32x32b_x16(tl + col_s(b) + k0 + 16 * q, sr);
+            tc_wait_ld();
+            mask(sr, k0 + 16 * q);
+          } else {
+            recompute_s(q, sr);
+          }
         }
+        if (lm) *lm = max16(sr, *lm);
         uint32_t th[8], tlo[8], t3[8];
 #pragma unroll
         for (int e = 0; e < 16; e += 2) {
@@ -1055,17 +1068,92 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
           else tc_st_32x32b_x8(tl + t3_col(kb >> 4), t3);
         }
       }
+      return true;
+    };
+    // the row's chunk maximum (log2 units) from the threads' entries
+    float *xm = xbuf + (c & 1) * (2 * kTcRows);
+    auto row_max = [&](float lm) {
+      xm[second * kTcRows + t] = lm;
+      named_bar_sync(1, kCW * 32);
+      float mx = lm;
+#pragma unroll
+      for (int j = 0; j < F; ++j)
+        mx = fmaxf(mx, fmaxf(xm[row + j * kRep], xm[kTcRows + row + j * kRep]));
+      return mx * sl2;
+    };
+
+    // The first chunk of an item (and every chunk of a repeated tile) takes
+    // its row maximum first and the exponentials against it, the running
+    // maximum moving up (and the sums rescaled) when the chunk's is 2^8
+    // larger.  Later chunks of 128-row tiles take the exponentials against
+    // the running maximum m_used in the same pass as the chunk's own maximum
+    // (one pass over S, one exchange after it):
+    //  - if the chunk's maximum exceeds m_used by more than 2^8, the running
+    //    maximum moves up after the chunk: its P and row sum are in the old
+    //    scale, so the rescale alpha_next is applied with its product, at the
+    //    next chunk;
+    //  - if it exceeds m_used by more than 2^64 (p could overflow), the
+    //    chunk's exponentials are taken again against its own maximum, from
+    //    S kept in registers or, in 128-row tiles, recomputed on CUDA cores.
+    unsigned long long lsum2 = 0ull;  // {0.f, 0.f}
+    float alpha_now = 1.f;   // rescale of acc and l_run before this chunk is added
+    float alpha_next = 1.f;  // rescale after this chunk (applied with its product)
+    float m_next = m_used;
+    if (first || F != 1) {
+      // (repeated tiles keep their S in registers: their maximum costs no
+      // second read, and the one-pass form measured slower for them)
+      float lm = -INFINITY;
+#pragma unroll
+      for (int q = 0; q < kSteps; ++q) {
+        uint32_t(&sr)[16] = sv[F == 1 ? 0 : q];
+        if (F == 1) {
+          tc_ld_32x32b_x16(tl + col_s(b) + k0 + 16 * q, sr);
+          tc_wait_ld();
+          mask(sr, k0 + 16 * q);
+        }
+        lm = max16(sr, lm);
+      }
+      const float mcs = row_max(lm);
+      if (real && mcs != -INFINITY) {
+        // the lazy rescale: keep the old maximum unless the chunk's is 2^8 larger
+        if (m_used == -INFINITY) {
+          m_used = m_next = mcs;
+        } else if (mcs > m_used + 8.f) {
+          alpha_now = ex2_approx(m_used - mcs);
+          m_used = m_next = mcs;
+        }
+      }
+      const float moff = (!real || m_used == -INFINITY) ? -INFINITY : -m_used;
+      if (!exp_pass(moff, 0, lsum2, nullptr)) return false;
+    } else {
+      float lm = -INFINITY;
+      const float moff = (!real || m_used == -INFINITY) ? -INFINITY : -m_used;
+      if (!exp_pass(moff, 0, lsum2, &lm)) return false;
+      const float mcs = row_max(lm);
+      if (real && mcs != -INFINITY) {
+        if (m_used == -INFINITY || mcs > m_used + 64.f) {
+          alpha_now = m_used == -INFINITY ? 0.f : ex2_approx(m_used - mcs);
+          m_used = m_next = mcs;
+          lsum2 = 0ull;
+          if (!exp_pass(-mcs, F == 1 ? 1 : 0, lsum2, nullptr)) return false;
+        } else if (mcs > m_used + 8.f) {
+          alpha_next = ex2_approx(m_used - mcs);
+          m_next = mcs;
+        }
+      }
     }
     // then the previous chunk's product into the registers (before this
-    // chunk's product overwrites O)
+    // chunk's product overwrites O), with the rescales decided since
     if (F == 1 && !wait_prev()) return false;
     if (F != 1) fence_proxy_async_smem();
-    if (!first) take_o(alpha);
+    if (!first) take_o(alpha_pend * alpha_now);
     {
       float a0, a1;
       f2_unpack(lsum2, a0, a1);
-      if (real) l_run = l_run * alpha + (a0 + a1);
+      if (real) l_run = (l_run * alpha_now + (a0 + a1)) * alpha_next;
     }
+    alpha_pend = alpha_next;
+    m_used = m_next;
     tc_wait_st();
     tc_fence_before();
     __syncwarp();
@@ -1078,7 +1166,7 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
   // ---- the last chunk's product, then the copies' sums into the first copy ----
   if (!wait_pv_done(c - 1)) return false;
   tc_fence_after();
-  take_o(1.f);
+  take_o(alpha_pend);
   // the other parity of the maximum exchange: its last readers (chunk c - 2)
   // have all passed chunk c - 1's barrier
   float *xl = xbuf + (c & 1) * (2 * kTcRows);
