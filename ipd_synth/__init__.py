@@ -89,6 +89,9 @@ class Spec:
     # K rows at absolute position p are scaled by 1 + key_growth * p / 128, so
     # that attention scores grow along the sequence (test workloads only)
     key_growth: float = 0.0
+    # ... and by key_jump from position key_jump_at on (a step in the scores)
+    key_jump_at: int = 0
+    key_jump: float = 1.0
 
 
 GB = 1 << 30
@@ -269,8 +272,8 @@ def make_workload(spec_or_index, seed: Optional[int] = None, device="cpu",
             v = torch.zeros_like(k) if device.type == "cpu" else torch.empty_like(k)
         _fill_pages(k, used, gd)
         _fill_pages(v, used, gd)
-        if spec.key_growth:
-            _grow_keys(k, pt, n_pages, spec.key_growth)
+        if spec.key_growth or spec.key_jump != 1.0:
+            _grow_keys(k, pt, n_pages, spec.key_growth, spec.key_jump_at, spec.key_jump)
         caches[name] = Cache(shape, k, v, pt)
 
     T = int(span.sum())
@@ -289,13 +292,17 @@ def make_workload(spec_or_index, seed: Optional[int] = None, device="cpu",
                     q_decode_s, q_decode_t, tokens, ls, lt)
 
 
-def _grow_keys(k, page_table, n_pages, growth: float):
+def _grow_keys(k, page_table, n_pages, growth: float, jump_at: int = 0, jump: float = 1.0):
     """Scales the K row at absolute position p of every request by
-    1 + growth * p / 128 (rounded to bf16)."""
+    1 + growth * p / 128, times `jump` from position jump_at on (rounded to
+    bf16)."""
     pos = torch.arange(PAGE_SIZE, dtype=torch.float32)
     for r in range(page_table.shape[0]):
         for j in range(int(n_pages[r])):
-            f = (1.0 + growth * (16 * j + pos) / 128.0).to(k.device)
+            p = 16 * j + pos
+            f = (1.0 + growth * p / 128.0) * torch.where(p >= jump_at, jump, 1.0) \
+                if jump_at else (1.0 + growth * p / 128.0)
+            f = f.to(k.device)
             page = int(page_table[r, j])
             k[page] = (k[page].float() * f[None, :, None]).to(torch.bfloat16)
 

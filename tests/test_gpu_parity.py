@@ -252,7 +252,8 @@ def test_empty_spans(lib):
     assert out["next_driver"].tolist() == [0, 1, 0]
 
 
-# Scores that grow along the sequence (K rows scaled by 1 + g p / 128): every
+# Scores that grow along the sequence (K rows scaled by 1 + g p / 128, or a
+# step in them): every
 # row's maximum moves up by more than 2^8 between some chunks, so the running
 # maximum is rescaled, on every tile path and both caches.  Scores of this
 # size (up to ~40 in log2 units) carry an fp32 rounding error in the exponent
@@ -266,6 +267,11 @@ GROWING = [
     ("short-spans", S.small_spec(n_req=6, ctx=(300, 1000), span=(1, 4), key_growth=0.8,
                                  direction="T"), 19),
     ("steep", S.small_spec(n_req=4, ctx=(700, 1300), span=(1, 16), key_growth=1.0), 20),
+    # a step: keys from position 520 on are 20 times larger, so a later chunk's
+    # maximum exceeds the running one by more than 2^64 (128-row tiles then
+    # recompute that chunk's scores on CUDA cores)
+    ("jump", S.small_spec(n_req=4, ctx=(700, 1100), span=(9, 16), direction="S", key_jump_at=520,
+                          key_jump=20.0), 21),
 ]
 
 
