@@ -645,6 +645,12 @@ __device__ void merge_split_row(const AttnParams &p, const Item &I, int r, int l
 // --------------------------------------------------------------------------
 // the attention kernel
 // --------------------------------------------------------------------------
+// V jobs handed from the K producer to the V producer.  The K producer
+// writes job i + kVJobs after the K slot of stage use i + kVJobs - kStages is
+// released, which the compute warps do only after the V of use
+// i + kVJobs - kStages - 1 >= i was issued: job i has been read by then.
+constexpr int kVJobs = 2 * kStages;
+
 struct Smem {
   static constexpr int off_stage = 0;                              // 3 x 64 KB, 1024-aligned
   // the P operand of a stacked tile, or the Q tile of a 128-row tile: two
@@ -656,12 +662,13 @@ struct Smem {
   static constexpr int off_x = off_p + 2 * kPHalf;                 // row-max / row-sum exchange [2][256]
   static constexpr int off_meta = off_x + 2 * 256 * 4;
   static constexpr int off_bar = off_meta + kStages * (int)sizeof(StageMeta);
-  static constexpr int n_bars = 3 * kStages + 7;
+  static constexpr int n_bars = 4 * kStages + 6 + kVJobs;
   static constexpr int off_misc = off_bar + n_bars * 8;
-  // per stage, the V boxes' coordinates for the second producer warp: eight
-  // page slots and the V tensor map's index (-1: stop)
+  // per stage use (a ring of kVJobs), the V boxes' coordinates for the
+  // second producer warp: eight page slots and the V tensor map's index
+  // (-1: stop)
   static constexpr int off_vjob = off_misc + 64;
-  static constexpr int total = off_vjob + kStages * 16 * 4;
+  static constexpr int total = off_vjob + kVJobs * 16 * 4;
   // CUDA-core path scratch (inside the P region, unused by that path)
   static constexpr int off_ccq = off_p;                              // fp32 [7][128]
   static constexpr int off_merge = off_ccq + kCcRows * kD * 4;       // fp32 [4][8][132]
@@ -674,13 +681,16 @@ static_assert(Smem::off_bar % 8 == 0, "mbarrier alignment");
 static_assert(Smem::total <= 227 * 1024, "shared memory");
 
 struct Bars {
-  uint64_t *full, *empty;  // KV ring
+  // KV ring: full = the stage's K (and its metadata) landed, vfull = its V
+  // landed; empty = its K slot free, vempty = its V slot free.  K is released
+  // once Q K^T has read it, V only after P V: K is refilled a chunk earlier.
+  uint64_t *full, *empty, *vfull, *vempty;
   uint64_t *q_ready;       // Q tile written to TMEM (one phase per tensor item)
   uint64_t *s_full;        // S = Q K^T landed, per S buffer (one phase per use)
   uint64_t *p_full;        // P of a chunk written (one phase per chunk)
   uint64_t *p_free;        // P V product of a chunk done: P read, O written (one phase per chunk)
   uint64_t *s_free;        // P V of a chunk done, per S buffer: the buffer may take the next Q K^T
-  uint64_t *v_go;          // per stage: its V boxes may be issued (one phase per stage use)
+  uint64_t *v_go;          // per V job slot: the job is written (one phase per use of the slot)
 };
 
 __device__ __forceinline__ Bars bars(uint8_t *smem) {
@@ -688,7 +698,9 @@ __device__ __forceinline__ Bars bars(uint8_t *smem) {
   Bars r;
   r.full = b;
   r.empty = b + kStages;
-  r.q_ready = b + 2 * kStages;
+  r.vfull = b + 2 * kStages;
+  r.vempty = b + 3 * kStages;
+  r.q_ready = b + 4 * kStages;
   r.s_full = r.q_ready + 1;
   r.p_full = r.s_full + 2;
   r.p_free = r.p_full + 1;
@@ -769,10 +781,13 @@ __device__ __forceinline__ const uint16_t *q_row(const ItemGeom &g, const Item &
 
 // Zero the V rows of stage s at or past the end of the sequence: unwritten
 // cache slots may hold non-finite bits, and a zero probability times NaN is NaN.
-__device__ __forceinline__ void zero_tail(const CompCtx &X, int s, int page0, int L, int nthreads,
-                                          int bar) {
+// Waits for the stage's V first (false on a time-out); V of a stage without
+// a tail is never touched by the compute warps.
+__device__ __forceinline__ bool zero_tail(const CompCtx &X, int s, uint32_t par, int page0, int L,
+                                          int nthreads, int bar) {
   const int tail0 = max(L - page0 * kPage, 0);  // first key slot at or past L
-  if (tail0 >= kStageKeys) return;
+  if (tail0 >= kStageKeys) return true;
+  if (!wait_or_abort(X, &bars(X.smem).vfull[s], par)) return false;
   uint8_t *vb = stage_v(X.smem, s);
   for (int e = X.ctid; e < (kStageKeys - tail0) * 16; e += nthreads) {
     const int row = tail0 + e / 16, cpart = e % 16;
@@ -781,6 +796,7 @@ __device__ __forceinline__ void zero_tail(const CompCtx &X, int s, int page0, in
   }
   fence_proxy_async_smem();
   named_bar_sync(bar, nthreads);
+  return true;
 }
 
 // ============================ tensor-core path ============================
@@ -824,6 +840,7 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
   constexpr int kRep = kTcRows / F;                 // rows of one copy (>= 32: a copy is warp-uniform)
   constexpr int kKT = 64 / F;                       // keys of a chunk per thread
   constexpr int kSteps = kKT / 16;                  // 16-key steps per thread
+  constexpr int kExpUnroll = F == 1 ? 1 : kSteps;  // exponential-pass steps unrolled
   const ItemGeom g = item_geom(p, I);
   const Bars &B = X.B;
   const int lb = X.warp & 3;                        // lane block of this warp
@@ -881,7 +898,7 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
     const int s = it % kStages;
     if (!wait_or_abort(X, &B.full[s], (it / kStages) & 1)) return false;
     const StageMeta M = X.meta[s];
-    zero_tail(X, s, M.page0, g.L, kCW * 32, 1);
+    if (!zero_tail(X, s, (it / kStages) & 1, M.page0, g.L, kCW * 32, 1)) return false;
     if (first) {
       const uint4 *src =
           reinterpret_cast<const uint4 *>(q_row(g, I, I.rb * kTcRows + row) + 64 * second);
@@ -922,8 +939,11 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
       __syncwarp();
       if (X.lane == 0) mbar_arrive(B.q_ready);
     }
+    // This warp is done with the stage's metadata and, unless the tile is a
+    // 128-row one (whose S may be recomputed from the stage's K below: its
+    // stage is released by its P V, which follows), with its K.
     __syncwarp();
-    if (X.lane == 0) mbar_arrive(&B.empty[s]);  // this warp is done with the stage
+    if (X.lane == 0) mbar_arrive(&B.empty[s]);
 
     const uint32_t b = c & 1;
     if (!wait_or_abort(X, &B.s_full[b], (c >> 1) & 1)) return false;
@@ -1018,7 +1038,9 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
       // the two bf16 halves of a packed pair as fp32 values
       auto lo_f = [](uint32_t w) { return __uint_as_float(w << 16); };
       auto hi_f = [](uint32_t w) { return __uint_as_float(w & 0xffff0000u); };
-#pragma unroll
+      // (a 128-row tile's four steps stay a loop: its hot code then fits the
+      // instruction cache)
+#pragma unroll kExpUnroll
       for (int q = 0; q < kSteps; ++q) {
         uint32_t(&sr)[16] = sv[F == 1 ? 0 : q];
         if (F == 1) {
@@ -1127,19 +1149,27 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
       if (!exp_pass(moff, 0, lsum2, nullptr)) return false;
     } else {
       float lm = -INFINITY;
-      const float moff = (!real || m_used == -INFINITY) ? -INFINITY : -m_used;
+      float moff = (!real || m_used == -INFINITY) ? -INFINITY : -m_used;
       if (!exp_pass(moff, 0, lsum2, &lm)) return false;
       const float mcs = row_max(lm);
+      bool redo = false;
       if (real && mcs != -INFINITY) {
         if (m_used == -INFINITY || mcs > m_used + 64.f) {
           alpha_now = m_used == -INFINITY ? 0.f : ex2_approx(m_used - mcs);
           m_used = m_next = mcs;
-          lsum2 = 0ull;
-          if (!exp_pass(-mcs, F == 1 ? 1 : 0, lsum2, nullptr)) return false;
+          moff = -mcs;
+          redo = true;
         } else if (mcs > m_used + 8.f) {
           alpha_next = ex2_approx(m_used - mcs);
           m_next = mcs;
         }
+      }
+      // TMEM loads and stores are warp-wide: the whole warp takes the second
+      // pass when one of its rows needs it (its other rows recompute their
+      // exponentials against their unchanged maximum)
+      if (__any_sync(0xffffffffu, redo)) {
+        lsum2 = 0ull;
+        if (!exp_pass(moff, F == 1 ? 1 : 0, lsum2, nullptr)) return false;
       }
     }
     // then the previous chunk's product into the registers (before this
@@ -1250,8 +1280,9 @@ __device__ __forceinline__ bool cc_item(const AttnParams &p, const CompCtx &X, c
   for (bool first = true;; first = false) {
     const int s = it % kStages;
     if (!wait_or_abort(X, &B.full[s], (it / kStages) & 1)) return false;
+    if (!wait_or_abort(X, &B.vfull[s], (it / kStages) & 1)) return false;
     const StageMeta M = X.meta[s];
-    zero_tail(X, s, M.page0, g.L, kCcW * 32, 3);
+    zero_tail(X, s, (it / kStages) & 1, M.page0, g.L, kCcW * 32, 3);
     if (first) {
       for (int e = X.ctid; e < nrow * (kD / 8); e += kCcW * 32) {
         const int rho = e / (kD / 8), c8 = e % (kD / 8);
@@ -1475,8 +1506,9 @@ __device__ __forceinline__ bool cc2_item(const AttnParams &p, const CompCtx &X, 
   for (;;) {
     const int s = it % kStages;
     if (!wait_or_abort(X, &B.full[s], (it / kStages) & 1)) return false;
+    if (!wait_or_abort(X, &B.vfull[s], (it / kStages) & 1)) return false;
     const StageMeta M = X.meta[s];
-    zero_tail(X, s, M.page0, g.L, kCcW * 32, 3);
+    zero_tail(X, s, (it / kStages) & 1, M.page0, g.L, kCcW * 32, 3);
     const uint8_t *kst = stage_k(X.smem, s);
     const uint8_t *vb = stage_v(X.smem, s);
     // ---- partial dot products of this lane's quarter for keys g * 8 + k ----
@@ -1647,14 +1679,17 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&B.full[s], 1);
-      mbar_init(&B.empty[s], 1 + kCW);  // the P V issuer and every compute warp
+      mbar_init(&B.vfull[s], 1);
+      mbar_init(&B.empty[s], 2 + kCW);  // both MMA issuers and every compute warp
+      // the P V of a tile of up to 64 rows, else the K producer (below)
+      mbar_init(&B.vempty[s], 1);
     }
     mbar_init(B.q_ready, kCW);
     for (int i = 0; i < 2; ++i) mbar_init(&B.s_full[i], 1);
     mbar_init(B.p_full, kCW);
     mbar_init(B.p_free, 1);
     for (int i = 0; i < 2; ++i) mbar_init(&B.s_free[i], 1);
-    for (int s = 0; s < kStages; ++s) mbar_init(&B.v_go[s], 1);
+    for (int j = 0; j < kVJobs; ++j) mbar_init(&B.v_go[j], 1);
     misc[1] = 0;
     fence_mbar_init();
   }
@@ -1685,7 +1720,13 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
     const uint64_t policy = l2_policy_evict_first();
     uint32_t it = 0;
     bool aborted = false;
-    int *vjob = reinterpret_cast<int *>(smem + Smem::off_vjob);  // [kStages][16]
+    // bit s: stage s's current use belongs to a 128-row tile or a CUDA-core
+    // item.  Such a stage is released whole (a 128-row tile's by its P V: an
+    // earlier refill of its K measured slower for these compute-bound tiles;
+    // a CUDA-core item's by the compute warps, which read V themselves), and
+    // this warp passes the V half of that release on to the V producer.
+    uint32_t joint = 0;
+    int *vjob = reinterpret_cast<int *>(smem + Smem::off_vjob);  // [kVJobs][16]
     // the next item's index: the atomic is issued at one stage and its value
     // taken at a later one, so that the producer does not wait for it
     int claim_v = 0;
@@ -1697,12 +1738,13 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
       claim_issue();
       return claim_take();
     };
-    // hands stage s's V boxes (or a stop, tm < 0) to the V producer warp
-    auto post_v = [&](int s, int w, int tm) {
-      if (lane < kStagePages) vjob[16 * s + lane] = w;
-      if (lane == 0) vjob[16 * s + 8] = tm;
+    // hands stage use `i`'s V boxes (or a stop, tm < 0) to the V producer warp
+    auto post_v = [&](uint32_t i, int w, int tm) {
+      const int j = i % kVJobs;
+      if (lane < kStagePages) vjob[16 * j + lane] = w;
+      if (lane == 0) vjob[16 * j + 8] = tm;
       __syncwarp();
-      if (lane == 0) mbar_arrive(&B.v_go[s]);
+      if (lane == 0) mbar_arrive(&B.v_go[j]);
     };
     // page id of page `page_lo + 32 * batch + lane`, or -1 past the item
     auto load_ids = [&](const Item &I, int batch) -> int {
@@ -1753,6 +1795,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
           aborted = true;
           break;
         }
+        if (lane == 0 && ((joint >> s) & 1)) mbar_arrive(&B.vempty[s]);
+        joint = (joint & ~(1u << s)) |
+                ((I.path == kPathTc1 || I.path == kPathCc ? 1u : 0u) << s);
         int w = oob_w;
         bool ok = false;
         if (lane < np) {
@@ -1770,10 +1815,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
           m.invalid = (~okmask) & ((1u << np) - 1u);
           m.path = I.path;
           meta[s] = m;
-          // both tensors' bytes, before either warp's copies can land
-          mbar_arrive_expect_tx(&B.full[s], kStageBytes);
+          mbar_arrive_expect_tx(&B.full[s], kTensorBytes);
         }
-        post_v(s, w, 2 * Bt.cache + 1);
+        post_v(it, w, 2 * Bt.cache + 1);
         if (lane < kStagePages)  // every page slot is written (zeros past the item)
           tma_load_4d(stage_k(smem, s) + lane * kPageBytes, tk, 0, 0, 0, w, &B.full[s], policy);
         ++it;
@@ -1796,7 +1840,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
       const int s = it % kStages;
       const uint32_t ph = (it / kStages) & 1;
       if (mbar_wait_bounded(&B.empty[s], ph ^ 1)) {
-        post_v(s, 0, -1);
+        post_v(it, 0, -1);
         if (lane == 0) {
           meta[s].item = -1;
           mbar_arrive(&B.full[s]);
@@ -1806,8 +1850,8 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
         aborted = true;
       }
     }
-    // (stage `it` has not been handed over: its v_go phase is free)
-    if (aborted) post_v(it % kStages, 0, -1);
+    // (stage use `it` has not been handed over: its v_go phase is free)
+    if (aborted) post_v(it, 0, -1);
     if (aborted) {
       // the consumers stopped: let this CTA's copies land before exiting
       if (lane == 0) atomicExch(&misc[1], 1u);
@@ -1819,23 +1863,38 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
 
   if (warp == kVLoadWarp) {
     // ---------------------------- V producer -------------------------------
-    // Issues each stage's V boxes as the K producer hands them over (the K
-    // producer has already waited for the stage to be free and registered
-    // both tensors' bytes on its barrier).
+    // Issues each stage's V boxes as the K producer hands them over, once the
+    // stage's V slot is free (its previous P V done).
     const uint64_t policy = l2_policy_evict_first();
     const int *vjob = reinterpret_cast<const int *>(smem + Smem::off_vjob);
-    for (uint32_t it = 0;; ++it) {
-      const int s = it % kStages;
-      if (!mbar_wait_bounded(&B.v_go[s], (it / kStages) & 1)) {
-        ipd_set_error(&g_attn_err, IPD_DEVERR_WAIT);
-        atomicExch(&misc[1], 1u);
+    uint32_t it = 0;
+    bool aborted = false;
+    for (;; ++it) {
+      const int s = it % kStages, j = it % kVJobs;
+      if (!mbar_wait_bounded(&B.v_go[j], (it / kVJobs) & 1)) {
+        aborted = true;
         break;
       }
-      const int tm = vjob[16 * s + 8];
+      const int tm = vjob[16 * j + 8];
       if (tm < 0) break;
+      if (!mbar_wait_bounded(&B.vempty[s], ((it / kStages) & 1) ^ 1)) {
+        aborted = true;
+        break;
+      }
+      if (lane == 0) mbar_arrive_expect_tx(&B.vfull[s], kTensorBytes);
+      __syncwarp();
       if (lane < kStagePages)
         tma_load_4d(stage_v(smem, s) + lane * kPageBytes, &p.tmap[tm], 0, 0, 0,
-                    vjob[16 * s + lane], &B.full[s], policy);
+                    vjob[16 * j + lane], &B.vfull[s], policy);
+    }
+    if (aborted) {
+      ipd_set_error(&g_attn_err, IPD_DEVERR_WAIT);
+      if (lane == 0) atomicExch(&misc[1], 1u);
+    }
+    if (aborted || *(volatile uint32_t *)&misc[1]) {
+      // the consumers stopped: let this CTA's copies land before exiting
+      for (uint32_t k = (it > (uint32_t)kStages ? it - kStages : 0); k < it; ++k)
+        (void)mbar_wait_bounded(&B.vfull[k % kStages], (k / kStages) & 1);
     }
     return;
   }
@@ -1870,8 +1929,11 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
       flags = __shfl_sync(0xffffffffu, flags, 0);
       path = __shfl_sync(0xffffffffu, path, 0);
       if (item < 0 || *(volatile uint32_t *)&misc[1]) break;
+      // the P V issuer has read the stage's metadata (the K producer may
+      // rewrite it once the K slot is free)
+      if (!is_qk && lane == 0 && path != kPathTc1) mbar_arrive(&B.empty[s]);
       if (path == kPathCc) {
-        if (!is_qk && lane == 0) mbar_arrive(&B.empty[s]);
+        if (is_qk && lane == 0) mbar_arrive(&B.empty[s]);
         __syncwarp();
         ++it;
         continue;
@@ -1908,10 +1970,13 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
             }
           }
           tc_commit(&B.s_full[c & 1]);
+          if (path != kPathTc1) tc_commit(&B.empty[s]);  // Q K^T has read the stage's K
+          else mbar_arrive(&B.empty[s]);
         }
         __syncwarp();
       } else {
         if (!mwait(B.p_full, c & 1)) break;
+        if (!mwait(&B.vfull[s], (it / kStages) & 1)) break;
         tc_fence_after();
         if (lane == 0) {
           // V keys 16kk.. as an MN-major operand: 64-dim halves 1 KB apart,
@@ -1944,7 +2009,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
           }
           tc_commit(B.p_free);
           tc_commit(&B.s_free[c & 1]);
-          tc_commit(&B.empty[s]);
+          tc_commit(path == kPathTc1 ? &B.empty[s] : &B.vempty[s]);
         }
         __syncwarp();
       }
