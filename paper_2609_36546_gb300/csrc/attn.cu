@@ -1096,7 +1096,11 @@ __device__ __forceinline__ bool tc_item(const AttnParams &p, const CompCtx &X, c
     float *xm = xbuf + (c & 1) * (2 * kTcRows);
     auto row_max = [&](float lm) {
       xm[second * kTcRows + t] = lm;
-      named_bar_sync(1, kCW * 32);
+      // only the warps holding copies of the thread's row meet: a 128-row
+      // tile's row lives in one lane block, a 64-row tile's in two
+      if (F == 1) named_bar_sync(4 + lb, 64);
+      else if (F == 2) named_bar_sync(8 + (lb & 1), 128);  // lane blocks lb and lb ^ 2
+      else named_bar_sync(1, kCW * 32);
       float mx = lm;
 #pragma unroll
       for (int j = 0; j < F; ++j)
