@@ -646,9 +646,11 @@ __device__ void merge_split_row(const AttnParams &p, const Item &I, int r, int l
 // the attention kernel
 // --------------------------------------------------------------------------
 // V jobs handed from the K producer to the V producer.  The K producer
-// writes job i + kVJobs after the K slot of stage use i + kVJobs - kStages is
-// released, which the compute warps do only after the V of use
-// i + kVJobs - kStages - 1 >= i was issued: job i has been read by then.
+// writes job i + kVJobs after the K slot of stage use i + kVJobs - kStages
+// is released, which the compute warps do only once they have finished use
+// i + kVJobs - kStages - 1; finishing a use means the V of the use before it
+// was issued (its P V, or the CUDA-core path's own wait, saw it land), so
+// job i + kVJobs - kStages - 2 >= i, and job i, have been read by then.
 constexpr int kVJobs = 2 * kStages;
 
 struct Smem {
@@ -682,8 +684,9 @@ static_assert(Smem::total <= 227 * 1024, "shared memory");
 
 struct Bars {
   // KV ring: full = the stage's K (and its metadata) landed, vfull = its V
-  // landed; empty = its K slot free, vempty = its V slot free.  K is released
-  // once Q K^T has read it, V only after P V: K is refilled a chunk earlier.
+  // landed; empty = its K slot free, vempty = its V slot free.  In tiles of
+  // up to 64 rows K is released once Q K^T has read it and V after P V, so
+  // K is refilled a chunk earlier; other stages are released whole.
   uint64_t *full, *empty, *vfull, *vempty;
   uint64_t *q_ready;       // Q tile written to TMEM (one phase per tensor item)
   uint64_t *s_full;        // S = Q K^T landed, per S buffer (one phase per use)
@@ -1908,7 +1911,8 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(const __grid_constant
     // Both issuers walk the same stages.  Warp kMmaWarp issues Q K^T of
     // tensor chunk j into S buffer j & 1 as soon as its stage has landed (and
     // the buffer's previous chunk, j - 2, has had its P V); warp kPvWarp
-    // issues P V of chunk j once its P is written, and releases the stage.
+    // issues P V of chunk j once its P is written and its V has landed, and
+    // releases the stage's V (a 128-row tile's whole stage).
     constexpr uint32_t idesc_s = idesc_bf16_f32(kTcRows, kStageKeys, 0);
     constexpr uint32_t idesc_o = idesc_bf16_f32(kTcRows, kD, 1);
     const uint32_t pa = smem_u32(smem + Smem::off_p);
