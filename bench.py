@@ -51,12 +51,14 @@ def _peaks():
         return HBM_FALLBACK_GBS, "fallback"
 
 
-def attn_code_key() -> str:
+ATTN_SRC = os.path.join(ROOT, "paper_2609_36546_gb300", "csrc", "attn.cu")
+
+
+def attn_code_key(src: str = ATTN_SRC) -> str:
     """Names the attention kernel's code: the first 16 hex digits of the
     SHA-256 of csrc/attn.cu with its // comments and blank lines removed, so
     that a comment edit does not retire an ncu record of the same code."""
     import hashlib
-    src = os.path.join(ROOT, "paper_2609_36546_gb300", "csrc", "attn.cu")
     lines = []
     for line in open(src, encoding="utf-8"):
         code = line.split("//", 1)[0].rstrip()
@@ -65,15 +67,16 @@ def attn_code_key() -> str:
     return hashlib.sha256("\n".join(lines).encode()).hexdigest()[:16]
 
 
-def _committed_traffic(cfg: int, attn_bytes: int):
+def _committed_traffic(cfg: int, attn_bytes: int, profiles: str = os.path.join(ROOT, "profiles"),
+                       src: str = ATTN_SRC):
     """DRAM bytes per attention launch from the committed ncu record of this
     workload, or None when the kernel's code has changed since it was taken.
     The record is a capture of a smaller case of the same shape; its ratio of
     DRAM bytes to algorithmic bytes scales to this launch's bytes."""
-    path = os.path.join(ROOT, "profiles", f"attn_traffic_cfg{cfg}.json")
+    path = os.path.join(profiles, f"attn_traffic_cfg{cfg}.json")
     try:
         rec = json.load(open(path))
-        if rec.get("attn_code_key") != attn_code_key():
+        if rec.get("attn_code_key") != attn_code_key(src):
             return None
         return int(round(rec["traffic_over_algorithmic"] * attn_bytes))
     except Exception:
