@@ -2,7 +2,9 @@
 
 One step = the whole hot path on one batch: ipd_verify_attn (span-verify
 attention on the verifier's cache co-launched with the proposer's decode
-attention), ipd_score_span (vocabulary pass + verdict) and ipd_split_loss.
+attention), the vocabulary pass + verdict (ipd_score_span_needed: the logits
+rows the verdict and the emitted positions need; --rows all: ipd_score_span,
+every row) and ipd_split_loss.
 Inputs are synthetic, seeded, resident in HBM and larger than L2, so every
 step streams its KV pages and logits from DRAM.
 
@@ -338,7 +340,7 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
-def measure_config(cfg, K, W, world, rank, stream, sampler=None):
+def measure_config(cfg, K, W, world, rank, stream, sampler=None, rows="needed"):
     """Device-timed steps of one workload: per-call events, the attention
     kernel's own events, and the step replayed from CUDA graphs.  Returns the
     step, the workload and a dict of figures (max over ranks)."""
@@ -347,7 +349,7 @@ def measure_config(cfg, K, W, world, rank, stream, sampler=None):
     from paper_2609_36546_gb300 import VerifyStep, ipd
 
     w = S.make_workload(cfg, seed=cfg + 1000 * rank, device="cuda")
-    step = VerifyStep.from_workload(w, device="cuda")
+    step = VerifyStep.from_workload(w, device="cuda", rows=rows)
     T_tok = step.T
     # warm-up (also yields the verdict used for the algorithmic byte count)
     for _ in range(W):
@@ -465,7 +467,8 @@ def run_gpu(args):
     K = args.steps
     sampler = ClockSampler(_smi_index(local)) if rank == 0 else None
     time.sleep(0.3 if sampler else 0.0)
-    step, w, fig = measure_config(cfg, K, max(3, args.warmup), world, rank, stream, sampler)
+    step, w, fig = measure_config(cfg, K, max(3, args.warmup), world, rank, stream, sampler,
+                                  rows=args.rows)
 
     # ---- end to end through host buffers ----
     e2e = run_e2e(step, w, min(K, args.e2e_steps), stream, world)
@@ -483,7 +486,7 @@ def run_gpu(args):
             if c == cfg:
                 continue
             st, wc, f = measure_config(c, min(K, args.per_config_steps), max(3, args.warmup),
-                                       world, rank, stream)
+                                       world, rank, stream, rows=args.rows)
             per_config[S.CONFIGS[c].name] = {
                 "workload": _workload_name(c), "value": f["value"], "unit": UNIT,
                 "ms_per_step": f["ms_per_step"],
@@ -504,6 +507,9 @@ def run_gpu(args):
         "config": {"workload": _workload_name(cfg), "seed": cfg,
                    "tokens_per_step": fig["tokens_per_step"], "requests": fig["requests"],
                    "l2": "inputs larger than L2 (no flush needed)",
+                   "vocab_pass": ("logits rows the verdict and the emitted positions need "
+                                  "(ipd_score_span_needed)" if args.rows == "needed" else
+                                  "every logits row (ipd_score_span)"),
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU"},
         "roofline": fig["roofline"], "step_hbm": fig["step_hbm"], "calls_ms": fig["calls_ms"],
         "ms_per_step_one_stream_graph": fig["ms_per_step_one_stream_graph"],
@@ -828,6 +834,9 @@ def main():
     ap.add_argument("--no-per-config", action="store_true",
                     help="skip the device-timed figures of the other workloads")
     ap.add_argument("--per-config-steps", type=int, default=100)
+    ap.add_argument("--rows", choices=["needed", "all"], default="needed",
+                    help="vocabulary pass of the step: only the logits rows the verdict and "
+                         "the emitted positions need, or every row")
     ap.add_argument("--next-rows", action="store_true",
                     help="time the calls beyond the step instead (one GPU)")
     ap.add_argument("--attn-only", action="store_true",

@@ -198,6 +198,34 @@ int ipd_score_span(const uint16_t *logits_student, const uint16_t *logits_teache
                    int32_t *new_len, uint8_t *done,
                    void *workspace, size_t workspace_bytes, ipd_stream_t stream);
 
+/* ipd_score_span reading only the logits rows the step needs: the verifier's
+ * rows up to each request's first transition and the proposer's rows of the
+ * emitted positions (Sec. 3.2.3: tokens after the transition are discarded,
+ * so neither model's row there enters the verdict or the loss).  Rows past a
+ * transition that is already known when their turn comes are not read; the
+ * rest are read as by ipd_score_span, position 0 of every request first.
+ *
+ * Arguments as for ipd_score_span, plus
+ *  max_span       an upper bound (1 .. 65535) on every request's span length;
+ *                 a longer span records IPD_DEVERR_SPAN and leaves that
+ *                 request's outputs undefined.
+ * Outputs: first_trans, n_emit, next_driver, new_len, done and source as
+ * ipd_score_span.  logp_s, logp_t, feedback, kl_rev and kl_fwd as
+ * ipd_score_span at every emitted position (source != 255), covered and
+ * margin at every position up to the request's first transition; at the other
+ * positions each of these is either ipd_score_span's value or, where a row
+ * was not read, NaN (covered 0).  Only the default (top-K) rules.  Workspace
+ * as for ipd_score_span (ipd_score_workspace_size). */
+int ipd_score_span_needed(const uint16_t *logits_student, const uint16_t *logits_teacher,
+                          const int32_t *tokens, const int32_t *cu_span, const uint8_t *driver,
+                          const int32_t *prefix_len, int num_reqs, int total_tokens, int vocab,
+                          int K, int eos_id, int max_span,
+                          float *logp_s, float *logp_t, float *feedback, float *kl_rev,
+                          float *kl_fwd, uint8_t *covered, float *margin, uint8_t *source,
+                          int32_t *first_trans, int32_t *n_emit, uint8_t *next_driver,
+                          int32_t *new_len, uint8_t *done,
+                          void *workspace, size_t workspace_bytes, ipd_stream_t stream);
+
 /* Takeover / handback rules (Sec. 3.2.1: top-K coverage is IPD's rule, but the
  * framework admits others, possibly different for takeover and handback, for
  * example a threshold on the entropy of either model; SKD is top-K takeover

@@ -37,7 +37,7 @@ struct RowOut {
   float m;  // maximum logit of the part (-inf if the part is empty)
   float s;  // sum over the part of exp(l - m)
   float u;  // sum over the part of exp(l - m) * l (entropy; 0 unless it was asked for)
-  int pad;
+  int skipped;  // needed-rows pass only: 1 if the row was not read (not needed)
   unsigned long long keys[IPD_MAX_K];  // the part's best keys, best first, 0 past the end
 };
 
@@ -132,10 +132,29 @@ __device__ __forceinline__ unsigned long long warp_top32_u64(unsigned long long 
 // Those groups are read again (from L2), their keys >= (tau, largest id) go
 // to the warp's buffer, which is cut back to its best K (by rank) when it
 // fills, and the warps' lists are merged by rank.
-template <bool kEntropy>  // also accumulate sum exp(l - m) l (entropies / entropy rules)
+// The needed-rows pass (kNeeded) reads only the rows that the verdict and the
+// emitted positions need.  Its grid is (2 R, max span): block (2 r + model,
+// i) takes row `model` of request r's span position i, so the blocks of
+// position 0 of every request are dispatched first, then position 1, and so
+// on.  A verifier row whose token decides the verdict (not covered under a
+// student-driven span, covered under a teacher-driven one) lowers the
+// request's transition bound trans[r]; a block whose position lies past the
+// bound it reads skips its row: the verifier's rows are needed up to the
+// first transition, the proposer's at the emitted positions before it (and
+// at it, for a handback).  The bound only ever falls towards the true first
+// transition, so no needed row is skipped.
+struct NeededRows {
+  const int32_t *tokens, *cu_span;
+  const uint8_t *driver;
+  int *trans;  // [R] lowest transition position seen so far (starts high)
+  int total_tokens;
+};
+
+template <bool kEntropy,  // also accumulate sum exp(l - m) l (entropies / entropy rules)
+          bool kNeeded>   // the needed-rows pass (one part per row)
 __global__ void __launch_bounds__(kRowThreads, kRowCtasPerSm) score_rows_kernel(
     const uint16_t *__restrict__ ls, const uint16_t *__restrict__ lt, int vocab, int K, int parts,
-    RowOut *__restrict__ out) {
+    RowOut *__restrict__ out, const NeededRows nr) {
   constexpr int U = 4;  // vectors per thread and iteration
   __shared__ uint16_t s_gmax[kMaxGroups][kRowThreads];  // group maxima (order codes, 0: none)
   __shared__ float s_sorted[kRowWarps][32];
@@ -146,7 +165,26 @@ __global__ void __launch_bounds__(kRowThreads, kRowCtasPerSm) score_rows_kernel(
   __shared__ int s_cand[kRowWarps][32 * kMaxGroupVecs];  // a round's candidate vectors
   __shared__ float s_m[kRowWarps], s_s[kRowWarps], s_u[kRowWarps];
 
-  const int row_id = blockIdx.x / parts, part = blockIdx.x % parts;
+  int row_id = blockIdx.x / parts, part = blockIdx.x % parts, oi = blockIdx.x;
+  int r = 0, pos = 0, drv = 0, ver = 0;
+  if (kNeeded) {
+    r = blockIdx.x >> 1;
+    pos = blockIdx.y;
+    const int t0 = nr.cu_span[r], k = nr.cu_span[r + 1] - t0;
+    // no such position (or offsets the epilogue reports as broken)
+    if (pos >= k || t0 < 0 || t0 + k > nr.total_tokens) return;
+    drv = nr.driver[r] ? 1 : 0;
+    ver = drv ? 0 : 1;  // the verifier's row: the teacher's when the student drives
+    row_id = 2 * (t0 + pos) + (int)(blockIdx.x & 1);
+    part = 0;
+    oi = row_id;
+    const int tr = *reinterpret_cast<volatile const int *>(nr.trans + r);
+    const bool need = (row_id & 1) == ver ? pos <= tr : (drv ? pos <= tr : pos < tr);
+    if (!need) {
+      if (threadIdx.x == 0) out[oi].skipped = 1;
+      return;
+    }
+  }
   const int t = row_id >> 1, model = row_id & 1;
   const uint16_t *row = (model ? lt : ls) + (size_t)t * vocab;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, tid = threadIdx.x;
@@ -358,15 +396,23 @@ __global__ void __launch_bounds__(kRowThreads, kRowCtasPerSm) score_rows_kernel(
     const float bs = warp_sum(lane < kRowWarps ? s_s[lane] * bf : 0.f);
     const float bu = warp_sum(lane < kRowWarps ? s_u[lane] * bf : 0.f);
     if (lane == 0) {
-      out[blockIdx.x].m = gm;
-      out[blockIdx.x].s = bs;
-      out[blockIdx.x].u = bu;
+      out[oi].m = gm;
+      out[oi].s = bs;
+      out[oi].u = bu;
+      if (kNeeded) out[oi].skipped = 0;
     }
     // the warps' lists (each sorted, 0 past its end) merged to the part's top K
     const unsigned long long a = warp_top32_u64(s_lists[0][lane], s_lists[1][lane], lane);
     const unsigned long long b = warp_top32_u64(s_lists[2][lane], s_lists[3][lane], lane);
     const unsigned long long c = warp_top32_u64(a, b, lane);
-    out[blockIdx.x].keys[lane] = lane < K ? c : 0ull;
+    out[oi].keys[lane] = lane < K ? c : 0ull;
+    if (kNeeded && model == ver) {
+      // coverage of the proposed token by this verifier row's Top_K
+      const int x = nr.tokens[t];
+      const bool hit = lane < K && x >= 0 && x < vocab && key_idx(c) == (uint32_t)x;
+      const bool cov = __ballot_sync(0xffffffffu, hit) != 0;
+      if (lane == 0 && (drv ? cov : !cov)) atomicMin(nr.trans + r, pos);
+    }
   }
 }
 
@@ -386,7 +432,7 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     float *feedback,
     float *kl_rev, float *kl_fwd, uint8_t *covered, float *margin, uint8_t *source,
     int32_t *first_trans, int32_t *n_emit, uint8_t *next_driver, int32_t *new_len, uint8_t *done,
-    int total_tokens, const EpiOpts opt) {
+    int total_tokens, const EpiOpts opt, int max_span = 0) {
   // No shared memory.  In a step that forks the vocabulary pass onto its
   // own stream, this kernel's CTAs take the SMs that the first attention
   // CTAs to finish leave free, so it runs inside the attention's tail.
@@ -399,6 +445,12 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     return;
   }
   const int k = t1 - t0;
+  // after a needed-rows pass (max_span > 0) a span longer than its bound was
+  // read only in part: its verdict would be wrong
+  if (max_span > 0 && k > max_span) {
+    if (threadIdx.x == 0) ipd_set_error(&g_score_err, IPD_DEVERR_SPAN);
+    return;
+  }
 
   for (int t = t0 + warp; t < t1; t += kEpiThreads / 32) {
     const int x = tokens[t];
@@ -510,15 +562,21 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     }
     // |Top_K(pi) n Top_K(q)|: teacher keys also in the student's list
     const int n_common = __popc(__ballot_sync(0xffffffffu, lane < K && dupT));
+    // a needed-rows pass leaves the rows past the transition unread: the
+    // values that would come from them are NaN (coverage 0)
+    const bool skip_s = max_span > 0 && rows[(size_t)2 * t * parts].skipped;
+    const bool skip_t = max_span > 0 && rows[(size_t)(2 * t + 1) * parts].skipped;
+    const bool skip_ver = drv ? skip_s : skip_t;
     if (lane == 0) {
       const float lps = lxS - logz[0], lpt = lxT - logz[1];
-      logp_s[t] = lps;
-      logp_t[t] = lpt;
-      feedback[t] = lpt - lps;
-      kl_rev[t] = kr;
-      kl_fwd[t] = kf;
-      covered[t] = cov ? 1 : 0;
-      margin[t] = mar;
+      const bool both = !skip_s && !skip_t;
+      logp_s[t] = both ? lps : nan;
+      logp_t[t] = both ? lpt : nan;
+      feedback[t] = both ? lpt - lps : nan;
+      kl_rev[t] = both ? kr : nan;
+      kl_fwd[t] = both ? kf : nan;
+      covered[t] = cov && !skip_ver ? 1 : 0;
+      margin[t] = skip_ver ? nan : mar;
       if (opt.entropy_s) opt.entropy_s[t] = ent[0];
       if (opt.entropy_t) opt.entropy_t[t] = ent[1];
       if (opt.topk_overlap) opt.topk_overlap[t] = (float)n_common / (float)K;
@@ -602,11 +660,18 @@ int row_parts(int total_tokens, int vocab, int max_parts) {
     if (2LL * total_tokens * q <= slots && vocab / 8 / q >= kRowThreads * 4) return q;
   return 1;
 }
+
+// the needed-rows pass's transition bounds, after the row records and the
+// sampler's partials
+size_t trans_offset(int num_reqs, int total_tokens, int vocab) {
+  return (rows_region(total_tokens) + ipd_internal_sample_ws(num_reqs, vocab) + 255) &
+         ~(size_t)255;
+}
 }  // namespace
 
 extern "C" size_t ipd_score_workspace_size(int num_reqs, int total_tokens, int vocab, int K) {
   if (num_reqs < 0 || total_tokens < 0 || vocab < 1 || K < 1) return 0;
-  return rows_region(total_tokens) + ipd_internal_sample_ws(num_reqs, vocab) + 256;
+  return trans_offset(num_reqs, total_tokens, vocab) + (size_t)num_reqs * sizeof(int) + 256;
 }
 
 namespace {
@@ -662,11 +727,11 @@ extern "C" int ipd_score_span_ex(const uint16_t *logits_student, const uint16_t 
                         opt.take_rule == IPD_RULE_ENTROPY_T || opt.hand_rule == IPD_RULE_ENTROPY_S ||
                         opt.hand_rule == IPD_RULE_ENTROPY_T;
     if (need_h)
-      score_rows_kernel<true><<<2 * parts * total_tokens, kRowThreads, 0, st>>>(
-          logits_student, logits_teacher, vocab, K, parts, rows);
+      score_rows_kernel<true, false><<<2 * parts * total_tokens, kRowThreads, 0, st>>>(
+          logits_student, logits_teacher, vocab, K, parts, rows, NeededRows{});
     else
-      score_rows_kernel<false><<<2 * parts * total_tokens, kRowThreads, 0, st>>>(
-          logits_student, logits_teacher, vocab, K, parts, rows);
+      score_rows_kernel<false, false><<<2 * parts * total_tokens, kRowThreads, 0, st>>>(
+          logits_student, logits_teacher, vocab, K, parts, rows, NeededRows{});
     if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   }
   score_epilogue_kernel<<<num_reqs, kEpiThreads, 0, st>>>(
@@ -696,6 +761,56 @@ extern "C" int ipd_score_span(const uint16_t *logits_student, const uint16_t *lo
                            kl_rev, kl_fwd, covered, margin, source, first_trans, n_emit,
                            next_driver, new_len, done, nullptr, workspace, workspace_bytes,
                            stream);
+}
+
+extern "C" int ipd_score_span_needed(const uint16_t *logits_student,
+                                     const uint16_t *logits_teacher, const int32_t *tokens,
+                                     const int32_t *cu_span, const uint8_t *driver,
+                                     const int32_t *prefix_len, int num_reqs, int total_tokens,
+                                     int vocab, int K, int eos_id, int max_span, float *logp_s,
+                                     float *logp_t, float *feedback, float *kl_rev,
+                                     float *kl_fwd, uint8_t *covered, float *margin,
+                                     uint8_t *source, int32_t *first_trans, int32_t *n_emit,
+                                     uint8_t *next_driver, int32_t *new_len, uint8_t *done,
+                                     void *workspace, size_t workspace_bytes,
+                                     ipd_stream_t stream) {
+  if (num_reqs < 0 || total_tokens < 0) return IPD_ERR_INVALID_ARG;
+  if (K < 1 || K > IPD_MAX_K) return IPD_ERR_UNSUPPORTED;
+  if (vocab < 8 || vocab % 8 || K > vocab) return IPD_ERR_UNSUPPORTED;
+  if (num_reqs == 0) return IPD_OK;
+  if (max_span < 1 || max_span > 65535) return IPD_ERR_INVALID_ARG;
+  if (!cu_span || !driver || !prefix_len || !first_trans || !n_emit || !next_driver || !new_len ||
+      !done)
+    return IPD_ERR_INVALID_ARG;
+  if (total_tokens > 0 &&
+      (!logits_student || !logits_teacher || !tokens || !logp_s || !logp_t || !feedback ||
+       !kl_rev || !kl_fwd || !covered || !margin || !source))
+    return IPD_ERR_INVALID_ARG;
+  if (((uintptr_t)logits_student | (uintptr_t)logits_teacher) & 15) return IPD_ERR_INVALID_ARG;
+  const size_t need = ipd_score_workspace_size(num_reqs, total_tokens, vocab, K);
+  if (total_tokens > 0 && (!workspace || workspace_bytes < need || ((uintptr_t)workspace & 15)))
+    return IPD_ERR_WORKSPACE;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  RowOut *rows = static_cast<RowOut *>(workspace);
+  int *trans = reinterpret_cast<int *>(static_cast<char *>(workspace) +
+                                       trans_offset(num_reqs, total_tokens, vocab));
+  if (total_tokens > 0) {
+    // every bound starts above any position (0x7f7f7f7f)
+    if (cudaMemsetAsync(trans, 0x7f, (size_t)num_reqs * sizeof(int), st) != cudaSuccess)
+      return IPD_ERR_CUDA;
+    score_rows_kernel<false, true><<<dim3(2 * num_reqs, max_span), kRowThreads, 0, st>>>(
+        logits_student, logits_teacher, vocab, K, 1, rows,
+        NeededRows{tokens, cu_span, driver, trans, total_tokens});
+    if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
+  }
+  score_epilogue_kernel<<<num_reqs, kEpiThreads, 0, st>>>(
+      logits_student, logits_teacher, tokens, cu_span, driver, prefix_len, vocab, K, eos_id, rows,
+      1, logp_s, logp_t, feedback, kl_rev, kl_fwd, covered, margin, source, first_trans, n_emit,
+      next_driver, new_len, done, total_tokens,
+      EpiOpts{IPD_RULE_TOPK, IPD_RULE_TOPK, 0.f, 0.f, nullptr, nullptr, nullptr, nullptr, nullptr},
+      max_span);
+  if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
+  return IPD_OK;
 }
 
 // ---------------------------------------------------------------------------
@@ -980,8 +1095,8 @@ extern "C" int ipd_score_span_static(const uint16_t *logits_student,
       total_tokens, vocab,
       total_tokens > 0 ? std::min(kMaxParts, IPD_STATIC_MAX_TOKENS / total_tokens) : 1);
   if (total_tokens > 0) {
-    score_rows_kernel<false><<<2 * parts * total_tokens, kRowThreads, 0, s>>>(
-        logits_student, logits_teacher, vocab, K, parts, rows);
+    score_rows_kernel<false, false><<<2 * parts * total_tokens, kRowThreads, 0, s>>>(
+        logits_student, logits_teacher, vocab, K, parts, rows, NeededRows{});
     if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   }
   score_epilogue_kernel<<<num_reqs, kEpiThreads, 0, s>>>(

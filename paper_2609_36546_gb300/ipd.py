@@ -31,7 +31,7 @@ LOSS_FIELDS = ("loss", "sum_on", "sum_off", "n_on", "n_off", "intervention_ratio
 EXPORTS = ("ipd_attn_workspace_size", "ipd_verify_attn", "ipd_decode_attn",
            "ipd_score_workspace_size", "ipd_score_span", "ipd_loss_workspace_size",
            "ipd_split_loss", "ipd_get_device_error", "ipd_status_string", "ipd_version",
-           "ipd_score_span_static", "ipd_score_span_ex", "ipd_full_kl",
+           "ipd_score_span_static", "ipd_score_span_ex", "ipd_score_span_needed", "ipd_full_kl",
            "ipd_loss_grad_workspace_size", "ipd_split_loss_grad", "ipd_sample_workspace_size",
            "ipd_sample", "ipd_kv_append", "ipd_kv_append_many", "ipd_set_attn_kernel_timing",
            "ipd_attn_kernel_time")
@@ -102,6 +102,8 @@ _lib.ipd_score_workspace_size.restype = c_sz
 _lib.ipd_score_workspace_size.argtypes = [c_i, c_i, c_i, c_i]
 _lib.ipd_score_span.restype = c_i
 _lib.ipd_score_span.argtypes = [c_p] * 6 + [c_i] * 5 + [c_p] * 13 + [c_p, c_sz, c_p]
+_lib.ipd_score_span_needed.restype = c_i
+_lib.ipd_score_span_needed.argtypes = [c_p] * 6 + [c_i] * 6 + [c_p] * 13 + [c_p, c_sz, c_p]
 _lib.ipd_score_span_ex.restype = c_i
 _lib.ipd_score_span_ex.argtypes = ([c_p] * 6 + [c_i] * 5 + [c_p] * 13 +
                                    [ctypes.POINTER(_ScoreExt), c_p, c_sz, c_p])
@@ -252,6 +254,22 @@ def score_span(logits_student, logits_teacher, tokens, cu_span, driver, prefix_l
         *[_ptr(out[n]) for n, _ in SCORE_REQ_OUTPUTS],
         _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)),
         "ipd_score_span")
+
+
+def score_span_needed(logits_student, logits_teacher, tokens, cu_span, driver, prefix_len,
+                      K: int, eos_id: int, max_span: int, out: dict, workspace: torch.Tensor,
+                      stream=None):
+    """ipd_score_span reading only the rows the verdict and the emitted
+    positions need; ``max_span`` bounds every request's span length."""
+    R = driver.numel()
+    T, V = logits_student.shape
+    _check(_lib.ipd_score_span_needed(
+        _ptr(logits_student), _ptr(logits_teacher), _ptr(tokens), _ptr(cu_span), _ptr(driver),
+        _ptr(prefix_len), R, T, V, K, eos_id, max_span,
+        *[_ptr(out[n]) for n, _ in SCORE_TOKEN_OUTPUTS],
+        *[_ptr(out[n]) for n, _ in SCORE_REQ_OUTPUTS],
+        _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)),
+        "ipd_score_span_needed")
 
 
 def score_span_ex(logits_student, logits_teacher, tokens, cu_span, driver, prefix_len, K: int,

@@ -101,9 +101,15 @@ class VerifyStep:
                  pt_teacher, pt_student, q_verify_t, q_verify_s, q_decode_s, q_decode_t, tokens,
                  logits_s, logits_t, K: int = 16, eos_id: int = -1, resp_len=None,
                  agg_mode: int = ipd.AGG_SEQ_MEAN_TOKEN_MEAN, dir_mode: int = ipd.DIR_SPLIT,
-                 scale: float = SCALE, device="cuda"):
+                 scale: float = SCALE, device="cuda", rows: str = "all"):
         dev = torch.device(device)
         self.device = dev
+        # "all": the vocabulary pass reads every logits row (ipd_score_span);
+        # "needed": only the rows the verdict and the emitted positions need
+        # (ipd_score_span_needed); the verdict, sources and loss are the same
+        if rows not in ("all", "needed"):
+            raise ValueError(f"rows must be 'all' or 'needed', not {rows!r}")
+        self.rows = rows
         self.K, self.eos_id, self.agg_mode, self.dir_mode, self.scale = K, eos_id, agg_mode, \
             dir_mode, scale
         ctx = ctx.to(torch.int32).cpu()
@@ -111,6 +117,7 @@ class VerifyStep:
         driver = driver.to(torch.uint8).cpu()
         self.R = int(ctx.numel())
         self.T = int(span.sum())
+        self.max_span = max(1, int(span.max())) if span.numel() else 1
         self.cache_t = ipd.KVCache(teacher_k, teacher_v)
         self.cache_s = ipd.KVCache(student_k, student_v)
         idx_s = torch.nonzero(driver == 0).flatten()   # student proposes, teacher verifies
@@ -180,9 +187,17 @@ class VerifyStep:
     def run_attention(self, stream=None):
         ipd.verify_attn(self.verify, self.decode, self.scale, self.ws_attn, stream)
 
+    def _score_call(self, ls, lt, tokens, cu_span, driver, prefix_len, out, stream):
+        if self.rows == "needed":
+            ipd.score_span_needed(ls, lt, tokens, cu_span, driver, prefix_len, self.K,
+                                  self.eos_id, self.max_span, out, self.ws_score, stream)
+        else:
+            ipd.score_span(ls, lt, tokens, cu_span, driver, prefix_len, self.K, self.eos_id, out,
+                           self.ws_score, stream)
+
     def run_score(self, stream=None):
-        ipd.score_span(self.logits_s, self.logits_t, self.tokens, self.cu_span, self.driver,
-                       self.prefix_len, self.K, self.eos_id, self.score, self.ws_score, stream)
+        self._score_call(self.logits_s, self.logits_t, self.tokens, self.cu_span, self.driver,
+                         self.prefix_len, self.score, stream)
 
     def run_loss(self, stream=None):
         s = self.score
@@ -298,9 +313,9 @@ class VerifyStep:
             sc.wait_event(ev)
             out = {n: self.score[n][t0:t1] for n, _ in ipd.SCORE_TOKEN_OUTPUTS}
             out.update({n: self.score[n][r0:r1] for n, _ in ipd.SCORE_REQ_OUTPUTS})
-            ipd.score_span(self.logits_s[t0:t1], self.logits_t[t0:t1], self.tokens[t0:t1],
-                           cu_chunk[off:off + r1 - r0 + 1], self.driver[r0:r1],
-                           self.prefix_len[r0:r1], self.K, self.eos_id, out, self.ws_score, sc)
+            self._score_call(self.logits_s[t0:t1], self.logits_t[t0:t1], self.tokens[t0:t1],
+                             cu_chunk[off:off + r1 - r0 + 1], self.driver[r0:r1],
+                             self.prefix_len[r0:r1], out, sc)
             off += r1 - r0 + 1
         main.wait_stream(sc)
         main.wait_stream(cp)

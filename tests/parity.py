@@ -104,10 +104,23 @@ def oracle_scores(step, requests):
     return res
 
 
-def check_scores(step, requests=None, orc=None):
+def needed_positions(source, first_trans, cu_span, r):
+    """For request r of a step's outputs (numpy): the mask of its emitted
+    positions and of the positions up to its first transition (the ones a
+    needed-rows pass defines: ipd_score_span_needed)."""
+    t0, t1 = int(cu_span[r]), int(cu_span[r + 1])
+    emitted = source[t0:t1] != 255
+    decided = np.arange(t1 - t0) <= int(first_trans[r])
+    return emitted, decided
+
+
+def check_scores(step, requests=None, orc=None, needed=False):
     """Compare the scores and decisions of the chosen requests (all by
     default) with the oracle's; `orc` may hold the oracle's results already
-    (request -> (t0, t1, score_span output))."""
+    (request -> (t0, t1, score_span output)).  needed=True compares the
+    per-token values only where a needed-rows pass defines them: log-probs,
+    feedback and KL at emitted positions, coverage and margin up to the first
+    transition (the decisions everywhere)."""
     R = step.R
     reqs = list(range(R)) if requests is None else [int(r) for r in requests]
     if orc is None:
@@ -122,18 +135,21 @@ def check_scores(step, requests=None, orc=None):
         sl = slice(t0, t1)
         st["score_positions"] += t1 - t0
         if t1 > t0:
-            st["max_logp_err"] = max(st["max_logp_err"],
-                                     float(np.abs(g["logp_s"][sl] - o["logp_s"]).max()),
-                                     float(np.abs(g["logp_t"][sl] - o["logp_t"]).max()))
-            st["max_fb_err"] = max(st["max_fb_err"],
-                                   float(np.abs(g["feedback"][sl] - o["feedback"]).max()))
+            em = dec = np.ones(t1 - t0, bool)
+            if needed:
+                em, dec = needed_positions(o["source"], o["first_trans"], np.array([0, t1 - t0]),
+                                           0)
+            def err_of(name, rel=0.0):
+                e = np.abs(g[name][sl] - o[name]) - rel * np.abs(o[name])
+                m = dec if name == "margin" else em
+                return float(e[m].max()) if m.any() else 0.0
+            st["max_logp_err"] = max(st["max_logp_err"], err_of("logp_s"), err_of("logp_t"))
+            st["max_fb_err"] = max(st["max_fb_err"], err_of("feedback"))
             for name in ("kl_rev", "kl_fwd"):
-                err = np.abs(g[name][sl] - o[name]) - KL_RTOL * np.abs(o[name])
-                st["max_kl_err"] = max(st["max_kl_err"], float(err.max()))
-            st["max_margin_err"] = max(st["max_margin_err"],
-                                       float(np.abs(g["margin"][sl] - o["margin"]).max()))
-            near = np.abs(o["margin"]) <= 1e-3
-            cov_mis = g["covered"][sl].astype(np.int64) != o["covered"]
+                st["max_kl_err"] = max(st["max_kl_err"], err_of(name, KL_RTOL))
+            st["max_margin_err"] = max(st["max_margin_err"], err_of("margin"))
+            near = (np.abs(o["margin"]) <= 1e-3) & dec
+            cov_mis = (g["covered"][sl].astype(np.int64) != o["covered"]) & dec
             src_mis = g["source"][sl].astype(np.int64) != o["source"]
             st["near_threshold"] += int(near.sum())
             st["near_threshold_mismatch"] += int((near & cov_mis).sum())
@@ -174,14 +190,14 @@ def check_loss(step, orc):
     return st
 
 
-def check_step(step, w=None, requests=None, attn_max_reqs=None, rng=None):
+def check_step(step, w=None, requests=None, attn_max_reqs=None, rng=None, needed=False):
     """Full comparison; requests=None checks every request and the loss.
 
     With a subset of requests the batch loss cannot be recomputed: the report
     then says loss_checked = False and `ok` covers attention and scores only."""
     rep = {}
     rep.update(check_attention(step, requests, attn_max_reqs, rng))
-    s, orc = check_scores(step, requests)
+    s, orc = check_scores(step, requests, needed=needed)
     rep.update(s)
     rep["loss_checked"] = requests is None
     if requests is None:

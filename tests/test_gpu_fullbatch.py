@@ -53,5 +53,25 @@ def test_full_batch_matches_oracle(lib, pool, cfg):
     assert int(emitted.sum()) == int(sc["n_emit"].sum())
     assert float(o8[3] + o8[4]) == float(emitted.sum())
     assert torch.all(sc["new_len"] == step.prefix_len.cpu() + sc["n_emit"])
+    # the needed-rows pass on the same step: rows are read whole by both
+    # passes at these sizes, so where it defines a value it is bit-identical
+    o8 = step.out8.cpu()
+    step.rows = "needed"
+    step.run_score()
+    step.run_loss()
+    torch.cuda.synchronize()
+    assert lib.device_error() == 0
+    got = {k: v.cpu() for k, v in step.score.items()}
+    for n in ("first_trans", "n_emit", "next_driver", "new_len", "done", "source"):
+        assert torch.equal(got[n], sc[n]), n
+    assert torch.equal(step.out8.cpu(), o8)
+    cu = step.cu_span.cpu()
+    pos = torch.arange(step.T) - torch.repeat_interleave(cu[:-1], cu[1:] - cu[:-1])
+    first = torch.repeat_interleave(sc["first_trans"], cu[1:] - cu[:-1])
+    dec = pos <= first
+    for n in ("logp_s", "logp_t", "feedback", "kl_rev", "kl_fwd"):
+        assert torch.equal(got[n][emitted], sc[n][emitted]), n
+    for n in ("covered", "margin"):
+        assert torch.equal(got[n][dec], sc[n][dec]), n
     del step, w
     torch.cuda.empty_cache()

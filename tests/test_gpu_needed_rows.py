@@ -1,0 +1,107 @@
+"""The needed-rows vocabulary pass (ipd_score_span_needed) on the GPU: only
+the verifier's rows up to each request's first transition and the
+proposer's rows of the emitted positions are defined, and must match the
+fp64 oracle there; the verdict, the sources and the loss must match too."""
+import numpy as np
+import pytest
+import torch
+
+import ipd_synth as S
+from tests import parity
+
+pytestmark = pytest.mark.gpu
+
+SCORE_REQ = ("first_trans", "n_emit", "next_driver", "new_len", "done")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_36546_gb300 import ipd
+    return ipd
+
+
+def _step(spec, seed, rows):
+    from paper_2609_36546_gb300 import VerifyStep
+    w = S.make_workload(spec, seed=seed, device="cpu")
+    step = VerifyStep.from_workload(w, device="cuda", rows=rows)
+    step.run()
+    torch.cuda.synchronize()
+    return w, step
+
+
+CASES = [
+    ("mixed", S.small_spec(), 0),
+    ("teacher-driving", S.small_spec(n_req=6, direction="T", span=(1, 16), ctx=(20, 700)), 4),
+    ("ties", S.small_spec(n_req=6, vocab=4096, sigma=3.0, tie_quantum=0.5, span=(2, 6)), 5),
+    ("accept-all", S.small_spec(n_req=5, force="accept", span=(3, 9)), 6),
+    ("reject-all", S.small_spec(n_req=5, force="reject", span=(3, 9)), 7),
+    ("mixed-eos", S.small_spec(n_req=10, force="mixed", eos_id=5, eos_prob=0.3, span=(2, 10)), 8),
+    ("K1", S.small_spec(n_req=4, K=1), 9),
+    ("K32", S.small_spec(n_req=4, K=32, vocab=8192), 10),
+    ("wide-vocab", S.small_spec(n_req=2, vocab=151936, sigma=3.0, logits="boost", span=(4, 8),
+                                ctx=(100, 400)), 12),
+    # enough rows for several waves of row CTAs: later positions find their
+    # request's transition already known and are skipped
+    ("many-rows", S.small_spec(n_req=160, vocab=4096, span=(8, 16), ctx=(16, 64), force="mixed"),
+     18),
+    ("many-rows-teacher", S.small_spec(n_req=160, vocab=4096, span=(8, 16), ctx=(16, 64),
+                                       direction="T"), 19),
+]
+
+
+@pytest.mark.parametrize("name,spec,seed", CASES, ids=[c[0] for c in CASES])
+def test_needed_rows_match_oracle(lib, name, spec, seed):
+    """Scores where defined, every decision, and the whole batch's loss (the
+    attention of these steps is the same launch the other tests check)."""
+    w, step = _step(spec, seed, "needed")
+    assert lib.device_error() == 0
+    rep, orc = parity.check_scores(step, None, needed=True)
+    rep.update(parity.check_loss(step, orc))
+    assert rep["score_ok"] and rep["loss_ok"], rep
+
+
+@pytest.mark.parametrize("name,spec,seed", CASES[-2:], ids=[c[0] for c in CASES[-2:]])
+def test_needed_rows_equal_all_rows_where_defined(lib, name, spec, seed):
+    """Every row is read in one part by both passes here, so the values a
+    needed-rows pass defines are bit-identical to the full pass's, and so are
+    the decisions and the loss; rows past known transitions were skipped."""
+    _, full = _step(spec, seed, "all")
+    ref = {k: v.cpu() for k, v in full.score.items()}
+    ref8 = full.out8.cpu()
+    full.rows = "needed"
+    full.run_score()
+    full.run_loss()
+    torch.cuda.synchronize()
+    assert lib.device_error() == 0
+    got = {k: v.cpu() for k, v in full.score.items()}
+    for n in SCORE_REQ + ("source",):
+        assert torch.equal(got[n], ref[n]), n
+    assert torch.equal(full.out8.cpu(), ref8)
+    cu = full.cu_span.cpu().numpy()
+    src, ft = ref["source"].numpy(), ref["first_trans"].numpy()
+    em = np.zeros(full.T, bool)
+    dec = np.zeros(full.T, bool)
+    for r in range(full.R):
+        e, d = parity.needed_positions(src, ft, cu, r)
+        em[cu[r]:cu[r + 1]] = e
+        dec[cu[r]:cu[r + 1]] = d
+    for n in ("logp_s", "logp_t", "feedback", "kl_rev", "kl_fwd"):
+        assert torch.equal(got[n][em], ref[n][em]), n
+    for n in ("covered", "margin"):
+        assert torch.equal(got[n][dec], ref[n][dec]), n
+    # positions past the transitions: some rows were not read at all
+    skipped = torch.isnan(got["logp_s"][~torch.from_numpy(dec)])
+    assert int(skipped.sum()) > 0
+
+
+def test_span_longer_than_the_bound_is_reported(lib):
+    w, step = _step(S.small_spec(n_req=4, span=(5, 9)), 21, "needed")
+    assert lib.device_error() == 0
+    step.max_span = int(w.span.max()) - 1
+    step.run_score()
+    torch.cuda.synchronize()
+    assert lib.device_error() == 6  # IPD_DEVERR_SPAN
