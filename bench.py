@@ -360,7 +360,17 @@ def measure_config(cfg, K, W, world, rank, stream, sampler=None, rows="needed"):
     attn_bytes = step.attn_bytes(w.ctx)
     logits_alg = step.logits_bytes_alg()
     logits_full = step.logits_bytes_full()
-    accept_rate = float(step.score["covered"].float().mean()) if T_tok else 0.0
+    # coverage among the positions up to each request's first transition (the
+    # ones both vocabulary passes decide; the needed-rows pass leaves later
+    # positions unread)
+    if T_tok:
+        cu = step.cu_span.cpu()
+        lens = cu[1:] - cu[:-1]
+        pos = torch.arange(T_tok) - torch.repeat_interleave(cu[:-1], lens)
+        dec = pos <= torch.repeat_interleave(step.score["first_trans"].cpu(), lens)
+        accept_rate = float(step.score["covered"].cpu()[dec].float().mean())
+    else:
+        accept_rate = 0.0
     emitted = int(step.score["n_emit"].sum())
 
     # ---- K steps call by call, per-call events on the launching stream ----
@@ -450,7 +460,8 @@ def measure_config(cfg, K, W, world, rank, stream, sampler=None, rows="needed"):
         "calls_ms": {"verify_attn": attn_ms, "score_span": score_ms, "split_loss": loss_ms},
         "ms_per_step_one_stream_graph": ms_step_one_stream,
         "ms_per_step_direct_calls": _max_over_ranks(el_direct_ms, world) / K,
-        "acceptance": {"coverage_rate": accept_rate, "emitted_tokens_per_step": emitted},
+        "acceptance": {"coverage_rate_to_transition": accept_rate,
+                       "emitted_tokens_per_step": emitted},
     }
     return step, w, fig
 

@@ -105,3 +105,50 @@ def test_span_longer_than_the_bound_is_reported(lib):
     step.run_score()
     torch.cuda.synchronize()
     assert lib.device_error() == 6  # IPD_DEVERR_SPAN
+
+
+def _defined(step, score):
+    """Masks of the positions a needed-rows pass defines, from its verdict."""
+    cu = step.cu_span.cpu()
+    lens = cu[1:] - cu[:-1]
+    pos = torch.arange(step.T) - torch.repeat_interleave(cu[:-1], lens)
+    dec = pos <= torch.repeat_interleave(score["first_trans"].cpu(), lens)
+    return score["source"].cpu() != 255, dec
+
+
+@pytest.mark.parametrize("graph", [False, True])
+def test_needed_rows_from_host_equals_direct_calls(lib, graph):
+    """The host-fed step (logits in request-aligned chunks, each scored as it
+    lands, directly or replayed from a graph) gives the direct step's
+    decisions, loss and defined values, bit for bit."""
+    w, step = _step(S.small_spec(n_req=40, ctx=(100, 900), span=(0, 16), vocab=4096), 45,
+                    "needed")
+    first = {k: v.cpu() for k, v in step.score.items()}
+    o8 = step.out8.cpu()
+    em, dec = _defined(step, first)
+    host = step.host_inputs(3)
+    results = step.host_results()
+    g = step.capture_from_host(host, results) if graph else None
+    for _ in range(2):
+        for v in step.score.values():
+            v.zero_()
+        step.logits_s.zero_()
+        step.logits_t.zero_()
+        step.out8.zero_()
+        step._in.buf.zero_()
+        if g is not None:
+            g.replay()
+        else:
+            step.run_from_host(host, results, torch.cuda.current_stream())
+        torch.cuda.synchronize()
+        got = {k: v.cpu() for k, v in step.score.items()}
+        for n in SCORE_REQ + ("source",):
+            assert torch.equal(got[n], first[n]), n
+            assert torch.equal(results[n], first[n]), n
+        for n in ("logp_s", "logp_t", "feedback", "kl_rev", "kl_fwd"):
+            assert torch.equal(got[n][em], first[n][em]), n
+        for n in ("covered", "margin"):
+            assert torch.equal(got[n][dec], first[n][dec]), n
+        assert torch.equal(step.out8.cpu(), o8)
+        assert torch.equal(results["out8"], o8)
+    assert lib.device_error() == 0
