@@ -15,6 +15,10 @@
  *                    teacher-feedback term, top-K coverage, union-support
  *                    top-K KL in both directions, the accept / takeover /
  *                    handback verdict and the new cache lengths.
+ *   ipd_score_span_needed  the same verdict and loss inputs from only the
+ *                    logits rows they need (the verifier's up to each
+ *                    request's first transition, the proposer's at the
+ *                    emitted positions).
  *   ipd_split_loss   the source-split objective of the step.
  *
  * Beyond the step itself: ipd_score_span_ex (other takeover / handback rules,
