@@ -208,6 +208,8 @@ int ipd_score_span(const uint16_t *logits_student, const uint16_t *logits_teache
  * so neither model's row there enters the verdict or the loss).  Rows past a
  * transition that is already known when their turn comes are not read; the
  * rest are read as by ipd_score_span, position 0 of every request first.
+ * A call whose rows all fit one wave of row CTAs reads every row (no
+ * transition is known before every row has started).
  *
  * Arguments as for ipd_score_span, plus
  *  max_span       an upper bound (1 .. 65535) on every request's span length;

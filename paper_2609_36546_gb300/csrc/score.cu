@@ -432,7 +432,7 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     float *feedback,
     float *kl_rev, float *kl_fwd, uint8_t *covered, float *margin, uint8_t *source,
     int32_t *first_trans, int32_t *n_emit, uint8_t *next_driver, int32_t *new_len, uint8_t *done,
-    int total_tokens, const EpiOpts opt, int max_span = 0) {
+    int total_tokens, const EpiOpts opt, int max_span = 0, bool needed_rows = false) {
   // No shared memory.  In a step that forks the vocabulary pass onto its
   // own stream, this kernel's CTAs take the SMs that the first attention
   // CTAs to finish leave free, so it runs inside the attention's tail.
@@ -445,8 +445,8 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     return;
   }
   const int k = t1 - t0;
-  // after a needed-rows pass (max_span > 0) a span longer than its bound was
-  // read only in part: its verdict would be wrong
+  // a span longer than the bound a needed-rows call was given (max_span > 0)
+  // would have been read only in part
   if (max_span > 0 && k > max_span) {
     if (threadIdx.x == 0) ipd_set_error(&g_score_err, IPD_DEVERR_SPAN);
     return;
@@ -564,8 +564,8 @@ __global__ void __launch_bounds__(kEpiThreads) score_epilogue_kernel(
     const int n_common = __popc(__ballot_sync(0xffffffffu, lane < K && dupT));
     // a needed-rows pass leaves the rows past the transition unread: the
     // values that would come from them are NaN (coverage 0)
-    const bool skip_s = max_span > 0 && rows[(size_t)2 * t * parts].skipped;
-    const bool skip_t = max_span > 0 && rows[(size_t)(2 * t + 1) * parts].skipped;
+    const bool skip_s = needed_rows && rows[(size_t)2 * t * parts].skipped;
+    const bool skip_t = needed_rows && rows[(size_t)(2 * t + 1) * parts].skipped;
     const bool skip_ver = drv ? skip_s : skip_t;
     if (lane == 0) {
       const float lps = lxS - logz[0], lpt = lxT - logz[1];
@@ -794,6 +794,29 @@ extern "C" int ipd_score_span_needed(const uint16_t *logits_student,
   RowOut *rows = static_cast<RowOut *>(workspace);
   int *trans = reinterpret_cast<int *>(static_cast<char *>(workspace) +
                                        trans_offset(num_reqs, total_tokens, vocab));
+  // When every row CTA fits one wave, every row starts before any transition
+  // is known: the full pass (rows in up to four parts) is then as fast or
+  // faster, and defines every position.
+  const int parts = row_parts(total_tokens, vocab, kMaxParts);
+  int dev = 0;
+  const bool one_wave = cudaGetDevice(&dev) == cudaSuccess && dev >= 0 && dev < 64 &&
+                        g_sms[dev] > 0 &&
+                        2LL * total_tokens <= (long long)kRowCtasPerSm * g_sms[dev];
+  if (one_wave) {
+    if (total_tokens > 0) {
+      score_rows_kernel<false, false><<<2 * parts * total_tokens, kRowThreads, 0, st>>>(
+          logits_student, logits_teacher, vocab, K, parts, rows, NeededRows{});
+      if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
+    }
+    score_epilogue_kernel<<<num_reqs, kEpiThreads, 0, st>>>(
+        logits_student, logits_teacher, tokens, cu_span, driver, prefix_len, vocab, K, eos_id,
+        rows, parts, logp_s, logp_t, feedback, kl_rev, kl_fwd, covered, margin, source,
+        first_trans, n_emit, next_driver, new_len, done, total_tokens,
+        EpiOpts{IPD_RULE_TOPK, IPD_RULE_TOPK, 0.f, 0.f, nullptr, nullptr, nullptr, nullptr,
+                nullptr},
+        max_span, false);
+    return cudaGetLastError() == cudaSuccess ? IPD_OK : IPD_ERR_CUDA;
+  }
   if (total_tokens > 0) {
     // every bound starts above any position (0x7f7f7f7f)
     if (cudaMemsetAsync(trans, 0x7f, (size_t)num_reqs * sizeof(int), st) != cudaSuccess)
@@ -808,7 +831,7 @@ extern "C" int ipd_score_span_needed(const uint16_t *logits_student,
       1, logp_s, logp_t, feedback, kl_rev, kl_fwd, covered, margin, source, first_trans, n_emit,
       next_driver, new_len, done, total_tokens,
       EpiOpts{IPD_RULE_TOPK, IPD_RULE_TOPK, 0.f, 0.f, nullptr, nullptr, nullptr, nullptr, nullptr},
-      max_span);
+      max_span, true);
   if (cudaGetLastError() != cudaSuccess) return IPD_ERR_CUDA;
   return IPD_OK;
 }

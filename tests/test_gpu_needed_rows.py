@@ -121,7 +121,8 @@ def test_needed_rows_from_host_equals_direct_calls(lib, graph):
     """The host-fed step (logits in request-aligned chunks, each scored as it
     lands, directly or replayed from a graph) gives the direct step's
     decisions, loss and defined values, bit for bit."""
-    w, step = _step(S.small_spec(n_req=40, ctx=(100, 900), span=(0, 16), vocab=4096), 45,
+    # chunks of more rows than one wave of row CTAs holds, so that rows are skipped
+    w, step = _step(S.small_spec(n_req=400, ctx=(20, 200), span=(0, 16), vocab=4096), 45,
                     "needed")
     first = {k: v.cpu() for k, v in step.score.items()}
     o8 = step.out8.cpu()
