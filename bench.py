@@ -11,6 +11,7 @@ step streams its KV pages and logits from DRAM.
   python bench.py [--gpus N] [--steps K] [--warmup W] [--config I] [--impl reference]
   python bench.py --next-rows [--config I] [--steps K]
   python bench.py --attn-only [--config I] [--requests R] [--direction S|T] [--span LO HI]
+  python bench.py --score-only [--config I] [--requests R] [--rows needed|all]
 
 The headline workload is the full rollout-step mix (1024 requests, lognormal
 contexts up to 32K, spans of 1-16 tokens, both directions, 120 GB of KV
@@ -785,19 +786,11 @@ def run_next_rows(args):
     print(json.dumps(line), flush=True)
 
 
-def run_attn_only(args):
-    """--attn-only: only the attention call (planner + attention launch) of a
-    workload shaped like configuration --config, optionally with fewer
-    requests (--requests; pools then hold only the pages used), one direction
-    (--direction S|T) or other span lengths (--span LO HI).  A small case of
-    this kind is what an ncu capture runs; it prints one JSON line with the
-    algorithmic bytes and the mean time of the attention launch."""
+def _reduced_workload(args):
+    """The workload of configuration --config with the --requests,
+    --direction and --span changes (pools then hold only the pages used)."""
     import dataclasses
-    import torch
-    import __graft_entry__
-    __graft_entry__.build()
     import ipd_synth as S
-    from paper_2609_36546_gb300 import VerifyStep, ipd
     spec = S.CONFIGS[args.config]
     changes = {}
     if args.requests:
@@ -810,7 +803,63 @@ def run_attn_only(args):
         spec = dataclasses.replace(spec, name=spec.name + " (shape kept, " +
                                    ", ".join(f"{k}={v}" for k, v in changes.items()) + ")",
                                    **changes)
-    w = S.make_workload(spec, seed=args.config, device="cuda")
+    return spec, S.make_workload(spec, seed=args.config, device="cuda")
+
+
+def run_score_only(args):
+    """--score-only: only the vocabulary pass and verdict of a workload shaped
+    like configuration --config (same changes as --attn-only), in the mode
+    --rows names; the case an ncu capture of the row kernel runs.  Prints one
+    JSON line: the rows read, the bytes they hold, and the mean call time."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_36546_gb300 import VerifyStep, ipd
+    spec, w = _reduced_workload(args)
+    step = VerifyStep.from_workload(w, device="cuda", rows=args.rows)
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        step.run_score(stream)
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        step.run_score(stream)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    if ipd.device_error() != 0:
+        raise RuntimeError("device-side check failed")
+    ms = t0.elapsed_time(t1) / max(args.steps, 1)
+    row_bytes = step.V * 2
+    # rows the last call read: the row records' "not read" flags (one record
+    # of 272 bytes per row; the needed-rows pass writes every flag of a call
+    # that spans several waves, a one-wave call reads every row)
+    n_rows = 2 * step.T
+    if args.rows == "needed":
+        rec = step.ws_score[:n_rows * 272].view(n_rows, 272)[:, 12:16].contiguous()
+        flags = rec.view(torch.int32).flatten()
+        read = int((flags == 0).sum()) if 2 * step.T > 8 * torch.cuda.get_device_properties(
+            0).multi_processor_count else n_rows
+    else:
+        read = n_rows
+    print(json.dumps({"workload": spec.name, "requests": spec.n_req, "rows": args.rows,
+                      "logits_rows": n_rows, "rows_read": read, "bytes_read": read * row_bytes,
+                      "emitted": int(step.score["n_emit"].sum()), "ms_per_call": ms,
+                      "calls": args.steps}), flush=True)
+
+
+def run_attn_only(args):
+    """--attn-only: only the attention call (planner + attention launch) of a
+    workload shaped like configuration --config, optionally with fewer
+    requests (--requests; pools then hold only the pages used), one direction
+    (--direction S|T) or other span lengths (--span LO HI).  A small case of
+    this kind is what an ncu capture runs; it prints one JSON line with the
+    algorithmic bytes and the mean time of the attention launch."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_36546_gb300 import VerifyStep, ipd
+    spec, w = _reduced_workload(args)
     step = VerifyStep.from_workload(w, device="cuda")
     stream = torch.cuda.current_stream()
     for _ in range(args.warmup):
@@ -852,18 +901,23 @@ def main():
                     help="time the calls beyond the step instead (one GPU)")
     ap.add_argument("--attn-only", action="store_true",
                     help="time only the attention call (profiling cases; one GPU)")
+    ap.add_argument("--score-only", action="store_true",
+                    help="time only the vocabulary pass and verdict (profiling cases; one GPU)")
     ap.add_argument("--requests", type=int, default=0,
-                    help="--attn-only: requests of the workload (pools sized to them)")
+                    help="--attn-only / --score-only: requests of the workload (pools sized "
+                         "to them)")
     ap.add_argument("--direction", choices=["S", "T", "half", "bernoulli"], default=None,
-                    help="--attn-only: which model proposes")
+                    help="--attn-only / --score-only: which model proposes")
     ap.add_argument("--span", type=int, nargs=2, default=None,
-                    help="--attn-only: span lengths drawn uniformly in [LO, HI]")
+                    help="--attn-only / --score-only: span lengths drawn uniformly in [LO, HI]")
     args = ap.parse_args()
     args.warmup = max(3, args.warmup)
     if args.next_rows:
         run_next_rows(args)
     elif args.attn_only:
         run_attn_only(args)
+    elif args.score_only:
+        run_score_only(args)
     elif args.impl == "reference":
         run_reference(args)
     else:
