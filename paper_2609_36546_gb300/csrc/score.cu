@@ -133,10 +133,11 @@ __device__ __forceinline__ unsigned long long warp_top32_u64(unsigned long long 
 // to the warp's buffer, which is cut back to its best K (by rank) when it
 // fills, and the warps' lists are merged by rank.
 // The needed-rows pass (kNeeded) reads only the rows that the verdict and the
-// emitted positions need.  Its grid is (2 R, max span): block (2 r + model,
-// i) takes row `model` of request r's span position i, so the blocks of
-// position 0 of every request are dispatched first, then position 1, and so
-// on.  A verifier row whose token decides the verdict (not covered under a
+// emitted positions need.  Its grid is (2 R, max span): block (r, i) takes
+// the verifier's row of request r's span position i and block (R + r, i) the
+// proposer's, so the blocks of position 0 of every request are dispatched
+// first (the verifiers' rows before the proposers'), then position 1, and
+// so on.  A verifier row whose token decides the verdict (not covered under a
 // student-driven span, covered under a teacher-driven one) lowers the
 // request's transition bound trans[r]; a block whose position lies past the
 // bound it reads skips its row: the verifier's rows are needed up to the
@@ -168,14 +169,19 @@ __global__ void __launch_bounds__(kRowThreads, kRowCtasPerSm) score_rows_kernel(
   int row_id = blockIdx.x / parts, part = blockIdx.x % parts, oi = blockIdx.x;
   int r = 0, pos = 0, drv = 0, ver = 0;
   if (kNeeded) {
-    r = blockIdx.x >> 1;
+    // blocks 0 .. R-1 of a position take the verifiers' rows, R .. 2R-1 the
+    // proposers', so a proposer's row starts after its verifier's when the
+    // position spans more than one wave
+    const int R = gridDim.x >> 1;
+    const bool is_ver = (int)blockIdx.x < R;
+    r = is_ver ? blockIdx.x : blockIdx.x - R;
     pos = blockIdx.y;
     const int t0 = nr.cu_span[r], k = nr.cu_span[r + 1] - t0;
     // no such position (or offsets the epilogue reports as broken)
     if (pos >= k || t0 < 0 || t0 + k > nr.total_tokens) return;
     drv = nr.driver[r] ? 1 : 0;
     ver = drv ? 0 : 1;  // the verifier's row: the teacher's when the student drives
-    row_id = 2 * (t0 + pos) + (int)(blockIdx.x & 1);
+    row_id = 2 * (t0 + pos) + (is_ver ? ver : 1 - ver);
     part = 0;
     oi = row_id;
     const int tr = *reinterpret_cast<volatile const int *>(nr.trans + r);
