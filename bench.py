@@ -831,17 +831,21 @@ def run_score_only(args):
         raise RuntimeError("device-side check failed")
     ms = t0.elapsed_time(t1) / max(args.steps, 1)
     row_bytes = step.V * 2
-    # rows the last call read: the row records' "not read" flags (one record
-    # of 272 bytes per row; the needed-rows pass writes every flag of a call
-    # that spans several waves, a one-wave call reads every row)
+    # rows one more call reads: the row records' "not read" flags (one record
+    # of 272 bytes per row, the flag at byte 12), preset to 2.  A needed-rows
+    # pass over several waves writes every flag (0 read, 1 skipped); a call
+    # that leaves them at 2 took the full pass and read every row.
     n_rows = 2 * step.T
-    if args.rows == "needed":
-        rec = step.ws_score[:n_rows * 272].view(n_rows, 272)[:, 12:16].contiguous()
-        flags = rec.view(torch.int32).flatten()
-        read = int((flags == 0).sum()) if 2 * step.T > 8 * torch.cuda.get_device_properties(
-            0).multi_processor_count else n_rows
-    else:
-        read = n_rows
+    read = n_rows
+    if args.rows == "needed" and n_rows:
+        flags = step.ws_score[:n_rows * 272].view(n_rows, 272)[:, 12:16]
+        flags.copy_(torch.tensor([2, 0, 0, 0], dtype=torch.uint8, device=flags.device)
+                    .expand_as(flags))
+        step.run_score(stream)
+        torch.cuda.synchronize()
+        f = flags.contiguous().view(torch.int32).flatten()
+        if not bool((f == 2).all()):
+            read = int((f == 0).sum())
     print(json.dumps({"workload": spec.name, "requests": spec.n_req, "rows": args.rows,
                       "logits_rows": n_rows, "rows_read": read, "bytes_read": read * row_bytes,
                       "emitted": int(step.score["n_emit"].sum()), "ms_per_call": ms,
