@@ -789,3 +789,42 @@ def test_kv_append_then_paged_attention_equals_sdpa_on_the_concatenation():
     kb, vb = O.kv_append(kp, vp, kn, vn, cu, [x + 1 for x in L], np.pad(table, ((0, 0), (0, 1)),
                                                                        constant_values=perm[-1]))
     assert not np.array_equal(O.gather_pages(kb, table[0], L[0]), np.concatenate([old_k[0], kn[0:3]]))
+
+
+@pytest.mark.parametrize("driver", [0, 1])
+def test_rows_past_the_transition_do_not_change_the_verdict_or_the_loss(driver):
+    """Reading R22: the verdict needs the verifier's rows up to the first
+    transition, the loss the emitted positions' rows.  Replacing every row the
+    reading calls unneeded (the verifier's past the transition, the proposer's
+    at positions not emitted) leaves the verdict, the sources and the loss of
+    the oracle unchanged."""
+    for seed in range(12):
+        ls, lt, toks = _span(10, V=32, seed=100 + seed)
+        o = _run_rules(ls, lt, toks, driver)
+        ft, n = int(o["first_trans"][0]), int(o["n_emit"][0])
+        g = np.random.default_rng(seed)
+        ls2, lt2 = ls.copy(), lt.copy()
+        ver, prop = (lt2, ls2) if driver == 0 else (ls2, lt2)
+        for i in range(10):
+            if i > ft:
+                ver[i] = _bf16_round(g.normal(size=32) * 2)
+            if i >= n:
+                prop[i] = _bf16_round(g.normal(size=32) * 2)
+        o2 = _run_rules(ls2, lt2, toks, driver)
+        for name in ("first_trans", "n_emit", "next_driver", "new_len", "done", "source"):
+            assert np.array_equal(o[name], o2[name]), name
+        em = o["source"] != O.SRC_DISCARDED
+        for name in ("kl_rev", "kl_fwd", "logp_s", "logp_t"):
+            assert np.array_equal(o[name][em], o2[name][em]), name
+        l1 = O.split_loss(o["kl_rev"], o["kl_fwd"], o["source"], np.array([0, 10]), o["n_emit"])
+        l2 = O.split_loss(o2["kl_rev"], o2["kl_fwd"], o2["source"], np.array([0, 10]),
+                          o2["n_emit"])
+        assert l1["loss"] == l2["loss"]
+    # and a row the reading does need changes the verdict when it is replaced
+    ls, lt, toks = _span(10, V=32, seed=7)
+    o = _run_rules(ls, lt, toks, 0)
+    ft = int(o["first_trans"][0])
+    assert ft < 10  # this span has a takeover
+    lt2 = lt.copy()
+    lt2[ft, toks[ft]] = 50.0  # the verifier's row at the transition now covers the token
+    assert _run_rules(ls, lt2, toks, 0)["first_trans"][0] != ft
