@@ -545,40 +545,74 @@ def run_gpu(args):
 def run_e2e(step, w, K, stream, world):
     """The same step through host buffers, via VerifyStep.run_from_host: the
     per-step inputs (queries and their metadata, both models' logits, tokens,
-    request metadata) are copied from pinned host memory, the step runs, and
-    its results (per-request verdict, per-token sources, loss record) are
-    copied back and read before the next step; the KV pools stay resident
-    (they are the cache state, not step inputs).  The attention starts when
-    the queries land and the logits are scored chunk by chunk as they land,
-    so the step's time is about the host-to-device transfer.  The step, its
+    request metadata) come from pinned host memory, the step runs, and its
+    results (per-request verdict, per-token sources, loss record) are copied
+    back and read before the next step; the KV pools stay resident (they are
+    the cache state, not step inputs).  Queries and metadata go in one copy
+    and the attention starts when they land.  With the needed-rows
+    vocabulary pass and logits the device can read in place, the pass reads
+    its rows straight from host memory, so only the rows it needs cross the
+    link (counted from the row records' "not read" flags); otherwise the
+    logits are copied in four chunks, each scored as it lands.  The step, its
     copies included, is replayed from one CUDA graph
     (VerifyStep.capture_from_host)."""
     import torch
+    from paper_2609_36546_gb300 import ipd
     host = step.host_inputs(n_chunks=4)
     results = step.host_results()
-    # bytes copied per step: the packed inputs, both models' logits, the packed results
-    h2d = host["_arena"].numel() + sum(host[k].numel() * host[k].element_size()
-                                       for k in ("logits_s", "logits_t"))
     d2h = results["_arena"].numel()
-    graph = step.capture_from_host(host, results)
-    for _ in range(2):
-        graph.replay()
+    in_place = step.rows == "needed" and ipd.device_readable(host["logits_s"]) and \
+        ipd.device_readable(host["logits_t"])
+
+    def timed(host_logits):
+        graph = step.capture_from_host(host, results, host_logits=host_logits)
+        for _ in range(2):
+            graph.replay()
+            stream.synchronize()
+        _barrier(world)
+        t0 = time.perf_counter()
+        for _ in range(K):
+            graph.replay()                # inputs in, the step, results out
+            stream.synchronize()          # the engine reads the verdict before the next step
+        el = _max_over_ranks(time.perf_counter() - t0, world)
+        del graph
+        return _sum_over_ranks(float(step.T * K), world) / el
+
+    row_bytes = step.V * 2
+    all_rows = 2 * step.T * row_bytes
+    copy_all = timed(False)
+    out = {"unit": UNIT, "d2h_bytes_per_step": d2h, "steps": K,
+           "copy_all_logits": {"value": copy_all,
+                               "h2d_bytes_per_step": host["_arena"].numel() + all_rows}}
+    if in_place:
+        value = timed(True)
+        # rows one more such step reads: the row records' flags (byte 12 of
+        # each 272-byte record), preset to 2; the pass sets 0 (read) or 1 (not
+        # read), or leaves them when it read every row in one wave
+        n = 2 * step.T
+        flags = step.ws_score[:n * 272].view(n, 272)[:, 12:16]
+        flags.copy_(torch.tensor([2, 0, 0, 0], dtype=torch.uint8, device=flags.device)
+                    .expand_as(flags))
+        step.run_from_host(host, results, stream, host_logits=True)
         stream.synchronize()
-    _barrier(world)
-    t0 = time.perf_counter()
-    for _ in range(K):
-        graph.replay()                # copies in, the step, results out
-        stream.synchronize()          # the engine reads the verdict before the next step
-    el = time.perf_counter() - t0
-    el = _max_over_ranks(el, world)
-    toks = _sum_over_ranks(float(step.T * K), world)
-    return {"value": toks / el, "unit": UNIT, "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h, "steps": K,
-            "note": "pinned host -> device inputs (Q, tokens and metadata in one copy, the "
-                    "logits in 4 chunks) and device -> host results (one copy) each step, "
-                    "synchronised per step; KV pools resident; the attention overlaps the logits "
-                    "transfer, and each chunk is scored as it lands; the step with its copies "
-                    "replayed from one CUDA graph"}
+        f = flags.contiguous().view(torch.int32).flatten()
+        read = n if bool((f == 2).all()) else int((f == 0).sum())
+        out.update({"value": value, "h2d_bytes_per_step": host["_arena"].numel() + read * row_bytes,
+                    "logits_rows_read_last_step": read, "logits_rows": n,
+                    "note": "pinned host inputs: queries, tokens and metadata in one copy; the "
+                            "vocabulary pass reads the logits rows it needs from pinned host "
+                            "memory in place (the rest never cross the link); results back in "
+                            "one copy; synchronised per step; KV pools resident; the step "
+                            "replayed from one CUDA graph. copy_all_logits: the same step "
+                            "copying both models' logits in four chunks first"})
+    else:
+        out.update({"value": copy_all, "h2d_bytes_per_step": host["_arena"].numel() + all_rows,
+                    "note": "pinned host -> device inputs (Q, tokens and metadata in one copy, "
+                            "the logits in 4 chunks) and device -> host results (one copy) each "
+                            "step, synchronised per step; KV pools resident; the attention "
+                            "overlaps the logits transfer, and each chunk is scored as it lands; "
+                            "the step with its copies replayed from one CUDA graph"})
+    return out
 
 
 # ---------------------------------------------------------------------------

@@ -483,6 +483,14 @@ const char *ipd_status_string(int status);
 /* Library version, e.g. 100 for 0.1.0. */
 int ipd_version(void);
 
+/* Whether the current device's kernels can read `ptr` at that same address:
+ * device memory of the current device, managed memory, or page-locked host
+ * memory mapped into the device's address space (cudaHostAlloc under unified
+ * addressing).  *readable = 1 or 0; a pointer CUDA does not know is 0.  Lets
+ * a caller hand host-resident inputs (for example logits rows) to the calls
+ * directly, so that only the bytes a kernel reads cross the host link. */
+int ipd_device_readable(const void *ptr, int *readable);
+
 #ifdef __cplusplus
 }
 #endif

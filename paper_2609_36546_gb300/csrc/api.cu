@@ -36,3 +36,20 @@ extern "C" const char *ipd_status_string(int status) {
 }
 
 extern "C" int ipd_version(void) { return 100; }
+
+extern "C" int ipd_device_readable(const void *ptr, int *readable) {
+  if (!readable) return IPD_ERR_INVALID_ARG;
+  *readable = 0;
+  if (!ptr) return IPD_OK;
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, ptr) != cudaSuccess) {
+    (void)cudaGetLastError();  // an unregistered host pointer is not an error state
+    return IPD_OK;
+  }
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return IPD_ERR_CUDA;
+  if (a.type == cudaMemoryTypeDevice) *readable = a.device == dev;
+  else if (a.type == cudaMemoryTypeManaged) *readable = 1;
+  else if (a.type == cudaMemoryTypeHost) *readable = a.devicePointer == ptr;
+  return IPD_OK;
+}

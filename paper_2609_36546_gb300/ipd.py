@@ -34,7 +34,7 @@ EXPORTS = ("ipd_attn_workspace_size", "ipd_verify_attn", "ipd_decode_attn",
            "ipd_score_span_static", "ipd_score_span_ex", "ipd_score_span_needed", "ipd_full_kl",
            "ipd_loss_grad_workspace_size", "ipd_split_loss_grad", "ipd_sample_workspace_size",
            "ipd_sample", "ipd_kv_append", "ipd_kv_append_many", "ipd_set_attn_kernel_timing",
-           "ipd_attn_kernel_time")
+           "ipd_attn_kernel_time", "ipd_device_readable")
 # takeover / handback rules (IPD_RULE_*)
 RULE_TOPK, RULE_ENTROPY_S, RULE_ENTROPY_T, RULE_ALWAYS, RULE_NEVER = 0, 1, 2, 3, 4
 # element type of the dense gradient (IPD_DTYPE_*)
@@ -102,6 +102,8 @@ _lib.ipd_score_workspace_size.restype = c_sz
 _lib.ipd_score_workspace_size.argtypes = [c_i, c_i, c_i, c_i]
 _lib.ipd_score_span.restype = c_i
 _lib.ipd_score_span.argtypes = [c_p] * 6 + [c_i] * 5 + [c_p] * 13 + [c_p, c_sz, c_p]
+_lib.ipd_device_readable.restype = c_i
+_lib.ipd_device_readable.argtypes = [c_p, ctypes.POINTER(c_i)]
 _lib.ipd_score_span_needed.restype = c_i
 _lib.ipd_score_span_needed.argtypes = [c_p] * 6 + [c_i] * 6 + [c_p] * 13 + [c_p, c_sz, c_p]
 _lib.ipd_score_span_ex.restype = c_i
@@ -254,6 +256,14 @@ def score_span(logits_student, logits_teacher, tokens, cu_span, driver, prefix_l
         *[_ptr(out[n]) for n, _ in SCORE_REQ_OUTPUTS],
         _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(stream)),
         "ipd_score_span")
+
+
+def device_readable(t: torch.Tensor) -> bool:
+    """Whether the library's kernels can read tensor t where it lives (device
+    memory, or pinned host memory mapped into the device's address space)."""
+    r = c_i(0)
+    _check(_lib.ipd_device_readable(_ptr(t), ctypes.byref(r)), "ipd_device_readable")
+    return bool(r.value)
 
 
 def score_span_needed(logits_student, logits_teacher, tokens, cu_span, driver, prefix_len,

@@ -271,7 +271,7 @@ class VerifyStep:
         out["_arena"] = arena.buf
         return out
 
-    def run_from_host(self, host: dict, results: dict, stream=None):
+    def run_from_host(self, host: dict, results: dict, stream=None, host_logits: bool = False):
         """One step whose inputs sit in pinned host memory (``host_inputs``)
         and whose results (verdict per request, source per token, loss
         record) are copied back into ``results``: ``host_results()``, read
@@ -283,7 +283,19 @@ class VerifyStep:
         a copy stream in request-aligned chunks, and each chunk is scored as
         soon as it lands, so that only the last chunk's scoring and the loss
         follow the transfer.  Every kernel sees the same data as in run(), so
-        the results are bit-identical."""
+        the results are bit-identical.
+
+        host_logits=True (needed-rows steps only, with pinned logits the
+        device can read in place): the logits are not copied at all; the
+        vocabulary pass reads its rows from host memory, so only the rows the
+        verdict and the emitted positions need cross the host link."""
+        if host_logits:
+            if self.rows != "needed":
+                raise ValueError("host_logits needs a step with rows='needed'")
+            if not (ipd.device_readable(host["logits_s"]) and
+                    ipd.device_readable(host["logits_t"])):
+                raise ValueError("the host logits are not readable by the device in place")
+            return self._run_from_host_logits(host, results, stream)
         main = stream if stream is not None else torch.cuda.current_stream(self.device)
         if getattr(self, "_copy", None) is None:
             self._copy = torch.cuda.Stream(device=self.device)
@@ -327,20 +339,45 @@ class VerifyStep:
                 for name, t in results.items():
                     t.copy_(self.out8 if name == "out8" else self.score[name], non_blocking=True)
 
-    def capture_from_host(self, host: dict, results: dict, warmup: int = 2
-                          ) -> "torch.cuda.CUDAGraph":
+    def _run_from_host_logits(self, host: dict, results: dict, stream=None):
+        main = stream if stream is not None else torch.cuda.current_stream(self.device)
+        if getattr(self, "_scorer", None) is None:
+            self._copy = torch.cuda.Stream(device=self.device)
+            self._scorer = torch.cuda.Stream(device=self.device)
+        sc = self._scorer
+        sc.wait_stream(main)
+        with torch.cuda.stream(main):
+            self._in.buf.copy_(host["_arena"], non_blocking=True)
+        meta = torch.cuda.Event()
+        meta.record(main)
+        self.run_attention(main)
+        sc.wait_event(meta)
+        self._score_call(host["logits_s"], host["logits_t"], self.tokens, self.cu_span,
+                         self.driver, self.prefix_len, self.score, sc)
+        main.wait_stream(sc)
+        self.run_loss(main)
+        with torch.cuda.stream(main):
+            if "_arena" in results:
+                results["_arena"].copy_(self._res.buf, non_blocking=True)
+            else:
+                for name, t in results.items():
+                    t.copy_(self.out8 if name == "out8" else self.score[name], non_blocking=True)
+
+    def capture_from_host(self, host: dict, results: dict, warmup: int = 2,
+                          host_logits: bool = False) -> "torch.cuda.CUDAGraph":
         """run_from_host recorded as one CUDA graph: every copy and kernel of
         the step, with the same pinned host buffers and device buffers at
         each replay, without the per-call host work of issuing them."""
         side = torch.cuda.Stream(device=self.device)
         side.wait_stream(torch.cuda.current_stream(self.device))
         for _ in range(warmup):
-            self.run_from_host(host, results, side)
+            self.run_from_host(host, results, side, host_logits=host_logits)
         side.synchronize()
         torch.cuda.current_stream(self.device).wait_stream(side)
         graph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(graph):
-            self.run_from_host(host, results, torch.cuda.current_stream(self.device))
+            self.run_from_host(host, results, torch.cuda.current_stream(self.device),
+                               host_logits=host_logits)
         return graph
 
     # -- bytes the step must move (algorithmic) --------------------------------

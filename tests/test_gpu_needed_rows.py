@@ -153,3 +153,42 @@ def test_needed_rows_from_host_equals_direct_calls(lib, graph):
         assert torch.equal(step.out8.cpu(), o8)
         assert torch.equal(results["out8"], o8)
     assert lib.device_error() == 0
+
+
+def test_host_fed_step_reading_logits_in_place(lib):
+    """run_from_host(host_logits=True): the vocabulary pass reads the pinned
+    host logits in place (the device copies are zeroed first, so any use of
+    them would show); decisions, loss and defined values equal the
+    device-resident step's, bit for bit."""
+    w, step = _step(S.small_spec(n_req=400, ctx=(20, 200), span=(0, 16), vocab=4096), 47,
+                    "needed")
+    host = step.host_inputs(3)
+    if not (lib.device_readable(host["logits_s"]) and lib.device_readable(host["logits_t"])):
+        pytest.skip("pinned host memory is not mapped for the device here")
+    first = {k: v.cpu() for k, v in step.score.items()}
+    o8 = step.out8.cpu()
+    em, dec = _defined(step, first)
+    results = step.host_results()
+    step.logits_s.zero_()
+    step.logits_t.zero_()
+    for graph in (False, True):
+        for v in step.score.values():
+            v.zero_()
+        step.out8.zero_()
+        if graph:
+            step.capture_from_host(host, results, host_logits=True).replay()
+        else:
+            step.run_from_host(host, results, torch.cuda.current_stream(), host_logits=True)
+        torch.cuda.synchronize()
+        got = {k: v.cpu() for k, v in step.score.items()}
+        for n in SCORE_REQ + ("source",):
+            assert torch.equal(got[n], first[n]), n
+            assert torch.equal(results[n], first[n]), n
+        for n in ("logp_s", "logp_t", "feedback", "kl_rev", "kl_fwd"):
+            assert torch.equal(got[n][em], first[n][em]), n
+        for n in ("covered", "margin"):
+            assert torch.equal(got[n][dec], first[n][dec]), n
+        assert torch.equal(step.out8.cpu(), o8)
+        assert torch.equal(results["out8"], o8)
+    assert lib.device_error() == 0
+    assert not lib.device_readable(torch.zeros(4))  # pageable host memory is not offered
