@@ -133,7 +133,8 @@ __device__ __forceinline__ unsigned long long warp_top32_u64(unsigned long long 
 // to the warp's buffer, which is cut back to its best K (by rank) when it
 // fills, and the warps' lists are merged by rank.
 // The needed-rows pass (kNeeded) reads only the rows that the verdict and the
-// emitted positions need.  Its grid is (2 R, max span): block (r, i) takes
+// emitted positions need (Sec. 3.2.3: the tokens after a request's first
+// state change are discarded; the loss sums over emitted tokens).  Its grid is (2 R, max span): block (r, i) takes
 // the verifier's row of request r's span position i and block (R + r, i) the
 // proposer's, so the blocks of position 0 of every request are dispatched
 // first (the verifiers' rows before the proposers'), then position 1, and
