@@ -1,4 +1,4 @@
-// Device helpers shared by the IPD kernels (sm_103a): mbarrier and bulk-copy
+// Device helpers shared by the IPD kernels (sm_103a): mbarrier, TMA and tcgen05
 // wrappers in inline PTX, bounded waits, bf16 unpacking.
 #pragma once
 #include <cuda_runtime.h>
@@ -87,26 +87,6 @@ IPD_DEVINL bool mbar_wait_bounded(uint64_t *bar, uint32_t parity) {
   return true;
 }
 
-// 1-D bulk copy global -> shared, completion signalled on an mbarrier
-// (transaction bytes).  src and dst 16-byte aligned, bytes a multiple of 16.
-IPD_DEVINL void bulk_g2s(void *dst_smem, const void *src_gmem, uint32_t bytes, uint64_t *bar) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
-          "r"(smem_u32(dst_smem)),
-      "l"(src_gmem), "r"(bytes), "r"(smem_u32(bar))
-      : "memory");
-}
-
-// Same, with an L2 eviction-priority hint (streamed data read exactly once).
-IPD_DEVINL void bulk_g2s_evict_first(void *dst_smem, const void *src_gmem, uint32_t bytes,
-                                     uint64_t *bar, uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], "
-      "[%1], %2, [%3], %4;" ::"r"(smem_u32(dst_smem)),
-      "l"(src_gmem), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
-      : "memory");
-}
-
 IPD_DEVINL uint64_t l2_policy_evict_first() {
   uint64_t p;
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
@@ -144,18 +124,9 @@ static constexpr float kLn2 = 0.6931471805599453f;
 // ---------------------------------------------------------------------------
 // TMA tensor copies and 5th-generation tensor cores (tcgen05, TMEM)
 // ---------------------------------------------------------------------------
-// 2-D tiled TMA load into shared memory; completion counted on an mbarrier.
-// The tensor map is a __grid_constant__ kernel parameter (generic address).
-IPD_DEVINL void tma_load_2d(void *dst_smem, const void *tmap, int x, int y, uint64_t *bar,
-                            uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(smem_u32(dst_smem)),
-      "l"(tmap), "r"(x), "r"(y), "r"(smem_u32(bar)), "l"(policy)
-      : "memory");
-}
-
-// 4-D tiled TMA load (coordinates x, y, z, w), same conventions as above.
+// 4-D tiled TMA load into shared memory (coordinates x, y, z, w); completion
+// counted on an mbarrier.  The tensor map is a __grid_constant__ kernel
+// parameter (generic address).
 IPD_DEVINL void tma_load_4d(void *dst_smem, const void *tmap, int x, int y, int z, int w,
                             uint64_t *bar, uint64_t policy) {
   asm volatile(
@@ -300,29 +271,12 @@ IPD_DEVINL void tc_st_32x32b_x32(uint32_t taddr, const uint32_t (&r)[32]) {
       : "memory");
 }
 
-// Each lane of the warp writes 16 consecutive 32-bit TMEM columns of its lane.
-IPD_DEVINL void tc_st_32x32b_x16(uint32_t taddr, const uint32_t (&r)[16]) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
-      "%14,%15,%16};" ::"r"(taddr),
-      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
-      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
-      "r"(r[15])
-      : "memory");
-}
-
 // Each lane of the warp writes 8 consecutive 32-bit TMEM columns of its lane.
 IPD_DEVINL void tc_st_32x32b_x8(uint32_t taddr, const uint32_t (&r)[8]) {
   asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr),
                "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]),
                "r"(r[7])
                : "memory");
-}
-
-// Two floats truncated to their upper 16 bits (bf16 rounded toward zero) and
-// packed, the first in the low half.  Integer byte permute only.
-IPD_DEVINL uint32_t pack_bf16x2_trunc(float lo, float hi) {
-  return __byte_perm(__float_as_uint(lo), __float_as_uint(hi), 0x7632);
 }
 
 // Packed fp32 pairs (Blackwell f32x2 arithmetic): a 64-bit register holds
@@ -374,25 +328,3 @@ IPD_DEVINL uint32_t pack_bf16x2(float lo, float hi) {
   return d;
 }
 
-// Non-blocking test of an mbarrier phase.
-IPD_DEVINL bool mbar_test(uint64_t *bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-
-// Lane 0 tests the phase and the warp follows its answer; on success every
-// lane then observes the (completed, so immediate) phase itself.
-IPD_DEVINL bool warp_test(uint64_t *bar, uint32_t parity) {
-  uint32_t r = 0;
-  if ((threadIdx.x & 31) == 0) r = mbar_test(bar, parity) ? 1u : 0u;
-  r = __shfl_sync(0xffffffffu, r, 0);
-  if (r) (void)mbar_try_wait(bar, parity);
-  return r != 0;
-}
