@@ -85,3 +85,32 @@ def test_checker_rejects_planted_mistakes(pool):
     step.out8[0] *= 1.001                # the loss 1e-3 off
     rep = check_step_full(step, pool=pool)
     assert rep["score_ok"] and not rep["loss_ok"]
+
+
+def test_needed_positions_checker():
+    """check_scores(needed=True) ignores the values a needed-rows pass leaves
+    undefined (NaN past each transition) and still catches a wrong value at
+    an emitted position or a wrong coverage up to the transition."""
+    step = _oracle_filled_step()
+    orc = parity.oracle_scores(step, range(step.R))
+    src = step.score["source"].numpy()
+    cu = step.cu_span.numpy()
+    ft = step.score["first_trans"].numpy()
+    em = np.zeros(step.T, bool)
+    dec = np.zeros(step.T, bool)
+    for r in range(step.R):
+        e, d = parity.needed_positions(src, ft, cu, r)
+        em[cu[r]:cu[r + 1]], dec[cu[r]:cu[r + 1]] = e, d
+    assert (~dec).any() and (~em).any()  # the case has positions past transitions
+    for k in ("logp_s", "logp_t", "feedback", "kl_rev", "kl_fwd"):
+        step.score[k][torch.from_numpy(~em)] = float("nan")
+    step.score["margin"][torch.from_numpy(~dec)] = float("nan")
+    step.score["covered"][torch.from_numpy(~dec)] = 0
+    st, _ = parity.check_scores(step, None, orc=orc, needed=True)
+    assert st["score_ok"], st
+    st, _ = parity.check_scores(step, None, orc=orc)  # the full comparison sees the NaNs
+    assert not st["score_ok"]
+    t = int(np.flatnonzero(em)[0])
+    step.score["kl_rev"][t] += 1e-2
+    st, _ = parity.check_scores(step, None, orc=orc, needed=True)
+    assert not st["score_ok"] and st["max_kl_err"] > 1e-3
